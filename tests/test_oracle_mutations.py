@@ -1,0 +1,69 @@
+"""Planted mistakes in a copy of the oracle must each fail a pin.
+
+Each case rewrites one line of the oracle's C source into a plausible bug
+(a dropped term, a wrong sign or index, a swapped operand), compiles the copy
+into a temporary directory, swaps it in for the real library and runs one
+pin from test_oracle_pins, expecting that pin to fail. CPU only.
+"""
+import ctypes
+import os
+import subprocess
+
+import pytest
+
+from oracle import oracle as orc
+import test_oracle_pins as pins
+
+MUTATIONS = [
+    # (name, original text, planted mistake, pin expected to fail, args)
+    ("hash_zero_is_set", "int bit = acc > 0.0f;", "int bit = acc >= 0.0f;",
+     pins.test_sort_keys_hand_built_2d, ()),
+    ("gray_rank_or", "k ^= c;", "k |= c;",
+     pins.test_gray_rank_matches_reflected_gray_sequence, ()),
+    ("unstable_merge", "if (key[perm[b]] < key[perm[a]])",
+     "if (key[perm[b]] <= key[perm[a]])",
+     pins.test_stable_argsort_matches_numpy_stable, (1000, 32)),
+    ("missing_scale", "z[j] = s * scale;\n        if (z[j] > zmax) zmax = z[j];\n    }\n    int literal",
+     "z[j] = s;\n        if (z[j] > zmax) zmax = z[j];\n    }\n    int literal",
+     pins.test_single_block_is_dense_softmax_attention, (64, 16, 0)),
+    ("dropped_eps_sparse", "o[e] /= (den + floor_);", "o[e] /= den;",
+     pins.test_zero_sort_bits_is_block_diagonal_local_attention, (16,)),
+    ("next_key_block",
+     "block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)blk * b, b,\n"
+     "                  scale, eps, O_rows",
+     "block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)((blk + 1) %"
+     " (N / b)) * b, b,\n                  scale, eps, O_rows",
+     pins.test_query_block_t_attends_exactly_key_block_t, ()),
+    ("dropped_table_average", "den /= (double)L;", "",
+     pins.test_race_beta_zero_closed_form, ()),
+    ("phi_from_values", "race_phi(K + (size_t)j * d_h, d_h, w_l, gamma",
+     "race_phi(V + (size_t)j * d_h, d_h, w_l, gamma",
+     pins.test_race_matches_brute_force_kernel_matrix, (1.0,)),
+    ("tanh_dropped", "u[bb] = tanh(a);", "u[bb] = a;",
+     pins.test_race_feature_softmax_equals_product_identity, ()),
+    ("lambda_dropped", "d_s[k] + lam[k] * d_lr[k] + eps", "d_s[k] + d_lr[k] + eps",
+     pins.test_multiplier_direct_equals_log_domain_and_in_unit_interval, ()),
+    ("gate_swapped", "g_lr[k] * O_lr[(size_t)k * d_h + e]",
+     "g_s[k] * O_lr[(size_t)k * d_h + e]",
+     pins.test_gates_select_branches_and_ablation_sets_m_to_one, ()),
+]
+
+
+@pytest.mark.parametrize("name,old,new,pin,args", MUTATIONS,
+                         ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_is_caught(tmp_path, name, old, new, pin, args):
+    src = open(orc._SRC).read()
+    assert src.count(old) == 1, name
+    mutated = tmp_path / "mutant.c"
+    mutated.write_text(src.replace(old, new))
+    so = tmp_path / "libmutant.so"
+    subprocess.check_call(["gcc", "-O1", "-ffp-contract=off", "-fPIC",
+                           "-shared", "-std=c11", "-o", str(so),
+                           str(mutated), "-lm"])
+    saved = orc.lib()
+    orc._lib = orc.configure(ctypes.CDLL(os.fspath(so)))
+    try:
+        with pytest.raises(AssertionError):
+            pin(*args)
+    finally:
+        orc._lib = saved
