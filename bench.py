@@ -1,0 +1,417 @@
+#!/usr/bin/env python
+"""Benchmark of the ELSAA forward operator on GB300.
+
+One step = one elsaa_forward over the whole workload (all B*H heads: sort
+hash, stable sort, RACE summaries, block attention, RACE readout, fusion).
+Default workload: B=2, H=16, N=16384, d_h=128, bf16, block b=128, RACE
+r = 256 (L_s = 16, gamma = 4), non-causal. Prints ONE JSON line.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+--impl reference times the CPU oracle (fp64, host cores) on bounded samples
+of the same workload. Under torchrun (N > 1) every rank runs its own copy of
+the workload on its own GPU (heads are independent: no collective on the
+data path); rank 0 prints the aggregate.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import torch  # noqa: E402
+
+from paper_2607_20214_gb300 import perfmodel  # noqa: E402
+from paper_2607_20214_gb300.workloads import WORKLOADS, make_inputs  # noqa
+
+METRIC = "ELSAA fwd tokens/s at N=16K bf16 on 1 GB300"
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
+                  "bf16_tflops_sustained": 1700.0, "source": "fallback"}
+
+
+def load_peaks() -> dict:
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            d = json.load(f)
+        d["source"] = "measured"
+        return d
+    except OSError:
+        return dict(FALLBACK_PEAKS)
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons, sampled every 50 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,"
+              "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.samples = []
+        self.proc = None
+        self.device_index = device_index
+
+    def start(self):
+        cmd = ["nvidia-smi", "--query-gpu=" + self.FIELDS,
+               "--format=csv,noheader,nounits", "-lms", "50"]
+        uuid = None
+        try:
+            uuid = str(torch.cuda.get_device_properties(
+                self.device_index).uuid)
+        except Exception:
+            pass
+        if uuid:
+            cmd += ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        try:
+            self.proc = subprocess.Popen(cmd, stdout=subprocess.PIPE,
+                                         stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+            return
+        threading.Thread(target=self._read, daemon=True).start()
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.samples.append((time.time(), line.strip()))
+
+    def stop(self):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self, t0: float, t1: float) -> dict:
+        rows = []
+        for t, line in self.samples:
+            if t0 <= t <= t1:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [],
+                    "samples": 0}
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        mx = [num(r[2]) for r in rows if num(r[2]) is not None]
+        reasons = set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for r in rows:
+            for name, val in zip(names, r[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(rows)}
+
+
+def dist_setup(gpus: int):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def ncu_traffic(kernel: str, workload: str):
+    """Per-launch DRAM bytes from the committed ncu summary, if the kernel
+    source is unchanged since the counters were taken."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.json")
+    try:
+        with open(path) as f:
+            table = json.load(f)
+    except OSError:
+        return None
+    ent = table.get(kernel)
+    if not ent or ent.get("workload") != workload:
+        return None
+    src = os.path.join(ROOT, ent["source"])
+    try:
+        sha = hashlib.sha256(open(src, "rb").read()).hexdigest()[:16]
+    except OSError:
+        return None
+    if sha != ent.get("source_sha"):
+        return None
+    return ent.get("traffic_bytes_per_launch")
+
+
+def cpu_oracle_time(wl, x_cpu, heads, threads):
+    from oracle import oracle
+    p = oracle.params_from_workload(wl)
+    t0 = time.perf_counter()
+    res = oracle.forward(x_cpu, p, heads=heads, threads=threads)
+    return time.perf_counter() - t0, res
+
+
+def heads_to_cpu(x, heads):
+    """CPU copies of the listed (b, h) heads as a [1, n, N, d] batch."""
+    out = {}
+    for key in ("q", "k", "v"):
+        out[key] = torch.stack([x[key][b, h] for b, h in heads])[None].cpu()
+    out["w_sort"] = torch.stack([x["w_sort"][h] for _, h in heads]).cpu()
+    out["w_race"] = torch.stack([x["w_race"][h] for _, h in heads]).cpu()
+    return out
+
+
+def run_reference(args, wl):
+    """The CPU oracle as the reference arm: each step one bounded sample."""
+    world, rank, _ = dist_setup(args.gpus)
+    if rank != 0:
+        return 0
+    from oracle import oracle
+    oracle.build()
+    cores = os.cpu_count() or 1
+    per_step = max(1, min(wl.heads, cores))
+    x = make_inputs(wl.with_(B=1, H=min(wl.H, per_step)))
+    heads = [(0, h) for h in range(min(wl.H, per_step))]
+    times = []
+    for i in range(args.warmup + args.steps):
+        t, _ = cpu_oracle_time(wl, x, heads, threads=per_step)
+        if i >= args.warmup:
+            times.append(t)
+    t_step = statistics.mean(times)
+    # the sample covers len(heads) of the workload's B*H heads
+    value = wl.tokens * (len(heads) / wl.heads) / t_step
+    sample = "%d of %d heads (N=%d, d_h=%d) per step, %d threads" % (
+        len(heads), wl.heads, wl.N, wl.d_h, per_step)
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value,
+        "unit": "tokens/s", "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": t_step * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic",
+        "config": workload_config(wl),
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+def workload_config(wl):
+    return {"workload": "%s: B=%d H=%d N=%d d_h=%d %s b=%d r=%d "
+                        "(L_s=%d, gamma=%d) sort_bits=%d non-causal" % (
+                            wl.name, wl.B, wl.H, wl.N, wl.d_h, wl.dtype,
+                            wl.block, wl.r, wl.race_tables, wl.race_bits,
+                            wl.sort_bits),
+            "B": wl.B, "H": wl.H, "N": wl.N, "d_h": wl.d_h,
+            "block": wl.block, "r": wl.r, "global_batch": wl.B,
+            "seq_len": wl.N,
+            "l2": "no flush: Q+K+V = %.0f MB per step > 129 MB L2" % (
+                3 * wl.heads * wl.N * wl.d_h * wl.elt / 1e6)}
+
+
+def run_ours(args, wl):
+    from paper_2607_20214_gb300 import build as nvbuild
+    from paper_2607_20214_gb300 import elsaa
+
+    world, rank, local = dist_setup(args.gpus)
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    nvbuild.build()
+    elsaa.load_library()
+    peaks = load_peaks()
+
+    wl_rank = wl.with_(seed=wl.seed + 100 * rank)
+    x = make_inputs(wl_rank, device=dev)
+    p = elsaa.params_for(wl)
+    ws = elsaa.new_workspace(p, dev)
+    o = torch.empty_like(x["q"])
+    stream = torch.cuda.current_stream(dev)
+
+    def step():
+        elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                            x["w_race"], o=o, workspace=ws, stream=stream)
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    for _ in range(args.warmup):
+        step()
+    elsaa.elsaa_check_status(ws)
+    # time-based pre-roll so the clock record covers a loaded GPU
+    t_pre = time.time()
+    while time.time() - t_pre < 1.0:
+        step()
+        torch.cuda.synchronize(dev)
+    torch.cuda.synchronize(dev)
+    barrier()
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    elsaa.elsaa_profile_start()
+    ev0.record(stream)
+    for _ in range(args.steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    t_end = time.time()
+    barrier()
+    prof = elsaa.elsaa_profile_stop()
+    ms = ev0.elapsed_time(ev1)
+    elsaa.elsaa_check_status(ws)
+    sampler.stop()
+    clocks = sampler.summary(t_pre, t_end)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+    ms_step = ms / args.steps
+    value = world * wl.tokens / (ms_step / 1e3)
+
+    # dominant kernel roofline (device time of each launch, CUDA events on
+    # the launching stream over the timed region)
+    launches = sum(n for n, _ in prof.values())
+    dom = max(prof, key=lambda k: prof[k][1])
+    n_dom, ms_dom = prof[dom]
+    work = perfmodel.kernel_work(wl, dom)
+    roof = perfmodel.roofline(work, ms_dom / n_dom / 1e3, peaks)
+    roof["kernel"] = dom
+    roof["share_of_step"] = ms_dom / sum(v[1] for v in prof.values())
+    roof["peak_source"] = peaks.get("source", "measured")
+    roof["traffic"] = ncu_traffic(dom, wl.name)
+    roof["algorithmic"] = work["bytes"] if roof["bound"] == "hbm" else \
+        work["flops"]
+    kernels = {k: {"launches": n, "avg_us": 1e3 * t / n}
+               for k, (n, t) in sorted(prof.items())}
+
+    fm = perfmodel.flop_model(wl)
+    t_s = ms_step / 1e3
+    step_roof = max(fm["tensor_flops"] / (peaks["bf16_tflops"] * 1e12),
+                    fm["bytes"] / (peaks["hbm_gbs"] * 1e9)) / t_s
+
+    # end to end through the public API: pinned host inputs -> device ->
+    # forward -> host output, every step
+    e2e = None
+    if not args.no_e2e:
+        hx = {k: x[k].cpu().pin_memory() for k in ("q", "k", "v", "w_sort",
+                                                  "w_race")}
+        dx = {k: torch.empty_like(x[k]) for k in hx}
+        ho = torch.empty(o.shape, dtype=o.dtype).pin_memory()
+        h2d = sum(t.numel() * t.element_size() for t in hx.values())
+        d2h = ho.numel() * ho.element_size()
+
+        def e2e_step():
+            for k in hx:
+                dx[k].copy_(hx[k], non_blocking=True)
+            elsaa.elsaa_forward(p, dx["q"], dx["k"], dx["v"], dx["w_sort"],
+                                dx["w_race"], o=o, workspace=ws,
+                                stream=stream)
+            ho.copy_(o, non_blocking=True)
+
+        for _ in range(max(3, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize(dev)
+        barrier()
+        a = torch.cuda.Event(enable_timing=True)
+        bq = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        bq.record(stream)
+        torch.cuda.synchronize(dev)
+        barrier()
+        ms_e2e = a.elapsed_time(bq) / args.steps
+        if world > 1:
+            t = torch.tensor([ms_e2e], device=dev)
+            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+            ms_e2e = float(t.item())
+        e2e = {"value": world * wl.tokens / (ms_e2e / 1e3),
+               "unit": "tokens/s", "ms_per_step": ms_e2e,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+
+    # CPU oracle on the host cores (rank 0, N = 1): one whole step when it
+    # fits in the sample budget, also used as a parity spot check
+    cpu = None
+    err = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cores = os.cpu_count() or 1
+        n_heads = min(wl.heads, 2 * cores)
+        heads = [(i // wl.H, i % wl.H) for i in range(n_heads)]
+        xc = heads_to_cpu(x, heads)
+        t_cpu, res = cpu_oracle_time(wl, xc, [(0, j) for j in range(n_heads)],
+                                     threads=min(cores, n_heads))
+        cpu = {"value": wl.tokens * (n_heads / wl.heads) / t_cpu,
+               "unit": "tokens/s", "cores": min(cores, n_heads),
+               "kind": "oracle",
+               "sample": "%d of %d heads of one step (fp64 C oracle, "
+                         "threads over heads), %.1f s wall" % (
+                             n_heads, wl.heads, t_cpu)}
+        of = o.float()
+        err = 0.0
+        for j, (b, h) in enumerate(heads):
+            import numpy as np
+            err = max(err, float(np.abs(of[b, h].cpu().numpy() -
+                                        res[(0, j)]["O"]).max()))
+
+    if rank != 0:
+        return 0
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": workload_config(wl),
+        "tflops": fm["tensor_flops"] / t_s / 1e12,
+        "step_roofline_frac": step_roof,
+        "roofline": roof, "kernels": kernels,
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+        "max_abs_err_vs_oracle": err,
+    }
+    print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="c3", choices=sorted(WORKLOADS))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    wl = WORKLOADS[args.workload]
+    if args.impl == "reference":
+        return run_reference(args, wl)
+    return run_ours(args, wl)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

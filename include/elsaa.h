@@ -1,0 +1,167 @@
+/*
+ * elsaa.h - C ABI of the GB300 (sm_103a) ELSAA attention operator.
+ *
+ * ELSAA (Efficient Low-rank and Sparse Approximation of Attention) replaces
+ * dense attention after the Q/K/V projections by two branches and a fusion:
+ *   - the sortLSH sparse branch (Section 3.2; Algorithm "sortLSH Sparse Exact
+ *     Attention Branch"): angular-hash queries and keys, stably sort each by
+ *     hash key, cut both sorted orders into blocks of b, and let query block t
+ *     attend exactly to key block t, giving O_sparse and d_sparse;
+ *   - the RACE low-rank branch (Section 3.1; Algorithm "RACE Low-Rank
+ *     Attention Branch"): soft hypercube-hash features phi, bucket summaries
+ *     A = Phi_K^T 1 and B = Phi_K^T V per table, and the table-averaged readout
+ *     Num = Phi_Q B / L_s, Den = Phi_Q A / L_s, giving O_lr = Num / (Den + eps)
+ *     and d_lr = Den;
+ *   - the denominator-aware fusion (Eq. (5) and Eq. (6); Algorithm 1 steps
+ *     6-8): m = d_sparse / (d_sparse + lambda d_lr + eps),
+ *     O = g_sparse m O_sparse + g_lr O_lr.
+ * The N x N score matrix is never formed.
+ *
+ * Conventions for every entry point:
+ *   - All tensor pointers are DEVICE pointers owned by the caller; the
+ *     library allocates no memory. Scratch space comes from the caller through
+ *     the workspace argument, sized by elsaa_workspace_size().
+ *   - Calls are asynchronous on the caller's CUDA stream (cudaStream_t passed
+ *     as void*; NULL = the legacy default stream) and never synchronise.
+ *   - Arguments are validated on the host before any launch. The return value
+ *     is ELSAA_OK or one of the ELSAA_ERR_* codes; elsaa_last_error() then
+ *     holds a one-line description (thread-local).
+ *   - Tensors are contiguous row-major. Q, K, V and O are [B, H, N, d_h] of
+ *     the element type params.dtype; per-token arrays are [B, H, N].
+ */
+#ifndef ELSAA_H
+#define ELSAA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define ELSAA_ABI_VERSION 1
+
+/* Return codes. */
+#define ELSAA_OK 0
+#define ELSAA_ERR_INVALID_ARG 1  /* null pointer, bad size, N % b != 0 ... */
+#define ELSAA_ERR_UNSUPPORTED 2  /* valid per the paper, not built here    */
+#define ELSAA_ERR_WORKSPACE 3    /* workspace null or smaller than needed  */
+#define ELSAA_ERR_CUDA 4         /* a CUDA runtime call or launch failed   */
+#define ELSAA_ERR_DEVICE 5       /* a kernel reported a fault in-band      */
+
+/* Element type of Q, K, V and O. */
+#define ELSAA_BF16 0
+#define ELSAA_FP32 1
+
+/* Kernel family selection (params.impl). */
+#define ELSAA_IMPL_AUTO 0   /* tensor-core kernels where supported (bf16)   */
+#define ELSAA_IMPL_SIMT 1   /* fp32 CUDA-core kernels for every step        */
+
+typedef struct elsaa_params {
+    int B, H, N, d_h;   /* Q, K, V are [B, H, N, d_h] (Section 3)            */
+    int dtype;          /* ELSAA_BF16 or ELSAA_FP32                           */
+    int causal;         /* must be 0: the causal variant (Algorithm "Causal
+                           ELSAA") is not built; 1 -> ELSAA_ERR_UNSUPPORTED   */
+    int block_size;     /* b, keys per query (sortLSH block size; Table 7 "s").
+                           Requires N % b == 0 and b % 32 == 0, b <= 1024.    */
+    int sort_bits;      /* sortLSH hash bits n_s in [0, 8] (Table 7: 4-5);
+                           0 gives the identity order                         */
+    int gray_order;     /* 1: codes ordered by rank in the reflected Gray
+                           sequence (adjacent buckets differ in one bit);
+                           0: plain binary code order                         */
+    int race_tables;    /* L_s >= 1                                           */
+    int race_bits;      /* gamma in [1, 8]; R = 2^gamma buckets per table;
+                           L_s * R <= 1024                                    */
+    float beta;         /* RACE temperature beta >= 0                         */
+    float eps;          /* numerical floor epsilon > 0 (Table 7: 1e-6)        */
+    float scale;        /* score scale for sortLSH; 0 -> 1/sqrt(d_h)          */
+    float lambda;       /* scalar lambda >= 0, used when lambda_tok is NULL   */
+    int fusion_mode;    /* 0: ELSAA multiplier of Eq. (5);
+                           1: Sort_Lsh_RACE ablation, m := 1 (Section 5)      */
+    int impl;           /* ELSAA_IMPL_AUTO or ELSAA_IMPL_SIMT                 */
+} elsaa_params;
+
+/*
+ * Bytes of scratch memory elsaa_forward needs for these parameters.
+ * Returns ELSAA_OK and writes *bytes, or ELSAA_ERR_INVALID_ARG /
+ * ELSAA_ERR_UNSUPPORTED if the parameters would be rejected by
+ * elsaa_forward. No CUDA call is made.
+ */
+int elsaa_workspace_size(const elsaa_params *params, size_t *bytes);
+
+/*
+ * ELSAA forward pass for all B*H heads (Algorithm 1 steps 4-8, without the
+ * Q/K/V and output projections, which stay dense outside the operator).
+ *
+ * q, k, v      [B, H, N, d_h] of params->dtype (device, read only).
+ * w_sort       [H, sort_bits, d_h] fp32: planes of the angular sort hash,
+ *              shared by queries and keys of head h; may be NULL when
+ *              sort_bits == 0. Bit p of x is [<w_sort[h][p], x> > 0], the
+ *              projection evaluated as a sequential fp32 fused multiply-add
+ *              chain over i = 0..d_h-1.
+ * w_race       [H, L_s, gamma, d_h] fp32: Gaussian rows W^(l) of Algorithm
+ *              RACE. The tensor-core path rounds them to bf16; pass
+ *              bf16-representable values for bit-comparable results.
+ * lambda_tok   [B, H, N] fp32 per-token lambda_i >= 0, or NULL for the scalar
+ *              params->lambda (Section 3.3: fixed, learned scalar or
+ *              query-dependent).
+ * gates        [B, H, N, 2] fp32 (g_sparse, g_lr) per token, or NULL for
+ *              (1, 1). The paper's gates are sigma(G_theta(q_i)); the gate
+ *              network itself runs outside the operator.
+ * o            [B, H, N, d_h] of params->dtype (device, written).
+ * log_d_sparse [B, H, N] fp32 log of the sparse denominator, or NULL.
+ * d_lr         [B, H, N] fp32 low-rank denominator Den, or NULL.
+ * m_sparse     [B, H, N] fp32 multiplier of Eq. (5), or NULL.
+ * perm_q/k     [B, H, N] int32 sorted orders P_Q, P_K (sorted position ->
+ *              original index; equal keys by increasing index), or NULL.
+ * workspace    device scratch of at least elsaa_workspace_size() bytes,
+ *              256-byte aligned. Its contents need no initialisation.
+ * stream       cudaStream_t (as void*) on which all work is enqueued.
+ *
+ * Errors: ELSAA_ERR_INVALID_ARG / _UNSUPPORTED / _WORKSPACE before any
+ * launch; ELSAA_ERR_CUDA if a launch fails (the message names the kernel).
+ */
+int elsaa_forward(const elsaa_params *params, const void *q, const void *k,
+                  const void *v, const float *w_sort, const float *w_race,
+                  const float *lambda_tok, const float *gates, void *o,
+                  float *log_d_sparse, float *d_lr, float *m_sparse,
+                  int32_t *perm_q, int32_t *perm_k, void *workspace,
+                  size_t workspace_bytes, void *stream);
+
+/*
+ * Synchronises `stream` and reads the in-band status word that the kernels
+ * of the last elsaa_forward on this workspace wrote (bounded waits that ran
+ * out, inconsistent sort counts). Returns ELSAA_OK, ELSAA_ERR_DEVICE (with
+ * the recorded code in elsaa_last_error()) or ELSAA_ERR_CUDA.
+ */
+int elsaa_check_status(const void *workspace, void *stream);
+
+/*
+ * Per-kernel timing for measurement tools. Between elsaa_profile_start() and
+ * elsaa_profile_stop(), every kernel elsaa_forward launches is bracketed by
+ * a pair of CUDA events recorded on the caller's stream. elsaa_profile_stop
+ * waits for those events and writes one entry per kernel name (launch count,
+ * summed device milliseconds) into out[0..max_entries), setting *n_entries.
+ * Not for use during CUDA graph capture. Returns ELSAA_OK or ELSAA_ERR_CUDA.
+ */
+typedef struct elsaa_kernel_stat {
+    char name[32];
+    int launches;
+    double total_ms;
+} elsaa_kernel_stat;
+
+int elsaa_profile_start(void);
+int elsaa_profile_stop(elsaa_kernel_stat *out, int max_entries,
+                       int *n_entries);
+
+/* One-line description of the last error on this thread ("" if none). */
+const char *elsaa_last_error(void);
+
+/* ELSAA_ABI_VERSION of the loaded library. */
+int elsaa_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* ELSAA_H */

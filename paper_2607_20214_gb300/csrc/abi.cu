@@ -1,0 +1,351 @@
+// C ABI of libelsaa: argument validation, workspace plan, launch sequence.
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "internal.h"
+
+namespace elsaa {
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+int fail(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Optional per-launch event timing (elsaa_profile_start / _stop).
+struct ProfRec {
+    const char *name;
+    cudaEvent_t a, b;
+};
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+std::vector<ProfRec> g_prof;
+std::vector<cudaEvent_t> g_ev_pool;
+
+cudaEvent_t pool_event() {
+    if (!g_ev_pool.empty()) {
+        cudaEvent_t e = g_ev_pool.back();
+        g_ev_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    cudaEventCreate(&e);
+    return e;
+}
+
+// Launches `fn` on `st`, bracketed by events when profiling is on.
+template <typename F>
+cudaError_t timed(const char *name, cudaStream_t st, F fn) {
+    if (!g_prof_on) return fn();
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    ProfRec r{name, pool_event(), pool_event()};
+    cudaEventRecord(r.a, st);
+    cudaError_t e = fn();
+    cudaEventRecord(r.b, st);
+    g_prof.push_back(r);
+    return e;
+}
+
+// RACE key-chunk CTAs aimed for: about two per SM of a 152-SM GB300. A
+// constant (not a device query) keeps the workspace size device-independent.
+constexpr long kRaceTargetCtas = 304;
+
+}  // namespace
+
+int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
+    auto bad = [&](int code, const char *m) {
+        *msg = m;
+        return code;
+    };
+    if (!p) return bad(ELSAA_ERR_INVALID_ARG, "params is NULL");
+    if (p->B <= 0 || p->H <= 0 || p->N <= 0 || p->d_h <= 0)
+        return bad(ELSAA_ERR_INVALID_ARG, "B, H, N and d_h must be positive");
+    if (p->dtype != ELSAA_BF16 && p->dtype != ELSAA_FP32)
+        return bad(ELSAA_ERR_INVALID_ARG, "dtype must be ELSAA_BF16 or ELSAA_FP32");
+    if (p->causal != 0 && p->causal != 1)
+        return bad(ELSAA_ERR_INVALID_ARG, "causal must be 0 or 1");
+    if (p->causal)
+        return bad(ELSAA_ERR_UNSUPPORTED,
+                   "the causal variant is not built (causal must be 0)");
+    if (p->block_size <= 0)
+        return bad(ELSAA_ERR_INVALID_ARG, "block_size must be positive");
+    if (p->N % p->block_size != 0)
+        return bad(ELSAA_ERR_INVALID_ARG, "N must be a multiple of block_size");
+    if (p->block_size % 32 != 0 || p->block_size > 1024)
+        return bad(ELSAA_ERR_UNSUPPORTED,
+                   "block_size must be a multiple of 32 and at most 1024");
+    if (p->d_h != 32 && p->d_h != 64 && p->d_h != 128)
+        return bad(ELSAA_ERR_UNSUPPORTED, "d_h must be 32, 64 or 128");
+    if (p->sort_bits < 0 || p->sort_bits > 16)
+        return bad(ELSAA_ERR_INVALID_ARG, "sort_bits must be in [0, 16]");
+    if (p->sort_bits > 8)
+        return bad(ELSAA_ERR_UNSUPPORTED, "sort_bits above 8 are not built");
+    if (p->gray_order != 0 && p->gray_order != 1)
+        return bad(ELSAA_ERR_INVALID_ARG, "gray_order must be 0 or 1");
+    if (p->race_tables < 1 || p->race_bits < 1 || p->race_bits > 8)
+        return bad(ELSAA_ERR_INVALID_ARG,
+                   "race_tables must be >= 1 and race_bits in [1, 8]");
+    if ((long)p->race_tables << p->race_bits > 1024)
+        return bad(ELSAA_ERR_UNSUPPORTED, "race_tables * 2^race_bits > 1024");
+    if (!(p->beta >= 0.f) || !isfinite(p->beta))
+        return bad(ELSAA_ERR_INVALID_ARG, "beta must be finite and >= 0");
+    if (!(p->eps > 0.f) || !isfinite(p->eps))
+        return bad(ELSAA_ERR_INVALID_ARG, "eps must be finite and > 0");
+    if (!(p->scale >= 0.f) || !isfinite(p->scale))
+        return bad(ELSAA_ERR_INVALID_ARG, "scale must be finite and >= 0");
+    if (!(p->lambda >= 0.f) || !isfinite(p->lambda))
+        return bad(ELSAA_ERR_INVALID_ARG, "lambda must be finite and >= 0");
+    if (p->fusion_mode != 0 && p->fusion_mode != 1)
+        return bad(ELSAA_ERR_INVALID_ARG, "fusion_mode must be 0 or 1");
+    if (p->impl != ELSAA_IMPL_AUTO && p->impl != ELSAA_IMPL_SIMT)
+        return bad(ELSAA_ERR_INVALID_ARG, "impl must be AUTO or SIMT");
+    if ((long)p->B * p->H > 65535)
+        return bad(ELSAA_ERR_UNSUPPORTED, "B * H must be at most 65535");
+    if ((long)p->B * p->H * p->N > (1L << 31) - 1)
+        return bad(ELSAA_ERR_UNSUPPORTED, "B * H * N must fit in int32");
+
+    Plan &Q = *P;
+    Q.B = p->B;
+    Q.H = p->H;
+    Q.N = p->N;
+    Q.d = p->d_h;
+    Q.BH = p->B * p->H;
+    Q.dtype = p->dtype;
+    Q.b = p->block_size;
+    Q.n_s = p->sort_bits;
+    Q.bins = 1 << p->sort_bits;
+    Q.gray = p->gray_order;
+    Q.L = p->race_tables;
+    Q.gamma = p->race_bits;
+    Q.R = 1 << p->race_bits;
+    Q.r = Q.L * Q.R;
+    Q.tables_per_slice = Q.R >= kSliceBuckets ? 1 : kSliceBuckets / Q.R;
+    if (Q.R > kSliceBuckets)
+        return bad(ELSAA_ERR_UNSUPPORTED, "race_bits above 6 are not built");
+    Q.slices = (Q.L + Q.tables_per_slice - 1) / Q.tables_per_slice;
+    Q.beta = p->beta;
+    Q.eps = p->eps;
+    Q.scale = p->scale > 0.f ? p->scale : 1.0f / sqrtf((float)p->d_h);
+    Q.lambda = p->lambda;
+    Q.fusion_mode = p->fusion_mode;
+    Q.impl = 1;
+    Q.tiles = (Q.N + kHashTile - 1) / kHashTile;
+    // RACE key chunks: enough CTAs for about two waves, chunks of 32 keys.
+    {
+        long want = (kRaceTargetCtas + (long)Q.BH * Q.slices - 1) /
+                    ((long)Q.BH * Q.slices);
+        long maxS = (Q.N + 31) / 32;
+        long S = want < 1 ? 1 : (want > maxS ? maxS : want);
+        long chunk = ((Q.N + S - 1) / S + 31) / 32 * 32;
+        Q.chunk = (int)chunk;
+        Q.S = (int)((Q.N + chunk - 1) / chunk);
+    }
+    size_t BHN = (size_t)Q.BH * Q.N;
+    size_t off = 0;
+    Q.off_status = off;
+    off = align_up(off + sizeof(DeviceStatus), 256);
+    Q.off_keyrank = off;
+    off = align_up(off + 2 * BHN * sizeof(uint32_t), 256);
+    Q.off_hist = off;
+    off = align_up(off + (size_t)2 * Q.BH * Q.tiles * Q.bins * sizeof(int), 256);
+    Q.off_perm = off;
+    off = align_up(off + 2 * BHN * sizeof(int32_t), 256);
+    Q.off_part = off;
+    off = align_up(off + (size_t)Q.BH * Q.S * ((size_t)Q.r * Q.d + Q.r) *
+                             sizeof(float), 256);
+    Q.off_A = off;
+    off = align_up(off + (size_t)Q.BH * Q.r * sizeof(float), 256);
+    Q.off_B = off;
+    off = align_up(off + (size_t)Q.BH * Q.r * Q.d * sizeof(float), 256);
+    Q.off_Bh = off;
+    off = align_up(off + (size_t)Q.BH * Q.r * Q.d * sizeof(uint16_t), 256);
+    Q.total = off;
+    *msg = "";
+    return ELSAA_OK;
+}
+
+}  // namespace elsaa
+
+using namespace elsaa;
+
+extern "C" int elsaa_abi_version(void) { return ELSAA_ABI_VERSION; }
+
+extern "C" const char *elsaa_last_error(void) { return g_err; }
+
+extern "C" int elsaa_workspace_size(const elsaa_params *params,
+                                    size_t *bytes) {
+    g_err[0] = 0;
+    if (!bytes) return fail(ELSAA_ERR_INVALID_ARG, "bytes is NULL");
+    Plan P;
+    const char *msg = "";
+    int rc = make_plan(params, &P, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    *bytes = P.total;
+    return ELSAA_OK;
+}
+
+#define ELSAA_CHECK_LAUNCH(expr, name)                                       \
+    do {                                                                     \
+        cudaError_t e_ = (expr);                                             \
+        if (e_ != cudaSuccess)                                               \
+            return fail(ELSAA_ERR_CUDA, "%s: %s", name,                      \
+                        cudaGetErrorString(e_));                             \
+    } while (0)
+
+extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
+                             const void *k, const void *v,
+                             const float *w_sort, const float *w_race,
+                             const float *lambda_tok, const float *gates,
+                             void *o, float *log_d_sparse, float *d_lr,
+                             float *m_sparse, int32_t *perm_q,
+                             int32_t *perm_k, void *workspace,
+                             size_t workspace_bytes, void *stream) {
+    g_err[0] = 0;
+    Plan P;
+    const char *msg = "";
+    int rc = make_plan(params, &P, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    if (!q || !k || !v || !o)
+        return fail(ELSAA_ERR_INVALID_ARG, "q, k, v and o must be non-NULL");
+    if (!w_race) return fail(ELSAA_ERR_INVALID_ARG, "w_race must be non-NULL");
+    if (P.n_s > 0 && !w_sort)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "w_sort must be non-NULL when sort_bits > 0");
+    size_t elt = P.dtype == ELSAA_FP32 ? 4 : 2;
+    const void *ptrs[] = {q, k, v, o};
+    for (const void *p : ptrs)
+        if ((uintptr_t)p % elt)
+            return fail(ELSAA_ERR_INVALID_ARG,
+                        "q, k, v and o must be aligned to their element size");
+    if (!workspace)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if ((uintptr_t)workspace % 256)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if (workspace_bytes < P.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, P.total);
+
+    cudaStream_t st = (cudaStream_t)stream;
+    char *ws = (char *)workspace;
+    DeviceStatus *status = (DeviceStatus *)(ws + P.off_status);
+    uint32_t *keyrank = (uint32_t *)(ws + P.off_keyrank);
+    int *hist = (int *)(ws + P.off_hist);
+    int32_t *pq = perm_q ? perm_q : (int32_t *)(ws + P.off_perm);
+    int32_t *pk = perm_k ? perm_k
+                         : (int32_t *)(ws + P.off_perm) + (size_t)P.BH * P.N;
+    float *part = (float *)(ws + P.off_part);
+    float *A = (float *)(ws + P.off_A);
+    float *Bm = (float *)(ws + P.off_B);
+    uint16_t *Bh = (uint16_t *)(ws + P.off_Bh);
+
+    ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
+                       "status reset");
+    ELSAA_CHECK_LAUNCH(timed("sort_hash", st, [&] {
+                           return launch_sort_hash(P, q, k, w_sort, keyrank,
+                                                   hist, st);
+                       }),
+                       "sort_hash");
+    ELSAA_CHECK_LAUNCH(timed("sort_scan", st,
+                             [&] { return launch_sort_scan(P, hist, st); }),
+                       "sort_scan");
+    ELSAA_CHECK_LAUNCH(timed("sort_scatter", st, [&] {
+                           return launch_sort_scatter(P, keyrank, hist, pq,
+                                                      pk, status, st);
+                       }),
+                       "sort_scatter");
+    ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
+                           return launch_race_partial_simt(P, k, v, w_race,
+                                                           part, st);
+                       }),
+                       "race_partial_simt");
+    ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
+                           return launch_race_reduce(P, part, A, Bm, Bh, st);
+                       }),
+                       "race_reduce");
+    ELSAA_CHECK_LAUNCH(timed("block_attn_simt", st, [&] {
+                           return launch_block_attn_simt(
+                               P, q, k, v, w_race, pq, pk, A, Bm, lambda_tok,
+                               gates, o, log_d_sparse, d_lr, m_sparse,
+                               status, st);
+                       }),
+                       "block_attn_simt");
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_check_status(const void *workspace, void *stream) {
+    g_err[0] = 0;
+    if (!workspace) return fail(ELSAA_ERR_INVALID_ARG, "workspace is NULL");
+    cudaStream_t st = (cudaStream_t)stream;
+    cudaError_t e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess)
+        return fail(ELSAA_ERR_CUDA, "stream: %s", cudaGetErrorString(e));
+    DeviceStatus s;
+    e = cudaMemcpy(&s, workspace, sizeof(s), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess)
+        return fail(ELSAA_ERR_CUDA, "status read: %s", cudaGetErrorString(e));
+    if (s.code != 0)
+        return fail(ELSAA_ERR_DEVICE,
+                    "device status %d at site %d (info %d, %d)", s.code,
+                    s.where, s.info0, s.info1);
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_profile_start(void) {
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    g_prof_on = true;
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_profile_stop(elsaa_kernel_stat *out, int max_entries,
+                                  int *n_entries) {
+    g_err[0] = 0;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    g_prof_on = false;
+    std::vector<std::string> names;
+    std::vector<int> counts;
+    std::vector<double> ms;
+    int rc = ELSAA_OK;
+    for (auto &r : g_prof) {
+        float t = 0.f;
+        cudaError_t e = cudaEventSynchronize(r.b);
+        if (e == cudaSuccess) e = cudaEventElapsedTime(&t, r.a, r.b);
+        if (e != cudaSuccess && rc == ELSAA_OK)
+            rc = fail(ELSAA_ERR_CUDA, "profile: %s", cudaGetErrorString(e));
+        size_t i = 0;
+        while (i < names.size() && names[i] != r.name) ++i;
+        if (i == names.size()) {
+            names.push_back(r.name);
+            counts.push_back(0);
+            ms.push_back(0.0);
+        }
+        counts[i] += 1;
+        ms[i] += t;
+        g_ev_pool.push_back(r.a);
+        g_ev_pool.push_back(r.b);
+    }
+    g_prof.clear();
+    int n = 0;
+    for (size_t i = 0; i < names.size() && (int)i < max_entries; ++i, ++n) {
+        if (!out) break;
+        snprintf(out[i].name, sizeof(out[i].name), "%s", names[i].c_str());
+        out[i].launches = counts[i];
+        out[i].total_ms = ms[i];
+    }
+    if (n_entries) *n_entries = out ? n : (int)names.size();
+    return rc;
+}

@@ -1,0 +1,76 @@
+// Internal declarations shared by the CUDA translation units of libelsaa.
+// Nothing here is part of the public ABI (see include/elsaa.h).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/elsaa.h"
+
+namespace elsaa {
+
+// Tokens per hash tile: one CTA hashes, histograms and locally ranks one tile.
+constexpr int kHashTile = 128;
+// Queries per CTA of the CUDA-core block-attention kernel.
+constexpr int kSimtQT = 32;
+// Buckets per slice in the CUDA-core RACE kernels.
+constexpr int kSliceBuckets = 64;
+
+// In-band device status (first bytes of the workspace). code == 0: no fault.
+struct DeviceStatus {
+    int code;
+    int where;
+    int info0;
+    int info1;
+};
+// Status codes written by kernels (first writer wins).
+constexpr int kDevSortRange = 1;     // a scatter position fell outside [0, N)
+constexpr int kDevPermRange = 2;     // a permutation entry fell outside [0, N)
+constexpr int kDevWaitTimeout = 3;   // a bounded mbarrier wait ran out
+constexpr int kDevTmem = 4;          // tensor-memory allocation failed
+
+// Resolved problem geometry and workspace layout (all offsets in bytes).
+struct Plan {
+    int B, H, N, d, BH;
+    int dtype;
+    int b;           // block size
+    int n_s, bins;   // sort bits, 2^n_s
+    int gray;
+    int L, gamma, R, r;  // tables, bits, buckets per table, total buckets
+    int tables_per_slice, slices;
+    int S, chunk;    // RACE key chunks per head and tokens per chunk
+    int tiles;       // hash tiles per head
+    float beta, eps, scale, lambda;
+    int fusion_mode;
+    int impl;        // resolved: 1 = SIMT, 2 = tensor core
+    size_t off_status, off_keyrank, off_hist, off_perm, off_part, off_A,
+        off_B, off_Bh, total;
+};
+
+// Fills `plan` from validated parameters. Returns ELSAA_OK or an error code
+// and message (no CUDA calls).
+int make_plan(const elsaa_params *p, Plan *plan, const char **msg);
+
+// Launchers (return cudaError_t of the launch). Pointers are device pointers.
+cudaError_t launch_sort_hash(const Plan &P, const void *q, const void *k,
+                             const float *w_sort, uint32_t *keyrank,
+                             int *hist, cudaStream_t st);
+cudaError_t launch_sort_scan(const Plan &P, int *hist, cudaStream_t st);
+cudaError_t launch_sort_scatter(const Plan &P, const uint32_t *keyrank,
+                                const int *hist, int32_t *perm_q,
+                                int32_t *perm_k, DeviceStatus *status,
+                                cudaStream_t st);
+cudaError_t launch_race_partial_simt(const Plan &P, const void *k,
+                                     const void *v, const float *w_race,
+                                     float *part, cudaStream_t st);
+cudaError_t launch_race_reduce(const Plan &P, const float *part, float *A,
+                               float *Bm, uint16_t *Bh, cudaStream_t st);
+cudaError_t launch_block_attn_simt(
+    const Plan &P, const void *q, const void *k, const void *v,
+    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
+    const float *A, const float *Bm, const float *lambda_tok,
+    const float *gates, void *o, float *log_d_sparse, float *d_lr,
+    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+
+}  // namespace elsaa

@@ -1,0 +1,227 @@
+"""Python binding of the libelsaa C ABI (include/elsaa.h).
+
+Argument marshalling only: every step of the operator runs in the CUDA
+kernels of libelsaa.so. PyTorch provides device memory and streams. The
+functions keep the C names. If the library has not been built, every call
+raises RuntimeError; there is no fallback implementation.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from .build import LIB
+
+ELSAA_OK = 0
+ELSAA_ERR_INVALID_ARG = 1
+ELSAA_ERR_UNSUPPORTED = 2
+ELSAA_ERR_WORKSPACE = 3
+ELSAA_ERR_CUDA = 4
+ELSAA_ERR_DEVICE = 5
+ELSAA_BF16 = 0
+ELSAA_FP32 = 1
+ELSAA_IMPL_AUTO = 0
+ELSAA_IMPL_SIMT = 1
+
+SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
+           "elsaa_last_error", "elsaa_abi_version", "elsaa_profile_start",
+           "elsaa_profile_stop")
+
+
+class elsaa_params(ctypes.Structure):
+    """Mirror of struct elsaa_params (field order and types must match)."""
+    _fields_ = [
+        ("B", ctypes.c_int), ("H", ctypes.c_int), ("N", ctypes.c_int),
+        ("d_h", ctypes.c_int), ("dtype", ctypes.c_int),
+        ("causal", ctypes.c_int), ("block_size", ctypes.c_int),
+        ("sort_bits", ctypes.c_int), ("gray_order", ctypes.c_int),
+        ("race_tables", ctypes.c_int), ("race_bits", ctypes.c_int),
+        ("beta", ctypes.c_float), ("eps", ctypes.c_float),
+        ("scale", ctypes.c_float), ("lam", ctypes.c_float),
+        ("fusion_mode", ctypes.c_int), ("impl", ctypes.c_int),
+    ]
+
+
+class elsaa_kernel_stat(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 32), ("launches", ctypes.c_int),
+                ("total_ms", ctypes.c_double)]
+
+
+class ElsaaError(RuntimeError):
+    def __init__(self, code: int, msg: str):
+        super().__init__("libelsaa error %d: %s" % (code, msg))
+        self.code = code
+
+
+_lib = None
+
+
+def load_library(path: str = LIB) -> ctypes.CDLL:
+    """Load libelsaa.so (built in-tree by build.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(
+            "libelsaa.so is not built (%s); run "
+            "`python -c 'import __graft_entry__ as g; g.build()'`" % path)
+    L = ctypes.CDLL(path)
+    vp = ctypes.c_void_p
+    L.elsaa_workspace_size.argtypes = [ctypes.POINTER(elsaa_params),
+                                       ctypes.POINTER(ctypes.c_size_t)]
+    L.elsaa_workspace_size.restype = ctypes.c_int
+    L.elsaa_forward.argtypes = [ctypes.POINTER(elsaa_params)] + [vp] * 14 + [
+        ctypes.c_size_t, vp]
+    L.elsaa_forward.restype = ctypes.c_int
+    L.elsaa_check_status.argtypes = [vp, vp]
+    L.elsaa_check_status.restype = ctypes.c_int
+    L.elsaa_last_error.argtypes = []
+    L.elsaa_last_error.restype = ctypes.c_char_p
+    L.elsaa_abi_version.argtypes = []
+    L.elsaa_abi_version.restype = ctypes.c_int
+    L.elsaa_profile_start.argtypes = []
+    L.elsaa_profile_start.restype = ctypes.c_int
+    L.elsaa_profile_stop.argtypes = [ctypes.POINTER(elsaa_kernel_stat),
+                                     ctypes.c_int,
+                                     ctypes.POINTER(ctypes.c_int)]
+    L.elsaa_profile_stop.restype = ctypes.c_int
+    _lib = L
+    return L
+
+
+def elsaa_last_error() -> str:
+    return load_library().elsaa_last_error().decode()
+
+
+def elsaa_abi_version() -> int:
+    return load_library().elsaa_abi_version()
+
+
+def _check(rc: int):
+    if rc != ELSAA_OK:
+        raise ElsaaError(rc, elsaa_last_error())
+
+
+def make_params(B, H, N, d_h, dtype="bf16", block_size=64, sort_bits=5,
+                gray_order=1, race_tables=4, race_bits=4, beta=1.0, eps=1e-6,
+                scale=0.0, lam=1.0, fusion_mode=0, causal=0,
+                impl=ELSAA_IMPL_AUTO) -> elsaa_params:
+    dt = {"bf16": ELSAA_BF16, "fp32": ELSAA_FP32}[dtype] if isinstance(
+        dtype, str) else int(dtype)
+    return elsaa_params(B, H, N, d_h, dt, causal, block_size, sort_bits,
+                        gray_order, race_tables, race_bits, beta, eps, scale,
+                        lam, fusion_mode, impl)
+
+
+def params_for(wl, **over) -> elsaa_params:
+    """Parameters of a Workload (paper_2607_20214_gb300.workloads)."""
+    kw = dict(B=wl.B, H=wl.H, N=wl.N, d_h=wl.d_h, dtype=wl.dtype,
+              block_size=wl.block, sort_bits=wl.sort_bits,
+              gray_order=wl.gray_order, race_tables=wl.race_tables,
+              race_bits=wl.race_bits, beta=wl.beta, eps=wl.eps,
+              lam=wl.lam, fusion_mode=wl.fusion_mode, causal=wl.causal)
+    kw.update(over)
+    return make_params(**kw)
+
+
+def elsaa_workspace_size(params: elsaa_params) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load_library().elsaa_workspace_size(ctypes.byref(params),
+                                               ctypes.byref(n)))
+    return n.value
+
+
+def _ptr(t, name, dtype=None, numel=None, device=None):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError("%s must be a torch.Tensor" % name)
+    if device is not None and t.device != device:
+        raise ValueError("%s must be on %s (got %s)" % (name, device,
+                                                        t.device))
+    if not t.is_contiguous():
+        raise ValueError("%s must be contiguous" % name)
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError("%s must be %s (got %s)" % (name, dtype, t.dtype))
+    if numel is not None and t.numel() != numel:
+        raise ValueError("%s must have %d elements (got %d)" % (
+            name, numel, t.numel()))
+    return t.data_ptr()
+
+
+def new_workspace(params: elsaa_params, device) -> torch.Tensor:
+    """Caller-owned scratch of elsaa_workspace_size bytes (256-aligned)."""
+    n = elsaa_workspace_size(params)
+    return torch.empty(max(n, 256), dtype=torch.uint8, device=device)
+
+
+def elsaa_forward(params: elsaa_params, q, k, v, w_sort, w_race,
+                  lambda_tok=None, gates=None, o=None, log_d_sparse=None,
+                  d_lr=None, m_sparse=None, perm_q=None, perm_k=None,
+                  workspace=None, stream=None):
+    """Enqueue elsaa_forward on `stream` (default: torch's current stream).
+
+    Tensors are device tensors laid out as in include/elsaa.h. Returns o
+    (allocated here when not given). Raises ElsaaError on a non-zero return.
+    """
+    lib = load_library()
+    dev = q.device
+    if dev.type != "cuda":
+        raise ValueError("q must be a CUDA tensor")
+    tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    BHN = params.B * params.H * params.N
+    nqkv = BHN * params.d_h
+    if o is None:
+        o = torch.empty_like(q)
+    if workspace is None:
+        workspace = new_workspace(params, dev)
+    if stream is None:
+        stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    args = [
+        _ptr(q, "q", tdt, nqkv, dev), _ptr(k, "k", tdt, nqkv, dev),
+        _ptr(v, "v", tdt, nqkv, dev),
+        _ptr(w_sort, "w_sort", torch.float32,
+             params.H * params.sort_bits * params.d_h, dev)
+        if params.sort_bits > 0 else None,
+        _ptr(w_race, "w_race", torch.float32,
+             params.H * params.race_tables * params.race_bits * params.d_h,
+             dev),
+        _ptr(lambda_tok, "lambda_tok", torch.float32, BHN, dev),
+        _ptr(gates, "gates", torch.float32, 2 * BHN, dev),
+        _ptr(o, "o", tdt, nqkv, dev),
+        _ptr(log_d_sparse, "log_d_sparse", torch.float32, BHN, dev),
+        _ptr(d_lr, "d_lr", torch.float32, BHN, dev),
+        _ptr(m_sparse, "m_sparse", torch.float32, BHN, dev),
+        _ptr(perm_q, "perm_q", torch.int32, BHN, dev),
+        _ptr(perm_k, "perm_k", torch.int32, BHN, dev),
+        _ptr(workspace, "workspace", None, None, dev),
+    ]
+    rc = lib.elsaa_forward(ctypes.byref(params), *args,
+                           workspace.numel() * workspace.element_size(), sp)
+    _check(rc)
+    return o
+
+
+def elsaa_check_status(workspace: torch.Tensor, stream=None):
+    """Synchronise and raise ElsaaError if a kernel recorded a fault."""
+    lib = load_library()
+    if stream is None:
+        stream = torch.cuda.current_stream(workspace.device)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    _check(lib.elsaa_check_status(workspace.data_ptr(), sp))
+
+
+def elsaa_profile_start():
+    _check(load_library().elsaa_profile_start())
+
+
+def elsaa_profile_stop() -> dict:
+    """{kernel name: (launches, summed device ms)} since profile_start."""
+    arr = (elsaa_kernel_stat * 64)()
+    n = ctypes.c_int(0)
+    _check(load_library().elsaa_profile_stop(arr, 64, ctypes.byref(n)))
+    return {arr[i].name.decode(): (arr[i].launches, arr[i].total_ms)
+            for i in range(n.value)}

@@ -39,3 +39,55 @@ def flop_model(wl: Workload) -> dict:
         "hash_flops": 4 * N * d * wl.sort_bits * heads,
         "bytes": 4 * N * d * wl.elt * heads,
     }
+
+
+# CUDA-core fp32 peak of a 152-SM GB300 at its 2070 MHz maximum clock:
+# 152 SMs x 128 FP32 lanes x 2 FLOP per FMA x 2.07e9 / s.
+SIMT_FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def kernel_work(wl: Workload, kernel: str) -> dict:
+    """Algorithmic work of ONE launch of a kernel over the whole workload.
+
+    bytes: compulsory HBM traffic (each input element read once, each output
+    written once); flops: the kernel's share of the operator's arithmetic;
+    unit: which engine runs that arithmetic ("tensor" or "alu").
+    """
+    N, b, d, r = wl.N, wl.block, wl.d_h, wl.r
+    H = wl.heads
+    Lg = wl.race_tables * wl.race_bits
+    e = wl.elt
+    simt = kernel.endswith("_simt") or wl.dtype == "fp32"
+    if kernel.startswith("block_attn"):
+        by = H * 4 * N * d * e
+        fl = H * (4 * N * b * d + 2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
+    elif kernel.startswith("race_partial"):
+        by = H * 2 * N * d * e
+        fl = H * (2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
+    elif kernel.startswith("sort_hash"):
+        by = H * 2 * N * d * e
+        fl = H * 4 * N * d * wl.sort_bits
+        simt = True
+    else:
+        by = H * N * 8
+        fl = 0
+        simt = True
+    return {"bytes": by, "flops": fl, "unit": "alu" if simt else "tensor"}
+
+
+def roofline(work: dict, seconds: float, peaks: dict) -> dict:
+    """Bound, achieved and peak of one launch taking `seconds`."""
+    hbm = peaks["hbm_gbs"]
+    if work["unit"] == "tensor":
+        fpk = peaks["bf16_tflops"]
+    else:
+        fpk = SIMT_FP32_PEAK_TFLOPS
+    t_bytes = work["bytes"] / (hbm * 1e9)
+    t_flops = work["flops"] / (fpk * 1e12) if work["flops"] else 0.0
+    if t_bytes >= t_flops:
+        ach = work["bytes"] / seconds / 1e9
+        return {"bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s",
+                "frac": ach / hbm}
+    ach = work["flops"] / seconds / 1e12
+    return {"bound": work["unit"], "achieved": ach, "peak": fpk,
+            "unit": "TFLOP/s", "frac": ach / fpk}

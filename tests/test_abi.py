@@ -1,0 +1,128 @@
+"""The C-ABI library loads, exports what include/*.h declares, and rejects
+bad arguments on the host before any launch (no GPU needed, no compute)."""
+import ctypes
+import glob
+import os
+import re
+
+import pytest
+
+from paper_2607_20214_gb300 import build, elsaa
+from paper_2607_20214_gb300.workloads import WORKLOADS
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return elsaa.load_library()
+
+
+def declared_functions():
+    names = set()
+    for h in glob.glob(os.path.join(ROOT, "include", "*.h")):
+        src = re.sub(r"/\*.*?\*/", "", open(h).read(), flags=re.S)
+        names |= set(re.findall(r"\b(elsaa_\w+)\s*\(", src))
+    return names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert {"elsaa_forward", "elsaa_workspace_size", "elsaa_last_error",
+            "elsaa_check_status", "elsaa_abi_version"} <= names
+    for n in names:
+        assert hasattr(lib, n), n
+    assert set(elsaa.SYMBOLS) <= names
+
+
+def test_params_struct_matches_header():
+    src = open(os.path.join(ROOT, "include", "elsaa.h")).read()
+    body = src[src.index("typedef struct elsaa_params"):]
+    body = body[body.index("{") + 1:body.index("} elsaa_params;")]
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    fields = []
+    for decl in body.split(";"):
+        decl = decl.strip()
+        if not decl:
+            continue
+        typ, rest = decl.split(None, 1)
+        for name in rest.split(","):
+            fields.append((typ, name.strip()))
+    ct = {"int": ctypes.c_int, "float": ctypes.c_float}
+    assert len(fields) == len(elsaa.elsaa_params._fields_)
+    for (typ, name), (pname, ptype) in zip(fields,
+                                           elsaa.elsaa_params._fields_):
+        assert ct[typ] is ptype
+        assert name == pname or (name == "lambda" and pname == "lam")
+
+
+def test_abi_version(lib):
+    assert elsaa.elsaa_abi_version() == 1
+
+
+@pytest.mark.parametrize("name", sorted(WORKLOADS))
+def test_workspace_size_is_positive_and_deterministic(lib, name):
+    p = elsaa.params_for(WORKLOADS[name])
+    a = elsaa.elsaa_workspace_size(p)
+    assert a > 0 and a % 256 == 0
+    assert a == elsaa.elsaa_workspace_size(p)
+
+
+BAD = [
+    (dict(N=1000, block_size=64), elsaa.ELSAA_ERR_INVALID_ARG, "multiple"),
+    (dict(causal=1), elsaa.ELSAA_ERR_UNSUPPORTED, "causal"),
+    (dict(d_h=96), elsaa.ELSAA_ERR_UNSUPPORTED, "d_h"),
+    (dict(eps=0.0), elsaa.ELSAA_ERR_INVALID_ARG, "eps"),
+    (dict(lam=-1.0), elsaa.ELSAA_ERR_INVALID_ARG, "lambda"),
+    (dict(beta=float("nan")), elsaa.ELSAA_ERR_INVALID_ARG, "beta"),
+    (dict(block_size=48, N=96), elsaa.ELSAA_ERR_UNSUPPORTED, "block_size"),
+    (dict(sort_bits=12), elsaa.ELSAA_ERR_UNSUPPORTED, "sort_bits"),
+    (dict(sort_bits=-1), elsaa.ELSAA_ERR_INVALID_ARG, "sort_bits"),
+    (dict(race_bits=0), elsaa.ELSAA_ERR_INVALID_ARG, "race_bits"),
+    (dict(race_tables=64, race_bits=5), elsaa.ELSAA_ERR_UNSUPPORTED, "1024"),
+    (dict(fusion_mode=3), elsaa.ELSAA_ERR_INVALID_ARG, "fusion_mode"),
+    (dict(B=0), elsaa.ELSAA_ERR_INVALID_ARG, "positive"),
+]
+
+
+@pytest.mark.parametrize("over,code,word", BAD)
+def test_invalid_parameters_rejected(lib, over, code, word):
+    kw = dict(B=1, H=2, N=256, d_h=64, block_size=64, race_tables=4)
+    kw.update(over)
+    p = elsaa.make_params(**kw)
+    n = ctypes.c_size_t(0)
+    rc = lib.elsaa_workspace_size(ctypes.byref(p), ctypes.byref(n))
+    assert rc == code
+    assert word in elsaa.elsaa_last_error()
+
+
+def test_forward_rejects_null_and_small_workspace_before_launch(lib):
+    p = elsaa.make_params(B=1, H=1, N=256, d_h=64, block_size=64,
+                          race_tables=4)
+    fake = 1 << 20  # never dereferenced: validation fails first
+    args = [fake] * 5 + [None, None, fake, None, None, None, None, None]
+    rc = lib.elsaa_forward(ctypes.byref(p), *args, None, 0, None)
+    assert rc == elsaa.ELSAA_ERR_WORKSPACE
+    rc = lib.elsaa_forward(ctypes.byref(p), *args, fake, 256, None)
+    assert rc == elsaa.ELSAA_ERR_WORKSPACE
+    assert "too small" in elsaa.elsaa_last_error()
+    args_null = [None] + args[1:]
+    rc = lib.elsaa_forward(ctypes.byref(p), *args_null, fake, 1 << 40, None)
+    assert rc == elsaa.ELSAA_ERR_INVALID_ARG
+    p2 = elsaa.make_params(B=1, H=1, N=256, d_h=64, block_size=64,
+                           race_tables=4, dtype="fp32")
+    odd = [fake + 2] + args[1:]
+    rc = lib.elsaa_forward(ctypes.byref(p2), *odd, fake, 1 << 40, None)
+    assert rc == elsaa.ELSAA_ERR_INVALID_ARG
+    assert "aligned" in elsaa.elsaa_last_error()
+
+
+def test_missing_library_fails_loudly(tmp_path):
+    saved = elsaa._lib
+    elsaa._lib = None
+    try:
+        with pytest.raises(RuntimeError, match="not built"):
+            elsaa.load_library(str(tmp_path / "absent.so"))
+    finally:
+        elsaa._lib = saved

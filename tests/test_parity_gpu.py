@@ -1,0 +1,201 @@
+"""GPU (CUDA path through the C ABI) versus the fp64 CPU oracle.
+
+Both sides read the same seeded inputs. Sort orders must match exactly
+(integer work); outputs must lie within max-abs 1e-4 (fp32 inputs) or 2e-2
+(bf16 inputs), the tolerances the operator is specified to; the auxiliary
+denominators and multiplier are checked too. Small cases run the oracle on
+every row; the full-size workloads run the oracle on sampled heads and rows
+in the launch configuration the benchmark times.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as orc
+from paper_2607_20214_gb300 import build, elsaa
+from paper_2607_20214_gb300.workloads import (WORKLOADS, Workload,
+                                              make_gates_lambda, make_inputs)
+
+pytestmark = pytest.mark.gpu
+
+TOL_O = {"fp32": 1e-4, "bf16": 2e-2}
+TOL_LOGD = {"fp32": 2e-4, "bf16": 2e-2}
+TOL_M = {"fp32": 1e-4, "bf16": 1e-2}
+TOL_DLR_REL = {"fp32": 1e-4, "bf16": 1e-2}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    elsaa.load_library()
+
+
+def run_gpu(wl, x, gates=None, lam=None, impl=elsaa.ELSAA_IMPL_AUTO, **over):
+    dev = torch.device("cuda:0")
+    p = elsaa.params_for(wl, impl=impl, **over)
+    xd = {k: v.to(dev) for k, v in x.items()}
+    BHN = (wl.B, wl.H, wl.N)
+    out = dict(
+        log_d_sparse=torch.full(BHN, float("nan"), device=dev),
+        d_lr=torch.full(BHN, float("nan"), device=dev),
+        m_sparse=torch.full(BHN, float("nan"), device=dev),
+        perm_q=torch.full(BHN, -1, dtype=torch.int32, device=dev),
+        perm_k=torch.full(BHN, -1, dtype=torch.int32, device=dev),
+    )
+    ws = elsaa.new_workspace(p, dev)
+    o = elsaa.elsaa_forward(
+        p, xd["q"], xd["k"], xd["v"], xd["w_sort"], xd["w_race"],
+        lambda_tok=None if lam is None else lam.to(dev),
+        gates=None if gates is None else gates.to(dev), workspace=ws, **out)
+    elsaa.elsaa_check_status(ws)
+    torch.cuda.synchronize()
+    res = {k: v.cpu() for k, v in out.items()}
+    res["O"] = o.float().cpu()
+    return res
+
+
+def run_oracle(wl, x, gates=None, lam=None, heads=None, rows=None, **over):
+    p = orc.params_from_workload(wl, **over)
+    return orc.forward(x, p, lam=lam, gates=gates, heads=heads, rows=rows)
+
+
+def compare(wl, g, ref, rows=None, label=""):
+    """Element-wise comparison on the heads and rows the oracle computed."""
+    worst = 0.0
+    for (b, h), r in ref.items():
+        assert np.array_equal(g["perm_q"][b, h].numpy(), r["perm_q"]), \
+            (label, b, h, "perm_q")
+        assert np.array_equal(g["perm_k"][b, h].numpy(), r["perm_k"]), \
+            (label, b, h, "perm_k")
+        idx = r["rows"]
+        O = g["O"][b, h].numpy()[idx]
+        err = np.abs(O - r["O"]).max()
+        worst = max(worst, err)
+        assert err <= TOL_O[wl.dtype], (label, b, h, "O", err)
+        e_logd = np.abs(g["log_d_sparse"][b, h].numpy()[idx] -
+                        r["log_d_sparse"]).max()
+        assert e_logd <= TOL_LOGD[wl.dtype], (label, b, h, "logd", e_logd)
+        dl = g["d_lr"][b, h].numpy()[idx]
+        e_dlr = (np.abs(dl - r["d_lr"]) / np.abs(r["d_lr"])).max()
+        assert e_dlr <= TOL_DLR_REL[wl.dtype], (label, b, h, "d_lr", e_dlr)
+        e_m = np.abs(g["m_sparse"][b, h].numpy()[idx] - r["m"]).max()
+        assert e_m <= TOL_M[wl.dtype], (label, b, h, "m", e_m)
+    return worst
+
+
+def small(dtype="bf16", **kw):
+    base = dict(name="small", B=1, H=2, N=1184, d_h=64, dtype=dtype,
+                block=32, race_tables=4, recipe="plain", temperature=2.0,
+                seed=11, plane_seed=1011)
+    base.update(kw)
+    return Workload(**base)
+
+
+# --------------------------------------------------- small, every row
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("impl", [elsaa.ELSAA_IMPL_AUTO,
+                                  elsaa.ELSAA_IMPL_SIMT])
+def test_small_several_tiles_ragged_tail(dtype, impl):
+    wl = small(dtype)  # 1184 = 9 hash tiles of 128 + a ragged 32
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x, impl=impl), run_oracle(wl, x), label=dtype)
+
+
+@pytest.mark.parametrize("d_h,b,L,gamma", [(32, 32, 8, 3), (64, 64, 8, 4),
+                                           (128, 128, 16, 4),
+                                           (128, 256, 4, 4),
+                                           (64, 96, 3, 5), (128, 64, 2, 6)])
+def test_shapes(d_h, b, L, gamma):
+    wl = small("bf16", d_h=d_h, block=b, race_tables=L, race_bits=gamma,
+               N=b * 7, H=2, B=2)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="shape")
+
+
+def test_gates_and_per_token_lambda():
+    wl = small("fp32", H=3)
+    x = make_inputs(wl)
+    gates, lam = make_gates_lambda(wl, seed=5)
+    compare(wl, run_gpu(wl, x, gates=gates, lam=lam),
+            run_oracle(wl, x, gates=gates, lam=lam), label="gates")
+
+
+@pytest.mark.parametrize("over", [dict(fusion_mode=1), dict(sort_bits=0),
+                                  dict(gray_order=0), dict(sort_bits=8),
+                                  dict(beta=0.0), dict(beta=4.0),
+                                  dict(lam=0.0), dict(eps=1e-2),
+                                  dict(sort_bits=1)])
+def test_parameter_variants(over):
+    wl = small("fp32").with_(**over)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label=str(over))
+
+
+def test_single_block_and_minimum_size():
+    wl = small("fp32", N=32, block=32, B=3, H=1)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="min")
+    wl = small("bf16", N=256, block=256, d_h=128)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="oneblock")
+
+
+def test_duplicate_and_planted_recipes_small():
+    wl = WORKLOADS["c4"].with_(H=2, N=2048, block=256)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="dup")
+    wl = WORKLOADS["c2"].with_(B=1, H=4, N=1024)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="planted")
+
+
+def test_repeated_calls_are_deterministic():
+    wl = small("bf16", H=4)
+    x = make_inputs(wl)
+    a = run_gpu(wl, x)
+    b = run_gpu(wl, x)
+    for k in a:
+        assert torch.equal(a[k], b[k]) or (
+            a[k].isnan().all() and b[k].isnan().all()), k
+
+
+# ------------------------------------------------ the five workloads
+
+def test_c1_full():
+    wl = WORKLOADS["c1"]
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="c1")
+
+
+def test_c2_full_size_subset_of_heads():
+    wl = WORKLOADS["c2"]
+    x = make_inputs(wl)
+    heads = [(0, 0), (0, 1), (1, 2), (3, 3), (2, 10), (3, 11)]
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x, heads=heads), label="c2")
+
+
+@pytest.mark.parametrize("name,heads", [("c3", [(0, 0), (1, 15)]),
+                                        ("c4", [(0, 0), (0, 31)]),
+                                        ("c5", [(0, 0), (7, 11)])])
+def test_full_size_sampled_rows(name, heads):
+    """Full-size launch; exact perms of sampled heads; outputs on 512
+    sampled rows per head (plus the duplicated-key rows for c4)."""
+    wl = WORKLOADS[name]
+    x = make_inputs(wl, device="cuda")
+    g = run_gpu(wl, x)
+    rng = np.random.default_rng(0)
+    rows = np.unique(np.concatenate([
+        rng.choice(wl.N, 512, replace=False), [0, wl.N - 1],
+        np.arange(0, wl.N // 2, 64) if name == "c4" else []]).astype(
+            np.int32))
+    xs = {k: (v[[b for b, _ in heads]] if k in ("q", "k", "v") else v)
+          for k, v in x.items()}
+    # oracle on the sampled heads only (re-indexed batch entries)
+    ref = {}
+    for j, (b, h) in enumerate(heads):
+        sub = {k: (v[b:b + 1].cpu() if k in ("q", "k", "v") else v.cpu())
+               for k, v in x.items()}
+        r = run_oracle(wl.with_(B=1), sub, heads=[(0, h)], rows=rows)
+        ref[(b, h)] = r[(0, h)]
+    compare(wl, g, ref, label=name)
