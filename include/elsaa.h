@@ -129,6 +129,42 @@ int elsaa_forward(const elsaa_params *params, const void *q, const void *k,
                   size_t workspace_bytes, void *stream);
 
 /*
+ * elsaa_forward for callers that cannot allocate device memory.
+ *
+ * Not part of the paper's method (the paper has no counterpart); it exists
+ * for deployment. Some callers have no way to obtain scratch memory: a
+ * plug-in whose host application owns every device buffer and offers no
+ * allocator, or code on a latency-critical path that must not call
+ * cudaMalloc / cudaFree because those calls can synchronise the whole
+ * device. Such callers still own and pass the inputs and outputs exactly as
+ * for elsaa_forward (same meaning, layout and errors), but no workspace.
+ *
+ * Scratch comes from one fixed array of ELSAA_STATIC_WORKSPACE_BYTES inside
+ * the library's device image. Every GPU on which the library's kernels are
+ * loaded reserves that memory until the process exits.
+ *  - The first call on each device looks up the array's device address
+ *    (with that device current) and caches it; make that first call before
+ *    any stream capture.
+ *  - Problems whose elsaa_workspace_size() exceeds the array are rejected
+ *    with ELSAA_ERR_WORKSPACE (the message gives both sizes); nothing is
+ *    launched.
+ *  - All calls share the one array and it keeps the previous call's
+ *    contents. The forward pass writes every scratch value before reading
+ *    it (the status word is cleared at the start of each call). Calls whose
+ *    GPU work overlaps (other streams, other host threads without ordering)
+ *    race on the array and produce wrong results: order them on one stream.
+ *  - Allocates nothing: no cudaMalloc, cudaFree or allocating library call.
+ */
+#define ELSAA_STATIC_WORKSPACE_BYTES ((size_t)64 << 20)
+
+int elsaa_forward_noalloc(const elsaa_params *params, const void *q,
+                          const void *k, const void *v, const float *w_sort,
+                          const float *w_race, const float *lambda_tok,
+                          const float *gates, void *o, float *log_d_sparse,
+                          float *d_lr, float *m_sparse, int32_t *perm_q,
+                          int32_t *perm_k, void *stream);
+
+/*
  * Synchronises `stream` and reads the in-band status word that the kernels
  * of the last elsaa_forward on this workspace wrote (bounded waits that ran
  * out, inconsistent sort counts). Returns ELSAA_OK, ELSAA_ERR_DEVICE (with

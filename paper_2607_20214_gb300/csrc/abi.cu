@@ -178,6 +178,14 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     return ELSAA_OK;
 }
 
+int set_last_error(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return code;
+}
+
 }  // namespace elsaa
 
 using namespace elsaa;

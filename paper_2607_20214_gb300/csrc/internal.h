@@ -48,6 +48,9 @@ struct Plan {
         off_B, off_Bh, total;
 };
 
+// Records a one-line error for elsaa_last_error() and returns `code`.
+int set_last_error(int code, const char *fmt, ...);
+
 // Fills `plan` from validated parameters. Returns ELSAA_OK or an error code
 // and message (no CUDA calls).
 int make_plan(const elsaa_params *p, Plan *plan, const char **msg);

@@ -27,7 +27,9 @@ ELSAA_IMPL_SIMT = 1
 
 SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_last_error", "elsaa_abi_version", "elsaa_profile_start",
-           "elsaa_profile_stop")
+           "elsaa_profile_stop", "elsaa_forward_noalloc")
+# Size of the fixed scratch array behind elsaa_forward_noalloc.
+ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
 
 class elsaa_params(ctypes.Structure):
@@ -81,6 +83,9 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
     L.elsaa_last_error.restype = ctypes.c_char_p
     L.elsaa_abi_version.argtypes = []
     L.elsaa_abi_version.restype = ctypes.c_int
+    L.elsaa_forward_noalloc.argtypes = [ctypes.POINTER(elsaa_params)] + [
+        vp] * 13 + [vp]
+    L.elsaa_forward_noalloc.restype = ctypes.c_int
     L.elsaa_profile_start.argtypes = []
     L.elsaa_profile_start.restype = ctypes.c_int
     L.elsaa_profile_stop.argtypes = [ctypes.POINTER(elsaa_kernel_stat),
@@ -225,3 +230,49 @@ def elsaa_profile_stop() -> dict:
     _check(load_library().elsaa_profile_stop(arr, 64, ctypes.byref(n)))
     return {arr[i].name.decode(): (arr[i].launches, arr[i].total_ms)
             for i in range(n.value)}
+
+
+def elsaa_forward_noalloc(params: elsaa_params, q, k, v, w_sort, w_race,
+                          lambda_tok=None, gates=None, o=None,
+                          log_d_sparse=None, d_lr=None, m_sparse=None,
+                          perm_q=None, perm_k=None, stream=None):
+    """elsaa_forward without a workspace, for callers that cannot allocate
+    device memory (a host application that owns every buffer, or a path
+    that must not risk the device-wide synchronisation of cudaMalloc).
+
+    Scratch comes from the library's fixed ELSAA_STATIC_WORKSPACE_BYTES
+    array, shared by all calls: order overlapping calls on one stream. The
+    first call on a device looks up that array and should precede any
+    stream capture. `o` must be given (nothing is allocated here either).
+    """
+    lib = load_library()
+    if o is None:
+        raise ValueError("o must be given: elsaa_forward_noalloc allocates "
+                         "nothing")
+    dev = q.device
+    tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    BHN = params.B * params.H * params.N
+    nqkv = BHN * params.d_h
+    if stream is None:
+        stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    args = [
+        _ptr(q, "q", tdt, nqkv, dev), _ptr(k, "k", tdt, nqkv, dev),
+        _ptr(v, "v", tdt, nqkv, dev),
+        _ptr(w_sort, "w_sort", torch.float32,
+             params.H * params.sort_bits * params.d_h, dev)
+        if params.sort_bits > 0 else None,
+        _ptr(w_race, "w_race", torch.float32,
+             params.H * params.race_tables * params.race_bits * params.d_h,
+             dev),
+        _ptr(lambda_tok, "lambda_tok", torch.float32, BHN, dev),
+        _ptr(gates, "gates", torch.float32, 2 * BHN, dev),
+        _ptr(o, "o", tdt, nqkv, dev),
+        _ptr(log_d_sparse, "log_d_sparse", torch.float32, BHN, dev),
+        _ptr(d_lr, "d_lr", torch.float32, BHN, dev),
+        _ptr(m_sparse, "m_sparse", torch.float32, BHN, dev),
+        _ptr(perm_q, "perm_q", torch.int32, BHN, dev),
+        _ptr(perm_k, "perm_k", torch.int32, BHN, dev),
+    ]
+    _check(lib.elsaa_forward_noalloc(ctypes.byref(params), *args, sp))
+    return o
