@@ -260,7 +260,7 @@ def run_ours(args, wl):
     elsaa.elsaa_check_status(ws)
     # time-based pre-roll so the clock record covers a loaded GPU
     t_pre = time.time()
-    while time.time() - t_pre < 1.0:
+    while not args.no_preroll and time.time() - t_pre < 1.0:
         step()
         torch.cuda.synchronize(dev)
     torch.cuda.synchronize(dev)
@@ -404,10 +404,16 @@ def main():
     ap.add_argument("--workload", default="c3", choices=sorted(WORKLOADS))
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override B (smaller cases for profiler captures)")
+    ap.add_argument("--no-preroll", action="store_true",
+                    help="skip the 1 s loaded pre-roll (profiler captures)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     wl = WORKLOADS[args.workload]
+    if args.batch:
+        wl = wl.with_(B=args.batch)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_ours(args, wl)
