@@ -144,8 +144,12 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     Q.fusion_mode = p->fusion_mode;
     Q.impl = 1;
     Q.tiles = (Q.N + kHashTile - 1) / kHashTile;
-    // RACE key chunks: enough CTAs for about two waves, chunks of 32 keys.
-    {
+    if (p->impl == ELSAA_IMPL_AUTO && tc_supported(Q)) {
+        // tensor-core path: one wave of 128-key-tile chunks per head
+        Q.impl = 2;
+        Q.S = tc_race_chunks(Q, &Q.chunk);
+    } else {
+        // RACE key chunks: enough CTAs for about two waves, 32-key steps.
         long want = (kRaceTargetCtas + (long)Q.BH * Q.slices - 1) /
                     ((long)Q.BH * Q.slices);
         long maxS = (Q.N + 31) / 32;
@@ -276,22 +280,40 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                                       pk, status, st);
                        }),
                        "sort_scatter");
-    ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
-                           return launch_race_partial_simt(P, k, v, w_race,
-                                                           part, st);
-                       }),
-                       "race_partial_simt");
+    if (P.impl == 2) {
+        ELSAA_CHECK_LAUNCH(timed("race_keys_tc", st, [&] {
+                               return launch_race_keys_tc(P, k, v, w_race,
+                                                          part, status, st);
+                           }),
+                           "race_keys_tc");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
+                               return launch_race_partial_simt(P, k, v, w_race,
+                                                               part, st);
+                           }),
+                           "race_partial_simt");
+    }
     ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
                            return launch_race_reduce(P, part, A, Bm, Bh, st);
                        }),
                        "race_reduce");
-    ELSAA_CHECK_LAUNCH(timed("block_attn_simt", st, [&] {
-                           return launch_block_attn_simt(
-                               P, q, k, v, w_race, pq, pk, A, Bm, lambda_tok,
-                               gates, o, log_d_sparse, d_lr, m_sparse,
-                               status, st);
-                       }),
-                       "block_attn_simt");
+    if (P.impl == 2) {
+        ELSAA_CHECK_LAUNCH(timed("block_attn_tc", st, [&] {
+                               return launch_block_attn_tc(
+                                   P, q, k, v, w_race, pq, pk, A, Bh,
+                                   lambda_tok, gates, o, log_d_sparse, d_lr,
+                                   m_sparse, status, st);
+                           }),
+                           "block_attn_tc");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("block_attn_simt", st, [&] {
+                               return launch_block_attn_simt(
+                                   P, q, k, v, w_race, pq, pk, A, Bm,
+                                   lambda_tok, gates, o, log_d_sparse, d_lr,
+                                   m_sparse, status, st);
+                           }),
+                           "block_attn_simt");
+    }
     return ELSAA_OK;
 }
 

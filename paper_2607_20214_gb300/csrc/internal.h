@@ -76,4 +76,18 @@ cudaError_t launch_block_attn_simt(
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
     float *m_sparse, DeviceStatus *status, cudaStream_t st);
 
+// Tensor-core (tcgen05) path for bf16 inputs.
+bool tc_supported(const Plan &P);
+// Chunks per head of the tensor-core RACE key kernel; writes tokens per chunk.
+int tc_race_chunks(const Plan &P, int *chunk);
+cudaError_t launch_race_keys_tc(const Plan &P, const void *k, const void *v,
+                                const float *w_race, float *part,
+                                DeviceStatus *status, cudaStream_t st);
+cudaError_t launch_block_attn_tc(
+    const Plan &P, const void *q, const void *k, const void *v,
+    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
+    const float *A, const uint16_t *Bh, const float *lambda_tok,
+    const float *gates, void *o, float *log_d_sparse, float *d_lr,
+    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+
 }  // namespace elsaa

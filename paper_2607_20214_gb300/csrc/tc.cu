@@ -1,0 +1,676 @@
+// Tensor-core (tcgen05 / TMEM, bf16 in, fp32 accumulate) kernels of the
+// ELSAA forward for bf16 inputs.
+//
+//   k_race_keys_tc   RACE key side (Algorithm "RACE Low-Rank Attention
+//                    Branch", steps 3-7) over one chunk of keys of one head:
+//                    projections W^(l) K_j (MMA), soft-hash features phi
+//                    (CUDA cores), then B += Phi_K^T V and A += Phi_K^T 1
+//                    (MMAs accumulating in TMEM across the chunk).
+//   k_block_attn_tc  one CTA = 128 consecutive sorted query positions:
+//                    sortLSH block attention (Algorithm "sortLSH Sparse
+//                    Exact Attention Branch", block step), the RACE query
+//                    readout (Algorithm RACE, steps 9-10) and the fusion of
+//                    Eq. (5)-(6), written at the queries' original rows.
+//
+// Fusion trick of k_block_attn_tc: the fused row is
+//   O_i = c1_i * (P V)_i + c2_i * (Phi_Q B)_i,
+//   c1 = g_s m / (l + eps e^-M)      (P = exp(z - M) unnormalised, l = sum P)
+//   c2 = g_lr / (L_s (Den + eps)),
+// so the features are pre-scaled by c2/c1 and both MMAs accumulate into ONE
+// TMEM accumulator; the epilogue multiplies the row by c1.
+#include <type_traits>
+
+#include "device_common.cuh"
+#include "tc_common.cuh"
+
+namespace elsaa {
+
+namespace {
+
+using namespace tc;
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+__device__ __forceinline__ uint32_t align1k(uint32_t x) {
+    return (x + 1023u) & ~1023u;
+}
+
+// RACE planes of one head as bf16 rows [Lg_pad x d] in the panel layout;
+// rows >= Lg are zero.
+__device__ void load_planes_bf16(uint32_t dst, const float *w, int Lg,
+                                 int Lg_pad, int d, int tid, int nthreads) {
+    const int chunks = d >> 3;
+    for (int i = tid; i < Lg_pad * chunks; i += nthreads) {
+        int row = i / chunks, c = i - row * chunks;
+        uint32_t addr = dst + panel_offset(row, c, Lg_pad);
+        if (row < Lg) {
+            const float4 *src =
+                reinterpret_cast<const float4 *>(w + (size_t)row * d + c * 8);
+            float4 a = src[0], b = src[1];
+            float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
+            st_shared_bf16x8(addr, v);
+        } else {
+            st_shared_zero16(addr);
+        }
+    }
+}
+
+// Loads the projection row of this thread's TMEM lane (64 columns) and
+// turns it into per-bit factors sp[j] = sigmoid(2 beta tanh(a_j)) for the
+// L*G columns in use (sp of columns >= L*G is left unspecified).
+template <int G>
+__device__ __forceinline__ void race_bits_from_tmem(uint32_t taddr, int Lg,
+                                                    int Lg_pad, float beta,
+                                                    float (&sp)[64]) {
+    uint32_t pr[64];
+    uint32_t (&lo)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pr[0]);
+    uint32_t (&hi)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pr[32]);
+    tmem_ld32(taddr, lo);
+    if (Lg_pad > 32) tmem_ld32(taddr + 32, hi);
+    tmem_wait_ld();
+#pragma unroll
+    for (int j = 0; j < 64; ++j) {
+        if (j < Lg) {
+            float a = __uint_as_float(pr[j]);
+            // sigmoid(2 beta u) = 1/2 + tanh(beta u)/2
+            float t = tanh_approx(beta * tanh_approx(a));
+            sp[j] = fmaf(0.5f, t, 0.5f);
+        } else {
+            sp[j] = 0.5f;
+        }
+    }
+}
+
+// Features of table l from its G per-bit factors: phi[r] = prod_b (bit b of
+// r ? sp[b] : 1 - sp[b]), r < 2^G.
+template <int G>
+__device__ __forceinline__ void table_phi(const float *sp, float *phi) {
+    phi[0] = 1.0f;
+#pragma unroll
+    for (int b = 0; b < G; ++b) {
+        const float p = sp[b], q = 1.0f - p;
+#pragma unroll
+        for (int r = 0; r < (1 << b); ++r) {
+            phi[r + (1 << b)] = phi[r] * p;
+            phi[r] *= q;
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// RACE key side.
+template <int G>
+__global__ void __launch_bounds__(128, 1)
+    k_race_keys_tc(const uint16_t *__restrict__ kx,
+                   const uint16_t *__restrict__ vx,
+                   const float *__restrict__ w_race, int N, int d, int H,
+                   int L, int r_pad, int Lg_pad, int chunk, float beta,
+                   uint32_t tmem_cols, float *__restrict__ part,
+                   DeviceStatus *status) {
+    constexpr int R = 1 << G;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mb_proj, mb_acc;
+    __shared__ uint32_t tbase;
+    const int s = blockIdx.x, bh = blockIdx.y, S = gridDim.x;
+    const int h = bh % H;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int Lg = L * G, r = L * R;
+    const int nM = r_pad >> 7;  // 128-row tiles of the bucket dimension
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t tileB = 128u * d * 2u;
+    const uint32_t sW = base;
+    const uint32_t sOnes = sW + align1k(Lg_pad * d * 2);
+    const uint32_t sK0 = sOnes + 4096;
+    const uint32_t sV0 = sK0 + 2 * tileB;
+    const uint32_t sPhi = sV0 + 2 * tileB;
+
+    // TMEM columns: B accumulators [nM][d], A accumulators [nM][16], proj.
+    const uint32_t colA = nM * d;
+    const uint32_t colP = colA + nM * 16;
+
+    if (warp == 0) tmem_alloc(&tbase, tmem_cols);
+    if (tid == 0) {
+        mbar_init(&mb_proj, 1);
+        mbar_init(&mb_acc, 1);
+        fence_mbar_init();
+    }
+    load_planes_bf16(sW, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid, 128);
+    for (int i = tid; i < 4096 / 16; i += 128) {
+        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                         sOnes + i * 16),
+                     "r"(0x3F803F80u)
+                     : "memory");
+    }
+    const int c0 = s * chunk;
+    const int c1 = min(N, c0 + chunk);
+    const int ntiles = c1 > c0 ? (c1 - c0 + 127) / 128 : 0;
+    const uint16_t *kh = kx + (size_t)bh * N * d;
+    const uint16_t *vh = vx + (size_t)bh * N * d;
+
+    auto issue_tile = [&](int it, int stage) {
+        const int n0 = c0 + it * 128;
+        const int chunks = d >> 3;
+        for (int i = tid; i < 128 * chunks; i += 128) {
+            int row = i / chunks, c = i - row * chunks;
+            int n = min(n0 + row, N - 1);  // rows past the chunk are zeroed
+            uint32_t off = panel_offset(row, c, 128);
+            cp_async16(sK0 + stage * tileB + off, kh + (size_t)n * d + c * 8);
+            cp_async16(sV0 + stage * tileB + off, vh + (size_t)n * d + c * 8);
+        }
+    };
+    if (ntiles > 0) issue_tile(0, 0);
+    cp_async_commit();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t t = tbase;
+    const uint32_t lane = (uint32_t)(warp * 32) << 16;
+    const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
+    const uint32_t id_b = idesc_bf16(128, d, true, true);
+    const uint32_t id_a = idesc_bf16(128, 16, true, false);
+    bool ok = true;
+
+    for (int it = 0; it < ntiles && ok; ++it) {
+        const int stage = it & 1;
+        const uint32_t sK = sK0 + stage * tileB, sV = sV0 + stage * tileB;
+        if (it + 1 < ntiles) {
+            issue_tile(it + 1, stage ^ 1);
+            cp_async_commit();
+            cp_async_wait<1>();
+        } else {
+            cp_async_wait<0>();
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0 && ok) {
+            for (int k = 0; k < d / 16; ++k) {
+                uint32_t oa = (k >> 2) * 128 * 128 + (k & 3) * 32;
+                uint32_t ow = (k >> 2) * Lg_pad * 128 + (k & 3) * 32;
+                mma_ss(t + colP, smem_desc(sK + oa, 16, 1024),
+                       smem_desc(sW + ow, 16, 1024), id_proj, k > 0);
+            }
+            mma_commit(&mb_proj);
+        }
+        ok = mbar_wait(&mb_proj, it & 1, status, 11);
+        tc_fence_after();
+        // features of key row tid -> Phi tile row tid (bf16, MN-major A)
+        float sp[64];
+        race_bits_from_tmem<G>(t + lane + colP, Lg, Lg_pad, beta, sp);
+        const bool valid = c0 + it * 128 + tid < c1;
+        float buf[8];
+#pragma unroll
+        for (int l = 0; l < 64 / G; ++l) {
+            if (l < L) {
+                float phi[R];
+                table_phi<G>(&sp[l * G], phi);
+#pragma unroll
+                for (int q = 0; q < R; ++q) {
+                    const int pcol = l * R + q;
+                    buf[pcol & 7] = valid ? phi[q] : 0.0f;
+                    if ((pcol & 7) == 7)
+                        st_shared_bf16x8(
+                            sPhi + panel_offset(tid, pcol >> 3, 128), buf);
+                }
+            }
+        }
+        if ((r & 7) != 0) {  // partial last chunk (tables of < 8 buckets)
+            for (int q = r & 7; q < 8; ++q) buf[q] = 0.0f;
+            st_shared_bf16x8(sPhi + panel_offset(tid, r >> 3, 128), buf);
+        }
+        for (int c = (r + 7) >> 3; c < (r_pad >> 3); ++c)
+            st_shared_zero16(sPhi + panel_offset(tid, c, 128));
+        fence_proxy_async_smem();
+        tc_fence_before();
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+        if (tid == 0 && ok) {
+            for (int m = 0; m < nM; ++m) {
+                for (int k = 0; k < 8; ++k) {  // 128 keys, 16 per step
+                    uint64_t a = smem_desc(sPhi + 2 * m * 16384 + k * 2048,
+                                           16384, 1024);
+                    uint32_t acc = (it > 0 || k > 0) ? 1u : 0u;
+                    mma_ss(t + m * d, a,
+                           smem_desc(sV + k * 2048, 128 * 128, 1024), id_b,
+                           acc);
+                    mma_ss(t + colA + m * 16, a,
+                           smem_desc(sOnes + (k >> 2) * 2048 + (k & 3) * 32,
+                                     16, 1024),
+                           id_a, acc);
+                }
+            }
+            mma_commit(&mb_acc);
+        }
+        ok = mbar_wait(&mb_acc, it & 1, status, 12) && ok;
+        tc_fence_after();
+        ok = __syncthreads_and(ok);  // CTA-uniform loop control
+    }
+
+    // write this chunk's partial summaries
+    float *out = part + ((size_t)bh * S + s) * ((size_t)r * d + r);
+    if (ok && ntiles > 0) {
+        for (int m = 0; m < nM; ++m) {
+            const int row = m * 128 + tid;
+            for (int c = 0; c < d; c += 32) {
+                uint32_t v[32];
+                tmem_ld32(t + lane + m * d + c, v);
+                tmem_wait_ld();
+                if (row < r) {
+                    float4 *dst =
+                        reinterpret_cast<float4 *>(out + (size_t)row * d + c);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        dst[j] = make_float4(
+                            __uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
+                            __uint_as_float(v[4 * j + 2]),
+                            __uint_as_float(v[4 * j + 3]));
+                }
+            }
+            uint32_t a16[16];
+            tmem_ld16(t + lane + colA + m * 16, a16);
+            tmem_wait_ld();
+            if (row < r) out[(size_t)r * d + row] = __uint_as_float(a16[0]);
+        }
+    } else if (ntiles == 0) {
+        for (int i = tid; i < r * d + r; i += 128) out[i] = 0.0f;
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(t, tmem_cols);
+}
+
+// ---------------------------------------------------------------------------
+// Writes the pre-scaled features phi * scale of this thread's query row for
+// buckets [lo, hi) as packed bf16 pairs into TMEM, bucket lo at `taddr`.
+// lo is a multiple of 32 and hi a multiple of 16; buckets are flushed in
+// groups of 32 (16 columns), a last half group padded with zeros.
+template <int G>
+__device__ __forceinline__ void write_phi_tmem(const float (&sp)[64], int L,
+                                               float scale, int lo, int hi,
+                                               uint32_t taddr) {
+    constexpr int R = 1 << G;
+    const int r = L * R;
+    uint32_t buf[16];
+#pragma unroll
+    for (int l = 0; l < 64 / G; ++l) {
+        if (l < L) {
+            float phi[R];
+            table_phi<G>(&sp[l * G], phi);
+#pragma unroll
+            for (int q = 0; q < R; q += 2) {
+                const int p = l * R + q;  // even bucket index
+                const int slot = (p >> 1) & 15;
+                buf[slot] = pack_bf16x2(phi[q] * scale, phi[q + 1] * scale);
+                const bool last = p + 2 == r;
+                if (slot == 15 || last) {
+                    if (last) {
+#pragma unroll
+                        for (int z = 0; z < 16; ++z)
+                            if (z > slot) buf[z] = 0u;
+                    }
+                    const int g = p - 2 * slot;  // first bucket of the group
+                    if (g >= lo && g < hi)
+                        tmem_st16(taddr + ((g - lo) >> 1), buf);
+                }
+            }
+        }
+    }
+}
+
+template <int G>
+__global__ void __launch_bounds__(128)
+    k_block_attn_tc(const uint16_t *__restrict__ qx,
+                    const uint16_t *__restrict__ kx,
+                    const uint16_t *__restrict__ vx,
+                    const float *__restrict__ w_race,
+                    const int32_t *__restrict__ perm_q,
+                    const int32_t *__restrict__ perm_k,
+                    const float *__restrict__ Ag,
+                    const uint16_t *__restrict__ Bh,
+                    const float *__restrict__ lambda_tok,
+                    const float *__restrict__ gates, uint16_t *__restrict__ ox,
+                    float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
+                    float *__restrict__ m_out, int N, int d, int H, int b,
+                    int nk, int L, int Lg_pad, float beta, float eps,
+                    float scale, float lambda, int mode, uint32_t tmem_cols,
+                    DeviceStatus *status) {
+    constexpr int R = 1 << G;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mb;
+    __shared__ uint32_t tbase;
+    __shared__ int qidx[128];
+    __shared__ int kidx[256];
+    const int p0 = blockIdx.x * 128, bh = blockIdx.y, h = bh % H;
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int Lg = L * G, r = L * R;
+    const int kpos0 = b >= 128 ? (p0 / b) * b : p0;
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t sQ = base;                  // later: B summary [r x d]
+    const uint32_t sK = sQ + 128u * d * 2u;
+    const uint32_t sV = sK + (uint32_t)nk * d * 2u;  // W first, then V
+
+    if (warp == 0) tmem_alloc(&tbase, tmem_cols);
+    if (tid == 0) {
+        mbar_init(&mb, 1);
+        fence_mbar_init();
+    }
+    const int32_t *pq = perm_q + (size_t)bh * N;
+    const int32_t *pk = perm_k + (size_t)bh * N;
+    {
+        int pos = min(p0 + tid, N - 1);
+        int i = pq[pos];
+        if (i < 0 || i >= N) {
+            report(status, kDevPermRange, 3, bh, i);
+            i = 0;
+        }
+        qidx[tid] = i;
+    }
+    for (int j = tid; j < nk; j += 128) {
+        int pos = min(kpos0 + j, N - 1);
+        int i = pk[pos];
+        if (i < 0 || i >= N) {
+            report(status, kDevPermRange, 4, bh, i);
+            i = 0;
+        }
+        kidx[j] = i;
+    }
+    __syncthreads();
+    const uint16_t *qh = qx + (size_t)bh * N * d;
+    const uint16_t *kh = kx + (size_t)bh * N * d;
+    const uint16_t *vh = vx + (size_t)bh * N * d;
+    gather_rows(sQ, qh, qidx, 128, d, d, tid, 128);
+    gather_rows(sK, kh, kidx, nk, d, d, tid, 128);
+    cp_async_commit();
+    load_planes_bf16(sV, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid,
+                     128);
+    cp_async_wait<0>();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t t = tbase;
+    const uint32_t lane = (uint32_t)(warp * 32) << 16;
+    const uint32_t colO = (uint32_t)nk;
+    if (tid == 0) {
+        const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
+        const uint32_t id_s = idesc_bf16(128, nk, false, false);
+        for (int k = 0; k < d / 16; ++k) {
+            uint32_t oq = (k >> 2) * 128 * 128 + (k & 3) * 32;
+            uint32_t ow = (k >> 2) * Lg_pad * 128 + (k & 3) * 32;
+            uint32_t ok_ = (k >> 2) * nk * 128 + (k & 3) * 32;
+            uint64_t aq = smem_desc(sQ + oq, 16, 1024);
+            mma_ss(t + colO, aq, smem_desc(sV + ow, 16, 1024), id_proj, k > 0);
+            mma_ss(t, aq, smem_desc(sK + ok_, 16, 1024), id_s, k > 0);
+        }
+        mma_commit(&mb);
+    }
+    bool ok = mbar_wait(&mb, 0, status, 21);
+    ok = __syncthreads_and(ok);  // CTA-uniform from here on
+    tc_fence_after();
+    // Q, K and W are consumed: stream V into its slot and the bf16 B
+    // summary of this head into the Q/K slots while the softmax runs.
+    gather_rows(sV, vh, kidx, nk, d, d, tid, 128);
+    load_rows(sQ, Bh + (size_t)bh * r * d, r, d, d, tid, 128);
+    cp_async_commit();
+
+    // ---- RACE features of query row tid and Den = (1/L) sum phi . A
+    float sp[64];
+    race_bits_from_tmem<G>(t + lane + colO, Lg, Lg_pad, beta, sp);
+    const float *Ah = Ag + (size_t)bh * r;
+    float den = 0.0f;
+#pragma unroll
+    for (int l = 0; l < 64 / G; ++l) {
+        if (l < L) {
+            float phi[R];
+            table_phi<G>(&sp[l * G], phi);
+#pragma unroll
+            for (int q = 0; q < R; ++q)
+                den = fmaf(phi[q], __ldg(Ah + l * R + q), den);
+        }
+    }
+    den *= 1.0f / (float)L;
+
+    // ---- sparse branch: softmax of this row over its key block
+    const float sl2e = scale * kLog2e;
+    // keys of this query's block: all nk when b >= 128, else [klo, khi)
+    const int klo = b < 128 ? (tid / b) * b : 0;
+    const int khi = b < 128 ? klo + b : nk;
+    float mx = -INFINITY;
+    for (int c = 0; c < nk; c += 32) {
+        uint32_t v[32];
+        tmem_ld32(t + lane + c, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j)
+            if (c + j >= klo && c + j < khi)
+                mx = fmaxf(mx, __uint_as_float(v[j]));
+    }
+    const float M2 = mx * sl2e;  // row max in log2 units
+    float lsum = 0.0f;
+    for (int c = 0; c < nk; c += 32) {
+        uint32_t v[32];
+        tmem_ld32(t + lane + c, v);
+        tmem_wait_ld();
+        uint32_t pk16[16];
+#pragma unroll
+        for (int j = 0; j < 32; j += 2) {
+            float p0v = 0.0f, p1v = 0.0f;
+            if (c + j >= klo && c + j < khi)
+                p0v = ex2_approx(fmaf(__uint_as_float(v[j]), sl2e, -M2));
+            if (c + j + 1 >= klo && c + j + 1 < khi)
+                p1v = ex2_approx(fmaf(__uint_as_float(v[j + 1]), sl2e, -M2));
+            lsum += p0v + p1v;
+            pk16[j >> 1] = pack_bf16x2(p0v, p1v);
+        }
+        tmem_st16(t + lane + (c >> 1), pk16);  // P over the read columns
+    }
+    tmem_wait_st();
+
+    // ---- fusion scalars (Eq. (5) in log-sum-exp form, Eq. (6))
+    const int qpos = p0 + tid;
+    const bool qvalid = qpos < N;
+    const int qi = qidx[tid];
+    const size_t tok = (size_t)bh * N + qi;
+    const float log_ds = M2 * kLn2 + logf(lsum);
+    const float lam = (lambda_tok && qvalid) ? lambda_tok[tok] : lambda;
+    const float gs = (gates && qvalid) ? gates[2 * tok] : 1.0f;
+    const float gl = (gates && qvalid) ? gates[2 * tok + 1] : 1.0f;
+    const float msp = fusion_multiplier(log_ds, lam, den, eps, mode);
+    const float c1 = gs * msp / (lsum + eps * ex2_approx(-M2));
+    const float c1e = fmaxf(c1, 1e-30f);
+    const float c2 = gl / ((float)L * (den + eps));
+    const float ratio = c2 / c1e;
+
+    const int r0 = min(r, nk);  // buckets of the first Num pass
+    write_phi_tmem<G>(sp, L, ratio, 0, r0, t + lane + (nk >> 1));
+    tmem_wait_st();
+    cp_async_wait<0>();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (tid == 0 && ok) {
+        const uint32_t id_o = idesc_bf16(128, d, false, true);
+        for (int k = 0; k < nk / 16; ++k)  // O = P V
+            mma_ts(t + colO, t + k * 8,
+                   smem_desc(sV + k * 2048, (uint32_t)nk * 128, 1024), id_o,
+                   k > 0);
+        for (int k = 0; k < r0 / 16; ++k)  // O += Phi' B (first buckets)
+            mma_ts(t + colO, t + (nk >> 1) + k * 8,
+                   smem_desc(sQ + k * 2048, (uint32_t)r * 128, 1024), id_o,
+                   1);
+        mma_commit(&mb);
+    }
+    ok = ok && mbar_wait(&mb, 1, status, 22);
+    ok = __syncthreads_and(ok);
+    tc_fence_after();
+    const int phase = 0;  // third completion of the barrier
+    if (r > nk) {  // remaining buckets reuse the P columns
+        write_phi_tmem<G>(sp, L, ratio, nk, r, t + lane);
+        tmem_wait_st();
+        tc_fence_before();
+        __syncthreads();
+        tc_fence_after();
+        if (tid == 0 && ok) {
+            const uint32_t id_o = idesc_bf16(128, d, false, true);
+            for (int k = 0; k < (r - nk) / 16; ++k)
+                mma_ts(t + colO, t + k * 8,
+                       smem_desc(sQ + (uint32_t)nk * 128 + k * 2048,
+                                 (uint32_t)r * 128, 1024),
+                       id_o, 1);
+            mma_commit(&mb);
+        }
+        ok = ok && mbar_wait(&mb, phase, status, 23);
+        ok = __syncthreads_and(ok);
+        tc_fence_after();
+    }
+
+    // ---- epilogue: O row = c1 * accumulator, at the original query index
+    if (ok) {
+        uint16_t *orow = ox + tok * d;
+        for (int c = 0; c < d; c += 32) {
+            uint32_t v[32];
+            tmem_ld32(t + lane + colO + c, v);
+            tmem_wait_ld();
+            if (qvalid) {
+                uint4 *dst = reinterpret_cast<uint4 *>(orow + c);
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    uint4 w;
+                    w.x = pack_bf16x2(c1e * __uint_as_float(v[8 * j]),
+                                      c1e * __uint_as_float(v[8 * j + 1]));
+                    w.y = pack_bf16x2(c1e * __uint_as_float(v[8 * j + 2]),
+                                      c1e * __uint_as_float(v[8 * j + 3]));
+                    w.z = pack_bf16x2(c1e * __uint_as_float(v[8 * j + 4]),
+                                      c1e * __uint_as_float(v[8 * j + 5]));
+                    w.w = pack_bf16x2(c1e * __uint_as_float(v[8 * j + 6]),
+                                      c1e * __uint_as_float(v[8 * j + 7]));
+                    dst[j] = w;
+                }
+            }
+        }
+        if (qvalid) {
+            if (log_ds_out) log_ds_out[tok] = log_ds;
+            if (dlr_out) dlr_out[tok] = den;
+            if (m_out) m_out[tok] = msp;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(t, tmem_cols);
+}
+
+uint32_t pow2_cols(uint32_t n) {
+    uint32_t c = 32;
+    while (c < n) c <<= 1;
+    return c;
+}
+
+template <typename F>
+cudaError_t dispatch_gamma(int gamma, F f) {
+    switch (gamma) {
+        case 1: return f(std::integral_constant<int, 1>());
+        case 2: return f(std::integral_constant<int, 2>());
+        case 3: return f(std::integral_constant<int, 3>());
+        case 4: return f(std::integral_constant<int, 4>());
+        case 5: return f(std::integral_constant<int, 5>());
+        case 6: return f(std::integral_constant<int, 6>());
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+constexpr int kSmemPerSM = 233472;  // 228 KB of shared memory per SM
+
+// Dynamic shared memory that also caps residency at what TMEM allows.
+size_t smem_for(size_t need, uint32_t tmem_cols) {
+    int fit = 512 / (int)tmem_cols;  // CTAs whose TMEM fits on one SM
+    size_t cap = (size_t)kSmemPerSM / (fit + 1) + 1;
+    return need > cap ? need : cap;
+}
+
+}  // namespace
+
+bool tc_supported(const Plan &P) {
+    if (P.dtype != ELSAA_BF16) return false;
+    if (P.d != 64 && P.d != 128) return false;
+    if (!(P.b == 32 || P.b == 64 || P.b == 128 || P.b == 256)) return false;
+    if (P.gamma > 6 || P.L * P.gamma > 64) return false;
+    if (P.r % 16 != 0 || P.r > 256) return false;
+    return true;
+}
+
+int tc_race_chunks(const Plan &P, int *chunk) {
+    // TMEM use decides CTAs per SM; one wave of chunks over all heads.
+    int r_pad = (P.r + 127) / 128 * 128;
+    int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
+    uint32_t cols = pow2_cols((r_pad / 128) * (P.d + 16) + 64);
+    int per_sm = 512 / (int)cols;
+    size_t smem = 1024 + ((P.L * P.gamma + 15) / 16 * 16) * P.d * 2 + 4096 +
+                  4 * 128 * P.d * 2 + 128 * r_pad * 2;
+    int by_smem = (int)(kSmemPerSM / (smem + 1024));
+    if (by_smem < per_sm) per_sm = by_smem;
+    if (per_sm < 1) per_sm = 1;
+    long slots = 152L * per_sm;
+    int tiles = (P.N + 127) / 128;
+    int S = (int)(slots / P.BH);
+    if (S < 1) S = 1;
+    if (S > tiles) S = tiles;
+    int tiles_per = (tiles + S - 1) / S;
+    *chunk = tiles_per * 128;
+    return (P.N + *chunk - 1) / *chunk;
+}
+
+cudaError_t launch_race_keys_tc(const Plan &P, const void *k, const void *v,
+                                const float *w_race, float *part,
+                                DeviceStatus *status, cudaStream_t st) {
+    const int r_pad = (P.r + 127) / 128 * 128;
+    const int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
+    const uint32_t cols = pow2_cols((r_pad / 128) * (P.d + 16) + 64);
+    size_t need = 1024 + (size_t)lg_pad * P.d * 2 + 4096 +
+                  4 * (size_t)128 * P.d * 2 + (size_t)128 * r_pad * 2;
+    size_t smem = smem_for(need, cols);
+    dim3 grid(P.S, P.BH);
+    return dispatch_gamma(P.gamma, [&](auto g) {
+        constexpr int G = decltype(g)::value;
+        auto kern = k_race_keys_tc<G>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<grid, 128, smem, st>>>(
+            (const uint16_t *)k, (const uint16_t *)v, w_race, P.N, P.d, P.H,
+            P.L, r_pad, lg_pad, P.chunk, P.beta, cols, part, status);
+        return cudaGetLastError();
+    });
+}
+
+cudaError_t launch_block_attn_tc(
+    const Plan &P, const void *q, const void *k, const void *v,
+    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
+    const float *A, const uint16_t *Bh, const float *lambda_tok,
+    const float *gates, void *o, float *log_d_sparse, float *d_lr,
+    float *m_sparse, DeviceStatus *status, cudaStream_t st) {
+    const int nk = P.b >= 128 ? P.b : 128;
+    const int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
+    const uint32_t cols = pow2_cols((uint32_t)(nk + P.d));
+    (void)0;
+    size_t need = 1024 + (size_t)(128 + 2 * nk) * P.d * 2;
+    size_t smem = smem_for(need, cols);
+    dim3 grid((P.N + 127) / 128, P.BH);
+    return dispatch_gamma(P.gamma, [&](auto g) {
+        constexpr int G = decltype(g)::value;
+        auto kern = k_block_attn_tc<G>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<grid, 128, smem, st>>>(
+            (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
+            w_race, perm_q, perm_k, A, Bh, lambda_tok, gates, (uint16_t *)o,
+            log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, nk, P.L, lg_pad,
+            P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, cols, status);
+        return cudaGetLastError();
+    });
+}
+
+}  // namespace elsaa
