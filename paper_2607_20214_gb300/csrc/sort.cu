@@ -11,8 +11,8 @@
 //   sort_hash    one CTA per 128-token tile of (head, Q|K): hash, tile
 //                histogram, rank of each token among equal keys of its tile.
 //   sort_scan    one CTA per (head, Q|K): exclusive scan of the tile
-//                histograms in (bin, tile) order -> start offset of every
-//                (tile, bin) run in the sorted order.
+//                histograms stored bin-major ([bin][tile]) -> start offset
+//                of every (tile, bin) run in the sorted order.
 //   sort_scatter one CTA per tile: pos = offset[tile][key] + local rank,
 //                perm[pos] = token.
 #include "device_common.cuh"
@@ -22,79 +22,151 @@ namespace elsaa {
 namespace {
 
 template <typename T>
+__device__ __forceinline__ void unpack8(const uint4 &u, float *x);
+template <>
+__device__ __forceinline__ void unpack8<__nv_bfloat16>(const uint4 &u,
+                                                       float *x) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+
+template <>
+__device__ __forceinline__ void unpack8<float>(const uint4 &u, float *x) {
+    x[0] = __uint_as_float(u.x);
+    x[1] = __uint_as_float(u.y);
+    x[2] = __uint_as_float(u.z);
+    x[3] = __uint_as_float(u.w);
+}
+
+// One CTA hashes one 128-token tile of (head, Q|K). The tile is staged in
+// shared memory with coalesced 16-byte loads (16-byte chunks of each row
+// XOR-swizzled by the row index, so a warp reading one chunk of 32 rows is
+// conflict-free). Each thread then evaluates the NS projections of its
+// token as NS interleaved FMA chains; each chain keeps the canonical
+// sequential order i = 0..d-1. Ranks among equal keys of the tile come from
+// warp match masks plus per-warp counts.
+template <typename T, int NS>
 __global__ void __launch_bounds__(kHashTile)
     k_sort_hash(const T *__restrict__ q, const T *__restrict__ k,
                 const float *__restrict__ w_sort, int N, int d, int H,
-                int n_s, int bins, int gray, int tiles,
-                uint32_t *__restrict__ keyrank, int *__restrict__ hist) {
-    extern __shared__ float smem[];
+                int bins, int gray, int tiles, uint32_t *__restrict__ keyrank,
+                int *__restrict__ hist) {
+    extern __shared__ __align__(16) unsigned char smem[];
     const int tile = blockIdx.x, bh = blockIdx.y, which = blockIdx.z;
     const int BH = gridDim.y;
-    const int tid = threadIdx.x;
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int h = bh % H;
-    const int ds = d + 1;  // padded row stride: conflict-free column walks
-    float *xs = smem;                      // [kHashTile][d + 1]
-    float *ws = xs + kHashTile * ds;       // [n_s][d]
-    int *keys = (int *)(ws + n_s * d);     // [kHashTile]
-    int *hs = keys + kHashTile;            // [bins]
+    constexpr int kEl = 16 / sizeof(T);          // elements per 16-byte chunk
+    const int cpr = d / kEl;                     // chunks per row
+    const int swz = cpr >= 8 ? 7 : cpr - 1;      // swizzle mask
+    uint4 *xs = reinterpret_cast<uint4 *>(smem);               // [128][cpr]
+    float *ws = reinterpret_cast<float *>(xs + kHashTile * cpr);  // [NS][d]
+    int *cnt = reinterpret_cast<int *>(ws + NS * d);  // [4 warps][bins]
 
     const T *x = (which ? k : q) + (size_t)bh * N * d;
     const int n0 = tile * kHashTile;
-    for (int i = tid; i < kHashTile * d; i += kHashTile) {
-        int row = i / d, col = i - row * d;
-        int n = n0 + row;
-        xs[row * ds + col] = n < N ? to_f32<T>(x[(size_t)n * d + col]) : 0.f;
+    const uint4 *src = reinterpret_cast<const uint4 *>(x + (size_t)n0 * d);
+    const int valid_rows = min(kHashTile, N - n0);
+    const uint32_t xs_s = static_cast<uint32_t>(__cvta_generic_to_shared(xs));
+    for (int i = tid; i < kHashTile * cpr; i += kHashTile) {
+        int row = i / cpr, c = i - row * cpr;
+        uint32_t dst = xs_s + 16u * (row * cpr + (c ^ (row & swz)));
+        if (row < valid_rows)
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst),
+                         "l"(src + (size_t)row * cpr + c)
+                         : "memory");
+        else
+            xs[row * cpr + (c ^ (row & swz))] = make_uint4(0u, 0u, 0u, 0u);
     }
-    for (int i = tid; i < n_s * d; i += kHashTile)
-        ws[i] = w_sort[(size_t)h * n_s * d + i];
-    for (int i = tid; i < bins; i += kHashTile) hs[i] = 0;
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    for (int i = tid; i < NS * d; i += kHashTile)
+        ws[i] = w_sort[(size_t)h * NS * d + i];
+    for (int i = tid; i < 4 * bins; i += kHashTile) cnt[i] = 0;
+    asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
     const int n = n0 + tid;
-    int key = -1;
-    if (n < N) {
-        uint32_t code = 0;
-        const float *xr = xs + tid * ds;
-        for (int p = 0; p < n_s; ++p) {
-            // canonical projection: sequential fp32 FMA chain, i = 0..d-1
-            float acc = 0.0f;
-            const float *wp = ws + p * d;
-            for (int e = 0; e < d; ++e) acc = __fmaf_rn(wp[e], xr[e], acc);
-            code |= (acc > 0.0f ? 1u : 0u) << p;
-        }
-        key = (int)(gray ? gray_rank(code) : code);
+    float acc[NS > 0 ? NS : 1];
+#pragma unroll
+    for (int p = 0; p < NS; ++p) acc[p] = 0.0f;
+    const uint4 *xr = xs + tid * cpr;
+    const float4 *ws4 = reinterpret_cast<const float4 *>(ws);
+    for (int c = 0; c < cpr; ++c) {
+        float xv[kEl];
+        unpack8<T>(xr[c ^ (tid & swz)], xv);
+        const int e0 = c * kEl;
+        float wv[NS > 0 ? NS : 1][kEl];
+#pragma unroll
+        for (int p = 0; p < NS; ++p)
+#pragma unroll
+            for (int j = 0; j < kEl / 4; ++j) {
+                float4 w4 = ws4[(p * d + e0) / 4 + j];  // same for all lanes
+                wv[p][4 * j] = w4.x;
+                wv[p][4 * j + 1] = w4.y;
+                wv[p][4 * j + 2] = w4.z;
+                wv[p][4 * j + 3] = w4.w;
+            }
+#pragma unroll
+        for (int e = 0; e < kEl; ++e)
+#pragma unroll
+            for (int p = 0; p < NS; ++p)
+                acc[p] = __fmaf_rn(wv[p][e], xv[e], acc[p]);
     }
-    keys[tid] = key;
+    uint32_t code = 0;
+#pragma unroll
+    for (int p = 0; p < NS; ++p) code |= (acc[p] > 0.0f ? 1u : 0u) << p;
+    const int key = (int)(gray ? gray_rank(code) : code);
+    // rank among equal keys of the tile (lower index first)
+    const bool in = n < N;
+    const unsigned act = __ballot_sync(0xffffffffu, in);
+    unsigned peers = __match_any_sync(0xffffffffu, in ? key : -1) & act;
+    const int rank_w = __popc(peers & ((1u << lane) - 1u));
+    if (in && rank_w == 0) cnt[wid * bins + key] = __popc(peers);
     __syncthreads();
-    if (n < N) {
-        int rank = 0;
-        for (int j = 0; j < tid; ++j) rank += keys[j] == key;
-        atomicAdd(&hs[key], 1);
+    if (in) {
+        int rank = rank_w;
+        for (int w = 0; w < wid; ++w) rank += cnt[w * bins + key];
         keyrank[((size_t)which * BH + bh) * N + n] =
             (uint32_t)key | ((uint32_t)rank << 16);
     }
-    __syncthreads();
-    int *hout = hist + (((size_t)which * BH + bh) * tiles + tile) * bins;
-    for (int i = tid; i < bins; i += kHashTile) hout[i] = hs[i];
+    // tile histogram, stored bin-major ([bins][tiles]) so that the scan
+    // walks one contiguous array
+    int *hout = hist + ((size_t)which * BH + bh) * tiles * bins;
+    for (int i = tid; i < bins; i += kHashTile)
+        hout[(size_t)i * tiles + tile] = cnt[i] + cnt[bins + i] +
+                                         cnt[2 * bins + i] + cnt[3 * bins + i];
 }
 
 constexpr int kScanThreads = 1024;
 
+// Exclusive scan of the [bins][tiles] histogram of one (head, Q|K) in place:
+// entry (bin, tile) becomes the sorted position where that tile's run of
+// `bin` keys starts. Each thread owns one contiguous segment.
 __global__ void __launch_bounds__(kScanThreads)
     k_sort_scan(int *__restrict__ hist, int tiles, int bins) {
     __shared__ int warp_tot[32];
     const int tid = threadIdx.x;
-    int *hst = hist + (size_t)blockIdx.x * tiles * bins;  // [tiles][bins]
-    const long E = (long)tiles * bins;                    // bin-major order
-    const long per = (E + kScanThreads - 1) / kScanThreads;
-    const long e0 = tid * per;
-    const long e1 = e0 + per < E ? e0 + per : E;
+    int *hst = hist + (size_t)blockIdx.x * tiles * bins;
+    const int E = tiles * bins;
+    const int per = (E + kScanThreads - 1) / kScanThreads;
+    const int e0 = min(E, tid * per);
+    const int e1 = min(E, e0 + per);
     int sum = 0;
-    for (long e = e0; e < e1; ++e) {
-        int bin = (int)(e / tiles), t = (int)(e - (long)bin * tiles);
-        sum += hst[(size_t)t * bins + bin];
+    // 16-byte vector path when every segment start and end is 16-byte
+    // aligned (E and per multiples of 4; the workspace is 256-byte aligned)
+    const bool vec = ((per | E) & 3) == 0;
+    if (vec) {
+        for (int e = e0; e < e1; e += 4) {
+            int4 v = *reinterpret_cast<const int4 *>(hst + e);
+            sum += v.x + v.y + v.z + v.w;
+        }
+    } else {
+        for (int e = e0; e < e1; ++e) sum += hst[e];
     }
-    // block exclusive scan of per-thread sums
     const int lane = tid & 31, wid = tid >> 5;
     int incl = sum;
 #pragma unroll
@@ -116,11 +188,23 @@ __global__ void __launch_bounds__(kScanThreads)
     }
     __syncthreads();
     int run = warp_tot[wid] + incl - sum;
-    for (long e = e0; e < e1; ++e) {
-        int bin = (int)(e / tiles), t = (int)(e - (long)bin * tiles);
-        int c = hst[(size_t)t * bins + bin];
-        hst[(size_t)t * bins + bin] = run;
-        run += c;
+    if (vec) {
+        for (int e = e0; e < e1; e += 4) {
+            int4 v = *reinterpret_cast<const int4 *>(hst + e);
+            int4 o;
+            o.x = run;
+            o.y = o.x + v.x;
+            o.z = o.y + v.y;
+            o.w = o.z + v.z;
+            run = o.w + v.w;
+            *reinterpret_cast<int4 *>(hst + e) = o;
+        }
+    } else {
+        for (int e = e0; e < e1; ++e) {
+            int c = hst[e];
+            hst[e] = run;
+            run += c;
+        }
     }
 }
 
@@ -135,7 +219,8 @@ __global__ void __launch_bounds__(kHashTile)
     if (n >= N) return;
     uint32_t kr = keyrank[((size_t)which * BH + bh) * N + n];
     int key = (int)(kr & 0xffffu), rank = (int)(kr >> 16);
-    int pos = hist[(((size_t)which * BH + bh) * tiles + tile) * bins + key] +
+    int pos = hist[((size_t)which * BH + bh) * tiles * bins +
+                   (size_t)key * tiles + tile] +
               rank;
     if (pos < 0 || pos >= N) {
         report(status, kDevSortRange, 0, bh, pos);
@@ -145,31 +230,46 @@ __global__ void __launch_bounds__(kHashTile)
     perm[pos] = n;
 }
 
+template <typename T, int NS>
+cudaError_t launch_hash_t(const Plan &P, const void *q, const void *k,
+                          const float *w_sort, uint32_t *keyrank, int *hist,
+                          cudaStream_t st) {
+    dim3 grid(P.tiles, P.BH, 2);
+    size_t smem = (size_t)kHashTile * P.d * sizeof(T) +
+                  sizeof(float) * (size_t)NS * P.d + sizeof(int) * 4 * P.bins;
+    auto kern = k_sort_hash<T, NS>;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    kern<<<grid, kHashTile, smem, st>>>((const T *)q, (const T *)k, w_sort,
+                                        P.N, P.d, P.H, P.bins, P.gray,
+                                        P.tiles, keyrank, hist);
+    return cudaGetLastError();
+}
+
+template <typename T>
+cudaError_t launch_hash_dtype(const Plan &P, const void *q, const void *k,
+                              const float *w_sort, uint32_t *keyrank,
+                              int *hist, cudaStream_t st) {
+    switch (P.n_s) {
+#define ELSAA_NS_CASE(n) \
+    case n: return launch_hash_t<T, n>(P, q, k, w_sort, keyrank, hist, st);
+        ELSAA_NS_CASE(0) ELSAA_NS_CASE(1) ELSAA_NS_CASE(2) ELSAA_NS_CASE(3)
+        ELSAA_NS_CASE(4) ELSAA_NS_CASE(5) ELSAA_NS_CASE(6) ELSAA_NS_CASE(7)
+        ELSAA_NS_CASE(8)
+#undef ELSAA_NS_CASE
+        default: return cudaErrorInvalidValue;
+    }
+}
+
 }  // namespace
 
 cudaError_t launch_sort_hash(const Plan &P, const void *q, const void *k,
                              const float *w_sort, uint32_t *keyrank,
                              int *hist, cudaStream_t st) {
-    dim3 grid(P.tiles, P.BH, 2);
-    size_t smem = sizeof(float) * ((size_t)kHashTile * (P.d + 1) +
-                                   (size_t)P.n_s * P.d) +
-                  sizeof(int) * (kHashTile + P.bins);
-    if (P.dtype == ELSAA_FP32) {
-        auto kern = k_sort_hash<float>;
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-        kern<<<grid, kHashTile, smem, st>>>(
-            (const float *)q, (const float *)k, w_sort, P.N, P.d, P.H, P.n_s,
-            P.bins, P.gray, P.tiles, keyrank, hist);
-    } else {
-        auto kern = k_sort_hash<__nv_bfloat16>;
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-        kern<<<grid, kHashTile, smem, st>>>(
-            (const __nv_bfloat16 *)q, (const __nv_bfloat16 *)k, w_sort, P.N,
-            P.d, P.H, P.n_s, P.bins, P.gray, P.tiles, keyrank, hist);
-    }
-    return cudaGetLastError();
+    if (P.dtype == ELSAA_FP32)
+        return launch_hash_dtype<float>(P, q, k, w_sort, keyrank, hist, st);
+    return launch_hash_dtype<__nv_bfloat16>(P, q, k, w_sort, keyrank, hist,
+                                            st);
 }
 
 cudaError_t launch_sort_scan(const Plan &P, int *hist, cudaStream_t st) {

@@ -56,26 +56,30 @@ __device__ void load_planes_bf16(uint32_t dst, const float *w, int Lg,
     }
 }
 
-// Loads the projection row of this thread's TMEM lane (64 columns) and
-// turns it into per-bit factors sp[j] = sigmoid(2 beta tanh(a_j)) for the
-// L*G columns in use (sp of columns >= L*G is left unspecified).
-template <int G>
-__device__ __forceinline__ void race_bits_from_tmem(uint32_t taddr, int Lg,
-                                                    int Lg_pad, float beta,
-                                                    float (&sp)[64]) {
-    uint32_t pr[64];
-    uint32_t (&lo)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pr[0]);
-    uint32_t (&hi)[32] = *reinterpret_cast<uint32_t(*)[32]>(&pr[32]);
-    tmem_ld32(taddr, lo);
-    if (Lg_pad > 32) tmem_ld32(taddr + 32, hi);
+// Two threads share each row (warps w and w + 4 read the same TMEM lanes).
+// The RACE tables of a row are split between them at table `split`, chosen
+// so that each half's buckets start on a 32-bucket boundary (whole TMEM
+// store groups) and each half reads at most 32 projection columns.
+__host__ __device__ inline int table_split(int L, int G) {
+    const int R = 1 << G;
+    const int unit = R >= 32 ? 1 : 32 / R;  // tables per 32 buckets
+    int split = ((L + 1) / 2 + unit - 1) / unit * unit;
+    return split > L ? L : split;
+}
+
+// Per-bit factors sp[j] = sigmoid(2 beta tanh(a_j)) of the projection
+// columns [col0, col0 + 32) of this thread's TMEM lane; entries past `ncols`
+// are set to 1/2 and not used.
+__device__ __forceinline__ void race_bits32(uint32_t taddr, int ncols,
+                                           float beta, float (&sp)[32]) {
+    uint32_t pr[32];
+    tmem_ld32(taddr, pr);
     tmem_wait_ld();
 #pragma unroll
-    for (int j = 0; j < 64; ++j) {
-        if (j < Lg) {
-            float a = __uint_as_float(pr[j]);
-            // sigmoid(2 beta u) = 1/2 + tanh(beta u)/2
-            float t = tanh_approx(beta * tanh_approx(a));
-            sp[j] = fmaf(0.5f, t, 0.5f);
+    for (int j = 0; j < 32; ++j) {
+        if (j < ncols) {
+            float t = tanh_approx(beta * tanh_approx(__uint_as_float(pr[j])));
+            sp[j] = fmaf(0.5f, t, 0.5f);  // 1/2 + tanh(beta u)/2
         } else {
             sp[j] = 0.5f;
         }
@@ -99,9 +103,12 @@ __device__ __forceinline__ void table_phi(const float *sp, float *phi) {
 }
 
 // ---------------------------------------------------------------------------
-// RACE key side.
+// RACE key side. 256 threads: thread pairs (tid, tid ^ 128) share a key row
+// (a TMEM lane) and split its tables at table_split().
+constexpr int kTcThreads = 256;
+
 template <int G>
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(kTcThreads, 1)
     k_race_keys_tc(const uint16_t *__restrict__ kx,
                    const uint16_t *__restrict__ vx,
                    const float *__restrict__ w_race, int N, int d, int H,
@@ -115,8 +122,12 @@ __global__ void __launch_bounds__(128, 1)
     const int s = blockIdx.x, bh = blockIdx.y, S = gridDim.x;
     const int h = bh % H;
     const int tid = threadIdx.x, warp = tid >> 5;
+    const int grp = warp & 3, half = warp >> 2;
+    const int row = grp * 32 + (tid & 31);  // key row of the tile = TMEM lane
     const int Lg = L * G, r = L * R;
     const int nM = r_pad >> 7;  // 128-row tiles of the bucket dimension
+    const int split = table_split(L, G);
+    const int l0 = half ? split : 0, l1 = half ? L : split;
 
     const uint32_t base = align1k(smem_u32(smem_raw));
     const uint32_t tileB = 128u * d * 2u;
@@ -136,8 +147,9 @@ __global__ void __launch_bounds__(128, 1)
         mbar_init(&mb_acc, 1);
         fence_mbar_init();
     }
-    load_planes_bf16(sW, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid, 128);
-    for (int i = tid; i < 4096 / 16; i += 128) {
+    load_planes_bf16(sW, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid,
+                     kTcThreads);
+    for (int i = tid; i < 4096 / 16; i += kTcThreads) {
         asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
                          sOnes + i * 16),
                      "r"(0x3F803F80u)
@@ -152,10 +164,10 @@ __global__ void __launch_bounds__(128, 1)
     auto issue_tile = [&](int it, int stage) {
         const int n0 = c0 + it * 128;
         const int chunks = d >> 3;
-        for (int i = tid; i < 128 * chunks; i += 128) {
-            int row = i / chunks, c = i - row * chunks;
-            int n = min(n0 + row, N - 1);  // rows past the chunk are zeroed
-            uint32_t off = panel_offset(row, c, 128);
+        for (int i = tid; i < 128 * chunks; i += kTcThreads) {
+            int rr = i / chunks, c = i - rr * chunks;
+            int n = min(n0 + rr, N - 1);  // rows past the chunk are zeroed
+            uint32_t off = panel_offset(rr, c, 128);
             cp_async16(sK0 + stage * tileB + off, kh + (size_t)n * d + c * 8);
             cp_async16(sV0 + stage * tileB + off, vh + (size_t)n * d + c * 8);
         }
@@ -166,10 +178,11 @@ __global__ void __launch_bounds__(128, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t t = tbase;
-    const uint32_t lane = (uint32_t)(warp * 32) << 16;
+    const uint32_t lane = (uint32_t)(grp * 32) << 16;
     const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
     const uint32_t id_b = idesc_bf16(128, d, true, true);
     const uint32_t id_a = idesc_bf16(128, 16, true, false);
+    const bool tail_owner = (l1 == L) && (l1 > l0 || half == 0);
     bool ok = true;
 
     for (int it = 0; it < ntiles && ok; ++it) {
@@ -197,32 +210,35 @@ __global__ void __launch_bounds__(128, 1)
         }
         ok = mbar_wait(&mb_proj, it & 1, status, 11);
         tc_fence_after();
-        // features of key row tid -> Phi tile row tid (bf16, MN-major A)
-        float sp[64];
-        race_bits_from_tmem<G>(t + lane + colP, Lg, Lg_pad, beta, sp);
-        const bool valid = c0 + it * 128 + tid < c1;
+        // features of key `row`, tables [l0, l1) -> Phi tile row (bf16)
+        float sp[32];
+        race_bits32(t + lane + colP + l0 * G, (l1 - l0) * G, beta, sp);
+        const bool valid = c0 + it * 128 + row < c1;
         float buf[8];
 #pragma unroll
-        for (int l = 0; l < 64 / G; ++l) {
-            if (l < L) {
+        for (int lt = 0; lt < 32 / G; ++lt) {
+            if (l0 + lt < l1) {
                 float phi[R];
-                table_phi<G>(&sp[l * G], phi);
+                table_phi<G>(&sp[lt * G], phi);
 #pragma unroll
                 for (int q = 0; q < R; ++q) {
-                    const int pcol = l * R + q;
-                    buf[pcol & 7] = valid ? phi[q] : 0.0f;
-                    if ((pcol & 7) == 7)
+                    const int prel = lt * R + q;  // l0 * R is 32-aligned
+                    buf[prel & 7] = valid ? phi[q] : 0.0f;
+                    if ((prel & 7) == 7)
                         st_shared_bf16x8(
-                            sPhi + panel_offset(tid, pcol >> 3, 128), buf);
+                            sPhi + panel_offset(row, (l0 * R + prel) >> 3, 128),
+                            buf);
                 }
             }
         }
-        if ((r & 7) != 0) {  // partial last chunk (tables of < 8 buckets)
-            for (int q = r & 7; q < 8; ++q) buf[q] = 0.0f;
-            st_shared_bf16x8(sPhi + panel_offset(tid, r >> 3, 128), buf);
+        if (tail_owner) {
+            if ((r & 7) != 0) {  // partial last chunk (tables of < 8 buckets)
+                for (int q = r & 7; q < 8; ++q) buf[q] = 0.0f;
+                st_shared_bf16x8(sPhi + panel_offset(row, r >> 3, 128), buf);
+            }
+            for (int c = (r + 7) >> 3; c < (r_pad >> 3); ++c)
+                st_shared_zero16(sPhi + panel_offset(row, c, 128));
         }
-        for (int c = (r + 7) >> 3; c < (r_pad >> 3); ++c)
-            st_shared_zero16(sPhi + panel_offset(tid, c, 128));
         fence_proxy_async_smem();
         tc_fence_before();
         ok = __syncthreads_and(ok);
@@ -249,33 +265,35 @@ __global__ void __launch_bounds__(128, 1)
         ok = __syncthreads_and(ok);  // CTA-uniform loop control
     }
 
-    // write this chunk's partial summaries
+    // write this chunk's partial summaries (each half: half the columns)
     float *out = part + ((size_t)bh * S + s) * ((size_t)r * d + r);
     if (ok && ntiles > 0) {
         for (int m = 0; m < nM; ++m) {
-            const int row = m * 128 + tid;
-            for (int c = 0; c < d; c += 32) {
+            const int rrow = m * 128 + row;
+            for (int c = half * (d >> 1); c < (half + 1) * (d >> 1); c += 32) {
                 uint32_t v[32];
                 tmem_ld32(t + lane + m * d + c, v);
                 tmem_wait_ld();
-                if (row < r) {
+                if (rrow < r) {
                     float4 *dst =
-                        reinterpret_cast<float4 *>(out + (size_t)row * d + c);
+                        reinterpret_cast<float4 *>(out + (size_t)rrow * d + c);
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
-                        dst[j] = make_float4(
-                            __uint_as_float(v[4 * j]), __uint_as_float(v[4 * j + 1]),
-                            __uint_as_float(v[4 * j + 2]),
-                            __uint_as_float(v[4 * j + 3]));
+                        dst[j] = make_float4(__uint_as_float(v[4 * j]),
+                                             __uint_as_float(v[4 * j + 1]),
+                                             __uint_as_float(v[4 * j + 2]),
+                                             __uint_as_float(v[4 * j + 3]));
                 }
             }
-            uint32_t a16[16];
-            tmem_ld16(t + lane + colA + m * 16, a16);
-            tmem_wait_ld();
-            if (row < r) out[(size_t)r * d + row] = __uint_as_float(a16[0]);
+            if (half == 0) {
+                uint32_t a16[16];
+                tmem_ld16(t + lane + colA + m * 16, a16);
+                tmem_wait_ld();
+                if (rrow < r) out[(size_t)r * d + rrow] = __uint_as_float(a16[0]);
+            }
         }
     } else if (ntiles == 0) {
-        for (int i = tid; i < r * d + r; i += 128) out[i] = 0.0f;
+        for (int i = tid; i < r * d + r; i += kTcThreads) out[i] = 0.0f;
     }
     tc_fence_before();
     __syncthreads();
@@ -283,27 +301,29 @@ __global__ void __launch_bounds__(128, 1)
 }
 
 // ---------------------------------------------------------------------------
-// Writes the pre-scaled features phi * scale of this thread's query row for
-// buckets [lo, hi) as packed bf16 pairs into TMEM, bucket lo at `taddr`.
-// lo is a multiple of 32 and hi a multiple of 16; buckets are flushed in
-// groups of 32 (16 columns), a last half group padded with zeros.
+// Writes the pre-scaled features phi * scale of tables [l0, l1) of this
+// thread's query row, for buckets [lo, hi), as packed bf16 pairs into TMEM
+// with bucket lo at `taddr`. l0 * R and lo are multiples of 32 and hi of 16;
+// buckets go out in groups of 32 (16 columns), the last half group padded
+// with zeros.
 template <int G>
-__device__ __forceinline__ void write_phi_tmem(const float (&sp)[64], int L,
-                                               float scale, int lo, int hi,
+__device__ __forceinline__ void write_phi_tmem(const float (&sp)[32], int l0,
+                                               int l1, int r, float scale,
+                                               int lo, int hi,
                                                uint32_t taddr) {
     constexpr int R = 1 << G;
-    const int r = L * R;
     uint32_t buf[16];
 #pragma unroll
-    for (int l = 0; l < 64 / G; ++l) {
-        if (l < L) {
+    for (int lt = 0; lt < 32 / G; ++lt) {
+        if (l0 + lt < l1) {
             float phi[R];
-            table_phi<G>(&sp[l * G], phi);
+            table_phi<G>(&sp[lt * G], phi);
 #pragma unroll
             for (int q = 0; q < R; q += 2) {
-                const int p = l * R + q;  // even bucket index
-                const int slot = (p >> 1) & 15;
+                const int prel = lt * R + q;     // even, relative to l0 * R
+                const int slot = (prel >> 1) & 15;
                 buf[slot] = pack_bf16x2(phi[q] * scale, phi[q + 1] * scale);
+                const int p = l0 * R + prel;      // absolute bucket
                 const bool last = p + 2 == r;
                 if (slot == 15 || last) {
                     if (last) {
@@ -320,8 +340,12 @@ __device__ __forceinline__ void write_phi_tmem(const float (&sp)[64], int L,
     }
 }
 
-template <int G>
-__global__ void __launch_bounds__(128)
+// Sparse block attention + RACE readout + fusion for 128 sorted queries.
+// 256 threads: thread pairs (tid, tid ^ 128) share a query row (a TMEM lane)
+// and split its key columns (softmax), RACE tables (features) and output
+// columns (epilogue). NK = keys per query tile (b rounded up to 128).
+template <int G, int NK>
+__global__ void __launch_bounds__(kTcThreads, NK == 128 ? 2 : 1)
     k_block_attn_tc(const uint16_t *__restrict__ qx,
                     const uint16_t *__restrict__ kx,
                     const uint16_t *__restrict__ vx,
@@ -334,19 +358,25 @@ __global__ void __launch_bounds__(128)
                     const float *__restrict__ gates, uint16_t *__restrict__ ox,
                     float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
                     float *__restrict__ m_out, int N, int d, int H, int b,
-                    int nk, int L, int Lg_pad, float beta, float eps,
-                    float scale, float lambda, int mode, uint32_t tmem_cols,
+                    int L, int Lg_pad, float beta, float eps, float scale,
+                    float lambda, int mode, uint32_t tmem_cols,
                     DeviceStatus *status) {
     constexpr int R = 1 << G;
+    constexpr int nk = NK;
     extern __shared__ unsigned char smem_raw[];
     __shared__ uint64_t mb;
     __shared__ uint32_t tbase;
     __shared__ int qidx[128];
-    __shared__ int kidx[256];
+    __shared__ int kidx[NK];
+    __shared__ float xmax[2][128], xsum[2][128], xden[2][128];
     const int p0 = blockIdx.x * 128, bh = blockIdx.y, h = bh % H;
     const int tid = threadIdx.x, warp = tid >> 5;
+    const int grp = warp & 3, half = warp >> 2;
+    const int row = grp * 32 + (tid & 31);  // query row of the tile
     const int Lg = L * G, r = L * R;
     const int kpos0 = b >= 128 ? (p0 / b) * b : p0;
+    const int split = table_split(L, G);
+    const int l0 = half ? split : 0, l1 = half ? L : split;
 
     const uint32_t base = align1k(smem_u32(smem_raw));
     const uint32_t sQ = base;                  // later: B summary [r x d]
@@ -360,7 +390,7 @@ __global__ void __launch_bounds__(128)
     }
     const int32_t *pq = perm_q + (size_t)bh * N;
     const int32_t *pk = perm_k + (size_t)bh * N;
-    {
+    if (tid < 128) {
         int pos = min(p0 + tid, N - 1);
         int i = pq[pos];
         if (i < 0 || i >= N) {
@@ -369,7 +399,7 @@ __global__ void __launch_bounds__(128)
         }
         qidx[tid] = i;
     }
-    for (int j = tid; j < nk; j += 128) {
+    for (int j = tid; j < nk; j += kTcThreads) {
         int pos = min(kpos0 + j, N - 1);
         int i = pk[pos];
         if (i < 0 || i >= N) {
@@ -382,18 +412,18 @@ __global__ void __launch_bounds__(128)
     const uint16_t *qh = qx + (size_t)bh * N * d;
     const uint16_t *kh = kx + (size_t)bh * N * d;
     const uint16_t *vh = vx + (size_t)bh * N * d;
-    gather_rows(sQ, qh, qidx, 128, d, d, tid, 128);
-    gather_rows(sK, kh, kidx, nk, d, d, tid, 128);
+    gather_rows(sQ, qh, qidx, 128, d, d, tid, kTcThreads);
+    gather_rows(sK, kh, kidx, nk, d, d, tid, kTcThreads);
     cp_async_commit();
     load_planes_bf16(sV, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid,
-                     128);
+                     kTcThreads);
     cp_async_wait<0>();
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t t = tbase;
-    const uint32_t lane = (uint32_t)(warp * 32) << 16;
+    const uint32_t lane = (uint32_t)(grp * 32) << 16;
     const uint32_t colO = (uint32_t)nk;
     if (tid == 0) {
         const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
@@ -413,67 +443,82 @@ __global__ void __launch_bounds__(128)
     tc_fence_after();
     // Q, K and W are consumed: stream V into its slot and the bf16 B
     // summary of this head into the Q/K slots while the softmax runs.
-    gather_rows(sV, vh, kidx, nk, d, d, tid, 128);
-    load_rows(sQ, Bh + (size_t)bh * r * d, r, d, d, tid, 128);
+    gather_rows(sV, vh, kidx, nk, d, d, tid, kTcThreads);
+    load_rows(sQ, Bh + (size_t)bh * r * d, r, d, d, tid, kTcThreads);
     cp_async_commit();
 
-    // ---- RACE features of query row tid and Den = (1/L) sum phi . A
-    float sp[64];
-    race_bits_from_tmem<G>(t + lane + colO, Lg, Lg_pad, beta, sp);
+    // ---- RACE features of this row's tables [l0, l1); partial Den
+    float sp[32];
+    race_bits32(t + lane + colO + l0 * G, (l1 - l0) * G, beta, sp);
     const float *Ah = Ag + (size_t)bh * r;
     float den = 0.0f;
 #pragma unroll
-    for (int l = 0; l < 64 / G; ++l) {
-        if (l < L) {
+    for (int lt = 0; lt < 32 / G; ++lt) {
+        if (l0 + lt < l1) {
             float phi[R];
-            table_phi<G>(&sp[l * G], phi);
+            table_phi<G>(&sp[lt * G], phi);
 #pragma unroll
             for (int q = 0; q < R; ++q)
-                den = fmaf(phi[q], __ldg(Ah + l * R + q), den);
+                den = fmaf(phi[q], __ldg(Ah + (l0 + lt) * R + q), den);
         }
     }
-    den *= 1.0f / (float)L;
 
-    // ---- sparse branch: softmax of this row over its key block
+    // ---- sparse branch: softmax over this half's key columns
     const float sl2e = scale * kLog2e;
-    // keys of this query's block: all nk when b >= 128, else [klo, khi)
-    const int klo = b < 128 ? (tid / b) * b : 0;
+    const int klo = b < 128 ? (row / b) * b : 0;  // the row's key block
     const int khi = b < 128 ? klo + b : nk;
+    const int cbeg = half * (nk / 2);
     float mx = -INFINITY;
-    for (int c = 0; c < nk; c += 32) {
+#pragma unroll
+    for (int cc = 0; cc < nk / 2; cc += 32) {
         uint32_t v[32];
-        tmem_ld32(t + lane + c, v);
+        tmem_ld32(t + lane + cbeg + cc, v);
         tmem_wait_ld();
 #pragma unroll
-        for (int j = 0; j < 32; ++j)
-            if (c + j >= klo && c + j < khi)
-                mx = fmaxf(mx, __uint_as_float(v[j]));
+        for (int j = 0; j < 32; ++j) {
+            const int key = cbeg + cc + j;
+            if (key >= klo && key < khi) mx = fmaxf(mx, __uint_as_float(v[j]));
+        }
     }
+    xmax[half][row] = mx;
+    xden[half][row] = den;
+    __syncthreads();
+    mx = fmaxf(xmax[0][row], xmax[1][row]);
+    den = (xden[0][row] + xden[1][row]) * (1.0f / (float)L);
     const float M2 = mx * sl2e;  // row max in log2 units
     float lsum = 0.0f;
-    for (int c = 0; c < nk; c += 32) {
+    uint32_t ppk[nk / 4];  // this half's P, packed bf16 pairs
+#pragma unroll
+    for (int cc = 0; cc < nk / 2; cc += 32) {
         uint32_t v[32];
-        tmem_ld32(t + lane + c, v);
+        tmem_ld32(t + lane + cbeg + cc, v);
         tmem_wait_ld();
-        uint32_t pk16[16];
 #pragma unroll
         for (int j = 0; j < 32; j += 2) {
-            float p0v = 0.0f, p1v = 0.0f;
-            if (c + j >= klo && c + j < khi)
-                p0v = ex2_approx(fmaf(__uint_as_float(v[j]), sl2e, -M2));
-            if (c + j + 1 >= klo && c + j + 1 < khi)
-                p1v = ex2_approx(fmaf(__uint_as_float(v[j + 1]), sl2e, -M2));
-            lsum += p0v + p1v;
-            pk16[j >> 1] = pack_bf16x2(p0v, p1v);
+            const int key = cbeg + cc + j;
+            float a0 = 0.0f, a1 = 0.0f;
+            if (key >= klo && key < khi)
+                a0 = ex2_approx(fmaf(__uint_as_float(v[j]), sl2e, -M2));
+            if (key + 1 >= klo && key + 1 < khi)
+                a1 = ex2_approx(fmaf(__uint_as_float(v[j + 1]), sl2e, -M2));
+            lsum += a0 + a1;
+            ppk[(cc + j) >> 1] = pack_bf16x2(a0, a1);
         }
-        tmem_st16(t + lane + (c >> 1), pk16);  // P over the read columns
     }
-    tmem_wait_st();
+    xsum[half][row] = lsum;
+    tc_fence_before();
+    __syncthreads();  // every S read is done: P may overwrite S
+    tc_fence_after();
+    lsum = xsum[0][row] + xsum[1][row];
+#pragma unroll
+    for (int cc = 0; cc < nk / 4; cc += 16)
+        tmem_st16(t + lane + (cbeg >> 1) + cc,
+                  *reinterpret_cast<uint32_t(*)[16]>(&ppk[cc]));
 
     // ---- fusion scalars (Eq. (5) in log-sum-exp form, Eq. (6))
-    const int qpos = p0 + tid;
+    const int qpos = p0 + row;
     const bool qvalid = qpos < N;
-    const int qi = qidx[tid];
+    const int qi = qidx[row];
     const size_t tok = (size_t)bh * N + qi;
     const float log_ds = M2 * kLn2 + logf(lsum);
     const float lam = (lambda_tok && qvalid) ? lambda_tok[tok] : lambda;
@@ -486,7 +531,7 @@ __global__ void __launch_bounds__(128)
     const float ratio = c2 / c1e;
 
     const int r0 = min(r, nk);  // buckets of the first Num pass
-    write_phi_tmem<G>(sp, L, ratio, 0, r0, t + lane + (nk >> 1));
+    write_phi_tmem<G>(sp, l0, l1, r, ratio, 0, r0, t + lane + (nk >> 1));
     tmem_wait_st();
     cp_async_wait<0>();
     fence_proxy_async_smem();
@@ -508,9 +553,8 @@ __global__ void __launch_bounds__(128)
     ok = ok && mbar_wait(&mb, 1, status, 22);
     ok = __syncthreads_and(ok);
     tc_fence_after();
-    const int phase = 0;  // third completion of the barrier
     if (r > nk) {  // remaining buckets reuse the P columns
-        write_phi_tmem<G>(sp, L, ratio, nk, r, t + lane);
+        write_phi_tmem<G>(sp, l0, l1, r, ratio, nk, r, t + lane);
         tmem_wait_st();
         tc_fence_before();
         __syncthreads();
@@ -524,7 +568,7 @@ __global__ void __launch_bounds__(128)
                        id_o, 1);
             mma_commit(&mb);
         }
-        ok = ok && mbar_wait(&mb, phase, status, 23);
+        ok = ok && mbar_wait(&mb, 0, status, 23);  // third completion
         ok = __syncthreads_and(ok);
         tc_fence_after();
     }
@@ -532,7 +576,7 @@ __global__ void __launch_bounds__(128)
     // ---- epilogue: O row = c1 * accumulator, at the original query index
     if (ok) {
         uint16_t *orow = ox + tok * d;
-        for (int c = 0; c < d; c += 32) {
+        for (int c = half * (d >> 1); c < (half + 1) * (d >> 1); c += 32) {
             uint32_t v[32];
             tmem_ld32(t + lane + colO + c, v);
             tmem_wait_ld();
@@ -553,7 +597,7 @@ __global__ void __launch_bounds__(128)
                 }
             }
         }
-        if (qvalid) {
+        if (qvalid && half == 0) {
             if (log_ds_out) log_ds_out[tok] = log_ds;
             if (dlr_out) dlr_out[tok] = den;
             if (m_out) m_out[tok] = msp;
@@ -600,6 +644,9 @@ bool tc_supported(const Plan &P) {
     if (!(P.b == 32 || P.b == 64 || P.b == 128 || P.b == 256)) return false;
     if (P.gamma > 6 || P.L * P.gamma > 64) return false;
     if (P.r % 16 != 0 || P.r > 256) return false;
+    // each half of a row's tables must fit in 32 projection columns
+    const int split = table_split(P.L, P.gamma);
+    if (split * P.gamma > 32 || (P.L - split) * P.gamma > 32) return false;
     return true;
 }
 
@@ -639,7 +686,7 @@ cudaError_t launch_race_keys_tc(const Plan &P, const void *k, const void *v,
         auto kern = k_race_keys_tc<G>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-        kern<<<grid, 128, smem, st>>>(
+        kern<<<grid, kTcThreads, smem, st>>>(
             (const uint16_t *)k, (const uint16_t *)v, w_race, P.N, P.d, P.H,
             P.L, r_pad, lg_pad, P.chunk, P.beta, cols, part, status);
         return cudaGetLastError();
@@ -655,21 +702,25 @@ cudaError_t launch_block_attn_tc(
     const int nk = P.b >= 128 ? P.b : 128;
     const int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
     const uint32_t cols = pow2_cols((uint32_t)(nk + P.d));
-    (void)0;
     size_t need = 1024 + (size_t)(128 + 2 * nk) * P.d * 2;
     size_t smem = smem_for(need, cols);
     dim3 grid((P.N + 127) / 128, P.BH);
     return dispatch_gamma(P.gamma, [&](auto g) {
         constexpr int G = decltype(g)::value;
-        auto kern = k_block_attn_tc<G>;
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-        kern<<<grid, 128, smem, st>>>(
-            (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
-            w_race, perm_q, perm_k, A, Bh, lambda_tok, gates, (uint16_t *)o,
-            log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, nk, P.L, lg_pad,
-            P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, cols, status);
-        return cudaGetLastError();
+        auto run = [&](auto kern) {
+            cudaFuncSetAttribute(kern,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem);
+            kern<<<grid, kTcThreads, smem, st>>>(
+                (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
+                w_race, perm_q, perm_k, A, Bh, lambda_tok, gates,
+                (uint16_t *)o, log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H,
+                P.b, P.L, lg_pad, P.beta, P.eps, P.scale, P.lambda,
+                P.fusion_mode, cols, status);
+            return cudaGetLastError();
+        };
+        return nk == 256 ? run(k_block_attn_tc<G, 256>)
+                         : run(k_block_attn_tc<G, 128>);
     });
 }
 
