@@ -4,6 +4,8 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <cudaTypedefs.h>
+
 #include <mutex>
 #include <string>
 #include <vector>
@@ -182,6 +184,33 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     return ELSAA_OK;
 }
 
+cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
+                              uint64_t rows, uint64_t cols,
+                              uint32_t box_rows) {
+    static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &fn,
+                                    cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    });
+    if (!encode) return cudaErrorNotSupported;
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+                        const_cast<void *>(base), dims, strides, box, estr,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE,
+                        CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                        CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
 int set_last_error(int code, const char *fmt, ...) {
     va_list ap;
     va_start(ap, fmt);
@@ -281,11 +310,11 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                        }),
                        "sort_scatter");
     if (P.impl == 2) {
-        ELSAA_CHECK_LAUNCH(timed("race_keys_tc", st, [&] {
-                               return launch_race_keys_tc(P, k, v, w_race,
+        ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
+                               return launch_race_keys_ws(P, k, v, w_race,
                                                           part, status, st);
                            }),
-                           "race_keys_tc");
+                           "race_keys_ws");
     } else {
         ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
                                return launch_race_partial_simt(P, k, v, w_race,
@@ -297,7 +326,15 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                            return launch_race_reduce(P, part, A, Bm, Bh, st);
                        }),
                        "race_reduce");
-    if (P.impl == 2) {
+    if (P.impl == 2 && ws_supported(P)) {
+        ELSAA_CHECK_LAUNCH(timed("block_attn_ws", st, [&] {
+                               return launch_block_attn_ws(
+                                   P, q, k, v, w_race, pq, pk, A, Bh,
+                                   lambda_tok, gates, o, log_d_sparse, d_lr,
+                                   m_sparse, status, st);
+                           }),
+                           "block_attn_ws");
+    } else if (P.impl == 2) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_tc", st, [&] {
                                return launch_block_attn_tc(
                                    P, q, k, v, w_race, pq, pk, A, Bh,

@@ -85,4 +85,17 @@ __device__ __forceinline__ float fusion_multiplier(float log_ds, float lam,
     return expf(a - (mx + logf(s)));
 }
 
+// fusion_multiplier with fast (approximate) log/exp, for the bf16 path.
+__device__ __forceinline__ float fusion_multiplier_fast(float log_ds, float lam,
+                                                        float dlr, float eps,
+                                                        int mode) {
+    if (mode == 1) return 1.0f;
+    float a = log_ds;
+    float b = (lam > 0.0f && dlr > 0.0f) ? __logf(lam * dlr) : -INFINITY;
+    float c = __logf(eps);
+    float mx = fmaxf(a, fmaxf(b, c));
+    float s = __expf(a - mx) + __expf(b - mx) + __expf(c - mx);
+    return __expf(a - mx) / s;
+}
+
 }  // namespace elsaa

@@ -2,6 +2,7 @@
 // Nothing here is part of the public ABI (see include/elsaa.h).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -84,6 +85,29 @@ cudaError_t launch_race_keys_tc(const Plan &P, const void *k, const void *v,
                                 const float *w_race, float *part,
                                 DeviceStatus *status, cudaStream_t st);
 cudaError_t launch_block_attn_tc(
+    const Plan &P, const void *q, const void *k, const void *v,
+    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
+    const float *A, const uint16_t *Bh, const float *lambda_tok,
+    const float *gates, void *o, float *log_d_sparse, float *d_lr,
+    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+
+// Row-major bf16 matrix [rows x cols] as a TMA tensor map with boxes of
+// 64 columns x box_rows rows and 128-byte swizzle (the panel layout).
+// Returns cudaSuccess or an error if the driver entry point is missing or
+// the encoding is rejected.
+cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
+                              uint64_t rows, uint64_t cols, uint32_t box_rows);
+
+// Warp-specialised RACE key summaries (tensor-core path).
+size_t race_keys_ws_smem(const Plan &P);
+uint32_t race_keys_ws_cols(const Plan &P);
+cudaError_t launch_race_keys_ws(const Plan &P, const void *k, const void *v,
+                                const float *w_race, float *part,
+                                DeviceStatus *status, cudaStream_t st);
+
+// Persistent warp-specialised block attention (key blocks of <= 128).
+bool ws_supported(const Plan &P);
+cudaError_t launch_block_attn_ws(
     const Plan &P, const void *q, const void *k, const void *v,
     const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const uint16_t *Bh, const float *lambda_tok,

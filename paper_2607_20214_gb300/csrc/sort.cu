@@ -8,8 +8,9 @@
 // original index). Consecutive runs of b sorted positions form the blocks.
 //
 // Three launches, all integer-exact after the hash:
-//   sort_hash    one CTA per 128-token tile of (head, Q|K): hash, tile
-//                histogram, rank of each token among equal keys of its tile.
+//   sort_hash    one CTA per two 128-token tiles of (head, Q|K): hash,
+//                tile histograms, rank of each token among equal keys of
+//                its tile.
 //   sort_scan    one CTA per (head, Q|K): exclusive scan of the tile
 //                histograms stored bin-major ([bin][tile]) -> start offset
 //                of every (tile, bin) run in the sorted order.
@@ -42,13 +43,28 @@ __device__ __forceinline__ void unpack8<float>(const uint4 &u, float *x) {
     x[3] = __uint_as_float(u.w);
 }
 
-// One CTA hashes one 128-token tile of (head, Q|K). The tile is staged in
-// shared memory with coalesced 16-byte loads (16-byte chunks of each row
-// XOR-swizzled by the row index, so a warp reading one chunk of 32 rows is
-// conflict-free). Each thread then evaluates the NS projections of its
-// token as NS interleaved FMA chains; each chain keeps the canonical
-// sequential order i = 0..d-1. Ranks among equal keys of the tile come from
-// warp match masks plus per-warp counts.
+// Two fp32 FMAs in one instruction: lanes (lo, hi) of d = a * b + c, each an
+// IEEE round-to-nearest fused multiply-add (bit-identical to fmaf).
+__device__ __forceinline__ unsigned long long fma2(unsigned long long a,
+                                                   unsigned long long b,
+                                                   unsigned long long c) {
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ unsigned long long pair2(float lo, float hi) {
+    return ((unsigned long long)__float_as_uint(hi) << 32) |
+           __float_as_uint(lo);
+}
+
+// One CTA hashes two 128-token tiles (A = 2 * blockIdx.x, B = A + 1) of one
+// (head, Q|K). The tiles are staged in shared memory with cp.async (16-byte
+// chunks of each row XOR-swizzled by the row index, so a warp reading one
+// chunk of 32 rows is conflict-free). Thread t evaluates the NS projections
+// of row t of both tiles with packed fma.rn.f32x2 (lane lo: tile A, lane
+// hi: tile B); every chain keeps the canonical sequential order
+// i = 0..d-1. Ranks among equal keys of a tile come from warp match masks
+// plus per-warp counts.
 template <typename T, int NS>
 __global__ void __launch_bounds__(kHashTile)
     k_sort_hash(const T *__restrict__ q, const T *__restrict__ k,
@@ -56,89 +72,108 @@ __global__ void __launch_bounds__(kHashTile)
                 int bins, int gray, int tiles, uint32_t *__restrict__ keyrank,
                 int *__restrict__ hist) {
     extern __shared__ __align__(16) unsigned char smem[];
-    const int tile = blockIdx.x, bh = blockIdx.y, which = blockIdx.z;
+    const int tile0 = 2 * blockIdx.x, bh = blockIdx.y, which = blockIdx.z;
     const int BH = gridDim.y;
     const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
     const int h = bh % H;
     constexpr int kEl = 16 / sizeof(T);          // elements per 16-byte chunk
     const int cpr = d / kEl;                     // chunks per row
     const int swz = cpr >= 8 ? 7 : cpr - 1;      // swizzle mask
-    uint4 *xs = reinterpret_cast<uint4 *>(smem);               // [128][cpr]
-    float *ws = reinterpret_cast<float *>(xs + kHashTile * cpr);  // [NS][d]
-    int *cnt = reinterpret_cast<int *>(ws + NS * d);  // [4 warps][bins]
+    uint4 *xs = reinterpret_cast<uint4 *>(smem);  // [2][128][cpr]
+    float *ws = reinterpret_cast<float *>(xs + 2 * kHashTile * cpr);  // [NS][d]
+    int *cnt = reinterpret_cast<int *>(ws + NS * d);  // [2][4 warps][bins]
 
     const T *x = (which ? k : q) + (size_t)bh * N * d;
-    const int n0 = tile * kHashTile;
-    const uint4 *src = reinterpret_cast<const uint4 *>(x + (size_t)n0 * d);
-    const int valid_rows = min(kHashTile, N - n0);
     const uint32_t xs_s = static_cast<uint32_t>(__cvta_generic_to_shared(xs));
-    for (int i = tid; i < kHashTile * cpr; i += kHashTile) {
-        int row = i / cpr, c = i - row * cpr;
-        uint32_t dst = xs_s + 16u * (row * cpr + (c ^ (row & swz)));
-        if (row < valid_rows)
-            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst),
-                         "l"(src + (size_t)row * cpr + c)
-                         : "memory");
-        else
-            xs[row * cpr + (c ^ (row & swz))] = make_uint4(0u, 0u, 0u, 0u);
+    for (int tt = 0; tt < 2; ++tt) {
+        const int n0 = (tile0 + tt) * kHashTile;
+        const int valid_rows = max(0, min(kHashTile, N - n0));
+        const uint4 *src = reinterpret_cast<const uint4 *>(x + (size_t)n0 * d);
+        for (int i = tid; i < kHashTile * cpr; i += kHashTile) {
+            int row = i / cpr, c = i - row * cpr;
+            int slot = (tt * kHashTile + row) * cpr + (c ^ (row & swz));
+            if (row < valid_rows)
+                asm volatile(
+                    "cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                        xs_s + 16u * slot),
+                    "l"(src + (size_t)row * cpr + c)
+                    : "memory");
+            else
+                xs[slot] = make_uint4(0u, 0u, 0u, 0u);
+        }
     }
     asm volatile("cp.async.commit_group;" ::: "memory");
     for (int i = tid; i < NS * d; i += kHashTile)
         ws[i] = w_sort[(size_t)h * NS * d + i];
-    for (int i = tid; i < 4 * bins; i += kHashTile) cnt[i] = 0;
+    for (int i = tid; i < 8 * bins; i += kHashTile) cnt[i] = 0;
     asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
 
-    const int n = n0 + tid;
-    float acc[NS > 0 ? NS : 1];
+    unsigned long long acc[NS > 0 ? NS : 1];
 #pragma unroll
-    for (int p = 0; p < NS; ++p) acc[p] = 0.0f;
-    const uint4 *xr = xs + tid * cpr;
+    for (int p = 0; p < NS; ++p) acc[p] = 0ull;
+    const uint4 *xa = xs + tid * cpr;
+    const uint4 *xb = xs + (kHashTile + tid) * cpr;
     const float4 *ws4 = reinterpret_cast<const float4 *>(ws);
     for (int c = 0; c < cpr; ++c) {
-        float xv[kEl];
-        unpack8<T>(xr[c ^ (tid & swz)], xv);
+        float va[kEl], vb[kEl];
+        unpack8<T>(xa[c ^ (tid & swz)], va);
+        unpack8<T>(xb[c ^ (tid & swz)], vb);
         const int e0 = c * kEl;
-        float wv[NS > 0 ? NS : 1][kEl];
 #pragma unroll
-        for (int p = 0; p < NS; ++p)
+        for (int j = 0; j < kEl / 4; ++j) {
+            float wv[NS > 0 ? NS : 1][4];
 #pragma unroll
-            for (int j = 0; j < kEl / 4; ++j) {
+            for (int p = 0; p < NS; ++p) {
                 float4 w4 = ws4[(p * d + e0) / 4 + j];  // same for all lanes
-                wv[p][4 * j] = w4.x;
-                wv[p][4 * j + 1] = w4.y;
-                wv[p][4 * j + 2] = w4.z;
-                wv[p][4 * j + 3] = w4.w;
+                wv[p][0] = w4.x;
+                wv[p][1] = w4.y;
+                wv[p][2] = w4.z;
+                wv[p][3] = w4.w;
             }
 #pragma unroll
-        for (int e = 0; e < kEl; ++e)
+            for (int e = 0; e < 4; ++e) {
+                const unsigned long long xp = pair2(va[4 * j + e], vb[4 * j + e]);
 #pragma unroll
-            for (int p = 0; p < NS; ++p)
-                acc[p] = __fmaf_rn(wv[p][e], xv[e], acc[p]);
+                for (int p = 0; p < NS; ++p)
+                    acc[p] = fma2(pair2(wv[p][e], wv[p][e]), xp, acc[p]);
+            }
+        }
     }
-    uint32_t code = 0;
-#pragma unroll
-    for (int p = 0; p < NS; ++p) code |= (acc[p] > 0.0f ? 1u : 0u) << p;
-    const int key = (int)(gray ? gray_rank(code) : code);
-    // rank among equal keys of the tile (lower index first)
-    const bool in = n < N;
-    const unsigned act = __ballot_sync(0xffffffffu, in);
-    unsigned peers = __match_any_sync(0xffffffffu, in ? key : -1) & act;
-    const int rank_w = __popc(peers & ((1u << lane) - 1u));
-    if (in && rank_w == 0) cnt[wid * bins + key] = __popc(peers);
-    __syncthreads();
-    if (in) {
-        int rank = rank_w;
-        for (int w = 0; w < wid; ++w) rank += cnt[w * bins + key];
-        keyrank[((size_t)which * BH + bh) * N + n] =
-            (uint32_t)key | ((uint32_t)rank << 16);
-    }
-    // tile histogram, stored bin-major ([bins][tiles]) so that the scan
-    // walks one contiguous array
     int *hout = hist + ((size_t)which * BH + bh) * tiles * bins;
-    for (int i = tid; i < bins; i += kHashTile)
-        hout[(size_t)i * tiles + tile] = cnt[i] + cnt[bins + i] +
-                                         cnt[2 * bins + i] + cnt[3 * bins + i];
+#pragma unroll
+    for (int tt = 0; tt < 2; ++tt) {
+        const int tile = tile0 + tt;
+        const int n = tile * kHashTile + tid;
+        uint32_t code = 0;
+#pragma unroll
+        for (int p = 0; p < NS; ++p) {
+            const float pr = __uint_as_float(
+                (uint32_t)(tt ? (acc[p] >> 32) : (acc[p] & 0xffffffffull)));
+            code |= (pr > 0.0f ? 1u : 0u) << p;
+        }
+        const int key = (int)(gray ? gray_rank(code) : code);
+        const bool in = n < N && tile < tiles;
+        const unsigned act = __ballot_sync(0xffffffffu, in);
+        unsigned peers = __match_any_sync(0xffffffffu, in ? key : -1) & act;
+        const int rank_w = __popc(peers & ((1u << lane) - 1u));
+        int *cw = cnt + tt * 4 * bins;
+        if (in && rank_w == 0) cw[wid * bins + key] = __popc(peers);
+        __syncthreads();
+        if (in) {
+            int rank = rank_w;
+            for (int w = 0; w < wid; ++w) rank += cw[w * bins + key];
+            keyrank[((size_t)which * BH + bh) * N + n] =
+                (uint32_t)key | ((uint32_t)rank << 16);
+        }
+        // tile histogram, stored bin-major ([bins][tiles]) so that the scan
+        // walks one contiguous array
+        if (tile < tiles)
+            for (int i = tid; i < bins; i += kHashTile)
+                hout[(size_t)i * tiles + tile] = cw[i] + cw[bins + i] +
+                                                 cw[2 * bins + i] +
+                                                 cw[3 * bins + i];
+    }
 }
 
 constexpr int kScanThreads = 1024;
@@ -234,9 +269,9 @@ template <typename T, int NS>
 cudaError_t launch_hash_t(const Plan &P, const void *q, const void *k,
                           const float *w_sort, uint32_t *keyrank, int *hist,
                           cudaStream_t st) {
-    dim3 grid(P.tiles, P.BH, 2);
-    size_t smem = (size_t)kHashTile * P.d * sizeof(T) +
-                  sizeof(float) * (size_t)NS * P.d + sizeof(int) * 4 * P.bins;
+    dim3 grid((P.tiles + 1) / 2, P.BH, 2);
+    size_t smem = 2 * (size_t)kHashTile * P.d * sizeof(T) +
+                  sizeof(float) * (size_t)NS * P.d + sizeof(int) * 8 * P.bins;
     auto kern = k_sort_hash<T, NS>;
     cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                          (int)smem);

@@ -22,85 +22,13 @@
 
 #include "device_common.cuh"
 #include "tc_common.cuh"
+#include "tc_race.cuh"
 
 namespace elsaa {
 
 namespace {
 
 using namespace tc;
-
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kLn2 = 0.6931471805599453f;
-
-__device__ __forceinline__ uint32_t align1k(uint32_t x) {
-    return (x + 1023u) & ~1023u;
-}
-
-// RACE planes of one head as bf16 rows [Lg_pad x d] in the panel layout;
-// rows >= Lg are zero.
-__device__ void load_planes_bf16(uint32_t dst, const float *w, int Lg,
-                                 int Lg_pad, int d, int tid, int nthreads) {
-    const int chunks = d >> 3;
-    for (int i = tid; i < Lg_pad * chunks; i += nthreads) {
-        int row = i / chunks, c = i - row * chunks;
-        uint32_t addr = dst + panel_offset(row, c, Lg_pad);
-        if (row < Lg) {
-            const float4 *src =
-                reinterpret_cast<const float4 *>(w + (size_t)row * d + c * 8);
-            float4 a = src[0], b = src[1];
-            float v[8] = {a.x, a.y, a.z, a.w, b.x, b.y, b.z, b.w};
-            st_shared_bf16x8(addr, v);
-        } else {
-            st_shared_zero16(addr);
-        }
-    }
-}
-
-// Two threads share each row (warps w and w + 4 read the same TMEM lanes).
-// The RACE tables of a row are split between them at table `split`, chosen
-// so that each half's buckets start on a 32-bucket boundary (whole TMEM
-// store groups) and each half reads at most 32 projection columns.
-__host__ __device__ inline int table_split(int L, int G) {
-    const int R = 1 << G;
-    const int unit = R >= 32 ? 1 : 32 / R;  // tables per 32 buckets
-    int split = ((L + 1) / 2 + unit - 1) / unit * unit;
-    return split > L ? L : split;
-}
-
-// Per-bit factors sp[j] = sigmoid(2 beta tanh(a_j)) of the projection
-// columns [col0, col0 + 32) of this thread's TMEM lane; entries past `ncols`
-// are set to 1/2 and not used.
-__device__ __forceinline__ void race_bits32(uint32_t taddr, int ncols,
-                                           float beta, float (&sp)[32]) {
-    uint32_t pr[32];
-    tmem_ld32(taddr, pr);
-    tmem_wait_ld();
-#pragma unroll
-    for (int j = 0; j < 32; ++j) {
-        if (j < ncols) {
-            float t = tanh_approx(beta * tanh_approx(__uint_as_float(pr[j])));
-            sp[j] = fmaf(0.5f, t, 0.5f);  // 1/2 + tanh(beta u)/2
-        } else {
-            sp[j] = 0.5f;
-        }
-    }
-}
-
-// Features of table l from its G per-bit factors: phi[r] = prod_b (bit b of
-// r ? sp[b] : 1 - sp[b]), r < 2^G.
-template <int G>
-__device__ __forceinline__ void table_phi(const float *sp, float *phi) {
-    phi[0] = 1.0f;
-#pragma unroll
-    for (int b = 0; b < G; ++b) {
-        const float p = sp[b], q = 1.0f - p;
-#pragma unroll
-        for (int r = 0; r < (1 << b); ++r) {
-            phi[r + (1 << b)] = phi[r] * p;
-            phi[r] *= q;
-        }
-    }
-}
 
 // ---------------------------------------------------------------------------
 // RACE key side. 256 threads: thread pairs (tid, tid ^ 128) share a key row
@@ -217,7 +145,22 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         float buf[8];
 #pragma unroll
         for (int lt = 0; lt < 32 / G; ++lt) {
-            if (l0 + lt < l1) {
+            if (G == 4 && l0 + lt < l1) {
+                // 16 features as an outer product, two 16-byte chunks
+                float u[4], w[4];
+                table_uw4(&sp[lt * G], valid ? 1.0f : 0.0f, u, w);
+                uint32_t pk[8];
+                table_pack4(u, w, pk);
+                const int c0 = (l0 * R + lt * R) >> 3;
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+                    asm volatile(
+                        "st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
+                            sPhi + panel_offset(row, c0 + h, 128)),
+                        "r"(pk[4 * h]), "r"(pk[4 * h + 1]), "r"(pk[4 * h + 2]),
+                        "r"(pk[4 * h + 3])
+                        : "memory");
+            } else if (l0 + lt < l1) {
                 float phi[R];
                 table_phi<G>(&sp[lt * G], phi);
 #pragma unroll
@@ -298,46 +241,6 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(t, tmem_cols);
-}
-
-// ---------------------------------------------------------------------------
-// Writes the pre-scaled features phi * scale of tables [l0, l1) of this
-// thread's query row, for buckets [lo, hi), as packed bf16 pairs into TMEM
-// with bucket lo at `taddr`. l0 * R and lo are multiples of 32 and hi of 16;
-// buckets go out in groups of 32 (16 columns), the last half group padded
-// with zeros.
-template <int G>
-__device__ __forceinline__ void write_phi_tmem(const float (&sp)[32], int l0,
-                                               int l1, int r, float scale,
-                                               int lo, int hi,
-                                               uint32_t taddr) {
-    constexpr int R = 1 << G;
-    uint32_t buf[16];
-#pragma unroll
-    for (int lt = 0; lt < 32 / G; ++lt) {
-        if (l0 + lt < l1) {
-            float phi[R];
-            table_phi<G>(&sp[lt * G], phi);
-#pragma unroll
-            for (int q = 0; q < R; q += 2) {
-                const int prel = lt * R + q;     // even, relative to l0 * R
-                const int slot = (prel >> 1) & 15;
-                buf[slot] = pack_bf16x2(phi[q] * scale, phi[q + 1] * scale);
-                const int p = l0 * R + prel;      // absolute bucket
-                const bool last = p + 2 == r;
-                if (slot == 15 || last) {
-                    if (last) {
-#pragma unroll
-                        for (int z = 0; z < 16; ++z)
-                            if (z > slot) buf[z] = 0u;
-                    }
-                    const int g = p - 2 * slot;  // first bucket of the group
-                    if (g >= lo && g < hi)
-                        tmem_st16(taddr + ((g - lo) >> 1), buf);
-                }
-            }
-        }
-    }
 }
 
 // Sparse block attention + RACE readout + fusion for 128 sorted queries.
@@ -651,13 +554,11 @@ bool tc_supported(const Plan &P) {
 }
 
 int tc_race_chunks(const Plan &P, int *chunk) {
-    // TMEM use decides CTAs per SM; one wave of chunks over all heads.
-    int r_pad = (P.r + 127) / 128 * 128;
-    int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
-    uint32_t cols = pow2_cols((r_pad / 128) * (P.d + 16) + 64);
+    // CTAs per SM from the TMEM and shared memory of the key kernel; one
+    // wave of chunks over all heads.
+    const uint32_t cols = race_keys_ws_cols(P);
     int per_sm = 512 / (int)cols;
-    size_t smem = 1024 + ((P.L * P.gamma + 15) / 16 * 16) * P.d * 2 + 4096 +
-                  4 * 128 * P.d * 2 + 128 * r_pad * 2;
+    const size_t smem = race_keys_ws_smem(P);
     int by_smem = (int)(kSmemPerSM / (smem + 1024));
     if (by_smem < per_sm) per_sm = by_smem;
     if (per_sm < 1) per_sm = 1;

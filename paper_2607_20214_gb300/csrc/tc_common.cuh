@@ -13,6 +13,7 @@
 // cols = M or N).
 #pragma once
 
+#include <cuda.h>  // CUtensorMap (type only; the library links no libcuda)
 #include <stdint.h>
 
 #include "internal.h"
@@ -20,9 +21,18 @@
 namespace elsaa {
 namespace tc {
 
-// Upper bound on mbarrier polls before a wait gives up and reports
-// kDevWaitTimeout (a healthy wait completes in far fewer).
-constexpr uint32_t kWaitLimit = 1u << 22;
+// A bounded mbarrier wait gives up after this many nanoseconds (of
+// %globaltimer) and reports kDevWaitTimeout; a healthy wait is microseconds.
+constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+// Suspend hint of one try_wait: the thread sleeps until the phase completes
+// or this many nanoseconds pass, instead of spinning on issue slots.
+constexpr uint32_t kSuspendHintNs = 1000000u;
+
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -51,25 +61,66 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{\n .reg .pred p;\n"
-        " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
         " selp.u32 %0, 1, 0, p;\n}\n"
         : "=r"(ok)
-        : "r"(smem_u32(bar)), "r"(parity)
+        : "r"(smem_u32(bar)), "r"(parity), "r"(kSuspendHintNs)
         : "memory");
     return ok != 0;
 }
 
-// Bounded wait; returns false (and records the site) if it ran out.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
-                                          DeviceStatus *st, int site) {
-    for (uint32_t i = 0; i < kWaitLimit; ++i)
-        if (mbar_try_wait(bar, parity)) return true;
+__device__ __forceinline__ void record_timeout(DeviceStatus *st, int site) {
     if (st && atomicCAS(&st->code, 0, kDevWaitTimeout) == 0) {
         st->where = site;
         st->info0 = blockIdx.x;
         st->info1 = blockIdx.y;
     }
-    return false;
+}
+
+// Bounded wait; returns false (and records the site) if it ran out.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          DeviceStatus *st, int site) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (global_ns() - t0 > kWaitLimitNs) {
+            record_timeout(st, site);
+            return false;
+        }
+    }
+    return true;
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(
+                     smem_u32(bar))
+                 : "memory");
+}
+
+// Bounded wait that also gives up as soon as another thread of the CTA has
+// set *abort (after its own wait ran out), so a stalled pipeline drains in
+// one wait limit instead of one per pending stage.
+__device__ __forceinline__ bool mbar_wait_or_abort(uint64_t *bar,
+                                                   uint32_t parity,
+                                                   volatile int *abort,
+                                                   DeviceStatus *st,
+                                                   int site) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    while (!mbar_try_wait(bar, parity)) {
+        if (*abort) return false;
+        if (global_ns() - t0 > kWaitLimitNs) {
+            *abort = 1;
+            record_timeout(st, site);
+            return false;
+        }
+    }
+    return true;
+}
+
+// Named barrier over `count` threads (id 0 is __syncthreads).
+__device__ __forceinline__ void named_sync(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
 // --------------------------------------------------------------- fences
@@ -223,6 +274,30 @@ __device__ __forceinline__ void mma_commit(uint64_t *bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 "
         "[%0];" ::"r"(smem_u32(bar))
+        : "memory");
+}
+
+// ------------------------------------------------------------------ TMA
+
+// Arrives on `bar` and raises its expected transaction count by `bytes`.
+__device__ __forceinline__ void mbar_expect_tx(uint64_t *bar, uint32_t bytes) {
+    asm volatile(
+        "mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(
+            smem_u32(bar)),
+        "r"(bytes)
+        : "memory");
+}
+
+// 2-D tiled TMA load of the box at (x = column, y = row) into shared memory;
+// completion is counted in bytes on `bar`. x * element size must be a
+// multiple of 16 bytes.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map,
+                                            int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx"
+        "::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y),
+        "r"(smem_u32(bar))
         : "memory");
 }
 
