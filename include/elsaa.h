@@ -93,7 +93,9 @@ int elsaa_workspace_size(const elsaa_params *params, size_t *bytes);
  * ELSAA forward pass for all B*H heads (Algorithm 1 steps 4-8, without the
  * Q/K/V and output projections, which stay dense outside the operator).
  *
- * q, k, v      [B, H, N, d_h] of params->dtype (device, read only).
+ * q, k, v      [B, H, N, d_h] of params->dtype (device, read only). q, k, v,
+ *              o and w_race must be 16-byte aligned (rows move in 16-byte
+ *              pieces); ELSAA_ERR_INVALID_ARG otherwise.
  * w_sort       [H, sort_bits, d_h] fp32: planes of the angular sort hash,
  *              shared by queries and keys of head h; may be NULL when
  *              sort_bits == 0. Bit p of x is [<w_sort[h][p], x> > 0], the

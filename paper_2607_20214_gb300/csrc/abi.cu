@@ -145,6 +145,7 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     Q.lambda = p->lambda;
     Q.fusion_mode = p->fusion_mode;
     Q.impl = 1;
+    Q.Lg_pad = (Q.L * Q.gamma + 15) / 16 * 16;
     Q.tiles = (Q.N + kHashTile - 1) / kHashTile;
     if (p->impl == ELSAA_IMPL_AUTO && tc_supported(Q)) {
         // tensor-core path: one wave of 128-key-tile chunks per head
@@ -179,6 +180,8 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     off = align_up(off + (size_t)Q.BH * Q.r * Q.d * sizeof(float), 256);
     Q.off_Bh = off;
     off = align_up(off + (size_t)Q.BH * Q.r * Q.d * sizeof(uint16_t), 256);
+    Q.off_W = off;
+    off = align_up(off + (size_t)Q.H * Q.Lg_pad * Q.d * sizeof(uint16_t), 256);
     Q.total = off;
     *msg = "";
     return ELSAA_OK;
@@ -266,12 +269,12 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     if (P.n_s > 0 && !w_sort)
         return fail(ELSAA_ERR_INVALID_ARG,
                     "w_sort must be non-NULL when sort_bits > 0");
-    size_t elt = P.dtype == ELSAA_FP32 ? 4 : 2;
-    const void *ptrs[] = {q, k, v, o};
+    // rows are moved in 16-byte pieces (cp.async, vector loads)
+    const void *ptrs[] = {q, k, v, o, w_race};
     for (const void *p : ptrs)
-        if ((uintptr_t)p % elt)
+        if ((uintptr_t)p % 16)
             return fail(ELSAA_ERR_INVALID_ARG,
-                        "q, k, v and o must be aligned to their element size");
+                        "q, k, v, o and w_race must be 16-byte aligned");
     if (!workspace)
         return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
     if ((uintptr_t)workspace % 256)
@@ -293,6 +296,7 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     float *A = (float *)(ws + P.off_A);
     float *Bm = (float *)(ws + P.off_B);
     uint16_t *Bh = (uint16_t *)(ws + P.off_Bh);
+    uint16_t *Wbf = (uint16_t *)(ws + P.off_W);
 
     ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
                        "status reset");
@@ -310,9 +314,13 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                        }),
                        "sort_scatter");
     if (P.impl == 2) {
+        ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
+                               return launch_prep_planes(P, w_race, Wbf, st);
+                           }),
+                           "prep_planes");
         ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
-                               return launch_race_keys_ws(P, k, v, w_race,
-                                                          part, status, st);
+                               return launch_race_keys_ws(P, k, v, Wbf, part,
+                                                          status, st);
                            }),
                            "race_keys_ws");
     } else {
@@ -329,7 +337,7 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     if (P.impl == 2 && ws_supported(P)) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_ws", st, [&] {
                                return launch_block_attn_ws(
-                                   P, q, k, v, w_race, pq, pk, A, Bh,
+                                   P, q, k, v, Wbf, pq, pk, A, Bh,
                                    lambda_tok, gates, o, log_d_sparse, d_lr,
                                    m_sparse, status, st);
                            }),

@@ -45,8 +45,9 @@ struct Plan {
     float beta, eps, scale, lambda;
     int fusion_mode;
     int impl;        // resolved: 1 = SIMT, 2 = tensor core
+    int Lg_pad;      // L * gamma rounded up to 16 (projection MMA width)
     size_t off_status, off_keyrank, off_hist, off_perm, off_part, off_A,
-        off_B, off_Bh, total;
+        off_B, off_Bh, off_W, total;
 };
 
 // Records a one-line error for elsaa_last_error() and returns `code`.
@@ -98,18 +99,23 @@ cudaError_t launch_block_attn_tc(
 cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
                               uint64_t rows, uint64_t cols, uint32_t box_rows);
 
+// RACE planes as bf16 rows [H][Lg_pad][d] (rows >= L * gamma zero), the
+// operand image the tensor-core kernels load with TMA.
+cudaError_t launch_prep_planes(const Plan &P, const float *w_race,
+                               uint16_t *w_bf16, cudaStream_t st);
+
 // Warp-specialised RACE key summaries (tensor-core path).
 size_t race_keys_ws_smem(const Plan &P);
 uint32_t race_keys_ws_cols(const Plan &P);
 cudaError_t launch_race_keys_ws(const Plan &P, const void *k, const void *v,
-                                const float *w_race, float *part,
+                                const uint16_t *w_bf16, float *part,
                                 DeviceStatus *status, cudaStream_t st);
 
 // Persistent warp-specialised block attention (key blocks of <= 128).
 bool ws_supported(const Plan &P);
 cudaError_t launch_block_attn_ws(
     const Plan &P, const void *q, const void *k, const void *v,
-    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
+    const uint16_t *w_bf16, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const uint16_t *Bh, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
     float *m_sparse, DeviceStatus *status, cudaStream_t st);

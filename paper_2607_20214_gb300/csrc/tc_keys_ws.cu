@@ -29,7 +29,7 @@ using namespace tc;
 constexpr int kKwThreads = 320;
 
 struct KwBars {
-    uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2], done;
+    uint64_t k_full[2], k_empty[2], v_full[2], v_empty[2], w_full, done;
     uint64_t proj_full[2];
     uint64_t phi_full[2], phi_empty[2];  // per row half
 };
@@ -38,7 +38,8 @@ template <int G>
 __global__ void __launch_bounds__(kKwThreads, 1)
     k_race_keys_ws(const __grid_constant__ CUtensorMap tmK,
                    const __grid_constant__ CUtensorMap tmV,
-                   const float *__restrict__ w_race, int N, int d, int H,
+                   const __grid_constant__ CUtensorMap tmW, int N, int d,
+                   int H,
                    int L, int r_pad, int Lg_pad, int chunk, float beta,
                    uint32_t tmem_cols, float *__restrict__ part,
                    DeviceStatus *status) {
@@ -70,6 +71,7 @@ __global__ void __launch_bounds__(kKwThreads, 1)
     if (warp == 1) tmem_alloc(&tbase, tmem_cols);
     if (tid == 0) {
         mbar_init(&bars.done, 1);
+        mbar_init(&bars.w_full, 1);
         for (int b = 0; b < 2; ++b) {
             mbar_init(&bars.k_full[b], 1);
             mbar_init(&bars.k_empty[b], 1);
@@ -82,8 +84,6 @@ __global__ void __launch_bounds__(kKwThreads, 1)
         abort_flag = 0;
         fence_mbar_init();
     }
-    load_planes_bf16(sW, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid,
-                     kKwThreads);
     for (int i = tid; i < 4096 / 16; i += kKwThreads)
         asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
                          sOnes + i * 16),
@@ -94,6 +94,13 @@ __global__ void __launch_bounds__(kKwThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t t = tbase;
+    // this head's bf16 planes (one TMA box of Lg_pad rows per 64 columns)
+    if (tid == 0) {
+        mbar_expect_tx(&bars.w_full, (uint32_t)Lg_pad * d * 2u);
+        for (int pnl = 0; pnl < d / 64; ++pnl)
+            tma_load_2d(sW + pnl * Lg_pad * 128, &tmW, 64 * pnl, h * Lg_pad,
+                        &bars.w_full);
+    }
 
     const int c0 = s * chunk;
     const int c1 = min(N, c0 + chunk);
@@ -183,7 +190,7 @@ __global__ void __launch_bounds__(kKwThreads, 1)
             // projections run two tiles ahead (both TMEM buffers); each
             // iteration issues the summary MMAs of tile i, then the
             // projection of tile i + 2
-            bool ok = true;
+            bool ok = mbar_wait_or_abort(&bars.w_full, 0, abort, status, 60);
             for (int it = 0; it < 2 && it < ntiles && ok; ++it) {
                 ok = mbar_wait_or_abort(&bars.k_full[it], 0, abort, status, 63);
                 if (ok) {
@@ -370,8 +377,33 @@ uint32_t race_keys_ws_cols(const Plan &P) {
     return pow2_cols_kw((r_pad / 128) * (P.d + 16) + 128);
 }
 
+namespace {
+__global__ void k_prep_planes(const float *__restrict__ w, int H, int Lg,
+                              int Lg_pad, int d, uint16_t *__restrict__ out) {
+    const long n = (long)H * Lg_pad * d;
+    for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n;
+         i += (long)gridDim.x * blockDim.x) {
+        const int c = (int)(i % d);
+        const long hr = i / d;
+        const int row = (int)(hr % Lg_pad), h = (int)(hr / Lg_pad);
+        const float x = row < Lg ? w[((long)h * Lg + row) * d + c] : 0.0f;
+        const __nv_bfloat16 b = __float2bfloat16_rn(x);
+        out[i] = *reinterpret_cast<const uint16_t *>(&b);
+    }
+}
+}  // namespace
+
+cudaError_t launch_prep_planes(const Plan &P, const float *w_race,
+                               uint16_t *w_bf16, cudaStream_t st) {
+    const long n = (long)P.H * P.Lg_pad * P.d;
+    const int blocks = (int)((n + 255) / 256 < 1024 ? (n + 255) / 256 : 1024);
+    k_prep_planes<<<blocks, 256, 0, st>>>(w_race, P.H, P.L * P.gamma,
+                                          P.Lg_pad, P.d, w_bf16);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_race_keys_ws(const Plan &P, const void *k, const void *v,
-                                const float *w_race, float *part,
+                                const uint16_t *w_bf16, float *part,
                                 DeviceStatus *status, cudaStream_t st) {
     const int r_pad = (P.r + 127) / 128 * 128;
     const int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
@@ -382,16 +414,19 @@ cudaError_t launch_race_keys_ws(const Plan &P, const void *k, const void *v,
     const size_t cap = (size_t)233472 / (fit + 1) + 1;
     const size_t smem = need > cap ? need : cap;
     dim3 grid(P.S, P.BH);
-    CUtensorMap tmK, tmV;
+    CUtensorMap tmK, tmV, tmW;
     const uint64_t rows = (uint64_t)P.BH * P.N;
     cudaError_t e = make_tma_map_bf16(&tmK, k, rows, P.d, 128);
     if (e == cudaSuccess) e = make_tma_map_bf16(&tmV, v, rows, P.d, 128);
+    if (e == cudaSuccess)
+        e = make_tma_map_bf16(&tmW, w_bf16, (uint64_t)P.H * P.Lg_pad, P.d,
+                              (uint32_t)P.Lg_pad);
     if (e != cudaSuccess) return e;
     auto launch = [&](auto kern) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         kern<<<grid, kKwThreads, smem, st>>>(
-            tmK, tmV, w_race, P.N, P.d, P.H, P.L, r_pad, lg_pad, P.chunk,
+            tmK, tmV, tmW, P.N, P.d, P.H, P.L, r_pad, lg_pad, P.chunk,
             P.beta, cols, part, status);
         return cudaGetLastError();
     };

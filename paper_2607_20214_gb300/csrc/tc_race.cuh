@@ -16,12 +16,16 @@ __device__ __forceinline__ uint32_t align1k(uint32_t x) {
 
 // RACE planes of one head as bf16 rows [Lg_pad x d] in the panel layout;
 // rows >= Lg are zero.
+// With row0 / prows: the planes are rows [row0, row0 + Lg_pad) of a panel
+// layout of prows rows (planes stacked under a key tile).
 __device__ inline void load_planes_bf16(uint32_t dst, const float *w, int Lg,
-                                 int Lg_pad, int d, int tid, int nthreads) {
+                                 int Lg_pad, int d, int tid, int nthreads,
+                                 int row0 = 0, int prows = 0) {
     const int chunks = d >> 3;
+    if (prows == 0) prows = Lg_pad;
     for (int i = tid; i < Lg_pad * chunks; i += nthreads) {
         int row = i / chunks, c = i - row * chunks;
-        uint32_t addr = dst + panel_offset(row, c, Lg_pad);
+        uint32_t addr = dst + panel_offset(row0 + row, c, prows);
         if (row < Lg) {
             const float4 *src =
                 reinterpret_cast<const float4 *>(w + (size_t)row * d + c * 8);
@@ -58,6 +62,24 @@ __device__ __forceinline__ void race_bits32(uint32_t taddr, int ncols,
         if (j < ncols) {
             float t = tanh_approx(beta * tanh_approx(__uint_as_float(pr[j])));
             sp[j] = fmaf(0.5f, t, 0.5f);  // 1/2 + tanh(beta u)/2
+        } else {
+            sp[j] = 0.5f;
+        }
+    }
+}
+
+// race_bits32 over 16 projection columns: sp[j] for j < 16, entries past
+// `ncols` set to 1/2. The TMEM load is waited for inside.
+__device__ __forceinline__ void race_bits16(uint32_t taddr, int ncols,
+                                           float beta, float *sp) {
+    uint32_t pr[16];
+    tmem_ld16(taddr, pr);
+    tmem_wait_ld();
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+        if (j < ncols) {
+            float t = tanh_approx(beta * tanh_approx(__uint_as_float(pr[j])));
+            sp[j] = fmaf(0.5f, t, 0.5f);
         } else {
             sp[j] = 0.5f;
         }
@@ -212,6 +234,71 @@ __device__ __forceinline__ void write_phi_tmem_q(const float (&sp)[32], int l0,
                     }
                 }
             }
+        }
+    }
+}
+
+// sum over tables t < nt of phi_t . A_t for the tables of one 64-bucket
+// chunk (at most TT of them; per-bit factors sp[t * G ..], A of the chunk's
+// first table at A). Four independent partial sums in acc.
+template <int G, int TT>
+__device__ __forceinline__ void chunk_den(const float *sp, int nt,
+                                          const float *A, float (&acc)[4]) {
+    constexpr int R = 1 << G;
+#pragma unroll
+    for (int t = 0; t < TT; ++t) {
+        if (t < nt) {
+            if constexpr (G == 4) {
+                float u[4], w[4];
+                table_uw4(&sp[t * G], 1.0f, u, w);
+                acc[t & 3] += table_dot4(u, w, A + t * R);
+            } else {
+                float phi[R];
+                table_phi<G>(&sp[t * G], phi);
+#pragma unroll
+                for (int q = 0; q < R; ++q)
+                    acc[q & 3] = fmaf(phi[q], A[t * R + q], acc[q & 3]);
+            }
+        }
+    }
+}
+
+// Writes the features phi * scale of the nt (<= TT) tables of one 64-bucket
+// chunk as packed bf16 pairs into TMEM: bucket pair (2k, 2k + 1) of the
+// chunk at column taddr + k, k < 32, in two stores of 16 columns (the second
+// only when the chunk holds more than 32 buckets). Pairs past the chunk's
+// last table are zero.
+template <int G, int TT>
+__device__ __forceinline__ void write_phi_chunk(const float *sp, int nt,
+                                                float scale, uint32_t taddr) {
+    constexpr int R = 1 << G;
+    static_assert(TT * R == 64, "a chunk is 64 buckets");
+    uint32_t buf[16];
+#pragma unroll
+    for (int t = 0; t < TT; ++t) {
+        uint32_t pk[R / 2];
+        if (t < nt) {
+            if constexpr (G == 4) {
+                float u[4], w[4];
+                table_uw4(&sp[t * G], scale, u, w);
+                table_pack4(u, w, pk);
+            } else {
+                float phi[R];
+                table_phi<G>(&sp[t * G], phi, scale);
+#pragma unroll
+                for (int q = 0; q < R; q += 2)
+                    pk[q >> 1] = pack_bf16x2(phi[q], phi[q + 1]);
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < R / 2; ++q) pk[q] = 0u;
+        }
+#pragma unroll
+        for (int q = 0; q < R / 2; ++q) {
+            const int k = t * (R / 2) + q;
+            buf[k & 15] = pk[q];
+            if ((k & 15) == 15 && (k < 16 || nt * R > 32))
+                tmem_st16(taddr + (uint32_t)(k - 15), buf);
         }
     }
 }

@@ -6,17 +6,21 @@
 // One CTA per SM walks a contiguous range of 128-query tiles (ordered by
 // head, then sorted position, so the per-head B summary, A summary and RACE
 // planes are loaded once per head). Roles:
-//   warp 0      loader: cp.async gathers of the tile's Q and K rows (one
-//               buffer), V rows (two buffers), and per head the RACE planes
-//               (as bf16), the bf16 B summary and the fp32 A summary.
-//   warp 1      allocates tensor memory and issues every MMA (lane 0).
-//   warps 2-9,  compute for TMEM slot 0 / slot 1 (256 columns each: scores,
-//   10-17       P and pre-scaled features, then the output accumulator);
+//   warps 0-7,  compute for TMEM slot 0 / slot 1 (256 columns each: scores,
+//   8-15        P and pre-scaled features, then the output accumulator);
 //               slot g takes the tiles of local index = g (mod 2), so one
 //               slot's softmax overlaps the other slot's MMAs and loads.
 //               Within a slot, warps w and w + 4 share TMEM lanes (lane
-//               group w mod 4) and split each row's key columns, RACE
-//               tables and output columns.
+//               group w mod 4) and split each row's key columns and output
+//               columns in halves; half h owns the RACE buckets of the
+//               64-bucket chunks h and h + 2, so both halves write features
+//               before and after the P V product.
+//   warp 16     allocates tensor memory and issues every MMA (lane 0).
+//   warps 17-19 loaders: cp.async gathers of the tile's Q rows (warp 17), K
+//               rows (warp 18, which also stages per head the RACE planes as
+//               bf16, the bf16 B summary and the fp32 A summary) and V rows
+//               (warp 19, two buffers). A gather's rate grows with the
+//               number of warps issuing it, hence one warp per operand.
 
 // Per tile: proj + S MMAs -> (group) features, Den, softmax, P and the
 // pre-scaled features into TMEM -> PV and Phi'B MMAs into one accumulator
@@ -32,8 +36,9 @@ namespace {
 
 using namespace tc;
 
-constexpr int kWsThreads = 576;   // loader, MMA and 16 compute warps
-constexpr int kWsLoaders = 32;    // warp 0
+constexpr int kWsThreads = 640;   // 16 compute, MMA and 3 loader warps
+constexpr int kWsMmaWarp = 16;
+constexpr int kWsLoaders = 32;    // threads of one loader warp
 constexpr int kWsNK = 128;        // keys per query tile
 // TMEM slot layout (256 columns): S/P/features region [0, 128) in four
 // 32-column quarters, output accumulator [128, 128 + d). P of keys
@@ -47,7 +52,8 @@ __device__ __forceinline__ uint32_t quarter_col(int k, int col0) {
 }
 
 struct WsBars {
-    uint64_t qk_full, qk_empty, wb_full, head_done;
+    uint64_t qk_full, wb_full, head_done;
+    uint64_t idx_full[2], idx_empty[2];
     uint64_t v_full[2], v_empty[2];
     uint64_t s_full[2], p_full[2], pv_done[2], p2_full[2], o_full[2];
     uint64_t tmem_empty[2];
@@ -58,11 +64,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     k_block_attn_ws(const uint16_t *__restrict__ qx,
                     const uint16_t *__restrict__ kx,
                     const uint16_t *__restrict__ vx,
-                    const float *__restrict__ w_race,
+                    const __grid_constant__ CUtensorMap tmW,
+                    const __grid_constant__ CUtensorMap tmB,
                     const int32_t *__restrict__ perm_q,
                     const int32_t *__restrict__ perm_k,
                     const float *__restrict__ Ag,
-                    const uint16_t *__restrict__ Bh,
                     const float *__restrict__ lambda_tok,
                     const float *__restrict__ gates, uint16_t *__restrict__ ox,
                     float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
@@ -77,6 +83,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     __shared__ uint32_t tbase;
     __shared__ int abort_flag;
     __shared__ float xmax[2][2][128], xsum[2][2][128], xden[2][2][128];
+    // global rows of a tile's queries / keys, per tile parity (written by
+    // the index warp, read by the slot that issues the tile's Q, K copies)
+    __shared__ __align__(16) int qkrow[2][2][128];
+    __shared__ __align__(16) int vrow[128];  // V loader: rows of its tile
+    __shared__ int orow[2][128];          // per slot: output row or -1
     volatile int *abort = &abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
     const int Lg = L * G, r = L * R;
@@ -86,21 +97,25 @@ __global__ void __launch_bounds__(kWsThreads, 1)
 
     const uint32_t tileB = (uint32_t)nk * d * 2u;  // one [128 x d] tile
     const uint32_t base = align1k(smem_u32(smem_raw));
+    // key tile and RACE planes stacked as one B operand of NR rows: the
+    // scores and the query projections come out of one MMA (N = NR) into
+    // TMEM columns [0, 128) and [128, 128 + Lg_pad)
+    const int NR = nk + Lg_pad;
     const uint32_t sQ = base;
-    const uint32_t sK = sQ + tileB;
-    const uint32_t sW = sK + tileB;
-    const uint32_t sV0 = sW + align1k(Lg_pad * d * 2);
+    const uint32_t sKW = sQ + tileB;
+    const uint32_t sV0 = sKW + align1k((uint32_t)NR * d * 2u);
     const uint32_t sB = sV0 + 2 * tileB;
     const uint32_t sA = sB + align1k(r * d * 2);  // fp32 [r]
     const float *Asm = reinterpret_cast<const float *>(smem_raw + (sA - smem_u32(smem_raw)));
 
-    if (warp == 1) tmem_alloc(&tbase, 512);
+    if (warp == kWsMmaWarp) tmem_alloc(&tbase, 512);
     if (tid == 0) {
-        mbar_init(&bars.qk_full, kWsLoaders);
-        mbar_init(&bars.qk_empty, 1);
-        mbar_init(&bars.wb_full, kWsLoaders);
+        mbar_init(&bars.qk_full, 256);  // the issuing slot's threads
+        mbar_init(&bars.wb_full, 1);
         mbar_init(&bars.head_done, 1);
         for (int s = 0; s < 2; ++s) {
+            mbar_init(&bars.idx_full[s], kWsLoaders);
+            mbar_init(&bars.idx_empty[s], 256);
             mbar_init(&bars.v_full[s], kWsLoaders);
             mbar_init(&bars.v_empty[s], 1);
             mbar_init(&bars.s_full[s], 1);
@@ -118,204 +133,264 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     tc_fence_after();
     const uint32_t tm = tbase;
 
-    auto tile_head = [=](int i) {
-        return (int)((t_begin + i) / tiles_per_head);
-    };
-    auto tile_p0 = [=](int i) {
-        return (int)((t_begin + i) % tiles_per_head) * 128;
-    };
+    // tile indices fit in int (checked on the host)
+    const int tb = (int)t_begin;
+    auto tile_head = [=](int i) { return (tb + i) / tiles_per_head; };
+    auto tile_p0 = [=](int i) { return (tb + i) % tiles_per_head * 128; };
     auto new_head = [=](int i) {
-        return i == 0 || tile_head(i) != tile_head(i - 1);
+        return i == 0 || (tb + i) % tiles_per_head == 0;
     };
-    auto head_last = [=](int i) {
-        return i == ntiles - 1 || tile_head(i + 1) != tile_head(i);
-    };
-    auto key_pos0 = [=](int p0) { return b >= 128 ? (p0 / b) * b : p0; };
-
-    if (warp == 0) {
-        // ------------------------------------------------------------- loader
-        const int lt = lane_id;
-        const int chunks = d >> 3;
-        constexpr int kRows = kWsNK / kWsLoaders;  // rows per loader thread
-        int hc = 0;           // heads loaded
-        int pending_v = -1;   // tile whose V copies are not yet signalled
-        // signal_v: the V copies of tile pending_v have landed (all but the
-        // newest copy group when keep_newest) -> arrive on its barrier
-#define ELSAA_SIGNAL_V(keep_newest)                       \
-    do {                                                  \
-        if (pending_v >= 0) {                             \
-            if (keep_newest)                              \
-                cp_async_wait<1>();                       \
-            else                                          \
-                cp_async_wait<0>();                       \
-            fence_proxy_async_smem();                     \
-            mbar_arrive(&bars.v_full[pending_v & 1]);     \
-            pending_v = -1;                               \
-        }                                                 \
-    } while (0)
-        auto clampi = [=](int i) { return (i < 0 || i >= N) ? 0 : i; };
-        auto copy_row = [=](uint32_t dst, int row, const uint16_t *g) {
-            for (int c = 0; c < chunks; ++c)
-                cp_async16(dst + panel_offset(row, c, nk), g + c * 8);
+    // global row numbers of the 4 sorted positions pos.. pos + 3 (the
+    // ragged end repeats the last row; those rows are never stored)
+    auto rows4 = [=](const int32_t *pm, int pos, int rowbase) {
+        int4 r;
+        if (pos + 3 < N && ((uintptr_t)(pm + pos) & 15u) == 0) {
+            r = *reinterpret_cast<const int4 *>(pm + pos);
+        } else {
+            r.x = pm[min(pos, N - 1)];
+            r.y = pm[min(pos + 1, N - 1)];
+            r.z = pm[min(pos + 2, N - 1)];
+            r.w = pm[min(pos + 3, N - 1)];
+        }
+        auto fix = [=](int v) {
+            return rowbase + ((v < 0 || v >= N) ? 0 : v);
         };
-        for (int i = 0; i < ntiles; ++i) {
-            const int bh = tile_head(i), p0 = tile_p0(i), kp0 = key_pos0(p0);
-            const int32_t *pq = perm_q + (size_t)bh * N;
-            const int32_t *pk = perm_k + (size_t)bh * N;
-            // row indices first (independent loads in flight together)
-            int iq[kRows], ik[kRows];
-#pragma unroll
-            for (int u = 0; u < kRows; ++u) {
-                iq[u] = pq[min(p0 + lt + u * kWsLoaders, N - 1)];
-                ik[u] = pk[min(kp0 + lt + u * kWsLoaders, N - 1)];
-            }
-            const uint16_t *qh = qx + (size_t)bh * N * d;
-            const uint16_t *kh = kx + (size_t)bh * N * d;
-            const uint16_t *vh = vx + (size_t)bh * N * d;
-            if (new_head(i)) {
-                ELSAA_SIGNAL_V(false);
-                if (i > 0 && !mbar_wait_or_abort(&bars.head_done, (hc - 1) & 1,
-                                                 abort, status, 31))
-                    break;
-                load_planes_bf16(sW, w_race + (size_t)(bh % H) * Lg * d, Lg,
-                                 Lg_pad, d, lt, kWsLoaders);
-                load_rows(sB, Bh + (size_t)bh * r * d, r, d, d, lt,
-                          kWsLoaders);
-                for (int c = lt; c < r / 4; c += kWsLoaders)
-                    cp_async16(sA + 16 * c, Ag + (size_t)bh * r + 4 * c);
-                cp_async_commit();
-                cp_async_wait<0>();
-                fence_proxy_async_smem();
-                mbar_arrive(&bars.wb_full);
-                ++hc;
-            }
-            if (i > 0 && !mbar_wait_or_abort(&bars.qk_empty, (i - 1) & 1,
-                                             abort, status, 32))
-                break;
-#pragma unroll
-            for (int u = 0; u < kRows; ++u) {
-                copy_row(sQ, lt + u * kWsLoaders, qh + (size_t)clampi(iq[u]) * d);
-                copy_row(sK, lt + u * kWsLoaders, kh + (size_t)clampi(ik[u]) * d);
-            }
-            cp_async_commit();
-            ELSAA_SIGNAL_V(true);
-            if (i >= 2 && !mbar_wait_or_abort(&bars.v_empty[i & 1],
-                                              ((i >> 1) - 1) & 1, abort,
-                                              status, 33))
-                break;
-            const uint32_t sV = sV0 + (i & 1) * tileB;
-#pragma unroll
-            for (int u = 0; u < kRows; ++u)
-                copy_row(sV, lt + u * kWsLoaders, vh + (size_t)clampi(ik[u]) * d);
-            cp_async_commit();
-            pending_v = i;
-            cp_async_wait<1>();
-            fence_proxy_async_smem();
-            mbar_arrive(&bars.qk_full);
-        }
-        ELSAA_SIGNAL_V(false);
-#undef ELSAA_SIGNAL_V
-        cp_async_wait<0>();
-    } else if (warp == 1) {
-        // ----------------------------------------------------------- MMA issue
-        if (lane_id == 0 && ntiles > 0) {
-            const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
-            const uint32_t id_s = idesc_bf16(128, nk, false, false);
-            const uint32_t id_o = idesc_bf16(128, d, false, true);
-            const int r0 = min(r, nk);
-            auto finish = [&](int j) -> bool {
-                const int s = j & 1, k = j >> 1;
-                const uint32_t so = tm + 256u * s;
-                if (!mbar_wait_or_abort(&bars.p_full[s], k & 1, abort, status,
-                                        41) ||
-                    !mbar_wait_or_abort(&bars.v_full[s], k & 1, abort, status,
-                                        42))
-                    return false;
-                tc_fence_after();
-                const uint32_t sV = sV0 + s * tileB;
-                for (int kk = 0; kk < nk / 16; ++kk)  // O = P V
-                    mma_ts(so + nk, so + quarter_col(kk, 0),
-                           smem_desc(sV + kk * 2048, (uint32_t)nk * 128, 1024),
-                           id_o, kk > 0);
-                for (int kk = 0; kk < r0 / 16; ++kk)  // O += Phi' B
-                    mma_ts(so + nk, so + quarter_col(kk, 32),
-                           smem_desc(sB + kk * 2048, (uint32_t)r * 128, 1024),
-                           id_o, 1);
-                mma_commit(&bars.v_empty[s]);
-                if (r > nk) {
-                    mma_commit(&bars.pv_done[s]);
-                    if (!mbar_wait_or_abort(&bars.p2_full[s], k & 1, abort,
-                                            status, 43))
-                        return false;
-                    tc_fence_after();
-                    for (int kk = 0; kk < (r - nk) / 16; ++kk)
-                        mma_ts(so + nk, so + quarter_col(kk, 0),
-                               smem_desc(sB + (uint32_t)nk * 128 + kk * 2048,
-                                         (uint32_t)r * 128, 1024),
-                               id_o, 1);
-                }
-                mma_commit(&bars.o_full[s]);
-                if (head_last(j)) mma_commit(&bars.head_done);
-                return true;
-            };
-            int hc = 0;
-            bool ok = true;
-            for (int i = 0; i < ntiles && ok; ++i) {
-                const int s = i & 1;
-                const uint32_t so = tm + 256u * s;
-                // at a head boundary the loaders wait for the previous
-                // head's MMAs (head_done) before loading the new planes and
-                // B summary: finish the previous tile first
-                if (i >= 1 && new_head(i)) ok = finish(i - 1);
-                if (!ok) break;
-                ok = mbar_wait_or_abort(&bars.qk_full, i & 1, abort, status,
-                                        44);
-                if (ok && new_head(i)) {
-                    ok = mbar_wait_or_abort(&bars.wb_full, hc & 1, abort,
-                                            status, 45);
-                    ++hc;
-                }
-                if (ok && i >= 2)
-                    ok = mbar_wait_or_abort(&bars.tmem_empty[s],
-                                            ((i >> 1) - 1) & 1, abort, status,
-                                            46);
-                if (!ok) break;
-                tc_fence_after();
-                for (int kk = 0; kk < d / 16; ++kk) {
-                    uint32_t oq = (kk >> 2) * 128 * 128 + (kk & 3) * 32;
-                    uint32_t ow = (kk >> 2) * Lg_pad * 128 + (kk & 3) * 32;
-                    uint64_t aq = smem_desc(sQ + oq, 16, 1024);
-                    mma_ss(so + nk, aq, smem_desc(sW + ow, 16, 1024), id_proj,
-                           kk > 0);
-                    mma_ss(so, aq, smem_desc(sK + oq, 16, 1024), id_s, kk > 0);
-                }
-                mma_commit(&bars.s_full[s]);
-                mma_commit(&bars.qk_empty);
-                if (i >= 1 && !new_head(i)) ok = finish(i - 1);
-            }
-            if (ok) finish(ntiles - 1);
-        }
-        __syncwarp();
-    } else {
-        // ------------------------------------------------------ compute groups
-        // warps 2-9: slot 0, warps 10-17: slot 1; within a slot, warps
-        // (w, w + 4) share TMEM lanes and split the row in two halves.
-        const int cw = warp - 2;
-        const int g = cw >> 3;                       // TMEM slot / tile parity
-        const int half = (cw >> 2) & 1;
-        const int row = (warp & 3) * 32 + lane_id;   // query row = TMEM lane
-        const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
-        const int split = table_split(L, G);
-        const int l0 = half ? split : 0, l1 = half ? L : split;
-        const float sl2e = scale * kLog2e;
-        const int r0 = min(r, nk);
-        const int kbeg = half * (nk / 2);
-        auto wwait = [=](uint64_t *bar, uint32_t par, int site) {
+        return make_int4(fix(r.x), fix(r.y), fix(r.z), fix(r.w));
+    };
+
+    if (warp > kWsMmaWarp) {
+        // ------------------------------------------------------------ loaders
+        // warp 17: global row numbers of each tile's queries and keys into
+        //          qkrow[tile & 1] (the copies themselves are issued by the
+        //          compute slot whose scores just freed the Q, K buffer);
+        // warp 18: per head, TMA loads of the bf16 RACE planes (under the
+        //          key rows), the bf16 B summary and the fp32 A summary;
+        // warp 19: V rows with cp.async (whole rows per instruction, into
+        //          the swizzled operand layout); completion reaches v_full
+        //          through cp.async's own mbarrier arrivals.
+        const int role = warp - kWsMmaWarp - 1;
+        const int lt = lane_id;
+        auto lwait = [=](uint64_t *bar, uint32_t par, int site) {
             return __all_sync(0xffffffffu,
                               mbar_wait_or_abort(bar, par, abort, status,
                                                  site));
         };
-        for (int j = g; j < ntiles; j += 2) {
+        if (role == 0) {
+            for (int i = 0; i < ntiles; ++i) {
+                const int bh = tile_head(i), p0 = tile_p0(i), t = i & 1;
+                if (i >= 2 &&
+                    !lwait(&bars.idx_empty[t], ((i >> 1) - 1) & 1, 30))
+                    break;
+                *reinterpret_cast<int4 *>(&qkrow[t][0][4 * lt]) =
+                    rows4(perm_q + (size_t)bh * N, p0 + 4 * lt, bh * N);
+                *reinterpret_cast<int4 *>(&qkrow[t][1][4 * lt]) =
+                    rows4(perm_k + (size_t)bh * N, p0 + 4 * lt, bh * N);
+                __syncwarp();
+                mbar_arrive(&bars.idx_full[t]);
+            }
+        } else if (role == 1) {
+            int hc = 0;
+            for (int i = 0; i < ntiles; ++i) {
+                if (!new_head(i)) continue;
+                const int bh = tile_head(i);
+                if (i > 0 && !lwait(&bars.head_done, (hc - 1) & 1, 31)) break;
+                if (lt == 0) {  // TMA: planes under the key rows, B, A
+                    mbar_expect_tx(&bars.wb_full,
+                                   (uint32_t)(Lg_pad + r) * d * 2u + r * 4u);
+                    for (int p = 0; p < (d >> 6); ++p) {
+                        tma_load_2d(sKW + p * NR * 128 + nk * 128, &tmW,
+                                    64 * p, (bh % H) * Lg_pad, &bars.wb_full);
+                        tma_load_2d(sB + p * r * 128, &tmB, 64 * p, bh * r,
+                                    &bars.wb_full);
+                    }
+                    bulk_load(sA, Ag + (size_t)bh * r, (uint32_t)r * 4u,
+                              &bars.wb_full);
+                }
+                __syncwarp();
+                ++hc;
+            }
+        } else {
+            const int cpr = d >> 3;    // 16-byte chunks per row
+            const int rpi = 32 / cpr;  // rows per instruction
+            const int lrow = lt / cpr, lc = lt - lrow * cpr;
+            for (int i = 0; i < ntiles; ++i) {
+                const int bh = tile_head(i), p0 = tile_p0(i);
+                __syncwarp();  // the previous tile's rows are all read
+                *reinterpret_cast<int4 *>(&vrow[4 * lt]) =
+                    rows4(perm_k + (size_t)bh * N, p0 + 4 * lt, bh * N);
+                __syncwarp();
+                // V of tile i goes to buffer i & 1 once the epilogue of
+                // tile i - 2 has copied its output out of there
+                if (i >= 2 &&
+                    !lwait(&bars.v_empty[i & 1], ((i >> 1) - 1) & 1, 33))
+                    break;
+                const uint32_t sV = sV0 + (i & 1) * tileB;
+                for (int row = lrow; row < nk; row += rpi)
+                    cp_async16(sV + panel_offset(row, lc, nk),
+                               vx + (size_t)vrow[row] * d + lc * 8);
+                cp_async_mbar_arrive(&bars.v_full[i & 1]);
+            }
+            cp_async_wait<0>();
+        }
+    } else if (warp == kWsMmaWarp) {
+        // ----------------------------------------------------------- MMA issue
+        // Event driven: each pass issues whichever MMA group is ready, the
+        // oldest tile's first (second feature part, then P V with the first
+        // part, then the next tile's projections and scores), so one slot's
+        // epilogue never holds back the other slot's products.
+        if (lane_id == 0 && ntiles > 0) {
+            const uint32_t id_sp = idesc_bf16(128, NR, false, false);
+            const uint32_t id_o = idesc_bf16(128, d, false, true);
+            const int r0 = min(r, nk);
+            const bool two_parts = r > nk;
+            int is = 0, ip = 0, i2 = 0;  // next tile for S, P V, part 2
+            // position of each cursor's tile within its head (advanced
+            // incrementally: no divisions in the issue loop)
+            const int tph = tiles_per_head;
+            int ps = (int)(t_begin % tph), pp = ps, p2 = ps;
+            auto adv = [tph](int q) { return q + 1 == tph ? 0 : q + 1; };
+            int hc = 0;                  // heads whose planes were consumed
+            unsigned long long t_last = global_ns();
+            while ((two_parts ? i2 : ip) < ntiles) {
+                bool did = false;
+                if (two_parts && i2 < ip) {
+                    const int s = i2 & 1;
+                    const uint32_t so = tm + 256u * s;
+                    if (mbar_test(&bars.p2_full[s], (i2 >> 1) & 1)) {
+                        tc_fence_after();
+                        for (int kk = 0; kk < (r - nk) / 16; ++kk)
+                            mma_ts(so + nk, so + quarter_col(kk, 0),
+                                   smem_desc(sB + (uint32_t)nk * 128 + kk * 2048,
+                                             (uint32_t)r * 128, 1024),
+                                   id_o, 1);
+                        mma_commit(&bars.o_full[s]);
+                        if (i2 == ntiles - 1 || p2 == tph - 1)
+                            mma_commit(&bars.head_done);
+                        ++i2;
+                        p2 = adv(p2);
+                        did = true;
+                    }
+                }
+                if (ip < is) {
+                    const int s = ip & 1;
+                    const uint32_t so = tm + 256u * s;
+                    if (mbar_test(&bars.p_full[s], (ip >> 1) & 1) &&
+                        mbar_test(&bars.v_full[s], (ip >> 1) & 1)) {
+                        fence_proxy_async_smem();  // cp.async data -> MMA
+                        tc_fence_after();
+                        const uint32_t sV = sV0 + s * tileB;
+                        for (int kk = 0; kk < nk / 16; ++kk)  // O = P V
+                            mma_ts(so + nk, so + quarter_col(kk, 0),
+                                   smem_desc(sV + kk * 2048, (uint32_t)nk * 128,
+                                             1024),
+                                   id_o, kk > 0);
+                        for (int kk = 0; kk < r0 / 16; ++kk)  // O += Phi' B
+                            mma_ts(so + nk, so + quarter_col(kk, 32),
+                                   smem_desc(sB + kk * 2048, (uint32_t)r * 128,
+                                             1024),
+                                   id_o, 1);
+                        if (two_parts) {
+                            mma_commit(&bars.pv_done[s]);
+                        } else {
+                            mma_commit(&bars.o_full[s]);
+                            if (ip == ntiles - 1 || pp == tph - 1)
+                                mma_commit(&bars.head_done);
+                        }
+                        ++ip;
+                        pp = adv(pp);
+                        did = true;
+                    }
+                }
+                // a new head's planes and B summary replace the old ones
+                // only after head_done: its first S waits for every MMA of
+                // the previous head to be issued
+                const bool nh = is == 0 || ps == 0;  // tile is starts a head
+                if (is < ntiles && !(nh && is > 0 &&
+                                     (two_parts ? i2 : ip) < is)) {
+                    const int s = is & 1;
+                    const uint32_t so = tm + 256u * s;
+                    bool ready = mbar_test(&bars.qk_full, is & 1) &&
+                                 (is < 2 || mbar_test(&bars.tmem_empty[s],
+                                                      ((is >> 1) - 1) & 1)) &&
+                                 (!nh || mbar_test(&bars.wb_full, hc & 1));
+                    if (ready) {
+                        if (nh) ++hc;
+                        fence_proxy_async_smem();  // cp.async data -> MMA
+                        tc_fence_after();
+                        for (int kk = 0; kk < d / 16; ++kk) {
+                            uint32_t oq = (kk >> 2) * 128 * 128 + (kk & 3) * 32;
+                            uint32_t okw = (kk >> 2) * NR * 128 + (kk & 3) * 32;
+                            mma_ss(so, smem_desc(sQ + oq, 16, 1024),
+                                   smem_desc(sKW + okw, 16, 1024), id_sp,
+                                   kk > 0);
+                        }
+                        mma_commit(&bars.s_full[s]);
+                        ++is;
+                        ps = adv(ps);
+                        did = true;
+                    }
+                }
+                if (did) {
+                    t_last = global_ns();
+                } else {
+                    if (*abort) break;
+                    if (global_ns() - t_last > kWaitLimitNs) {
+                        *abort = 1;
+                        record_timeout(status, 41);
+                        break;
+                    }
+                }
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------ compute groups
+        // warps 0-7: slot 0, warps 8-15: slot 1; within a slot, warps
+        // (w, w + 4) share TMEM lanes and split the row in two halves.
+        const int cw = warp;
+        const int g = cw >> 3;                       // TMEM slot / tile parity
+        const int half = (cw >> 2) & 1;
+        const int row = (warp & 3) * 32 + lane_id;   // query row = TMEM lane
+        const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
+        // RACE buckets of this half: the 64-bucket chunks c = half (written
+        // with P, before the P V product) and c = half + 2 (written after
+        // it); chunk c holds tables [c T, c T + T)
+        constexpr int T = R >= 64 ? 1 : 64 / R;
+        const int ta0 = min(half * T, L), nt0 = min(ta0 + T, L) - ta0;
+        const int ta1 = min((half + 2) * T, L), nt1 = min(ta1 + T, L) - ta1;
+        const uint32_t cb0 = half ? 96u : 32u, cb1 = half ? 64u : 0u;
+        const float sl2e = scale * kLog2e;
+        const int kbeg = half * (nk / 2);
+        // a slot's 256 threads leave a wait with one verdict (an abort
+        // seen by some warps only would strand the others at the slot's
+        // named barriers)
+        auto wwait = [=](uint64_t *bar, uint32_t par, int site) {
+            const bool ok = mbar_wait_or_abort(bar, par, abort, status, site);
+            return named_sync_and(1 + g, 256, ok);
+        };
+        // The Q, K copies of tile t are issued by the other slot (the one
+        // of tile t - 1) as soon as the scores of tile t - 1 free the Q, K
+        // buffer: 256 threads, whole rows per warp instruction; completion
+        // reaches qk_full through cp.async's own mbarrier arrivals.
+        const int ct = (cw & 7) * 32 + lane_id;  // 0..255 within the slot
+        auto issue_qk = [&](int t) -> bool {
+            if (!wwait(&bars.idx_full[t & 1], (t >> 1) & 1, 54)) return false;
+            const int cpr = d >> 3, rpp = 256 / cpr;
+            const int crow = ct / cpr, cc = ct - crow * cpr;
+            const int *qr = qkrow[t & 1][0], *kr = qkrow[t & 1][1];
+            for (int rr = crow; rr < nk; rr += rpp) {
+                cp_async16(sQ + panel_offset(rr, cc, nk),
+                           qx + (size_t)qr[rr] * d + cc * 8);
+                cp_async16(sKW + panel_offset(rr, cc, NR),
+                           kx + (size_t)kr[rr] * d + cc * 8);
+            }
+            cp_async_mbar_arrive(&bars.qk_full);
+            mbar_arrive(&bars.idx_empty[t & 1]);
+            return true;
+        };
+        bool started = true;
+        if (g == 1 && ntiles > 0) started = issue_qk(0);
+        for (int j = g; started && j < ntiles; j += 2) {
             const int k = j >> 1;
             const uint32_t so = tm + 256u * g + lane;
             const int bh = tile_head(j), p0 = tile_p0(j);
@@ -324,37 +399,36 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             int qi = perm_q[(size_t)bh * N + min(qpos, N - 1)];  // prefetch
             if (!wwait(&bars.s_full[g], k & 1, 51)) break;
             tc_fence_after();
-            // RACE features of this half's tables and partial Den (A from
-            // shared memory: the loaders stage it with the planes; the MMA
-            // warp only starts tile j after that head's stage completed)
+            // the A summary (read below) came by TMA: acquire its head's
+            // stage (complete already, since S of this tile waited for it)
+            if ((j < 2 || tile_head(j) != tile_head(j - 2)) &&
+                !wwait(&bars.wb_full, (tile_head(j) - tile_head(0)) & 1, 55))
+                break;
+            if (j + 1 < ntiles && !issue_qk(j + 1)) break;
+            // per-bit factors of this half's tables (sp[0, 16): chunk half,
+            // up to 32 when the chunk has more projection columns and no
+            // second chunk exists; sp[16, 32): chunk half + 2) and partial
+            // Den (A from shared memory: the loaders stage it with the
+            // planes; the MMA warp only starts tile j after that head's
+            // stage completed)
             float sp[32];
-            race_bits32(so + nk + l0 * G, (l1 - l0) * G, beta, sp);
+            if (nt0 * G > 16)
+                race_bits32(so + nk + ta0 * G, nt0 * G, beta, sp);
+            else
+                race_bits16(so + nk + ta0 * G, nt0 * G, beta, sp);
             float dacc[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // independent chains
+            chunk_den<G, T>(sp, nt0, Asm + ta0 * R, dacc);
+            // the second chunk's factors wait for the P V product: kept as
+            // fp16 pairs (factors lie in (0.11, 0.89); relative rounding
+            // 2^-11, below the bf16 rounding of the features they make)
+            uint32_t sp1[8];
+            if constexpr (T * G <= 16) {
+                if (nt1 > 0) {
+                    race_bits16(so + nk + ta1 * G, nt1 * G, beta, sp + 16);
+                    chunk_den<G, T>(sp + 16, nt1, Asm + ta1 * R, dacc);
 #pragma unroll
-            for (int lt = 0; lt < 32 / G; ++lt) {
-                if (G == 4 && l0 + lt < l1) {
-                    float u[4], w[4];
-                    table_uw4(&sp[lt * G], 1.0f, u, w);
-                    dacc[lt & 3] += table_dot4(u, w, Asm + (l0 + lt) * R);
-                } else if (l0 + lt < l1) {
-                    float phi[R];
-                    table_phi<G>(&sp[lt * G], phi);
-                    const float *a = Asm + (l0 + lt) * R;
-                    if (R >= 4) {
-#pragma unroll
-                        for (int q = 0; q < R; q += 4) {
-                            const float4 a4 =
-                                *reinterpret_cast<const float4 *>(a + q);
-                            dacc[0] = fmaf(phi[q], a4.x, dacc[0]);
-                            dacc[1] = fmaf(phi[q + 1], a4.y, dacc[1]);
-                            dacc[2] = fmaf(phi[q + 2], a4.z, dacc[2]);
-                            dacc[3] = fmaf(phi[q + 3], a4.w, dacc[3]);
-                        }
-                    } else {
-#pragma unroll
-                        for (int q = 0; q < R; ++q)
-                            dacc[q & 3] = fmaf(phi[q], a[q], dacc[q & 3]);
-                    }
+                    for (int q = 0; q < 8; ++q)
+                        sp1[q] = pack_f16x2(sp[16 + 2 * q], sp[17 + 2 * q]);
                 }
             }
             const float den = (dacc[0] + dacc[1]) + (dacc[2] + dacc[3]);
@@ -364,28 +438,15 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             const bool masked = b < 128;
 #pragma unroll
-            for (int c = 0; c < nk / 2; c += 32) {
-                uint32_t v0[16], v1[16];
-                tmem_ld16(so + kbeg + c, v0);
-                tmem_ld16(so + kbeg + c + 16, v1);
+            for (int c = 0; c < nk / 2; c += 16) {
+                uint32_t v[16];
+                tmem_ld16(so + kbeg + c, v);
                 tmem_wait_ld();
-                if (!masked) {
 #pragma unroll
-                    for (int jj = 0; jj < 16; ++jj)
-                        mxa[jj & 3] = fmaxf(mxa[jj & 3],
-                                            fmaxf(__uint_as_float(v0[jj]),
-                                                  __uint_as_float(v1[jj])));
-                } else {
-#pragma unroll
-                    for (int jj = 0; jj < 16; ++jj) {
-                        const int key0 = kbeg + c + jj, key1 = key0 + 16;
-                        if (key0 >= klo && key0 < khi)
-                            mxa[jj & 3] =
-                                fmaxf(mxa[jj & 3], __uint_as_float(v0[jj]));
-                        if (key1 >= klo && key1 < khi)
-                            mxa[jj & 3] =
-                                fmaxf(mxa[jj & 3], __uint_as_float(v1[jj]));
-                    }
+                for (int jj = 0; jj < 16; ++jj) {
+                    const int key = kbeg + c + jj;
+                    if (!masked || (key >= klo && key < khi))
+                        mxa[jj & 3] = fmaxf(mxa[jj & 3], __uint_as_float(v[jj]));
                 }
             }
             float mx = fmaxf(fmaxf(mxa[0], mxa[1]), fmaxf(mxa[2], mxa[3]));
@@ -399,20 +460,19 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
             for (int c = 0; c < nk / 2; c += 32) {
-                uint32_t v[2][16];
-                tmem_ld16(so + kbeg + c, v[0]);
-                tmem_ld16(so + kbeg + c + 16, v[1]);
-                tmem_wait_ld();
                 uint32_t pk16[16];
 #pragma unroll
                 for (int hh = 0; hh < 2; ++hh) {
+                    uint32_t v[16];
+                    tmem_ld16(so + kbeg + c + 16 * hh, v);
+                    tmem_wait_ld();
 #pragma unroll
                     for (int jj = 0; jj < 16; jj += 2) {
                         const int key = kbeg + c + 16 * hh + jj;
                         float a0 = ex2_approx(
-                            fmaf(__uint_as_float(v[hh][jj]), sl2e, -M2));
+                            fmaf(__uint_as_float(v[jj]), sl2e, -M2));
                         float a1 = ex2_approx(
-                            fmaf(__uint_as_float(v[hh][jj + 1]), sl2e, -M2));
+                            fmaf(__uint_as_float(v[jj + 1]), sl2e, -M2));
                         if (masked) {
                             a0 = (key >= klo && key < khi) ? a0 : 0.0f;
                             a1 = (key + 1 >= klo && key + 1 < khi) ? a1 : 0.0f;
@@ -444,70 +504,100 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             const float c1e = fmaxf(c1, 1e-30f);
             const float ratio =
                 __fdividef(gl, (float)L * (denf + eps) * c1e);
-            const int b0 = l0 * R, b1 = l1 * R;  // this half's buckets
-            if (b0 < r0 && b1 > b0)
-                write_phi_tmem_q<G>(sp, l0, l1, r, ratio, 0, r0, so + 32);
+            if (nt0 > 0) write_phi_chunk<G, T>(sp, nt0, ratio, so + cb0);
             tmem_wait_st();
             tc_fence_before();
             mbar_arrive(&bars.p_full[g]);
             if (r > nk) {
                 if (!wwait(&bars.pv_done[g], k & 1, 52)) break;
                 tc_fence_after();
-                if (b1 > nk && b1 > b0)
-                    write_phi_tmem_q<G>(sp, l0, l1, r, ratio, nk, r, so);
+                if constexpr (T * G <= 16) {
+                    if (nt1 > 0) {
+                        float f1[16];
+#pragma unroll
+                        for (int q = 0; q < 8; ++q)
+                            unpack_f16x2(sp1[q], f1[2 * q], f1[2 * q + 1]);
+                        write_phi_chunk<G, T>(f1, nt1, ratio, so + cb1);
+                    }
+                }
                 tmem_wait_st();
                 tc_fence_before();
                 mbar_arrive(&bars.p2_full[g]);
             }
             if (!wwait(&bars.o_full[g], k & 1, 53)) break;
             tc_fence_after();
-            uint16_t *orow = ox + tok * d;
-            for (int c = half * (d >> 1); c < (half + 1) * (d >> 1); c += 32) {
-                uint32_t v[32];
-                tmem_ld16(so + nk + c, *reinterpret_cast<uint32_t(*)[16]>(&v[0]));
-                tmem_ld16(so + nk + c + 16,
-                          *reinterpret_cast<uint32_t(*)[16]>(&v[16]));
-                tmem_wait_ld();
-                if (qvalid) {
-                    uint4 *dst = reinterpret_cast<uint4 *>(orow + c);
+            // O = c1 acc as bf16, this half's d / 2 columns, staged in this
+            // slot's V buffer (the P V product of the tile is complete) in
+            // the swizzled panel layout, then copied out by the slot's 256
+            // threads in whole rows (coalesced 16-byte stores)
+            const uint32_t sVg = sV0 + g * tileB;
+            constexpr int kMaxHalf = 64;  // d / 2 for d = 128
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        uint4 w;
-                        w.x = pack_bf16x2(c1e * __uint_as_float(v[8 * q]),
-                                          c1e * __uint_as_float(v[8 * q + 1]));
-                        w.y = pack_bf16x2(c1e * __uint_as_float(v[8 * q + 2]),
-                                          c1e * __uint_as_float(v[8 * q + 3]));
-                        w.z = pack_bf16x2(c1e * __uint_as_float(v[8 * q + 4]),
-                                          c1e * __uint_as_float(v[8 * q + 5]));
-                        w.w = pack_bf16x2(c1e * __uint_as_float(v[8 * q + 6]),
-                                          c1e * __uint_as_float(v[8 * q + 7]));
-                        dst[q] = w;
-                    }
+            for (int c = 0; c < kMaxHalf; c += 16) {
+                if (c < (d >> 1)) {
+                    uint32_t v[16], ob[8];
+                    tmem_ld16(so + nk + half * (d >> 1) + c, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        ob[q] = pack_bf16x2(c1e * __uint_as_float(v[2 * q]),
+                                            c1e * __uint_as_float(v[2 * q + 1]));
+                    const int cidx = (half * (d >> 1) + c) >> 3;  // 16-B chunk
+                    st_shared_v4(sVg + panel_offset(row, cidx, nk), ob[0],
+                                 ob[1], ob[2], ob[3]);
+                    st_shared_v4(sVg + panel_offset(row, cidx + 1, nk), ob[4],
+                                 ob[5], ob[6], ob[7]);
                 }
-            }
-            if (qvalid && half == 0) {
-                if (log_ds_out) log_ds_out[tok] = log_ds;
-                if (dlr_out) dlr_out[tok] = denf;
-                if (m_out) m_out[tok] = msp;
             }
             tc_fence_before();
             mbar_arrive(&bars.tmem_empty[g]);
+            if (half == 0) {
+                orow[g][row] = qvalid ? (int)tok : -1;
+                if (qvalid) {
+                    if (log_ds_out) log_ds_out[tok] = log_ds;
+                    if (dlr_out) dlr_out[tok] = denf;
+                    if (m_out) m_out[tok] = msp;
+                }
+            }
+            named_sync(1 + g, 256);
+            {
+                const int ct = (cw & 7) * 32 + lane_id;  // 0..255
+                const int cpr = d >> 3, rpp = 256 / cpr;
+                const int crow = ct / cpr, cc = ct - crow * cpr;
+                for (int rr = crow; rr < nk; rr += rpp) {
+                    const int orr = orow[g][rr];
+                    if (orr >= 0) {
+                        const uint4 val =
+                            ld_shared_v4(sVg + panel_offset(rr, cc, nk));
+                        *reinterpret_cast<uint4 *>(ox + (size_t)orr * d +
+                                                   cc * 8) = val;
+                    }
+                }
+            }
+            named_sync(1 + g, 256);  // the staging buffer is read
+            if (cw == 8 * g && lane_id == 0) mbar_arrive(&bars.v_empty[g]);
         }
+        cp_async_wait<0>();
     }
     tc_fence_before();
     __syncthreads();
-    if (warp == 1) tmem_dealloc(tm, 512);
+    if (warp == kWsMmaWarp) tmem_dealloc(tm, 512);
 }
 
 }  // namespace
 
 bool ws_supported(const Plan &P) {
-    return tc_supported(P) && P.b <= 128;
+    // a half's chunks: the first may use up to 32 projection columns, the
+    // second (buckets past 128) at most 16, i.e. gamma >= 4 when r > 128;
+    // row numbers in int
+    const long rows = (long)P.N * P.BH;  // row numbers are int
+    return tc_supported(P) && P.b <= 128 && (P.gamma >= 4 || P.r <= 128) &&
+           rows < (1L << 31);
 }
 
 cudaError_t launch_block_attn_ws(
     const Plan &P, const void *q, const void *k, const void *v,
-    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
+    const uint16_t *w_bf16, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const uint16_t *Bh, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
     float *m_sparse, DeviceStatus *status, cudaStream_t st) {
@@ -524,12 +614,19 @@ cudaError_t launch_block_attn_ws(
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = (int)(total < sms ? total : sms);
     const int lg = lg_pad;
+    CUtensorMap tmW, tmB;
+    cudaError_t e = make_tma_map_bf16(&tmW, w_bf16, (uint64_t)P.H * P.Lg_pad,
+                                      P.d, (uint32_t)P.Lg_pad);
+    if (e == cudaSuccess)
+        e = make_tma_map_bf16(&tmB, Bh, (uint64_t)P.BH * P.r, P.d,
+                              (uint32_t)P.r);
+    if (e != cudaSuccess) return e;
     auto launch = [&](auto kern) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         kern<<<grid, kWsThreads, smem, st>>>(
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
-            w_race, perm_q, perm_k, A, Bh, lambda_tok, gates, (uint16_t *)o,
+            tmW, tmB, perm_q, perm_k, A, lambda_tok, gates, (uint16_t *)o,
             log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, P.L, lg, P.beta,
             P.eps, P.scale, P.lambda, P.fusion_mode, tiles_per_head, total,
             status);

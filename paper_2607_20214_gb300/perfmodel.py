@@ -61,9 +61,13 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
     if kernel.startswith("block_attn"):
         by = H * 4 * N * d * e
         fl = H * (4 * N * b * d + 2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
-    elif kernel.startswith("race_partial"):
+    elif kernel.startswith(("race_partial", "race_keys")):
         by = H * 2 * N * d * e
         fl = H * (2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
+    elif kernel.startswith("race_reduce"):
+        by = H * r * (d + 1) * 4  # the summaries A and B, written once
+        fl = 0
+        simt = True
     elif kernel.startswith("sort_hash"):
         by = H * 2 * N * d * e
         fl = H * 4 * N * d * wl.sort_bits

@@ -116,6 +116,13 @@ def test_forward_rejects_null_and_small_workspace_before_launch(lib):
     rc = lib.elsaa_forward(ctypes.byref(p2), *odd, fake, 1 << 40, None)
     assert rc == elsaa.ELSAA_ERR_INVALID_ARG
     assert "aligned" in elsaa.elsaa_last_error()
+    # element-aligned but not 16-byte aligned (q, then w_race)
+    for pos in (0, 4):
+        odd = list(args)
+        odd[pos] = fake + 8
+        rc = lib.elsaa_forward(ctypes.byref(p), *odd, fake, 1 << 40, None)
+        assert rc == elsaa.ELSAA_ERR_INVALID_ARG
+        assert "16-byte" in elsaa.elsaa_last_error()
 
 
 def test_missing_library_fails_loudly(tmp_path):
