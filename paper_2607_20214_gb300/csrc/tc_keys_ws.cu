@@ -1,12 +1,14 @@
 // Warp-specialised RACE key side (Algorithm "RACE Low-Rank Attention
 // Branch", steps 3-7) for bf16 inputs: one CTA accumulates the partial
 // bucket summaries B += Phi_K^T V and A += Phi_K^T 1 of one chunk of keys of
-// one head in tensor memory.
+// one head in tensor memory. A comes out of the same MMAs as B: the value
+// tile is followed in shared memory by a panel of ones, so each MMA has
+// N = d + 16 and its last 16 columns accumulate Phi^T 1.
 //
 // Roles (320 threads):
-//   warp 0      loader (lane 0): TMA loads of key and value tiles into two
-//               buffers each, running up to two tiles ahead; completion is
-//               counted in bytes on the buffers' mbarriers.
+//   warp 0      loader (lane 0): TMA loads of key tiles (two buffers) and
+//               value tiles (one buffer, one tile behind the keys);
+//               completion is counted in bytes on the buffers' mbarriers.
 //   warp 1      allocates tensor memory and issues the MMAs (lane 0): the
 //               projections W^(l) K of tile i+1 (double-buffered in TMEM)
 //               are issued before the summary MMAs of tile i.
@@ -58,15 +60,14 @@ __global__ void __launch_bounds__(kKwThreads, 1)
     const uint32_t base = align1k(smem_u32(smem_raw));
     const uint32_t tileB = 128u * d * 2u;
     const uint32_t sW = base;
-    const uint32_t sOnes = sW + align1k(Lg_pad * d * 2);
-    const uint32_t sK0 = sOnes + 4096;       // two key tiles
-    const uint32_t sV0 = sK0 + 2 * tileB;    // two value tiles
-    const uint32_t sPhi = sV0 + 2 * tileB;   // one feature tile
+    const uint32_t sK0 = sW + align1k(Lg_pad * d * 2);  // two key tiles
+    const uint32_t sV = sK0 + 2 * tileB;  // value tile, then a ones panel
+    const uint32_t sPhi = sV + tileB + 16384u;  // one feature tile
 
-    // TMEM columns: B accumulators [nM][d], A accumulators [nM][16], two
-    // projection buffers of 64 columns.
-    const uint32_t colA = nM * d;
-    const uint32_t colP = colA + nM * 16;
+    // TMEM columns: per M-tile an accumulator of d + 16 columns (B, then A
+    // repeated 16 times), then two projection buffers of 64 columns.
+    const uint32_t accN = (uint32_t)d + 16u;
+    const uint32_t colP = nM * accN;
 
     if (warp == 1) tmem_alloc(&tbase, tmem_cols);
     if (tid == 0) {
@@ -84,9 +85,9 @@ __global__ void __launch_bounds__(kKwThreads, 1)
         abort_flag = 0;
         fence_mbar_init();
     }
-    for (int i = tid; i < 4096 / 16; i += kKwThreads)
+    for (int i = tid; i < 16384 / 16; i += kKwThreads)  // bf16 ones
         asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
-                         sOnes + i * 16),
+                         sV + tileB + i * 16),
                      "r"(0x3F803F80u)
                      : "memory");
     fence_proxy_async_smem();
@@ -126,7 +127,7 @@ __global__ void __launch_bounds__(kKwThreads, 1)
         // ------------------------------------------------------------- loader
         if (lane_id == 0) {
             // K(i) needs the projection of tile i-2 done, V(i) the summary
-            // MMAs of tile i-2; K runs ahead of V
+            // MMAs of tile i-1; K runs ahead of V
             int iv = 0;
             for (int i = 0; i < ntiles; ++i) {
                 const int b = i & 1;
@@ -143,28 +144,25 @@ __global__ void __launch_bounds__(kKwThreads, 1)
                                 y, &bars.k_full[b]);
                 // values up to tile i - 1 (one tile behind the keys)
                 for (; iv < i; ++iv) {
-                    const int bv = iv & 1;
-                    if (iv >= 2 && !mbar_wait_or_abort(&bars.v_empty[bv],
-                                                       ((iv >> 1) - 1) & 1,
-                                                       abort, status, 62))
+                    if (iv >= 1 && !mbar_wait_or_abort(&bars.v_empty[0],
+                                                       (iv - 1) & 1, abort,
+                                                       status, 62))
                         break;
-                    mbar_expect_tx(&bars.v_full[bv], tileB);
+                    mbar_expect_tx(&bars.v_full[0], tileB);
                     for (int pnl = 0; pnl < d / 64; ++pnl)
-                        tma_load_2d(sV0 + bv * tileB + pnl * 16384, &tmV,
-                                    64 * pnl, bh * N + c0 + iv * 128,
-                                    &bars.v_full[bv]);
+                        tma_load_2d(sV + pnl * 16384, &tmV, 64 * pnl,
+                                    bh * N + c0 + iv * 128, &bars.v_full[0]);
                 }
             }
             for (; iv < ntiles; ++iv) {
-                const int bv = iv & 1;
-                if (iv >= 2 && !mbar_wait_or_abort(&bars.v_empty[bv],
-                                                   ((iv >> 1) - 1) & 1, abort,
+                if (iv >= 1 && !mbar_wait_or_abort(&bars.v_empty[0],
+                                                   (iv - 1) & 1, abort,
                                                    status, 62))
                     break;
-                mbar_expect_tx(&bars.v_full[bv], tileB);
+                mbar_expect_tx(&bars.v_full[0], tileB);
                 for (int pnl = 0; pnl < d / 64; ++pnl)
-                    tma_load_2d(sV0 + bv * tileB + pnl * 16384, &tmV, 64 * pnl,
-                                bh * N + c0 + iv * 128, &bars.v_full[bv]);
+                    tma_load_2d(sV + pnl * 16384, &tmV, 64 * pnl,
+                                bh * N + c0 + iv * 128, &bars.v_full[0]);
             }
         }
         __syncwarp();
@@ -172,8 +170,7 @@ __global__ void __launch_bounds__(kKwThreads, 1)
         // ----------------------------------------------------------- MMA issue
         if (lane_id == 0 && ntiles > 0) {
             const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
-            const uint32_t id_b = idesc_bf16(128, d, true, true);
-            const uint32_t id_a = idesc_bf16(128, 16, true, false);
+            const uint32_t id_b = idesc_bf16(128, d + 16, true, true);
             const int last0 = last_mtile(0), last1 = last_mtile(1);
             auto proj = [=](int it) {
                 const uint32_t sK = sK0 + (it & 1) * tileB;
@@ -200,10 +197,9 @@ __global__ void __launch_bounds__(kKwThreads, 1)
             }
             for (int i = 0; i < ntiles && ok; ++i) {
                 const int b = i & 1;
-                ok = mbar_wait_or_abort(&bars.v_full[b], (i >> 1) & 1, abort,
+                ok = mbar_wait_or_abort(&bars.v_full[0], i & 1, abort,
                                         status, 66);
                 bool got0 = false, got1 = false;
-                const uint32_t sV = sV0 + b * tileB;
                 for (int m = 0; m < nM && ok; ++m) {
                     if (tile_needs(m, 0) && !got0)
                         got0 = ok = mbar_wait_or_abort(&bars.phi_full[0], i & 1,
@@ -217,19 +213,15 @@ __global__ void __launch_bounds__(kKwThreads, 1)
                         uint64_t a = smem_desc(sPhi + 2 * m * 16384 + k * 2048,
                                                16384, 1024);
                         uint32_t acc = (i > 0 || k > 0) ? 1u : 0u;
-                        mma_ss(t + m * d, a,
+                        mma_ss(t + m * accN, a,
                                smem_desc(sV + k * 2048, 128 * 128, 1024), id_b,
                                acc);
-                        mma_ss(t + colA + m * 16, a,
-                               smem_desc(sOnes + (k >> 2) * 2048 + (k & 3) * 32,
-                                         16, 1024),
-                               id_a, acc);
                     }
                     if (m == last0) mma_commit(&bars.phi_empty[0]);
                     if (m == last1) mma_commit(&bars.phi_empty[1]);
                 }
                 if (!ok) break;
-                mma_commit(&bars.v_empty[b]);
+                mma_commit(&bars.v_empty[0]);
                 if (i + 2 < ntiles) {
                     // the features of tile i have read projection buffer b
                     ok = mbar_wait_or_abort(&bars.k_full[b],
@@ -326,7 +318,7 @@ __global__ void __launch_bounds__(kKwThreads, 1)
                 for (int c = half * (d >> 1); c < (half + 1) * (d >> 1);
                      c += 32) {
                     uint32_t v[32];
-                    tmem_ld32(t + lane + m * d + c, v);
+                    tmem_ld32(t + lane + m * accN + c, v);
                     tmem_wait_ld();
                     if (rrow < r) {
                         float4 *dst = reinterpret_cast<float4 *>(
@@ -342,7 +334,7 @@ __global__ void __launch_bounds__(kKwThreads, 1)
                 }
                 if (half == 0) {
                     uint32_t a16[16];
-                    tmem_ld16(t + lane + colA + m * 16, a16);
+                    tmem_ld16(t + lane + m * accN + d, a16);
                     tmem_wait_ld();
                     if (rrow < r)
                         out[(size_t)r * d + rrow] = __uint_as_float(a16[0]);
@@ -368,8 +360,8 @@ uint32_t pow2_cols_kw(uint32_t n) {
 size_t race_keys_ws_smem(const Plan &P) {
     const size_t r_pad = (P.r + 127) / 128 * 128;
     const size_t lg_pad = (P.L * P.gamma + 15) / 16 * 16;
-    return 1024 + (lg_pad * P.d * 2 + 1023) / 1024 * 1024 + 4096 +
-           4 * (size_t)128 * P.d * 2 + 128 * r_pad * 2;
+    return 1024 + (lg_pad * P.d * 2 + 1023) / 1024 * 1024 +
+           3 * (size_t)128 * P.d * 2 + 16384 + 128 * r_pad * 2;
 }
 
 uint32_t race_keys_ws_cols(const Plan &P) {
