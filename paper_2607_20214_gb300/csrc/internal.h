@@ -82,9 +82,6 @@ cudaError_t launch_block_attn_simt(
 bool tc_supported(const Plan &P);
 // Chunks per head of the tensor-core RACE key kernel; writes tokens per chunk.
 int tc_race_chunks(const Plan &P, int *chunk);
-cudaError_t launch_race_keys_tc(const Plan &P, const void *k, const void *v,
-                                const float *w_race, float *part,
-                                DeviceStatus *status, cudaStream_t st);
 cudaError_t launch_block_attn_tc(
     const Plan &P, const void *q, const void *k, const void *v,
     const float *w_race, const int32_t *perm_q, const int32_t *perm_k,

@@ -1,11 +1,7 @@
-// Tensor-core (tcgen05 / TMEM, bf16 in, fp32 accumulate) kernels of the
-// ELSAA forward for bf16 inputs.
+// Tensor-core (tcgen05 / TMEM, bf16 in, fp32 accumulate) block attention for
+// bf16 inputs whose key blocks span 256 keys (the persistent kernel in
+// tc_ws.cu covers b <= 128), plus the support checks of the tensor-core path.
 //
-//   k_race_keys_tc   RACE key side (Algorithm "RACE Low-Rank Attention
-//                    Branch", steps 3-7) over one chunk of keys of one head:
-//                    projections W^(l) K_j (MMA), soft-hash features phi
-//                    (CUDA cores), then B += Phi_K^T V and A += Phi_K^T 1
-//                    (MMAs accumulating in TMEM across the chunk).
 //   k_block_attn_tc  one CTA = 128 consecutive sorted query positions:
 //                    sortLSH block attention (Algorithm "sortLSH Sparse
 //                    Exact Attention Branch", block step), the RACE query
@@ -30,218 +26,7 @@ namespace {
 
 using namespace tc;
 
-// ---------------------------------------------------------------------------
-// RACE key side. 256 threads: thread pairs (tid, tid ^ 128) share a key row
-// (a TMEM lane) and split its tables at table_split().
 constexpr int kTcThreads = 256;
-
-template <int G>
-__global__ void __launch_bounds__(kTcThreads, 1)
-    k_race_keys_tc(const uint16_t *__restrict__ kx,
-                   const uint16_t *__restrict__ vx,
-                   const float *__restrict__ w_race, int N, int d, int H,
-                   int L, int r_pad, int Lg_pad, int chunk, float beta,
-                   uint32_t tmem_cols, float *__restrict__ part,
-                   DeviceStatus *status) {
-    constexpr int R = 1 << G;
-    extern __shared__ unsigned char smem_raw[];
-    __shared__ uint64_t mb_proj, mb_acc;
-    __shared__ uint32_t tbase;
-    const int s = blockIdx.x, bh = blockIdx.y, S = gridDim.x;
-    const int h = bh % H;
-    const int tid = threadIdx.x, warp = tid >> 5;
-    const int grp = warp & 3, half = warp >> 2;
-    const int row = grp * 32 + (tid & 31);  // key row of the tile = TMEM lane
-    const int Lg = L * G, r = L * R;
-    const int nM = r_pad >> 7;  // 128-row tiles of the bucket dimension
-    const int split = table_split(L, G);
-    const int l0 = half ? split : 0, l1 = half ? L : split;
-
-    const uint32_t base = align1k(smem_u32(smem_raw));
-    const uint32_t tileB = 128u * d * 2u;
-    const uint32_t sW = base;
-    const uint32_t sOnes = sW + align1k(Lg_pad * d * 2);
-    const uint32_t sK0 = sOnes + 4096;
-    const uint32_t sV0 = sK0 + 2 * tileB;
-    const uint32_t sPhi = sV0 + 2 * tileB;
-
-    // TMEM columns: B accumulators [nM][d], A accumulators [nM][16], proj.
-    const uint32_t colA = nM * d;
-    const uint32_t colP = colA + nM * 16;
-
-    if (warp == 0) tmem_alloc(&tbase, tmem_cols);
-    if (tid == 0) {
-        mbar_init(&mb_proj, 1);
-        mbar_init(&mb_acc, 1);
-        fence_mbar_init();
-    }
-    load_planes_bf16(sW, w_race + (size_t)h * Lg * d, Lg, Lg_pad, d, tid,
-                     kTcThreads);
-    for (int i = tid; i < 4096 / 16; i += kTcThreads) {
-        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
-                         sOnes + i * 16),
-                     "r"(0x3F803F80u)
-                     : "memory");
-    }
-    const int c0 = s * chunk;
-    const int c1 = min(N, c0 + chunk);
-    const int ntiles = c1 > c0 ? (c1 - c0 + 127) / 128 : 0;
-    const uint16_t *kh = kx + (size_t)bh * N * d;
-    const uint16_t *vh = vx + (size_t)bh * N * d;
-
-    auto issue_tile = [&](int it, int stage) {
-        const int n0 = c0 + it * 128;
-        const int chunks = d >> 3;
-        for (int i = tid; i < 128 * chunks; i += kTcThreads) {
-            int rr = i / chunks, c = i - rr * chunks;
-            int n = min(n0 + rr, N - 1);  // rows past the chunk are zeroed
-            uint32_t off = panel_offset(rr, c, 128);
-            cp_async16(sK0 + stage * tileB + off, kh + (size_t)n * d + c * 8);
-            cp_async16(sV0 + stage * tileB + off, vh + (size_t)n * d + c * 8);
-        }
-    };
-    if (ntiles > 0) issue_tile(0, 0);
-    cp_async_commit();
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t t = tbase;
-    const uint32_t lane = (uint32_t)(grp * 32) << 16;
-    const uint32_t id_proj = idesc_bf16(128, Lg_pad, false, false);
-    const uint32_t id_b = idesc_bf16(128, d, true, true);
-    const uint32_t id_a = idesc_bf16(128, 16, true, false);
-    const bool tail_owner = (l1 == L) && (l1 > l0 || half == 0);
-    bool ok = true;
-
-    for (int it = 0; it < ntiles && ok; ++it) {
-        const int stage = it & 1;
-        const uint32_t sK = sK0 + stage * tileB, sV = sV0 + stage * tileB;
-        if (it + 1 < ntiles) {
-            issue_tile(it + 1, stage ^ 1);
-            cp_async_commit();
-            cp_async_wait<1>();
-        } else {
-            cp_async_wait<0>();
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        __syncthreads();
-        tc_fence_after();
-        if (tid == 0 && ok) {
-            for (int k = 0; k < d / 16; ++k) {
-                uint32_t oa = (k >> 2) * 128 * 128 + (k & 3) * 32;
-                uint32_t ow = (k >> 2) * Lg_pad * 128 + (k & 3) * 32;
-                mma_ss(t + colP, smem_desc(sK + oa, 16, 1024),
-                       smem_desc(sW + ow, 16, 1024), id_proj, k > 0);
-            }
-            mma_commit(&mb_proj);
-        }
-        ok = mbar_wait(&mb_proj, it & 1, status, 11);
-        tc_fence_after();
-        // features of key `row`, tables [l0, l1) -> Phi tile row (bf16)
-        float sp[32];
-        race_bits32(t + lane + colP + l0 * G, (l1 - l0) * G, beta, sp);
-        const bool valid = c0 + it * 128 + row < c1;
-        float buf[8];
-#pragma unroll
-        for (int lt = 0; lt < 32 / G; ++lt) {
-            if (G == 4 && l0 + lt < l1) {
-                // 16 features as an outer product, two 16-byte chunks
-                float u[4], w[4];
-                table_uw4(&sp[lt * G], valid ? 1.0f : 0.0f, u, w);
-                uint32_t pk[8];
-                table_pack4(u, w, pk);
-                const int c0 = (l0 * R + lt * R) >> 3;
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-                    asm volatile(
-                        "st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(
-                            sPhi + panel_offset(row, c0 + h, 128)),
-                        "r"(pk[4 * h]), "r"(pk[4 * h + 1]), "r"(pk[4 * h + 2]),
-                        "r"(pk[4 * h + 3])
-                        : "memory");
-            } else if (l0 + lt < l1) {
-                float phi[R];
-                table_phi<G>(&sp[lt * G], phi);
-#pragma unroll
-                for (int q = 0; q < R; ++q) {
-                    const int prel = lt * R + q;  // l0 * R is 32-aligned
-                    buf[prel & 7] = valid ? phi[q] : 0.0f;
-                    if ((prel & 7) == 7)
-                        st_shared_bf16x8(
-                            sPhi + panel_offset(row, (l0 * R + prel) >> 3, 128),
-                            buf);
-                }
-            }
-        }
-        if (tail_owner) {
-            if ((r & 7) != 0) {  // partial last chunk (tables of < 8 buckets)
-                for (int q = r & 7; q < 8; ++q) buf[q] = 0.0f;
-                st_shared_bf16x8(sPhi + panel_offset(row, r >> 3, 128), buf);
-            }
-            for (int c = (r + 7) >> 3; c < (r_pad >> 3); ++c)
-                st_shared_zero16(sPhi + panel_offset(row, c, 128));
-        }
-        fence_proxy_async_smem();
-        tc_fence_before();
-        ok = __syncthreads_and(ok);
-        tc_fence_after();
-        if (tid == 0 && ok) {
-            for (int m = 0; m < nM; ++m) {
-                for (int k = 0; k < 8; ++k) {  // 128 keys, 16 per step
-                    uint64_t a = smem_desc(sPhi + 2 * m * 16384 + k * 2048,
-                                           16384, 1024);
-                    uint32_t acc = (it > 0 || k > 0) ? 1u : 0u;
-                    mma_ss(t + m * d, a,
-                           smem_desc(sV + k * 2048, 128 * 128, 1024), id_b,
-                           acc);
-                    mma_ss(t + colA + m * 16, a,
-                           smem_desc(sOnes + (k >> 2) * 2048 + (k & 3) * 32,
-                                     16, 1024),
-                           id_a, acc);
-                }
-            }
-            mma_commit(&mb_acc);
-        }
-        ok = mbar_wait(&mb_acc, it & 1, status, 12) && ok;
-        tc_fence_after();
-        ok = __syncthreads_and(ok);  // CTA-uniform loop control
-    }
-
-    // write this chunk's partial summaries (each half: half the columns)
-    float *out = part + ((size_t)bh * S + s) * ((size_t)r * d + r);
-    if (ok && ntiles > 0) {
-        for (int m = 0; m < nM; ++m) {
-            const int rrow = m * 128 + row;
-            for (int c = half * (d >> 1); c < (half + 1) * (d >> 1); c += 32) {
-                uint32_t v[32];
-                tmem_ld32(t + lane + m * d + c, v);
-                tmem_wait_ld();
-                if (rrow < r) {
-                    float4 *dst =
-                        reinterpret_cast<float4 *>(out + (size_t)rrow * d + c);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        dst[j] = make_float4(__uint_as_float(v[4 * j]),
-                                             __uint_as_float(v[4 * j + 1]),
-                                             __uint_as_float(v[4 * j + 2]),
-                                             __uint_as_float(v[4 * j + 3]));
-                }
-            }
-            if (half == 0) {
-                uint32_t a16[16];
-                tmem_ld16(t + lane + colA + m * 16, a16);
-                tmem_wait_ld();
-                if (rrow < r) out[(size_t)r * d + rrow] = __uint_as_float(a16[0]);
-            }
-        }
-    } else if (ntiles == 0) {
-        for (int i = tid; i < r * d + r; i += kTcThreads) out[i] = 0.0f;
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (warp == 0) tmem_dealloc(t, tmem_cols);
-}
 
 // Sparse block attention + RACE readout + fusion for 128 sorted queries.
 // 256 threads: thread pairs (tid, tid ^ 128) share a query row (a TMEM lane)
@@ -570,28 +355,6 @@ int tc_race_chunks(const Plan &P, int *chunk) {
     int tiles_per = (tiles + S - 1) / S;
     *chunk = tiles_per * 128;
     return (P.N + *chunk - 1) / *chunk;
-}
-
-cudaError_t launch_race_keys_tc(const Plan &P, const void *k, const void *v,
-                                const float *w_race, float *part,
-                                DeviceStatus *status, cudaStream_t st) {
-    const int r_pad = (P.r + 127) / 128 * 128;
-    const int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
-    const uint32_t cols = pow2_cols((r_pad / 128) * (P.d + 16) + 64);
-    size_t need = 1024 + (size_t)lg_pad * P.d * 2 + 4096 +
-                  4 * (size_t)128 * P.d * 2 + (size_t)128 * r_pad * 2;
-    size_t smem = smem_for(need, cols);
-    dim3 grid(P.S, P.BH);
-    return dispatch_gamma(P.gamma, [&](auto g) {
-        constexpr int G = decltype(g)::value;
-        auto kern = k_race_keys_tc<G>;
-        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)smem);
-        kern<<<grid, kTcThreads, smem, st>>>(
-            (const uint16_t *)k, (const uint16_t *)v, w_race, P.N, P.d, P.H,
-            P.L, r_pad, lg_pad, P.chunk, P.beta, cols, part, status);
-        return cudaGetLastError();
-    });
 }
 
 cudaError_t launch_block_attn_tc(

@@ -64,6 +64,11 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
     elif kernel.startswith(("race_partial", "race_keys")):
         by = H * 2 * N * d * e
         fl = H * (2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
+    elif kernel.startswith("prep_planes"):
+        lg = wl.race_tables * wl.race_bits
+        by = wl.H * lg * d * 4 + wl.H * ((lg + 15) // 16 * 16) * d * 2
+        fl = 0
+        simt = True
     elif kernel.startswith("race_reduce"):
         by = H * r * (d + 1) * 4  # the summaries A and B, written once
         fl = 0
