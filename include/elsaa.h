@@ -167,6 +167,42 @@ int elsaa_forward_noalloc(const elsaa_params *params, const void *q,
                           int32_t *perm_k, void *stream);
 
 /*
+ * Backward pass: gradients of a loss L with respect to Q, K, V (and
+ * optionally the gates and the per-token lambda), given dO = dL/dO.
+ *
+ * The paper trains ELSAA end to end but prints no backward pass; this is
+ * the derivative of the forward definitions (Algorithm "sortLSH Sparse
+ * Exact Attention Branch" block step, Algorithm "RACE Low-Rank Attention
+ * Branch", Eq. (5)-(6)). The hash and the sort are piecewise constant and
+ * carry no gradient: the caller passes the permutations perm_q, perm_k that
+ * elsaa_forward returned for the same inputs (required, not recomputed).
+ * Everything else (block scores, features, A and B) is recomputed.
+ *
+ * params, q, k, v, w_sort, w_race, lambda_tok, gates: as for elsaa_forward
+ *              (w_sort is not read).
+ * d_o          [B, H, N, d_h] of params->dtype: dL/dO (device, read only).
+ * perm_q/k     [B, H, N] int32 from elsaa_forward (device, read only).
+ * dq, dk, dv   [B, H, N, d_h] fp32 (device, written).
+ * d_gates      [B, H, N, 2] fp32 dL/d(g_sparse, g_lr), or NULL.
+ * d_lambda     [B, H, N] fp32 dL/dlambda_i, or NULL.
+ * workspace    at least elsaa_backward_workspace_size() bytes, 256-byte
+ *              aligned (a different size from the forward workspace).
+ *
+ * Computed on CUDA cores in fp32 (all dtypes). Supported: the forward's
+ * shapes with b * (4 d_h + b + r + 2) * 4 bytes of block state <= 200 KiB
+ * (e.g. b = 64, d_h = 64, r = 128); ELSAA_ERR_UNSUPPORTED otherwise.
+ * Errors as for elsaa_forward.
+ */
+int elsaa_backward_workspace_size(const elsaa_params *params, size_t *bytes);
+int elsaa_backward(const elsaa_params *params, const void *q, const void *k,
+                   const void *v, const float *w_sort, const float *w_race,
+                   const float *lambda_tok, const float *gates,
+                   const void *d_o, const int32_t *perm_q,
+                   const int32_t *perm_k, float *dq, float *dk, float *dv,
+                   float *d_gates, float *d_lambda, void *workspace,
+                   size_t workspace_bytes, void *stream);
+
+/*
  * Synchronises `stream` and reads the in-band status word that the kernels
  * of the last elsaa_forward on this workspace wrote (bounded waits that ran
  * out, inconsistent sort counts). Returns ELSAA_OK, ELSAA_ERR_DEVICE (with

@@ -362,6 +362,151 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     return ELSAA_OK;
 }
 
+// ---------------------------------------------------------------- backward
+
+namespace {
+
+// Backward workspace: status | RACE chunk partials (A, B, then gA, gB) |
+// A | B | gA | gB | gNum / L [B*H][N][d_h] | gDen / L [B*H][N].
+struct BwdPlan {
+    Plan P;  // forward geometry with CUDA-core RACE chunking
+    size_t off_status, off_part, off_A, off_B, off_gA, off_gB, off_gnum,
+        off_gden, total;
+};
+
+int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
+    elsaa_params q = *p;
+    q.impl = ELSAA_IMPL_SIMT;  // the backward runs on CUDA cores
+    int rc = make_plan(&q, &Bp->P, msg);
+    if (rc != ELSAA_OK) return rc;
+    const Plan &P = Bp->P;
+    if (!bwd_supported(P)) {
+        *msg = "backward: this block size, d_h and r need more shared "
+               "memory than an SM has";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
+    const size_t BHN = (size_t)P.BH * P.N;
+    const size_t per = (size_t)P.r * P.d + P.r;
+    size_t off = 0;
+    Bp->off_status = off;
+    off = align_up(off + sizeof(DeviceStatus), 256);
+    Bp->off_part = off;
+    off = align_up(off + (size_t)P.BH * P.S * per * sizeof(float), 256);
+    Bp->off_A = off;
+    off = align_up(off + (size_t)P.BH * P.r * sizeof(float), 256);
+    Bp->off_B = off;
+    off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(float), 256);
+    Bp->off_gA = off;
+    off = align_up(off + (size_t)P.BH * P.r * sizeof(float), 256);
+    Bp->off_gB = off;
+    off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(float), 256);
+    Bp->off_gnum = off;
+    off = align_up(off + BHN * P.d * sizeof(float), 256);
+    Bp->off_gden = off;
+    off = align_up(off + BHN * sizeof(float), 256);
+    Bp->total = off;
+    return ELSAA_OK;
+}
+
+}  // namespace
+
+extern "C" int elsaa_backward_workspace_size(const elsaa_params *params,
+                                             size_t *bytes) {
+    g_err[0] = 0;
+    if (!bytes) return fail(ELSAA_ERR_INVALID_ARG, "bytes is NULL");
+    BwdPlan Bp;
+    const char *msg = "";
+    int rc = make_bwd_plan(params, &Bp, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    *bytes = Bp.total;
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
+                              const void *k, const void *v,
+                              const float *w_sort, const float *w_race,
+                              const float *lambda_tok, const float *gates,
+                              const void *d_o, const int32_t *perm_q,
+                              const int32_t *perm_k, float *dq, float *dk,
+                              float *dv, float *d_gates, float *d_lambda,
+                              void *workspace, size_t workspace_bytes,
+                              void *stream) {
+    (void)w_sort;  // the permutations are given
+    g_err[0] = 0;
+    BwdPlan Bp;
+    const char *msg = "";
+    int rc = make_bwd_plan(params, &Bp, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    const Plan &P = Bp.P;
+    if (!q || !k || !v || !d_o || !dq || !dk || !dv)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "q, k, v, d_o, dq, dk and dv must be non-NULL");
+    if (!w_race) return fail(ELSAA_ERR_INVALID_ARG, "w_race must be non-NULL");
+    if (!perm_q || !perm_k)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "perm_q and perm_k (from elsaa_forward) are required");
+    const void *ptrs[] = {q, k, v, d_o, w_race, dq, dk, dv};
+    for (const void *p : ptrs)
+        if ((uintptr_t)p % 16)
+            return fail(ELSAA_ERR_INVALID_ARG,
+                        "q, k, v, d_o, w_race, dq, dk and dv must be 16-byte "
+                        "aligned");
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if ((uintptr_t)workspace % 256)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if (workspace_bytes < Bp.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, Bp.total);
+
+    cudaStream_t st = (cudaStream_t)stream;
+    char *ws = (char *)workspace;
+    DeviceStatus *status = (DeviceStatus *)(ws + Bp.off_status);
+    float *part = (float *)(ws + Bp.off_part);
+    float *A = (float *)(ws + Bp.off_A);
+    float *Bm = (float *)(ws + Bp.off_B);
+    float *gA = (float *)(ws + Bp.off_gA);
+    float *gB = (float *)(ws + Bp.off_gB);
+    float *gnum = (float *)(ws + Bp.off_gnum);
+    float *gden = (float *)(ws + Bp.off_gden);
+
+    ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
+                       "status reset");
+    ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
+                           return launch_race_partial_simt(P, k, v, w_race,
+                                                           part, st);
+                       }),
+                       "race_partial_simt");
+    ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
+                           return launch_race_reduce(P, part, A, Bm, nullptr,
+                                                     st);
+                       }),
+                       "race_reduce");
+    ELSAA_CHECK_LAUNCH(timed("bwd_block", st, [&] {
+                           return launch_bwd_block(
+                               P, q, k, v, d_o, w_race, A, Bm, perm_q, perm_k,
+                               lambda_tok, gates, dq, dk, dv, d_gates,
+                               d_lambda, gnum, gden, st);
+                       }),
+                       "bwd_block");
+    ELSAA_CHECK_LAUNCH(timed("bwd_race_sums", st, [&] {
+                           return launch_race_partial_weighted(
+                               P, q, gnum, gden, w_race, part, st);
+                       }),
+                       "bwd_race_sums");
+    ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
+                           return launch_race_reduce(P, part, gA, gB, nullptr,
+                                                     st);
+                       }),
+                       "race_reduce");
+    ELSAA_CHECK_LAUNCH(timed("bwd_keys", st, [&] {
+                           return launch_bwd_keys(P, k, v, w_race, gA, gB, dk,
+                                                  dv, st);
+                       }),
+                       "bwd_keys");
+    return ELSAA_OK;
+}
+
 extern "C" int elsaa_check_status(const void *workspace, void *stream) {
     g_err[0] = 0;
     if (!workspace) return fail(ELSAA_ERR_INVALID_ARG, "workspace is NULL");

@@ -69,6 +69,12 @@ cudaError_t launch_sort_scatter(const Plan &P, const uint32_t *keyrank,
 cudaError_t launch_race_partial_simt(const Plan &P, const void *k,
                                      const void *v, const float *w_race,
                                      float *part, cudaStream_t st);
+// k_race_partial with fp32 values and per-token A weights (backward pass:
+// gB = sum phi(x_i) vals_i^T, gA = sum phi(x_i) wA_i).
+cudaError_t launch_race_partial_weighted(const Plan &P, const void *x,
+                                         const float *vals, const float *wA,
+                                         const float *w_race, float *part,
+                                         cudaStream_t st);
 cudaError_t launch_race_reduce(const Plan &P, const float *part, float *A,
                                float *Bm, uint16_t *Bh, cudaStream_t st);
 cudaError_t launch_block_attn_simt(
@@ -88,6 +94,23 @@ cudaError_t launch_block_attn_tc(
     const float *A, const uint16_t *Bh, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
     float *m_sparse, DeviceStatus *status, cudaStream_t st);
+
+// Backward pass (bwd.cu), CUDA cores.
+size_t bwd_block_smem(const Plan &P);
+size_t bwd_keys_smem(const Plan &P);
+bool bwd_supported(const Plan &P);
+cudaError_t launch_bwd_block(const Plan &P, const void *q, const void *k,
+                             const void *v, const void *d_o,
+                             const float *w_race, const float *A,
+                             const float *Bm, const int32_t *perm_q,
+                             const int32_t *perm_k, const float *lambda_tok,
+                             const float *gates, float *dq, float *dk,
+                             float *dv, float *d_gates, float *d_lambda,
+                             float *gnum, float *gden, cudaStream_t st);
+cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
+                            const float *w_race, const float *gA,
+                            const float *gB, float *dk, float *dv,
+                            cudaStream_t st);
 
 // Row-major bf16 matrix [rows x cols] as a TMA tensor map with boxes of
 // 64 columns x box_rows rows and 128-byte swizzle (the panel layout).

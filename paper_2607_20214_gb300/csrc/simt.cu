@@ -13,12 +13,16 @@ namespace {
 // partial bucket summaries A^(l) = Phi_K^T 1 and B^(l) = Phi_K^T V over one
 // chunk of keys, for one slice of at most 64 buckets (whole tables).
 // Grid (S chunks, slices, BH heads); output part[bh][s] = [r x d] B then [r] A.
+// The same kernel forms the backward pass's gB = sum_i phi(Q_i) gNum_i^T and
+// gA = sum_i phi(Q_i) gDen_i: values of type TV (fp32 there) and an optional
+// per-token weight wA of the A sum (NULL: 1).
 constexpr int kRaceThreads = 256;
 constexpr int kRaceTok = 32;  // keys staged per iteration
 
-template <typename T>
+template <typename T, typename TV>
 __global__ void __launch_bounds__(kRaceThreads)
-    k_race_partial(const T *__restrict__ kx, const T *__restrict__ vx,
+    k_race_partial(const T *__restrict__ kx, const TV *__restrict__ vx,
+                   const float *__restrict__ wA,
                    const float *__restrict__ w_race, int N, int d, int H,
                    int L, int gamma, int tps, int chunk, float beta,
                    float *__restrict__ part) {
@@ -37,6 +41,7 @@ __global__ void __launch_bounds__(kRaceThreads)
     float *vt = kt + kRaceTok * ds;    // [kRaceTok][d]
     float *ph = vt + kRaceTok * d;     // [kRaceTok][64]
     float *wr = ph + kRaceTok * 64;    // [tables in slice][gamma][d]
+    __shared__ float wt[kRaceTok];     // A weights of the staged tokens
 
     for (int i = tid; i < (t1 - t0) * gamma * d; i += kRaceThreads)
         wr[i] = w_race[((size_t)h * L + t0) * gamma * d + i];
@@ -51,7 +56,7 @@ __global__ void __launch_bounds__(kRaceThreads)
     float accA = 0.f;
 
     const T *kh = kx + (size_t)bh * N * d;
-    const T *vh = vx + (size_t)bh * N * d;
+    const TV *vh = vx + (size_t)bh * N * d;
     const int c0 = s * chunk;
     const int c1 = min(N, c0 + chunk);
     for (int base = c0; base < c1; base += kRaceTok) {
@@ -61,7 +66,11 @@ __global__ void __launch_bounds__(kRaceThreads)
             int n = base + row;
             bool ok = n < c1;
             kt[row * ds + col] = ok ? to_f32<T>(kh[(size_t)n * d + col]) : 0.f;
-            vt[row * d + col] = ok ? to_f32<T>(vh[(size_t)n * d + col]) : 0.f;
+            vt[row * d + col] = ok ? to_f32<TV>(vh[(size_t)n * d + col]) : 0.f;
+        }
+        if (tid < kRaceTok) {
+            const int n = base + tid;
+            wt[tid] = n < c1 ? (wA ? wA[(size_t)bh * N + n] : 1.f) : 0.f;
         }
         __syncthreads();
         // features: one task per (token, table)
@@ -96,7 +105,7 @@ __global__ void __launch_bounds__(kRaceThreads)
                 int rb = grp + j * ngrp;
                 if (j < nacc && rb < nb) acc[j] = fmaf(pr[rb], vv, acc[j]);
             }
-            if (tid < nb) accA += pr[tid];
+            if (tid < nb) accA = fmaf(pr[tid], wt[tok], accA);
         }
     }
     float *out = part + ((size_t)bh * S + s) * ((size_t)r * d + r);
@@ -336,20 +345,47 @@ cudaError_t launch_race_partial_simt(const Plan &P, const void *k,
                    (size_t)kRaceTok * 64 +
                    (size_t)P.tables_per_slice * P.gamma * P.d);
     if (P.dtype == ELSAA_FP32) {
-        auto kern = k_race_partial<float>;
+        auto kern = k_race_partial<float, float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         kern<<<grid, kRaceThreads, smem, st>>>(
-            (const float *)k, (const float *)v, w_race, P.N, P.d, P.H, P.L,
-            P.gamma, P.tables_per_slice, P.chunk, P.beta, part);
+            (const float *)k, (const float *)v, nullptr, w_race, P.N, P.d,
+            P.H, P.L, P.gamma, P.tables_per_slice, P.chunk, P.beta, part);
     } else {
-        auto kern = k_race_partial<__nv_bfloat16>;
+        auto kern = k_race_partial<__nv_bfloat16, __nv_bfloat16>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         kern<<<grid, kRaceThreads, smem, st>>>(
-            (const __nv_bfloat16 *)k, (const __nv_bfloat16 *)v, w_race, P.N,
-            P.d, P.H, P.L, P.gamma, P.tables_per_slice, P.chunk, P.beta,
-            part);
+            (const __nv_bfloat16 *)k, (const __nv_bfloat16 *)v, nullptr,
+            w_race, P.N, P.d, P.H, P.L, P.gamma, P.tables_per_slice, P.chunk,
+            P.beta, part);
+    }
+    return cudaGetLastError();
+}
+
+cudaError_t launch_race_partial_weighted(const Plan &P, const void *x,
+                                         const float *vals, const float *wA,
+                                         const float *w_race, float *part,
+                                         cudaStream_t st) {
+    dim3 grid(P.S, P.slices, P.BH);
+    size_t smem = sizeof(float) *
+                  ((size_t)kRaceTok * (P.d + 1) + (size_t)kRaceTok * P.d +
+                   (size_t)kRaceTok * 64 +
+                   (size_t)P.tables_per_slice * P.gamma * P.d);
+    if (P.dtype == ELSAA_FP32) {
+        auto kern = k_race_partial<float, float>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<grid, kRaceThreads, smem, st>>>(
+            (const float *)x, vals, wA, w_race, P.N, P.d, P.H, P.L, P.gamma,
+            P.tables_per_slice, P.chunk, P.beta, part);
+    } else {
+        auto kern = k_race_partial<__nv_bfloat16, float>;
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<grid, kRaceThreads, smem, st>>>(
+            (const __nv_bfloat16 *)x, vals, wA, w_race, P.N, P.d, P.H, P.L,
+            P.gamma, P.tables_per_slice, P.chunk, P.beta, part);
     }
     return cudaGetLastError();
 }

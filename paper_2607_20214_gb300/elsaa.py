@@ -27,7 +27,8 @@ ELSAA_IMPL_SIMT = 1
 
 SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_last_error", "elsaa_abi_version", "elsaa_profile_start",
-           "elsaa_profile_stop", "elsaa_forward_noalloc")
+           "elsaa_profile_stop", "elsaa_forward_noalloc",
+           "elsaa_backward_workspace_size", "elsaa_backward")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -92,6 +93,12 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
                                      ctypes.c_int,
                                      ctypes.POINTER(ctypes.c_int)]
     L.elsaa_profile_stop.restype = ctypes.c_int
+    L.elsaa_backward_workspace_size.argtypes = [
+        ctypes.POINTER(elsaa_params), ctypes.POINTER(ctypes.c_size_t)]
+    L.elsaa_backward_workspace_size.restype = ctypes.c_int
+    L.elsaa_backward.argtypes = [ctypes.POINTER(elsaa_params)] + [vp] * 16 + [
+        ctypes.c_size_t, vp]
+    L.elsaa_backward.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -208,6 +215,63 @@ def elsaa_forward(params: elsaa_params, q, k, v, w_sort, w_race,
                            workspace.numel() * workspace.element_size(), sp)
     _check(rc)
     return o
+
+
+def elsaa_backward_workspace_size(params: elsaa_params) -> int:
+    n = ctypes.c_size_t(0)
+    _check(load_library().elsaa_backward_workspace_size(ctypes.byref(params),
+                                                        ctypes.byref(n)))
+    return n.value
+
+
+def elsaa_backward(params: elsaa_params, q, k, v, w_sort, w_race, d_o,
+                   perm_q, perm_k, lambda_tok=None, gates=None, dq=None,
+                   dk=None, dv=None, d_gates=None, d_lambda=None,
+                   workspace=None, stream=None):
+    """Enqueue elsaa_backward on `stream`; returns (dq, dk, dv) (fp32,
+    allocated here when not given). perm_q, perm_k come from elsaa_forward
+    on the same inputs."""
+    lib = load_library()
+    dev = q.device
+    if dev.type != "cuda":
+        raise ValueError("q must be a CUDA tensor")
+    tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    BHN = params.B * params.H * params.N
+    nqkv = BHN * params.d_h
+    shape = tuple(q.shape)
+    dq = torch.empty(shape, dtype=torch.float32, device=dev) if dq is None else dq
+    dk = torch.empty(shape, dtype=torch.float32, device=dev) if dk is None else dk
+    dv = torch.empty(shape, dtype=torch.float32, device=dev) if dv is None else dv
+    if workspace is None:
+        n = elsaa_backward_workspace_size(params)
+        workspace = torch.empty(max(n, 256), dtype=torch.uint8, device=dev)
+    if stream is None:
+        stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    args = [
+        _ptr(q, "q", tdt, nqkv, dev), _ptr(k, "k", tdt, nqkv, dev),
+        _ptr(v, "v", tdt, nqkv, dev),
+        _ptr(w_sort, "w_sort", torch.float32, None, dev)
+        if w_sort is not None else None,
+        _ptr(w_race, "w_race", torch.float32,
+             params.H * params.race_tables * params.race_bits * params.d_h,
+             dev),
+        _ptr(lambda_tok, "lambda_tok", torch.float32, BHN, dev),
+        _ptr(gates, "gates", torch.float32, 2 * BHN, dev),
+        _ptr(d_o, "d_o", tdt, nqkv, dev),
+        _ptr(perm_q, "perm_q", torch.int32, BHN, dev),
+        _ptr(perm_k, "perm_k", torch.int32, BHN, dev),
+        _ptr(dq, "dq", torch.float32, nqkv, dev),
+        _ptr(dk, "dk", torch.float32, nqkv, dev),
+        _ptr(dv, "dv", torch.float32, nqkv, dev),
+        _ptr(d_gates, "d_gates", torch.float32, 2 * BHN, dev),
+        _ptr(d_lambda, "d_lambda", torch.float32, BHN, dev),
+        _ptr(workspace, "workspace", None, None, dev),
+    ]
+    rc = lib.elsaa_backward(ctypes.byref(params), *args,
+                            workspace.numel() * workspace.element_size(), sp)
+    _check(rc)
+    return dq, dk, dv
 
 
 def elsaa_check_status(workspace: torch.Tensor, stream=None):

@@ -1,0 +1,123 @@
+"""GPU backward (elsaa_backward through the C ABI) versus the oracle's
+analytic fp64 gradient on the same seeded inputs.
+
+The permutations come from the GPU forward and must equal the oracle's
+(integer work, bit-exact). Gradients are compared relative to the largest
+reference magnitude of each tensor: the GPU accumulates in fp32 over at most
+b + r terms per element (b <= 128, r <= 256), so its error stays near
+1e-6 of that magnitude; the bound written here is 1e-3.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import backward as bwd
+from oracle import oracle as orc
+from paper_2607_20214_gb300 import build, elsaa
+from paper_2607_20214_gb300.workloads import (WORKLOADS, Workload,
+                                              make_gates_lambda, make_inputs)
+
+pytestmark = pytest.mark.gpu
+
+TOL_REL = 1e-3
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    elsaa.load_library()
+
+
+def run_gpu(wl, x, gates=None, lam=None):
+    dev = torch.device("cuda:0")
+    p = elsaa.params_for(wl)
+    xd = {k: v.to(dev) for k, v in x.items()}
+    BHN = (wl.B, wl.H, wl.N)
+    perm_q = torch.empty(BHN, dtype=torch.int32, device=dev)
+    perm_k = torch.empty(BHN, dtype=torch.int32, device=dev)
+    g = None if gates is None else gates.to(dev)
+    lt = None if lam is None else lam.to(dev)
+    elsaa.elsaa_forward(p, xd["q"], xd["k"], xd["v"], xd["w_sort"],
+                        xd["w_race"], lambda_tok=lt, gates=g,
+                        perm_q=perm_q, perm_k=perm_k)
+    d_gates = torch.full(BHN + (2,), float("nan"), device=dev)
+    d_lambda = torch.full(BHN, float("nan"), device=dev)
+    dq, dk, dv = elsaa.elsaa_backward(
+        p, xd["q"], xd["k"], xd["v"], xd["w_sort"], xd["w_race"], xd["do"],
+        perm_q, perm_k, lambda_tok=lt, gates=g, d_gates=d_gates,
+        d_lambda=d_lambda)
+    torch.cuda.synchronize()
+    return dict(dQ=dq.cpu(), dK=dk.cpu(), dV=dv.cpu(),
+                dgates=d_gates.cpu(), dlam=d_lambda.cpu(),
+                perm_q=perm_q.cpu(), perm_k=perm_k.cpu())
+
+
+def oracle_head(wl, x, b, h, gates=None, lam=None):
+    f32 = lambda t: t[b, h].float().cpu().numpy()
+    p = orc.params_from_workload(wl)
+    lam_h = None if lam is None else lam[b, h].double().numpy()
+    gates_h = None if gates is None else gates[b, h].double().numpy()
+    if lam_h is None:
+        lam_h = np.full(wl.N, wl.lam)
+    return bwd.backward_head(
+        f32(x["q"]), f32(x["k"]), f32(x["v"]),
+        x["w_sort"][h].float().cpu().numpy(),
+        x["w_race"][h].double().cpu().numpy(), f32(x["do"]), p, lam=lam_h,
+        gates=gates_h)
+
+
+def compare(wl, g, x, heads, gates=None, lam=None):
+    worst = {}
+    for (b, h) in heads:
+        r = oracle_head(wl, x, b, h, gates, lam)
+        assert np.array_equal(g["perm_q"][b, h].numpy(), r["perm_q"])
+        assert np.array_equal(g["perm_k"][b, h].numpy(), r["perm_k"])
+        for name in ("dQ", "dK", "dV"):
+            ref = r[name]
+            err = np.abs(g[name][b, h].numpy() - ref).max() / np.abs(ref).max()
+            worst[name] = max(worst.get(name, 0.0), err)
+            assert err <= TOL_REL, (name, b, h, err)
+        ref = r["dgates"]
+        err = np.abs(g["dgates"][b, h].numpy() - ref).max() / np.abs(ref).max()
+        assert err <= TOL_REL, ("dgates", b, h, err)
+        if wl.fusion_mode == 0:
+            ref = r["dlam"]
+            err = (np.abs(g["dlam"][b, h].numpy() - ref).max()
+                   / max(np.abs(ref).max(), 1e-30))
+            assert err <= TOL_REL, ("dlam", b, h, err)
+    return worst
+
+
+def small(dtype="bf16", **kw):
+    base = dict(name="small", B=1, H=2, N=384, d_h=64, dtype=dtype, block=64,
+                race_tables=4, recipe="plain", temperature=2.0, seed=21,
+                plane_seed=1021, backward=True)
+    base.update(kw)
+    return Workload(**base)
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_small_backward_matches_oracle(dtype):
+    wl = small(dtype)
+    x = make_inputs(wl)
+    gates, lam = make_gates_lambda(wl, seed=3)
+    compare(wl, run_gpu(wl, x, gates, lam), x, [(0, 0), (0, 1)], gates, lam)
+
+
+@pytest.mark.parametrize("over", [dict(fusion_mode=1), dict(block=32),
+                                  dict(d_h=32, race_bits=3, race_tables=6),
+                                  dict(block=128, d_h=32, race_tables=2)])
+def test_backward_variants(over):
+    wl = small("bf16").with_(**over)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), x, [(0, 0), (0, 1)])
+
+
+def test_c5_full_size_sampled_heads():
+    """The training workload at full size (96 heads); the oracle checks
+    two whole heads."""
+    wl = WORKLOADS["c5"]
+    x = make_inputs(wl, device="cuda")
+    g = run_gpu(wl, x)
+    xc = {k: v.cpu() for k, v in x.items()}
+    compare(wl, g, xc, [(0, 0), (7, 11)])
