@@ -35,6 +35,7 @@ from paper_2607_20214_gb300 import perfmodel  # noqa: E402
 from paper_2607_20214_gb300.workloads import WORKLOADS, make_inputs  # noqa
 
 METRIC = "ELSAA fwd tokens/s at N=16K bf16 on 1 GB300"
+METRIC_BWD = "ELSAA bwd tokens/s (dQ, dK, dV fp32) on 1 GB300"
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
                   "bf16_tflops_sustained": 1700.0, "source": "fallback"}
 
@@ -239,6 +240,8 @@ def run_ours(args, wl):
     peaks = load_peaks()
 
     wl_rank = wl.with_(seed=wl.seed + 100 * rank)
+    if args.backward:
+        wl_rank = wl_rank.with_(backward=True)
     x = make_inputs(wl_rank, device=dev)
     p = elsaa.params_for(wl)
     ws = elsaa.new_workspace(p, dev)
@@ -248,6 +251,26 @@ def run_ours(args, wl):
     def step():
         elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
                             x["w_race"], o=o, workspace=ws, stream=stream)
+
+    if args.backward:
+        # the backward pass of the same inputs: permutations from one
+        # forward (outside the timed region), then elsaa_backward per step
+        BHN = (wl.B, wl.H, wl.N)
+        perm_q = torch.empty(BHN, dtype=torch.int32, device=dev)
+        perm_k = torch.empty(BHN, dtype=torch.int32, device=dev)
+        elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                            x["w_race"], o=o, perm_q=perm_q, perm_k=perm_k,
+                            workspace=ws, stream=stream)
+        wsb = torch.empty(max(elsaa.elsaa_backward_workspace_size(p), 256),
+                          dtype=torch.uint8, device=dev)
+        grads = [torch.empty(x["q"].shape, dtype=torch.float32, device=dev)
+                 for _ in range(3)]
+
+        def step():
+            elsaa.elsaa_backward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                                 x["w_race"], x["do"], perm_q, perm_k,
+                                 dq=grads[0], dk=grads[1], dv=grads[2],
+                                 workspace=wsb, stream=stream)
 
     def barrier():
         if world > 1:
@@ -277,7 +300,7 @@ def run_ours(args, wl):
     barrier()
     prof = elsaa.elsaa_profile_stop()
     ms = ev0.elapsed_time(ev1)
-    elsaa.elsaa_check_status(ws)
+    elsaa.elsaa_check_status(wsb if args.backward else ws)
     sampler.stop()
     clocks = sampler.summary(t_pre, t_end)
     if world > 1:
@@ -311,7 +334,44 @@ def run_ours(args, wl):
     # end to end through the public API: pinned host inputs -> device ->
     # forward -> host output, every step
     e2e = None
-    if not args.no_e2e:
+    if args.backward and not args.no_e2e:
+        names = ("q", "k", "v", "w_race", "do")
+        hx = {k: x[k].cpu().pin_memory() for k in names}
+        hp = [perm_q.cpu().pin_memory(), perm_k.cpu().pin_memory()]
+        dx = {k: torch.empty_like(x[k]) for k in hx}
+        dp = [torch.empty_like(perm_q), torch.empty_like(perm_k)]
+        hg = [torch.empty(g.shape, dtype=g.dtype).pin_memory() for g in grads]
+        h2d = sum(t.numel() * t.element_size() for t in hx.values()) + sum(
+            t.numel() * t.element_size() for t in hp)
+        d2h = sum(t.numel() * t.element_size() for t in hg)
+
+        def e2e_step():
+            for k in hx:
+                dx[k].copy_(hx[k], non_blocking=True)
+            for dd, hh in zip(dp, hp):
+                dd.copy_(hh, non_blocking=True)
+            elsaa.elsaa_backward(p, dx["q"], dx["k"], dx["v"], None,
+                                 dx["w_race"], dx["do"], dp[0], dp[1],
+                                 dq=grads[0], dk=grads[1], dv=grads[2],
+                                 workspace=wsb, stream=stream)
+            for hh, g in zip(hg, grads):
+                hh.copy_(g, non_blocking=True)
+
+        for _ in range(max(3, args.warmup)):
+            e2e_step()
+        torch.cuda.synchronize(dev)
+        a = torch.cuda.Event(enable_timing=True)
+        bq = torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(args.steps):
+            e2e_step()
+        bq.record(stream)
+        torch.cuda.synchronize(dev)
+        ms_e2e = a.elapsed_time(bq) / args.steps
+        e2e = {"value": world * wl.tokens / (ms_e2e / 1e3),
+               "unit": "tokens/s", "ms_per_step": ms_e2e,
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
+    if not args.no_e2e and not args.backward:
         hx = {k: x[k].cpu().pin_memory() for k in ("q", "k", "v", "w_sort",
                                                   "w_race")}
         dx = {k: torch.empty_like(x[k]) for k in hx}
@@ -352,7 +412,35 @@ def run_ours(args, wl):
     # fits in the sample budget, also used as a parity spot check
     cpu = None
     err = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if args.backward and rank == 0 and world == 1 and \
+            not args.no_cpu_baseline:
+        # the oracle's fp64 gradient of whole heads on one host core, also a
+        # parity spot check (relative to the largest reference gradient)
+        import numpy as np
+        from oracle import backward as obwd
+        from oracle import oracle as orc
+        po = orc.params_from_workload(wl)
+        heads = [(0, 0), (wl.B - 1, wl.H - 1)]
+        t0 = time.perf_counter()
+        err = 0.0
+        for (b, h) in heads:
+            f32 = lambda t: t[b, h].float().cpu().numpy()
+            r = obwd.backward_head(
+                f32(x["q"]), f32(x["k"]), f32(x["v"]),
+                x["w_sort"][h].float().cpu().numpy(),
+                x["w_race"][h].double().cpu().numpy(), f32(x["do"]), po,
+                lam=np.full(wl.N, wl.lam))
+            for name, g in zip(("dQ", "dK", "dV"), grads):
+                ref = r[name]
+                err = max(err, float(np.abs(g[b, h].cpu().numpy() - ref).max()
+                                     / np.abs(ref).max()))
+        t_cpu = time.perf_counter() - t0
+        cpu = {"value": wl.N * len(heads) / t_cpu, "unit": "tokens/s",
+               "cores": 1, "kind": "oracle",
+               "sample": "%d of %d heads (fp64 numpy gradient, one thread), "
+                         "%.1f s wall" % (len(heads), wl.heads, t_cpu)}
+    if rank == 0 and world == 1 and not args.no_cpu_baseline and \
+            not args.backward:
         cores = os.cpu_count() or 1
         n_heads = min(wl.heads, 2 * cores)
         heads = [(i // wl.H, i % wl.H) for i in range(n_heads)]
@@ -375,7 +463,8 @@ def run_ours(args, wl):
     if rank != 0:
         return 0
     line = {
-        "metric": METRIC, "value": value, "unit": "tokens/s",
+        "metric": METRIC_BWD if args.backward else METRIC, "value": value,
+        "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
@@ -387,7 +476,8 @@ def run_ours(args, wl):
         "clocks": clocks,
         "e2e": e2e,
         "cpu_baseline": cpu,
-        "max_abs_err_vs_oracle": err,
+        ("max_rel_grad_err_vs_oracle" if args.backward else
+         "max_abs_err_vs_oracle"): err,
     }
     print(json.dumps(line))
     if world > 1:
@@ -408,6 +498,9 @@ def main():
                     help="override B (smaller cases for profiler captures)")
     ap.add_argument("--no-preroll", action="store_true",
                     help="skip the 1 s loaded pre-roll (profiler captures)")
+    ap.add_argument("--backward", action="store_true",
+                    help="time elsaa_backward (dQ, dK, dV) instead of the "
+                         "forward; use with --workload c5")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3

@@ -369,9 +369,10 @@ namespace {
 // Backward workspace: status | RACE chunk partials (A, B, then gA, gB) |
 // A | B | gA | gB | gNum / L [B*H][N][d_h] | gDen / L [B*H][N].
 struct BwdPlan {
-    Plan P;  // forward geometry with CUDA-core RACE chunking
+    Plan P;    // forward geometry with CUDA-core RACE chunking
+    Plan Pf;   // the forward's own plan (tensor-core key summaries if bf16)
     size_t off_status, off_part, off_A, off_B, off_gA, off_gB, off_gnum,
-        off_gden, total;
+        off_gden, off_W, total;
 };
 
 int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
@@ -379,7 +380,10 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     q.impl = ELSAA_IMPL_SIMT;  // the backward runs on CUDA cores
     int rc = make_plan(&q, &Bp->P, msg);
     if (rc != ELSAA_OK) return rc;
+    rc = make_plan(p, &Bp->Pf, msg);  // A, B as the forward makes them
+    if (rc != ELSAA_OK) return rc;
     const Plan &P = Bp->P;
+    const int S = P.S > Bp->Pf.S ? P.S : Bp->Pf.S;
     if (!bwd_supported(P)) {
         *msg = "backward: this block size, d_h and r need more shared "
                "memory than an SM has";
@@ -391,7 +395,7 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     Bp->off_status = off;
     off = align_up(off + sizeof(DeviceStatus), 256);
     Bp->off_part = off;
-    off = align_up(off + (size_t)P.BH * P.S * per * sizeof(float), 256);
+    off = align_up(off + (size_t)P.BH * S * per * sizeof(float), 256);
     Bp->off_A = off;
     off = align_up(off + (size_t)P.BH * P.r * sizeof(float), 256);
     Bp->off_B = off;
@@ -404,6 +408,8 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     off = align_up(off + BHN * P.d * sizeof(float), 256);
     Bp->off_gden = off;
     off = align_up(off + BHN * sizeof(float), 256);
+    Bp->off_W = off;
+    off = align_up(off + (size_t)P.H * P.Lg_pad * P.d * sizeof(uint16_t), 256);
     Bp->total = off;
     return ELSAA_OK;
 }
@@ -472,13 +478,29 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
 
     ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
                        "status reset");
-    ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
-                           return launch_race_partial_simt(P, k, v, w_race,
-                                                           part, st);
-                       }),
-                       "race_partial_simt");
+    // A, B exactly as the forward made them
+    const Plan &Pf = Bp.Pf;
+    if (Pf.impl == 2) {
+        uint16_t *Wbf = (uint16_t *)(ws + Bp.off_W);
+        ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
+                               return launch_prep_planes(Pf, w_race, Wbf, st);
+                           }),
+                           "prep_planes");
+        ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
+                               return launch_race_keys_ws(Pf, k, v, Wbf, part,
+                                                          status, st);
+                           }),
+                           "race_keys_ws");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
+                               return launch_race_partial_simt(Pf, k, v,
+                                                               w_race, part,
+                                                               st);
+                           }),
+                           "race_partial_simt");
+    }
     ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
-                           return launch_race_reduce(P, part, A, Bm, nullptr,
+                           return launch_race_reduce(Pf, part, A, Bm, nullptr,
                                                      st);
                        }),
                        "race_reduce");

@@ -29,6 +29,7 @@ namespace elsaa {
 namespace {
 
 constexpr int kBwdThreads = 256;
+constexpr int kKeyThreads = 256;
 constexpr int kBwdMaxB = 1024;
 constexpr int kKeyTile = 32;
 
@@ -37,6 +38,44 @@ __device__ __forceinline__ float lse2(float a, float b) {
     const float mx = fmaxf(a, b);
     if (mx == -INFINITY) return -INFINITY;
     return mx + logf(expf(a - mx) + expf(b - mx));
+}
+
+// C = A B on 4 x 4 register tiles spread over the CTA's threads. Element
+// (m, k) of A is A[m * am + k * ak] and (k, n) of B is B[k * bk + n * bn]
+// (shared or global memory: transposes are stride swaps); epi(m, n, value)
+// receives every element of C with m < M, n < N.
+template <int TM = 4, typename Epi>
+__device__ __forceinline__ void tile_gemm(int M, int N, int K,
+                                          const float *A, int am, int ak,
+                                          const float *B, int bk, int bn,
+                                          Epi epi) {
+    const int tn = (N + 3) >> 2, tm = (M + TM - 1) / TM;
+    for (int t = threadIdx.x; t < tm * tn; t += blockDim.x) {
+        const int m0 = (t / tn) * TM, n0 = (t % tn) * 4;
+        float c[TM][4];
+#pragma unroll
+        for (int u = 0; u < TM; ++u)
+#pragma unroll
+            for (int w = 0; w < 4; ++w) c[u][w] = 0.f;
+        for (int k = 0; k < K; ++k) {
+            float a[TM], bb[4];
+#pragma unroll
+            for (int u = 0; u < TM; ++u)
+                a[u] = (m0 + u < M) ? A[(m0 + u) * am + k * ak] : 0.f;
+#pragma unroll
+            for (int w = 0; w < 4; ++w)
+                bb[w] = (n0 + w < N) ? B[k * bk + (n0 + w) * bn] : 0.f;
+#pragma unroll
+            for (int u = 0; u < TM; ++u)
+#pragma unroll
+                for (int w = 0; w < 4; ++w) c[u][w] = fmaf(a[u], bb[w], c[u][w]);
+        }
+#pragma unroll
+        for (int u = 0; u < TM; ++u)
+#pragma unroll
+            for (int w = 0; w < 4; ++w)
+                if (m0 + u < M && n0 + w < N) epi(m0 + u, n0 + w, c[u][w]);
+    }
 }
 
 // u_b = tanh(<w_b, x>) for the G planes of table l, and phi_r of that table
@@ -128,12 +167,8 @@ __global__ void __launch_bounds__(kBwdThreads)
     }
     __syncthreads();
     // z_ij = scale <Q_i, K_j>
-    for (int x = tid; x < b * b; x += kBwdThreads) {
-        const int i = x / b, j = x - i * b;
-        float a = 0.f;
-        for (int e = 0; e < d; ++e) a = fmaf(Qs[i * dp + e], Ks[j * dp + e], a);
-        Es[i * bp + j] = scale * a;
-    }
+    tile_gemm(b, b, d, Qs, dp, 1, Ks, 1, dp,
+              [&](int i, int j, float v) { Es[i * bp + j] = scale * v; });
     __syncthreads();
     for (int i = tid; i < b; i += kBwdThreads) {
         float mx = -INFINITY;
@@ -146,15 +181,13 @@ __global__ void __launch_bounds__(kBwdThreads)
         }
         sM[i] = mx;
         sl[i] = l;
+        sfN[i] = 1.f / (l + eps * expf(-mx));  // (d_s + eps)^-1 e^M
     }
     __syncthreads();
     // O_s = sum_j e^(z - M) V_j / (l + eps e^-M)
-    for (int x = tid; x < b * d; x += kBwdThreads) {
-        const int i = x / d, e = x - i * d;
-        float a = 0.f;
-        for (int j = 0; j < b; ++j) a = fmaf(Es[i * bp + j], Vs[j * dp + e], a);
-        Xs[i * dp + e] = a / (sl[i] + eps * expf(-sM[i]));
-    }
+    tile_gemm(b, d, b, Es, bp, 1, Vs, dp, 1, [&](int i, int e, float v) {
+        Xs[i * dp + e] = v * sfN[i];
+    });
     // RACE features of the queries
     for (int x = tid; x < b * L; x += kBwdThreads) {
         const int i = x / L, l = x - i * L;
@@ -165,13 +198,9 @@ __global__ void __launch_bounds__(kBwdThreads)
     const float *Bh_ = Bg + (size_t)bh * r * d;
     const float *Ah = Ag + (size_t)bh * r;
     // Num = (1/L) sum phi B, Den = (1/L) sum phi . A
-    for (int x = tid; x < b * d; x += kBwdThreads) {
-        const int i = x / d, e = x - i * d;
-        float a = 0.f;
-        for (int rr = 0; rr < r; ++rr)
-            a = fmaf(Ph[i * r + rr], Bh_[(size_t)rr * d + e], a);
-        Ys[i * dp + e] = a / (float)L;
-    }
+    tile_gemm(b, d, r, Ph, r, 1, Bh_, d, 1, [&](int i, int e, float v) {
+        Ys[i * dp + e] = v / (float)L;
+    });
     for (int i = tid; i < b; i += kBwdThreads) {
         float a = 0.f;
         for (int rr = 0; rr < r; ++rr) a = fmaf(Ph[i * r + rr], Ah[rr], a);
@@ -220,28 +249,18 @@ __global__ void __launch_bounds__(kBwdThreads)
     }
     __syncthreads();
     // dV_j (sparse) = sum_i e^(z_ij - M_i) gN_s,i e^(M_i)
-    for (int x = tid; x < b * d; x += kBwdThreads) {
-        const int j = x / d, e = x - j * d;
-        float a = 0.f;
-        for (int i = 0; i < b; ++i) a = fmaf(Es[i * bp + j], Xs[i * dp + e], a);
-        dv[(base + ki[j]) * d + e] = a;
-    }
+    tile_gemm(b, d, b, Es, 1, bp, Xs, dp, 1, [&](int j, int e, float v) {
+        dv[(base + ki[j]) * d + e] = v;
+    });
     __syncthreads();
     // dZ_ij = e^(z - M) (gN_s e^M . V_j + e^M dL/dd_s)
-    for (int x = tid; x < b * b; x += kBwdThreads) {
-        const int i = x / b, j = x - i * b;
-        float a = 0.f;
-        for (int e = 0; e < d; ++e) a = fmaf(Xs[i * dp + e], Vs[j * dp + e], a);
-        Es[i * bp + j] *= (a + sgdsE[i]);
-    }
+    tile_gemm(b, b, d, Xs, dp, 1, Vs, 1, dp, [&](int i, int j, float v) {
+        Es[i * bp + j] *= (v + sgdsE[i]);
+    });
     // dL/dphi(Q_i) = (B gNum_i + A dL/dDen_i) / L
-    for (int x = tid; x < b * r; x += kBwdThreads) {
-        const int i = x / r, rr = x - i * r;
-        float a = 0.f;
-        for (int e = 0; e < d; ++e)
-            a = fmaf(Bh_[(size_t)rr * d + e], Ys[i * dp + e], a);
-        Gp[i * r + rr] = (a + Ah[rr] * sgDen[i]) / (float)L;
-    }
+    tile_gemm(b, r, d, Ys, dp, 1, Bh_, 1, d, [&](int i, int rr, float v) {
+        Gp[i * r + rr] = (v + Ah[rr] * sgDen[i]) / (float)L;
+    });
     __syncthreads();
     for (int x = tid; x < b * L; x += kBwdThreads) {
         const int i = x / L, l = x - i * L;
@@ -249,26 +268,21 @@ __global__ void __launch_bounds__(kBwdThreads)
                        Us + i * LG + l * G);
     }
     // dK_j (sparse) = scale sum_i dZ_ij Q_i
-    for (int x = tid; x < b * d; x += kBwdThreads) {
-        const int j = x / d, e = x - j * d;
-        float a = 0.f;
-        for (int i = 0; i < b; ++i) a = fmaf(Es[i * bp + j], Qs[i * dp + e], a);
-        dk[(base + ki[j]) * d + e] = scale * a;
-    }
+    tile_gemm(b, d, b, Es, 1, bp, Qs, dp, 1, [&](int j, int e, float v) {
+        dk[(base + ki[j]) * d + e] = scale * v;
+    });
+    // dQ_i = scale sum_j dZ_ij K_j (into Xs, free after dZ)
+    tile_gemm(b, d, b, Es, bp, 1, Ks, dp, 1, [&](int i, int e, float v) {
+        Xs[i * dp + e] = scale * v;
+    });
     __syncthreads();
-    // dQ_i = scale sum_j dZ_ij K_j + sum_(l,b) W_lb dL/d(W q)_lb
+    // ... + sum_(l,b) W_lb dL/d(W q)_lb
     const float *wh = w_race + (size_t)h * LG * d;
-    for (int x = tid; x < b * d; x += kBwdThreads) {
-        const int i = x / d, e = x - i * d;
-        float a = 0.f;
-        for (int j = 0; j < b; ++j) a = fmaf(Es[i * bp + j], Ks[j * dp + e], a);
-        float c = 0.f;
-        for (int lb = 0; lb < LG; ++lb)
-            c = fmaf(wh[(size_t)lb * d + e], Us[i * LG + lb], c);
+    tile_gemm(b, d, LG, Us, LG, 1, wh, d, 1, [&](int i, int e, float v) {
         const size_t row = base + qi[i];
-        dq[row * d + e] = scale * a + c;
+        dq[row * d + e] = Xs[i * dp + e] + v;
         gnum[row * d + e] = Ys[i * dp + e] / (float)L;
-    }
+    });
     for (int i = tid; i < b; i += kBwdThreads)
         gden[base + qi[i]] = sgDen[i] / (float)L;
 }
@@ -276,7 +290,7 @@ __global__ void __launch_bounds__(kBwdThreads)
 // Key side of RACE: dV_j += phi(K_j)^T gB, dL/dphi(K_j) = gB V_j + gA, then
 // back through the features into dK_j. Grid (ceil(N / 32), B*H).
 template <typename T>
-__global__ void __launch_bounds__(kBwdThreads)
+__global__ void __launch_bounds__(kKeyThreads)
     k_bwd_keys(const T *__restrict__ kx, const T *__restrict__ vx,
                const float *__restrict__ w_race, const float *__restrict__ gA,
                const float *__restrict__ gB, int N, int d, int H, int L,
@@ -293,13 +307,13 @@ __global__ void __launch_bounds__(kBwdThreads)
     float *Gp = Ph + kKeyTile * r;   // [32][r]
     float *Us = Gp + kKeyTile * r;   // [32][L*G]
     const size_t base = (size_t)bh * N + j0;
-    for (int x = tid; x < nk * d; x += kBwdThreads) {
+    for (int x = tid; x < nk * d; x += kKeyThreads) {
         const int j = x / d, e = x - j * d;
         Ks[j * dp + e] = to_f32<T>(kx[(base + j) * d + e]);
         Vs[j * dp + e] = to_f32<T>(vx[(base + j) * d + e]);
     }
     __syncthreads();
-    for (int x = tid; x < nk * L; x += kBwdThreads) {
+    for (int x = tid; x < nk * L; x += kKeyThreads) {
         const int j = x / L, l = x - j * L;
         table_features<6>(w_race + ((size_t)h * L + l) * G * d, Ks + j * dp, d,
                           G, beta, Us + j * LG + l * G, Ph + j * r + l * R);
@@ -307,35 +321,23 @@ __global__ void __launch_bounds__(kBwdThreads)
     __syncthreads();
     const float *gBh = gB + (size_t)bh * r * d;
     const float *gAh = gA + (size_t)bh * r;
-    for (int x = tid; x < nk * d; x += kBwdThreads) {
-        const int j = x / d, e = x - j * d;
-        float a = 0.f;
-        for (int rr = 0; rr < r; ++rr)
-            a = fmaf(Ph[j * r + rr], gBh[(size_t)rr * d + e], a);
-        dv[(base + j) * d + e] += a;
-    }
-    for (int x = tid; x < nk * r; x += kBwdThreads) {
-        const int j = x / r, rr = x - j * r;
-        float a = 0.f;
-        for (int e = 0; e < d; ++e)
-            a = fmaf(gBh[(size_t)rr * d + e], Vs[j * dp + e], a);
-        Gp[j * r + rr] = a + gAh[rr];
-    }
+    tile_gemm(nk, d, r, Ph, r, 1, gBh, d, 1, [&](int j, int e, float v) {
+        dv[(base + j) * d + e] += v;
+    });
+    tile_gemm(nk, r, d, Vs, dp, 1, gBh, 1, d, [&](int j, int rr, float v) {
+        Gp[j * r + rr] = v + gAh[rr];
+    });
     __syncthreads();
-    for (int x = tid; x < nk * L; x += kBwdThreads) {
+    for (int x = tid; x < nk * L; x += kKeyThreads) {
         const int j = x / L, l = x - j * L;
         table_backward(Ph + j * r + l * R, Gp + j * r + l * R, G, beta,
                        Us + j * LG + l * G);
     }
     __syncthreads();
     const float *wh = w_race + (size_t)h * LG * d;
-    for (int x = tid; x < nk * d; x += kBwdThreads) {
-        const int j = x / d, e = x - j * d;
-        float c = 0.f;
-        for (int lb = 0; lb < LG; ++lb)
-            c = fmaf(wh[(size_t)lb * d + e], Us[j * LG + lb], c);
-        dk[(base + j) * d + e] += c;
-    }
+    tile_gemm(nk, d, LG, Us, LG, 1, wh, d, 1, [&](int j, int e, float v) {
+        dk[(base + j) * d + e] += v;
+    });
 }
 
 }  // namespace
@@ -397,14 +399,14 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
         auto kern = k_bwd_keys<float>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-        kern<<<grid, kBwdThreads, smem, st>>>(
+        kern<<<grid, kKeyThreads, smem, st>>>(
             (const float *)k, (const float *)v, w_race, gA, gB, P.N, P.d, P.H,
             P.L, P.gamma, P.beta, dk, dv);
     } else {
         auto kern = k_bwd_keys<__nv_bfloat16>;
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-        kern<<<grid, kBwdThreads, smem, st>>>(
+        kern<<<grid, kKeyThreads, smem, st>>>(
             (const __nv_bfloat16 *)k, (const __nv_bfloat16 *)v, w_race, gA, gB,
             P.N, P.d, P.H, P.L, P.gamma, P.beta, dk, dv);
     }

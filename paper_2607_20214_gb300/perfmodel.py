@@ -64,6 +64,21 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
     elif kernel.startswith(("race_partial", "race_keys")):
         by = H * 2 * N * d * e
         fl = H * (2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
+    elif kernel.startswith("bwd_block"):
+        # recompute scores and O_s, dZ, dV, dK, dQ (12 N b d) and the query
+        # side of RACE (4 N r d + 4 N d Lg); reads Q, K, V, dO, writes dQ,
+        # dK, dV and gNum in fp32
+        by = H * (4 * N * d * e + 4 * N * d * 4)
+        fl = H * (12 * N * b * d + 4 * N * r * d + 4 * N * d * Lg)
+        simt = True
+    elif kernel.startswith("bwd_keys"):
+        by = H * (2 * N * d * e + 4 * N * d * 4)
+        fl = H * (4 * N * r * d + 4 * N * d * Lg)
+        simt = True
+    elif kernel.startswith("bwd_race_sums"):
+        by = H * (N * d * e + N * d * 4)
+        fl = H * (2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
+        simt = True
     elif kernel.startswith("prep_planes"):
         lg = wl.race_tables * wl.race_bits
         by = wl.H * lg * d * 4 + wl.H * ((lg + 15) // 16 * 16) * d * 2
