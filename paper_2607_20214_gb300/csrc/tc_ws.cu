@@ -54,12 +54,14 @@ __device__ __forceinline__ uint32_t quarter_col(int k, int col0) {
 struct WsBars {
     uint64_t qk_full, wb_full, head_done;
     uint64_t idx_full[2], idx_empty[2];
-    uint64_t v_full[2], v_empty[2];
+    uint64_t v_full[2], v_empty[2], pv0_done[2];
     uint64_t s_full[2], p_full[2], pv_done[2], p2_full[2], o_full[2];
     uint64_t tmem_empty[2];
 };
 
-template <int G>
+// NPASS = 2 for key blocks of 256 (two 128-key halves per query tile,
+// online softmax across them), 1 for b <= 128.
+template <int G, int NPASS>
 __global__ void __launch_bounds__(kWsThreads, 1)
     k_block_attn_ws(const uint16_t *__restrict__ qx,
                     const uint16_t *__restrict__ kx,
@@ -85,7 +87,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     __shared__ float xmax[2][2][128], xsum[2][2][128], xden[2][2][128];
     // global rows of a tile's queries / keys, per tile parity (written by
     // the index warp, read by the slot that issues the tile's Q, K copies)
-    __shared__ __align__(16) int qkrow[2][2][128];
+    __shared__ __align__(16) int qkrow[2][1 + NPASS][128];
     __shared__ __align__(16) int vrow[128];  // V loader: rows of its tile
     __shared__ int orow[2][128];          // per slot: output row or -1
     volatile int *abort = &abort_flag;
@@ -115,7 +117,8 @@ __global__ void __launch_bounds__(kWsThreads, 1)
         mbar_init(&bars.head_done, 1);
         for (int s = 0; s < 2; ++s) {
             mbar_init(&bars.idx_full[s], kWsLoaders);
-            mbar_init(&bars.idx_empty[s], 256);
+            mbar_init(&bars.idx_empty[s], 256 * NPASS);
+            mbar_init(&bars.pv0_done[s], 1);
             mbar_init(&bars.v_full[s], kWsLoaders);
             mbar_init(&bars.v_empty[s], 1);
             mbar_init(&bars.s_full[s], 1);
@@ -139,6 +142,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     auto tile_p0 = [=](int i) { return (tb + i) % tiles_per_head * 128; };
     auto new_head = [=](int i) {
         return i == 0 || (tb + i) % tiles_per_head == 0;
+    };
+    // sorted position of key column 0 of pass p of the tile starting at
+    // query position p0 (key blocks of 256: the block's two 128-key halves)
+    auto key_pos = [=](int p0, int p) {
+        return NPASS == 1 ? p0 : (p0 / (128 * NPASS)) * (128 * NPASS) + 128 * p;
     };
     // global row numbers of the 4 sorted positions pos.. pos + 3 (the
     // ragged end repeats the last row; those rows are never stored)
@@ -183,8 +191,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     break;
                 *reinterpret_cast<int4 *>(&qkrow[t][0][4 * lt]) =
                     rows4(perm_q + (size_t)bh * N, p0 + 4 * lt, bh * N);
-                *reinterpret_cast<int4 *>(&qkrow[t][1][4 * lt]) =
-                    rows4(perm_k + (size_t)bh * N, p0 + 4 * lt, bh * N);
+#pragma unroll
+                for (int ps = 0; ps < NPASS; ++ps)
+                    *reinterpret_cast<int4 *>(&qkrow[t][1 + ps][4 * lt]) =
+                        rows4(perm_k + (size_t)bh * N,
+                              key_pos(p0, ps) + 4 * lt, bh * N);
                 __syncwarp();
                 mbar_arrive(&bars.idx_full[t]);
             }
@@ -213,22 +224,31 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             const int cpr = d >> 3;    // 16-byte chunks per row
             const int rpi = 32 / cpr;  // rows per instruction
             const int lrow = lt / cpr, lc = lt - lrow * cpr;
-            for (int i = 0; i < ntiles; ++i) {
+            bool go = true;
+            for (int i = 0; i < ntiles && go; ++i) {
                 const int bh = tile_head(i), p0 = tile_p0(i);
-                __syncwarp();  // the previous tile's rows are all read
-                *reinterpret_cast<int4 *>(&vrow[4 * lt]) =
-                    rows4(perm_k + (size_t)bh * N, p0 + 4 * lt, bh * N);
-                __syncwarp();
-                // V of tile i goes to buffer i & 1 once the epilogue of
-                // tile i - 2 has copied its output out of there
-                if (i >= 2 &&
-                    !lwait(&bars.v_empty[i & 1], ((i >> 1) - 1) & 1, 33))
-                    break;
-                const uint32_t sV = sV0 + (i & 1) * tileB;
-                for (int row = lrow; row < nk; row += rpi)
-                    cp_async16(sV + panel_offset(row, lc, nk),
-                               vx + (size_t)vrow[row] * d + lc * 8);
-                cp_async_mbar_arrive(&bars.v_full[i & 1]);
+                for (int ps = 0; ps < NPASS; ++ps) {
+                    __syncwarp();  // the previous rows are all read
+                    *reinterpret_cast<int4 *>(&vrow[4 * lt]) =
+                        rows4(perm_k + (size_t)bh * N,
+                              key_pos(p0, ps) + 4 * lt, bh * N);
+                    __syncwarp();
+                    // buffer i & 1 serves the passes of tiles i, i + 2, ...
+                    // in turn; a pass's V goes in once the previous user is
+                    // done (its P V product, or the epilogue of the last
+                    // pass, which stages O there)
+                    const int ub = (i >> 1) * NPASS + ps;
+                    if (ub >= 1 &&
+                        !lwait(&bars.v_empty[i & 1], (ub - 1) & 1, 33)) {
+                        go = false;
+                        break;
+                    }
+                    const uint32_t sV = sV0 + (i & 1) * tileB;
+                    for (int row = lrow; row < nk; row += rpi)
+                        cp_async16(sV + panel_offset(row, lc, nk),
+                                   vx + (size_t)vrow[row] * d + lc * 8);
+                    cp_async_mbar_arrive(&bars.v_full[i & 1]);
+                }
             }
             cp_async_wait<0>();
         }
@@ -238,12 +258,20 @@ __global__ void __launch_bounds__(kWsThreads, 1)
         // oldest tile's first (second feature part, then P V with the first
         // part, then the next tile's projections and scores), so one slot's
         // epilogue never holds back the other slot's products.
+        // Units: (tile, pass); with NPASS = 2 the second score product of
+        // a tile waits until its first P V product is complete (it reuses
+        // the S columns), and the first P V product releases the V buffer
+        // for the second key half.
         if (lane_id == 0 && ntiles > 0) {
             const uint32_t id_sp = idesc_bf16(128, NR, false, false);
+            const uint32_t id_s = idesc_bf16(128, nk, false, false);
             const uint32_t id_o = idesc_bf16(128, d, false, true);
             const int r0 = min(r, nk);
             const bool two_parts = r > nk;
-            int is = 0, ip = 0, i2 = 0;  // next tile for S, P V, part 2
+            const int nunits = ntiles * NPASS;
+            int us = 0, up = 0, i2 = 0;  // next unit for S, unit for P V, tile
+                                         // for part 2
+            int tiles_pv = 0;            // tiles whose last P V is issued
             // position of each cursor's tile within its head (advanced
             // incrementally: no divisions in the issue loop)
             const int tph = tiles_per_head;
@@ -251,9 +279,9 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             auto adv = [tph](int q) { return q + 1 == tph ? 0 : q + 1; };
             int hc = 0;                  // heads whose planes were consumed
             unsigned long long t_last = global_ns();
-            while ((two_parts ? i2 : ip) < ntiles) {
+            while ((two_parts ? i2 : tiles_pv) < ntiles) {
                 bool did = false;
-                if (two_parts && i2 < ip) {
+                if (two_parts && i2 < tiles_pv) {
                     const int s = i2 & 1;
                     const uint32_t so = tm + 256u * s;
                     if (mbar_test(&bars.p2_full[s], (i2 >> 1) & 1)) {
@@ -271,48 +299,60 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                         did = true;
                     }
                 }
-                if (ip < is) {
-                    const int s = ip & 1;
+                if (up < us) {
+                    const int t = up / NPASS, pass = up - t * NPASS;
+                    const int s = t & 1;
+                    const int su = (t >> 1) * NPASS + pass;  // unit in slot
                     const uint32_t so = tm + 256u * s;
-                    if (mbar_test(&bars.p_full[s], (ip >> 1) & 1) &&
-                        mbar_test(&bars.v_full[s], (ip >> 1) & 1)) {
+                    if (mbar_test(&bars.p_full[s], su & 1) &&
+                        mbar_test(&bars.v_full[s], su & 1)) {
                         fence_proxy_async_smem();  // cp.async data -> MMA
                         tc_fence_after();
                         const uint32_t sV = sV0 + s * tileB;
-                        for (int kk = 0; kk < nk / 16; ++kk)  // O = P V
+                        for (int kk = 0; kk < nk / 16; ++kk)  // O (+)= P V
                             mma_ts(so + nk, so + quarter_col(kk, 0),
                                    smem_desc(sV + kk * 2048, (uint32_t)nk * 128,
                                              1024),
-                                   id_o, kk > 0);
-                        for (int kk = 0; kk < r0 / 16; ++kk)  // O += Phi' B
-                            mma_ts(so + nk, so + quarter_col(kk, 32),
-                                   smem_desc(sB + kk * 2048, (uint32_t)r * 128,
-                                             1024),
-                                   id_o, 1);
-                        if (two_parts) {
-                            mma_commit(&bars.pv_done[s]);
+                                   id_o, pass > 0 || kk > 0);
+                        if (pass < NPASS - 1) {
+                            mma_commit(&bars.pv0_done[s]);
+                            mma_commit(&bars.v_empty[s]);
                         } else {
-                            mma_commit(&bars.o_full[s]);
-                            if (ip == ntiles - 1 || pp == tph - 1)
-                                mma_commit(&bars.head_done);
+                            for (int kk = 0; kk < r0 / 16; ++kk)  // + Phi' B
+                                mma_ts(so + nk, so + quarter_col(kk, 32),
+                                       smem_desc(sB + kk * 2048,
+                                                 (uint32_t)r * 128, 1024),
+                                       id_o, 1);
+                            if (two_parts) {
+                                mma_commit(&bars.pv_done[s]);
+                            } else {
+                                mma_commit(&bars.o_full[s]);
+                                if (t == ntiles - 1 || pp == tph - 1)
+                                    mma_commit(&bars.head_done);
+                            }
+                            ++tiles_pv;
+                            pp = adv(pp);
                         }
-                        ++ip;
-                        pp = adv(pp);
+                        ++up;
                         did = true;
                     }
                 }
                 // a new head's planes and B summary replace the old ones
                 // only after head_done: its first S waits for every MMA of
                 // the previous head to be issued
-                const bool nh = is == 0 || ps == 0;  // tile is starts a head
-                if (is < ntiles && !(nh && is > 0 &&
-                                     (two_parts ? i2 : ip) < is)) {
-                    const int s = is & 1;
+                const int ts = us / NPASS, spass = us - ts * NPASS;
+                const bool nh = spass == 0 && (ts == 0 || ps == 0);
+                if (us < nunits &&
+                    !(nh && ts > 0 && (two_parts ? i2 : tiles_pv) < ts)) {
+                    const int s = ts & 1;
                     const uint32_t so = tm + 256u * s;
-                    bool ready = mbar_test(&bars.qk_full, is & 1) &&
-                                 (is < 2 || mbar_test(&bars.tmem_empty[s],
-                                                      ((is >> 1) - 1) & 1)) &&
-                                 (!nh || mbar_test(&bars.wb_full, hc & 1));
+                    bool ready = mbar_test(&bars.qk_full, us & 1);
+                    if (ready && spass == 0)
+                        ready = (ts < 2 || mbar_test(&bars.tmem_empty[s],
+                                                     ((ts >> 1) - 1) & 1)) &&
+                                (!nh || mbar_test(&bars.wb_full, hc & 1));
+                    if (ready && spass > 0)  // S columns hold P of pass 0
+                        ready = mbar_test(&bars.pv0_done[s], (ts >> 1) & 1);
                     if (ready) {
                         if (nh) ++hc;
                         fence_proxy_async_smem();  // cp.async data -> MMA
@@ -320,13 +360,15 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                         for (int kk = 0; kk < d / 16; ++kk) {
                             uint32_t oq = (kk >> 2) * 128 * 128 + (kk & 3) * 32;
                             uint32_t okw = (kk >> 2) * NR * 128 + (kk & 3) * 32;
+                            // pass 0: scores and projections (N = NR);
+                            // later passes: scores only
                             mma_ss(so, smem_desc(sQ + oq, 16, 1024),
-                                   smem_desc(sKW + okw, 16, 1024), id_sp,
-                                   kk > 0);
+                                   smem_desc(sKW + okw, 16, 1024),
+                                   spass == 0 ? id_sp : id_s, kk > 0);
                         }
                         mma_commit(&bars.s_full[s]);
-                        ++is;
-                        ps = adv(ps);
+                        ++us;
+                        if (spass == NPASS - 1) ps = adv(ps);
                         did = true;
                     }
                 }
@@ -388,6 +430,20 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             mbar_arrive(&bars.idx_empty[t & 1]);
             return true;
         };
+        // keys of pass ps >= 1 of tile t (the queries stay): issued by the
+        // tile's own slot once the previous pass's scores are done
+        auto issue_k = [&](int t, int ps) -> bool {
+            if (!wwait(&bars.idx_full[t & 1], (t >> 1) & 1, 57)) return false;
+            const int cpr = d >> 3, rpp = 256 / cpr;
+            const int crow = ct / cpr, cc = ct - crow * cpr;
+            const int *kr = qkrow[t & 1][1 + ps];
+            for (int rr = crow; rr < nk; rr += rpp)
+                cp_async16(sKW + panel_offset(rr, cc, NR),
+                           kx + (size_t)kr[rr] * d + cc * 8);
+            cp_async_mbar_arrive(&bars.qk_full);
+            mbar_arrive(&bars.idx_empty[t & 1]);
+            return true;
+        };
         bool started = true;
         if (g == 1 && ntiles > 0) started = issue_qk(0);
         for (int j = g; started && j < ntiles; j += 2) {
@@ -397,14 +453,18 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             const int qpos = p0 + row;
             const bool qvalid = qpos < N;
             int qi = perm_q[(size_t)bh * N + min(qpos, N - 1)];  // prefetch
-            if (!wwait(&bars.s_full[g], k & 1, 51)) break;
+            if (!wwait(&bars.s_full[g], (k * NPASS) & 1, 51)) break;
             tc_fence_after();
             // the A summary (read below) came by TMA: acquire its head's
             // stage (complete already, since S of this tile waited for it)
             if ((j < 2 || tile_head(j) != tile_head(j - 2)) &&
                 !wwait(&bars.wb_full, (tile_head(j) - tile_head(0)) & 1, 55))
                 break;
-            if (j + 1 < ntiles && !issue_qk(j + 1)) break;
+            if constexpr (NPASS > 1) {
+                if (!issue_k(j, 1)) break;
+            } else {
+                if (j + 1 < ntiles && !issue_qk(j + 1)) break;
+            }
             // per-bit factors of this half's tables (sp[0, 16): chunk half,
             // up to 32 when the chunk has more projection columns and no
             // second chunk exists; sp[16, 32): chunk half + 2) and partial
@@ -456,7 +516,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             mx = fmaxf(xmax[g][0][row], xmax[g][1][row]);
             const float denf =
                 (xden[g][0][row] + xden[g][1][row]) * (1.0f / (float)L);
-            const float M2 = mx * sl2e;
+            float M2 = mx * sl2e;
             float ls[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
             for (int c = 0; c < nk / 2; c += 32) {
@@ -490,6 +550,81 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             named_sync(1 + g, 256);  // every S read of the slot is done
             tc_fence_after();
             lsum = xsum[g][0][row] + xsum[g][1][row];
+            if constexpr (NPASS > 1) {
+                // pass 0's P goes to its P V product; pass 1 scores the
+                // second key half into the same columns
+                tmem_wait_st();
+                tc_fence_before();
+                mbar_arrive(&bars.p_full[g]);
+                if (!wwait(&bars.s_full[g], (k * NPASS + 1) & 1, 56)) break;
+                tc_fence_after();
+                if (j + 1 < ntiles && !issue_qk(j + 1)) break;
+                float mxb[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+#pragma unroll
+                for (int c = 0; c < nk / 2; c += 16) {
+                    uint32_t v[16];
+                    tmem_ld16(so + kbeg + c, v);
+                    tmem_wait_ld();
+#pragma unroll
+                    for (int jj = 0; jj < 16; ++jj)
+                        mxb[jj & 3] = fmaxf(mxb[jj & 3], __uint_as_float(v[jj]));
+                }
+                xmax[g][half][row] =
+                    fmaxf(fmaxf(mxb[0], mxb[1]), fmaxf(mxb[2], mxb[3]));
+                named_sync(1 + g, 256);
+                const float M2b =
+                    fmaxf(xmax[g][0][row], xmax[g][1][row]) * sl2e;
+                // online softmax: keep pass 0's reference unless the row's
+                // max grew by more than 2^8; then rescale the accumulator
+                // (P V of pass 0 is complete: S of pass 1 waited for it)
+                // and the running sum
+                const bool need = M2b > M2 + 8.0f;
+                const float f = need ? ex2_approx(M2 - M2b) : 1.0f;
+                if (__any_sync(0xffffffffu, need)) {
+#pragma unroll
+                    for (int c = 0; c < 64; c += 16) {
+                        if (c < (d >> 1)) {
+                            uint32_t v[16];
+                            tmem_ld16(so + nk + half * (d >> 1) + c, v);
+                            tmem_wait_ld();
+#pragma unroll
+                            for (int q = 0; q < 16; ++q)
+                                v[q] = __float_as_uint(__uint_as_float(v[q]) * f);
+                            tmem_st16(so + nk + half * (d >> 1) + c, v);
+                        }
+                    }
+                }
+                if (need) {
+                    lsum *= f;
+                    M2 = M2b;
+                }
+                float lb[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+#pragma unroll
+                for (int c = 0; c < nk / 2; c += 32) {
+                    uint32_t pk16[16];
+#pragma unroll
+                    for (int hh = 0; hh < 2; ++hh) {
+                        uint32_t v[16];
+                        tmem_ld16(so + kbeg + c + 16 * hh, v);
+                        tmem_wait_ld();
+#pragma unroll
+                        for (int jj = 0; jj < 16; jj += 2) {
+                            const float a0 = ex2_approx(
+                                fmaf(__uint_as_float(v[jj]), sl2e, -M2));
+                            const float a1 = ex2_approx(
+                                fmaf(__uint_as_float(v[jj + 1]), sl2e, -M2));
+                            lb[(jj >> 1) & 3] += a0 + a1;
+                            pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
+                        }
+                    }
+                    tmem_st16(so + kbeg + (c >> 1), pk16);
+                }
+                xsum[g][half][row] = (lb[0] + lb[1]) + (lb[2] + lb[3]);
+                tc_fence_before();
+                named_sync(1 + g, 256);
+                tc_fence_after();
+                lsum += xsum[g][0][row] + xsum[g][1][row];
+            }
             // fusion scalars (Eq. (5) in log-sum-exp form, Eq. (6))
             qi = (qi < 0 || qi >= N) ? 0 : qi;
             const size_t tok = (size_t)bh * N + qi;
@@ -591,7 +726,7 @@ bool ws_supported(const Plan &P) {
     // second (buckets past 128) at most 16, i.e. gamma >= 4 when r > 128;
     // row numbers in int
     const long rows = (long)P.N * P.BH;  // row numbers are int
-    return tc_supported(P) && P.b <= 128 && (P.gamma >= 4 || P.r <= 128) &&
+    return tc_supported(P) && P.b <= 256 && (P.gamma >= 4 || P.r <= 128) &&
            rows < (1L << 31);
 }
 
@@ -633,12 +768,12 @@ cudaError_t launch_block_attn_ws(
         return cudaGetLastError();
     };
     switch (P.gamma) {
-        case 1: return launch(k_block_attn_ws<1>);
-        case 2: return launch(k_block_attn_ws<2>);
-        case 3: return launch(k_block_attn_ws<3>);
-        case 4: return launch(k_block_attn_ws<4>);
-        case 5: return launch(k_block_attn_ws<5>);
-        case 6: return launch(k_block_attn_ws<6>);
+        case 1: return P.b > 128 ? launch(k_block_attn_ws<1, 2>) : launch(k_block_attn_ws<1, 1>);
+        case 2: return P.b > 128 ? launch(k_block_attn_ws<2, 2>) : launch(k_block_attn_ws<2, 1>);
+        case 3: return P.b > 128 ? launch(k_block_attn_ws<3, 2>) : launch(k_block_attn_ws<3, 1>);
+        case 4: return P.b > 128 ? launch(k_block_attn_ws<4, 2>) : launch(k_block_attn_ws<4, 1>);
+        case 5: return P.b > 128 ? launch(k_block_attn_ws<5, 2>) : launch(k_block_attn_ws<5, 1>);
+        case 6: return P.b > 128 ? launch(k_block_attn_ws<6, 2>) : launch(k_block_attn_ws<6, 1>);
         default: return cudaErrorInvalidValue;
     }
 }

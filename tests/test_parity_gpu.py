@@ -108,7 +108,7 @@ def test_small_several_tiles_ragged_tail(dtype, impl):
                                            (64, 96, 3, 5), (128, 64, 2, 6),
                                            (64, 128, 8, 5), (64, 64, 16, 3),
                                            (128, 128, 32, 2), (64, 64, 5, 4),
-                                           (128, 128, 14, 4)])
+                                           (128, 128, 14, 4), (64, 64, 18, 3)])
 def test_shapes(d_h, b, L, gamma):
     wl = small("bf16", d_h=d_h, block=b, race_tables=L, race_bits=gamma,
                N=b * 7, H=2, B=2)
