@@ -227,6 +227,7 @@ def workload_config(wl):
 def run_ours(args, wl):
     from paper_2607_20214_gb300 import build as nvbuild
     from paper_2607_20214_gb300 import elsaa
+    from paper_2607_20214_gb300 import multirank
 
     world, rank, local = dist_setup(args.gpus)
     if world > 1:
@@ -239,7 +240,7 @@ def run_ours(args, wl):
     elsaa.load_library()
     peaks = load_peaks()
 
-    wl_rank = wl.with_(seed=wl.seed + 100 * rank)
+    wl_rank = multirank.rank_workload(wl, rank)
     if args.backward:
         wl_rank = wl_rank.with_(backward=True)
     x = make_inputs(wl_rank, device=dev)
@@ -272,9 +273,7 @@ def run_ours(args, wl):
                                  dq=grads[0], dk=grads[1], dv=grads[2],
                                  workspace=wsb, stream=stream)
 
-    def barrier():
-        if world > 1:
-            torch.distributed.barrier()
+    barrier = multirank.barrier
 
     sampler = ClockSampler(local)
     sampler.start()
@@ -303,12 +302,9 @@ def run_ours(args, wl):
     elsaa.elsaa_check_status(wsb if args.backward else ws)
     sampler.stop()
     clocks = sampler.summary(t_pre, t_end)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = multirank.max_over_ranks(ms, dev)
     ms_step = ms / args.steps
-    value = world * wl.tokens / (ms_step / 1e3)
+    value = multirank.job_throughput(world, wl.tokens, ms_step)
 
     # dominant kernel roofline (device time of each launch, CUDA events on
     # the launching stream over the timed region)
@@ -399,12 +395,9 @@ def run_ours(args, wl):
         bq.record(stream)
         torch.cuda.synchronize(dev)
         barrier()
-        ms_e2e = a.elapsed_time(bq) / args.steps
-        if world > 1:
-            t = torch.tensor([ms_e2e], device=dev)
-            torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-            ms_e2e = float(t.item())
-        e2e = {"value": world * wl.tokens / (ms_e2e / 1e3),
+        ms_e2e = multirank.max_over_ranks(a.elapsed_time(bq) / args.steps,
+                                          dev)
+        e2e = {"value": multirank.job_throughput(world, wl.tokens, ms_e2e),
                "unit": "tokens/s", "ms_per_step": ms_e2e,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
 
