@@ -187,9 +187,11 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     return ELSAA_OK;
 }
 
-cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
-                              uint64_t rows, uint64_t cols,
-                              uint32_t box_rows) {
+namespace {
+
+cudaError_t encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t rows,
+                           uint64_t cols, uint32_t box_cols,
+                           uint32_t box_rows, CUtensorMapSwizzle swizzle) {
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     static std::once_flag once;
     std::call_once(once, [] {
@@ -203,15 +205,36 @@ cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
     if (!encode) return cudaErrorNotSupported;
     cuuint64_t dims[2] = {cols, rows};
     cuuint64_t strides[1] = {cols * 2};
-    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t box[2] = {box_cols, box_rows};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
                         const_cast<void *>(base), dims, strides, box, estr,
-                        CU_TENSOR_MAP_INTERLEAVE_NONE,
-                        CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                         CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
+                              uint64_t rows, uint64_t cols,
+                              uint32_t box_rows) {
+    return encode_bf16_2d(map, base, rows, cols, 64, box_rows,
+                          CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+cudaError_t make_tma_map_bf16_narrow(CUtensorMap *map, const void *base,
+                                     uint64_t rows, uint64_t cols,
+                                     uint32_t box_cols, uint32_t box_rows) {
+    CUtensorMapSwizzle sw;
+    switch (box_cols) {
+        case 16: sw = CU_TENSOR_MAP_SWIZZLE_32B; break;
+        case 32: sw = CU_TENSOR_MAP_SWIZZLE_64B; break;
+        case 64: sw = CU_TENSOR_MAP_SWIZZLE_128B; break;
+        default: return cudaErrorInvalidValue;
+    }
+    return encode_bf16_2d(map, base, rows, cols, box_cols, box_rows, sw);
 }
 
 int set_last_error(int code, const char *fmt, ...) {
@@ -302,7 +325,7 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                        "status reset");
     ELSAA_CHECK_LAUNCH(timed("sort_hash", st, [&] {
                            return launch_sort_hash(P, q, k, w_sort, keyrank,
-                                                   hist, st);
+                                                   hist, status, st);
                        }),
                        "sort_hash");
     ELSAA_CHECK_LAUNCH(timed("sort_scan", st,

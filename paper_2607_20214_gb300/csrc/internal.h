@@ -60,7 +60,8 @@ int make_plan(const elsaa_params *p, Plan *plan, const char **msg);
 // Launchers (return cudaError_t of the launch). Pointers are device pointers.
 cudaError_t launch_sort_hash(const Plan &P, const void *q, const void *k,
                              const float *w_sort, uint32_t *keyrank,
-                             int *hist, cudaStream_t st);
+                             int *hist, DeviceStatus *status,
+                             cudaStream_t st);
 cudaError_t launch_sort_scan(const Plan &P, int *hist, cudaStream_t st);
 cudaError_t launch_sort_scatter(const Plan &P, const uint32_t *keyrank,
                                 const int *hist, int32_t *perm_q,
@@ -118,6 +119,13 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
 // the encoding is rejected.
 cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
                               uint64_t rows, uint64_t cols, uint32_t box_rows);
+// The same with boxes of box_cols = 16, 32 or 64 columns (32, 64 or 128
+// bytes per row) and the swizzle of that width (32, 64 or 128 bytes): the
+// 16-byte chunk c of box row r lands at chunk c ^ ((r / (8 / (box_cols / 8)))
+// mod (box_cols / 8)).
+cudaError_t make_tma_map_bf16_narrow(CUtensorMap *map, const void *base,
+                                     uint64_t rows, uint64_t cols,
+                                     uint32_t box_cols, uint32_t box_rows);
 
 // RACE planes as bf16 rows [H][Lg_pad][d] (rows >= L * gamma zero), the
 // operand image the tensor-core kernels load with TMA.

@@ -17,6 +17,7 @@
 //   sort_scatter one CTA per tile: pos = offset[tile][key] + local rank,
 //                perm[pos] = token.
 #include "device_common.cuh"
+#include "tc_common.cuh"
 
 namespace elsaa {
 
@@ -176,6 +177,212 @@ __global__ void __launch_bounds__(kHashTile)
     }
 }
 
+// k_sort_hash_tma: warps 0-3 hash, warp 4 streams the inputs with TMA.
+// A work item is four consecutive 128-token tiles (512 rows) of one
+// (head, Q|K); a job is one 32-column panel of an item (64 bytes per row,
+// 64-byte swizzle: 16-byte chunk c of row r sits at chunk c ^ ((r >> 1) & 3)),
+// loaded as two 256-row boxes into one stage of a three-stage ring. Two
+// CTAs share an SM.
+constexpr int kHashStages = 3;
+constexpr int kHashItemTiles = 4;
+constexpr int kHashRows = kHashItemTiles * kHashTile;
+constexpr int kHashBoxRows = 256;
+constexpr int kHashCols = 32;
+constexpr uint32_t kHashStageBytes = kHashRows * kHashCols * 2;
+constexpr int kHashThreads = kHashTile + 32;
+
+// bf16 inputs with d in {64, 128}: the same hash, ranks and histograms as
+// k_sort_hash, from persistent CTAs whose producer warp keeps the next
+// panels in flight while the hashing warps work. CTA c owns a contiguous
+// range of items (items of one head are adjacent, so the planes are
+// reloaded only when the head changes). Hashing thread t evaluates rows
+// t, 128 + t, 256 + t and 384 + t of the item as two packed chains
+// (fma.rn.f32x2 lanes: tiles 0|1 and tiles 2|3); the planes sit in shared
+// memory as duplicated pairs (w, w), so one 16-byte load feeds four packed
+// FMAs. Every chain keeps the canonical sequential order i = 0..d-1.
+template <int NS>
+__global__ void __launch_bounds__(kHashThreads, 2)
+    k_sort_hash_tma(const __grid_constant__ CUtensorMap tmQ,
+                    const __grid_constant__ CUtensorMap tmK,
+                    const float *__restrict__ w_sort, int N, int d, int H,
+                    int BH, int bins, int gray, int tiles, int quads,
+                    int items, int per_cta, uint32_t *__restrict__ keyrank,
+                    int *__restrict__ hist, DeviceStatus *status) {
+    using namespace tc;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t full[kHashStages], empty[kHashStages];
+    __shared__ int abort_flag;
+    // 512-byte aligned start, the period of the 64-byte swizzle (pointer
+    // arithmetic on the shared array keeps every access an ld.shared)
+    unsigned char *smem =
+        smem_raw + ((512u - (smem_u32(smem_raw) & 511u)) & 511u);
+    const uint32_t stage0 = smem_u32(smem);
+    float2 *ws2 = reinterpret_cast<float2 *>(smem + kHashStages *
+                                             kHashStageBytes);  // [NS][d]
+    int *cnt = reinterpret_cast<int *>(ws2 + NS * d);  // [4 tiles][4 w][bins]
+    const int tid = threadIdx.x, lane = tid & 31, wid = tid >> 5;
+    const int P = d / kHashCols;  // panels per row
+    const int i0 = blockIdx.x * per_cta;
+    const int i1 = min(items, i0 + per_cta);
+    if (i0 >= i1) return;
+    const int njobs = (i1 - i0) * P;
+
+    if (tid == 0) {
+        for (int s = 0; s < kHashStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], kHashTile / 32);
+        }
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    __syncthreads();
+
+    if (wid == kHashTile / 32) {
+        // ---- producer warp: job j = panel (j mod P) of item i0 + j / P
+        if (lane == 0) {
+            int it = i0, pnl = 0;
+            int issued = 0;
+            for (int j = 0; j < njobs; ++j) {
+                const int s = j % kHashStages;
+                if (j >= kHashStages &&
+                    !mbar_wait_or_abort(&empty[s],
+                                        ((j / kHashStages) - 1) & 1,
+                                        &abort_flag, status, 0x5002))
+                    break;
+                const int bw = it / quads, quad = it - bw * quads;
+                const int which = bw & 1, bh = bw >> 1;
+                const int row = bh * N + quad * kHashRows;
+                const uint32_t dst = stage0 + s * kHashStageBytes;
+                const CUtensorMap *map = which ? &tmK : &tmQ;
+                mbar_expect_tx(&full[s], kHashStageBytes);
+                tma_load_2d(dst, map, pnl * kHashCols, row, &full[s]);
+                tma_load_2d(dst + kHashStageBytes / 2, map, pnl * kHashCols,
+                            row + kHashBoxRows, &full[s]);
+                ++issued;
+                if (++pnl == P) {
+                    pnl = 0;
+                    ++it;
+                }
+            }
+            // never leave with copies in flight into this CTA's stages:
+            // wait (bounded) for the last job issued into every stage
+            for (int s = 0; s < kHashStages; ++s) {
+                int last = issued - 1 - ((issued - 1 - s) % kHashStages +
+                                         kHashStages) % kHashStages;
+                if (last >= 0 && last < issued)
+                    mbar_wait(&full[s], (last / kHashStages) & 1, nullptr, 0);
+            }
+        }
+        return;
+    }
+
+    // ---- hashing warps
+    int cur_h = -1;
+    int j = 0;
+    bool ok = true;
+    for (int it = i0; it < i1 && ok; ++it) {
+        const int bw = it / quads, quad = it - bw * quads;
+        const int which = bw & 1, bh = bw >> 1;
+        const int h = bh % H;
+        if (h != cur_h) {  // uniform: planes of the new head, as (w, w)
+            for (int i = tid; i < NS * d; i += kHashTile) {
+                const float w = w_sort[(size_t)h * NS * d + i];
+                ws2[i] = make_float2(w, w);
+            }
+            cur_h = h;
+        }
+        for (int i = tid; i < 4 * 4 * bins; i += kHashTile) cnt[i] = 0;
+        named_sync(1, kHashTile);
+
+        unsigned long long acc0[NS > 0 ? NS : 1], acc1[NS > 0 ? NS : 1];
+#pragma unroll
+        for (int p = 0; p < NS; ++p) acc0[p] = acc1[p] = 0ull;
+        const int sw = (tid >> 1) & 3;  // same for rows 128k + t
+        for (int pnl = 0; pnl < P; ++pnl, ++j) {
+            const int s = j % kHashStages;
+            ok = mbar_wait_or_abort(&full[s], (j / kHashStages) & 1,
+                                    &abort_flag, status, 0x5001);
+            if (!ok) break;
+            const unsigned char *st = smem + s * kHashStageBytes;
+            const uint4 *x0p = reinterpret_cast<const uint4 *>(
+                st + tid * (kHashCols * 2));
+            constexpr int kTileU4 = kHashTile * kHashCols * 2 / 16;
+            // (w_i, w_i) and (w_i+1, w_i+1) as two packed operands
+            const ulonglong2 *w4 = reinterpret_cast<const ulonglong2 *>(ws2);
+#pragma unroll
+            for (int c = 0; c < kHashCols / 8; ++c) {
+                float v0[8], v1[8], v2[8], v3[8];
+                unpack8<__nv_bfloat16>(x0p[(c ^ sw)], v0);
+                unpack8<__nv_bfloat16>(x0p[kTileU4 + (c ^ sw)], v1);
+                unpack8<__nv_bfloat16>(x0p[2 * kTileU4 + (c ^ sw)], v2);
+                unpack8<__nv_bfloat16>(x0p[3 * kTileU4 + (c ^ sw)], v3);
+                const int e0 = pnl * kHashCols + c * 8;
+#pragma unroll
+                for (int e2 = 0; e2 < 4; ++e2) {
+                    const unsigned long long xa0 =
+                        pair2(v0[2 * e2], v1[2 * e2]);
+                    const unsigned long long xa1 =
+                        pair2(v0[2 * e2 + 1], v1[2 * e2 + 1]);
+                    const unsigned long long xb0 =
+                        pair2(v2[2 * e2], v3[2 * e2]);
+                    const unsigned long long xb1 =
+                        pair2(v2[2 * e2 + 1], v3[2 * e2 + 1]);
+#pragma unroll
+                    for (int p = 0; p < NS; ++p) {
+                        // same address in every lane (broadcast)
+                        const ulonglong2 wq = w4[(p * d + e0) / 2 + e2];
+                        acc0[p] = fma2(wq.x, xa0, acc0[p]);
+                        acc1[p] = fma2(wq.x, xb0, acc1[p]);
+                        acc0[p] = fma2(wq.y, xa1, acc0[p]);
+                        acc1[p] = fma2(wq.y, xb1, acc1[p]);
+                    }
+                }
+            }
+            // this warp is done reading stage s
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[s]);
+        }
+        ok = named_sync_and(1, kHashTile, ok);
+        if (!ok) break;
+
+        int *hout = hist + ((size_t)which * BH + bh) * tiles * bins;
+#pragma unroll
+        for (int tt = 0; tt < kHashItemTiles; ++tt) {
+            const int tile = kHashItemTiles * quad + tt;
+            const int n = tile * kHashTile + tid;
+            const unsigned long long *acc = tt < 2 ? acc0 : acc1;
+            uint32_t code = 0;
+#pragma unroll
+            for (int p = 0; p < NS; ++p) {
+                const float pr = __uint_as_float((uint32_t)(
+                    (tt & 1) ? (acc[p] >> 32) : (acc[p] & 0xffffffffull)));
+                code |= (pr > 0.0f ? 1u : 0u) << p;
+            }
+            const int key = (int)(gray ? gray_rank(code) : code);
+            const bool in = n < N && tile < tiles;
+            const unsigned act = __ballot_sync(0xffffffffu, in);
+            unsigned peers =
+                __match_any_sync(0xffffffffu, in ? key : -1) & act;
+            const int rank_w = __popc(peers & ((1u << lane) - 1u));
+            int *cw = cnt + tt * 4 * bins;
+            if (in && rank_w == 0) cw[wid * bins + key] = __popc(peers);
+            named_sync(1, kHashTile);
+            if (in) {
+                int rank = rank_w;
+                for (int w = 0; w < wid; ++w) rank += cw[w * bins + key];
+                keyrank[((size_t)which * BH + bh) * N + n] =
+                    (uint32_t)key | ((uint32_t)rank << 16);
+            }
+            if (tile < tiles)
+                for (int i = tid; i < bins; i += kHashTile)
+                    hout[(size_t)i * tiles + tile] =
+                        cw[i] + cw[bins + i] + cw[2 * bins + i] +
+                        cw[3 * bins + i];
+        }
+        named_sync(1, kHashTile);  // counts and planes may be overwritten
+    }
+}
+
 constexpr int kScanThreads = 1024;
 
 // Exclusive scan of the [bins][tiles] histogram of one (head, Q|K) in place:
@@ -281,6 +488,39 @@ cudaError_t launch_hash_t(const Plan &P, const void *q, const void *k,
     return cudaGetLastError();
 }
 
+template <int NS>
+cudaError_t launch_hash_tma(const Plan &P, const void *q, const void *k,
+                            const float *w_sort, uint32_t *keyrank, int *hist,
+                            DeviceStatus *status, cudaStream_t st) {
+    const uint64_t rows = (uint64_t)P.BH * P.N;
+    CUtensorMap tmQ, tmK;
+    cudaError_t e =
+        make_tma_map_bf16_narrow(&tmQ, q, rows, P.d, kHashCols, kHashBoxRows);
+    if (e == cudaSuccess)
+        e = make_tma_map_bf16_narrow(&tmK, k, rows, P.d, kHashCols,
+                                     kHashBoxRows);
+    if (e != cudaSuccess) return e;
+    const int quads = (P.tiles + kHashItemTiles - 1) / kHashItemTiles;
+    const int items = 2 * P.BH * quads;
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess)
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int slots = 2 * sms;  // two CTAs per SM
+    const int per = (items + slots - 1) / slots;
+    const int grid = (items + per - 1) / per;
+    const size_t smem = 512 + (size_t)kHashStages * kHashStageBytes +
+                        sizeof(float2) * (size_t)NS * P.d +
+                        sizeof(int) * 16 * P.bins;
+    auto kern = k_sort_hash_tma<NS>;
+    cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                         (int)smem);
+    kern<<<grid, kHashThreads, smem, st>>>(tmQ, tmK, w_sort, P.N, P.d, P.H,
+                                           P.BH, P.bins, P.gray, P.tiles,
+                                           quads, items, per, keyrank, hist,
+                                           status);
+    return cudaGetLastError();
+}
+
 template <typename T>
 cudaError_t launch_hash_dtype(const Plan &P, const void *q, const void *k,
                               const float *w_sort, uint32_t *keyrank,
@@ -298,9 +538,28 @@ cudaError_t launch_hash_dtype(const Plan &P, const void *q, const void *k,
 
 }  // namespace
 
+bool hash_tma_supported(const Plan &P) {
+    return P.dtype == ELSAA_BF16 && (P.d == 64 || P.d == 128) &&
+           P.n_s >= 1 && P.n_s <= 8 && (long)P.BH * P.N >= kHashBoxRows &&
+           (long)P.BH * P.N < (1l << 31);
+}
+
 cudaError_t launch_sort_hash(const Plan &P, const void *q, const void *k,
                              const float *w_sort, uint32_t *keyrank,
-                             int *hist, cudaStream_t st) {
+                             int *hist, DeviceStatus *status,
+                             cudaStream_t st) {
+    if (hash_tma_supported(P)) {
+        switch (P.n_s) {
+#define ELSAA_NS_CASE(n)                                                   \
+    case n:                                                                \
+        return launch_hash_tma<n>(P, q, k, w_sort, keyrank, hist, status, st);
+            ELSAA_NS_CASE(1) ELSAA_NS_CASE(2) ELSAA_NS_CASE(3)
+            ELSAA_NS_CASE(4) ELSAA_NS_CASE(5) ELSAA_NS_CASE(6)
+            ELSAA_NS_CASE(7) ELSAA_NS_CASE(8)
+#undef ELSAA_NS_CASE
+            default: break;
+        }
+    }
     if (P.dtype == ELSAA_FP32)
         return launch_hash_dtype<float>(P, q, k, w_sort, keyrank, hist, st);
     return launch_hash_dtype<__nv_bfloat16>(P, q, k, w_sort, keyrank, hist,

@@ -135,6 +135,16 @@ def test_parameter_variants(over):
     compare(wl, run_gpu(wl, x), run_oracle(wl, x), label=str(over))
 
 
+@pytest.mark.parametrize("over", [dict(sort_bits=8), dict(sort_bits=1),
+                                  dict(sort_bits=3), dict(gray_order=0)])
+def test_bf16_hash_variants(over):
+    """bf16 inputs take the TMA-streamed hash kernel (four tiles per work
+    item; N = 1184 leaves a ragged item that reads into the next head)."""
+    wl = small("bf16", H=3).with_(**over)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label=str(over))
+
+
 def test_single_block_and_minimum_size():
     wl = small("fp32", N=32, block=32, B=3, H=1)
     x = make_inputs(wl)
