@@ -191,3 +191,33 @@ def make_gates_lambda(wl: Workload, seed: int, device="cpu"):
     lam = torch.rand((wl.B, wl.H, wl.N), generator=g, device=device,
                      dtype=torch.float32) * 1.5 + 0.3
     return gates.contiguous(), lam.contiguous()
+
+
+def make_gate_mlp(wl: Workload, hidden: int = 64, seed: int = 7,
+                  device="cpu", w_lambda_std: float = 0.05) -> dict:
+    """Parameters of the token-wise gate MLP and of the query-dependent
+    lambda, per head (Section 3.3; Appendix D "gate hidden dim" 64 or 128;
+    Appendix E for lambda).
+
+    w1 [H, g, d] and w_lambda [H, d] hold bf16-representable fp32 values
+    (like the RACE planes); w1 ~ N(0, 1/d), b1 ~ 0.1 N(0, 1),
+    w2 [H, 2, g] ~ N(0, 1/g), b2 [H, 2] ~ 0.5 N(0, 1). lambda: c = 0.3 and
+    b = 0 (so c + sigmoid(b) = 0.8, the paper's initial average target),
+    w_lambda ~ w_lambda_std N(0, 1) (the paper initialises it at std 1e-3;
+    tests use a larger spread so the lambda path varies), lambda_min = 1e-6.
+    """
+    g = _gen(seed, device)
+    d = wl.d_h
+    w1 = _randn((wl.H, hidden, d), g, device) / float(d) ** 0.5
+    w1 = w1.to(torch.bfloat16).to(torch.float32)
+    b1 = 0.1 * _randn((wl.H, hidden), g, device)
+    w2 = _randn((wl.H, 2, hidden), g, device) / float(hidden) ** 0.5
+    b2 = 0.5 * _randn((wl.H, 2), g, device)
+    w_lambda = w_lambda_std * _randn((wl.H, d), g, device)
+    w_lambda = w_lambda.to(torch.bfloat16).to(torch.float32)
+    b_lambda = torch.zeros(wl.H, device=device)
+    c_lambda = torch.full((wl.H,), 0.3, device=device)
+    return dict(hidden=hidden, w1=w1.contiguous(), b1=b1.contiguous(),
+                w2=w2.contiguous(), b2=b2.contiguous(),
+                w_lambda=w_lambda.contiguous(), b_lambda=b_lambda,
+                c_lambda=c_lambda, lambda_min=1e-6)
