@@ -32,7 +32,8 @@ if ROOT not in sys.path:
 import torch  # noqa: E402
 
 from paper_2607_20214_gb300 import perfmodel  # noqa: E402
-from paper_2607_20214_gb300.workloads import WORKLOADS, make_inputs  # noqa
+from paper_2607_20214_gb300.workloads import (WORKLOADS,  # noqa: E402
+                                              make_gate_mlp, make_inputs)
 
 METRIC = "ELSAA fwd tokens/s at N=16K bf16 on 1 GB300"
 METRIC_BWD = "ELSAA bwd tokens/s (dQ, dK, dV fp32) on 1 GB300"
@@ -253,6 +254,23 @@ def run_ours(args, wl):
         elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
                             x["w_race"], o=o, workspace=ws, stream=stream)
 
+    if args.gate_mlp:
+        # learned gates and query-dependent lambda (elsaa_gates) feeding the
+        # fusion: both calls run in every step
+        mlp = make_gate_mlp(wl_rank, hidden=args.gate_mlp, device=dev)
+        BHN = (wl.B, wl.H, wl.N)
+        gts = torch.empty(BHN + (2,), dtype=torch.float32, device=dev)
+        lam = torch.empty(BHN, dtype=torch.float32, device=dev)
+        wsg = torch.empty(max(elsaa.elsaa_gates_workspace_size(p, mlp), 256),
+                          dtype=torch.uint8, device=dev)
+
+        def step():
+            elsaa.elsaa_gates(p, mlp, x["q"], gates=gts, lambda_tok=lam,
+                              workspace=wsg, stream=stream)
+            elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                                x["w_race"], lambda_tok=lam, gates=gts, o=o,
+                                workspace=ws, stream=stream)
+
     if args.backward:
         # the backward pass of the same inputs: permutations from one
         # forward (outside the timed region), then elsaa_backward per step
@@ -367,7 +385,7 @@ def run_ours(args, wl):
         e2e = {"value": world * wl.tokens / (ms_e2e / 1e3),
                "unit": "tokens/s", "ms_per_step": ms_e2e,
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h}
-    if not args.no_e2e and not args.backward:
+    if not args.no_e2e and not args.backward and not args.gate_mlp:
         hx = {k: x[k].cpu().pin_memory() for k in ("q", "k", "v", "w_sort",
                                                   "w_race")}
         dx = {k: torch.empty_like(x[k]) for k in hx}
@@ -433,7 +451,7 @@ def run_ours(args, wl):
                "sample": "%d of %d heads (fp64 numpy gradient, one thread), "
                          "%.1f s wall" % (len(heads), wl.heads, t_cpu)}
     if rank == 0 and world == 1 and not args.no_cpu_baseline and \
-            not args.backward:
+            not args.backward and not args.gate_mlp:
         cores = os.cpu_count() or 1
         n_heads = min(wl.heads, 2 * cores)
         heads = [(i // wl.H, i % wl.H) for i in range(n_heads)]
@@ -461,7 +479,9 @@ def run_ours(args, wl):
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": ms_step, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": workload_config(wl),
+        "config": dict(workload_config(wl),
+                       **({"gate_mlp_hidden": args.gate_mlp}
+                          if args.gate_mlp else {})),
         "tflops": fm["tensor_flops"] / t_s / 1e12,
         "step_roofline_frac": step_roof,
         "roofline": roof, "kernels": kernels,
@@ -491,6 +511,10 @@ def main():
                     help="override B (smaller cases for profiler captures)")
     ap.add_argument("--no-preroll", action="store_true",
                     help="skip the 1 s loaded pre-roll (profiler captures)")
+    ap.add_argument("--gate-mlp", type=int, default=0, metavar="HIDDEN",
+                    help="also run the gate MLP / lambda kernel (hidden "
+                         "width HIDDEN, e.g. 64) in every step; its gates "
+                         "and lambda feed the fusion")
     ap.add_argument("--backward", action="store_true",
                     help="time elsaa_backward (dQ, dK, dV) instead of the "
                          "forward; use with --workload c5")

@@ -203,6 +203,58 @@ int elsaa_backward(const elsaa_params *params, const void *q, const void *k,
                    size_t workspace_bytes, void *stream);
 
 /*
+ * Token-wise gates and query-dependent lambda, the learned inputs of the
+ * fusion (Section 3.3: (g_sparse,i, g_lr,i) = sigma(G_theta(q_i)); the
+ * model-setup appendix: G_theta is a two-layer MLP with a SiLU hidden layer
+ * and two independent sigmoid outputs; the lambda appendix: the
+ * input-dependent coefficient lambda_i = c + sigma(w^T q_i + b), floored at
+ * lambda_min). For every query row q_i of head h:
+ *     a_i         = SiLU(W1[h] q_i + b1[h])            (width g)
+ *     gates[i]    = sigmoid(W2[h] a_i + b2[h])         (2 values)
+ *     lambda_tok[i] = max(c[h] + sigmoid(w_lambda[h] . q_i + b_lambda[h]),
+ *                         lambda_min)
+ * with SiLU(x) = x sigmoid(x). The outputs have exactly the layouts of
+ * elsaa_forward's `gates` and `lambda_tok` arguments: enqueue elsaa_gates
+ * and then elsaa_forward on one stream for the full fusion with learned
+ * gates. Parameter gradients of the MLP are not computed (elsaa_backward
+ * returns dL/dgates and dL/dlambda, from which they follow).
+ */
+typedef struct elsaa_gate_mlp {
+    int hidden;              /* g, a multiple of 16 in [16, 128]
+                                (the paper uses 64 or 128)                  */
+    const float *w1;         /* [H, g, d_h]; the tensor-core path rounds it
+                                to bf16: pass bf16-representable values     */
+    const float *b1;         /* [H, g]                                      */
+    const float *w2;         /* [H, 2, g]: rows for g_sparse, g_lr          */
+    const float *b2;         /* [H, 2]                                      */
+    const float *w_lambda;   /* [H, d_h] (bf16-representable), or NULL for
+                                no lambda output                            */
+    const float *b_lambda;   /* [H]; required with w_lambda                 */
+    const float *c_lambda;   /* [H], >= 0; required with w_lambda           */
+    float lambda_min;        /* > 0 (the paper: 1e-6)                       */
+} elsaa_gate_mlp;
+
+/*
+ * q           [B, H, N, d_h] of params->dtype (device, 16-byte aligned).
+ * gates       [B, H, N, 2] fp32 (device, written, 8-byte aligned).
+ * lambda_tok  [B, H, N] fp32 (device, written); required when
+ *             mlp->w_lambda != NULL, ignored otherwise.
+ * workspace   at least elsaa_gates_workspace_size() bytes, 256-byte
+ *             aligned (holds the bf16 image of W1 and w_lambda and the
+ *             status word that elsaa_check_status reads).
+ * All parameter arrays are device pointers. params is validated as for
+ * elsaa_forward. bf16 inputs with d_h in {64, 128} run on the tensor cores
+ * (tcgen05, fp32 accumulation); other shapes and fp32 inputs on CUDA cores
+ * in fp32. Errors: ELSAA_ERR_INVALID_ARG / _UNSUPPORTED / _WORKSPACE before
+ * any launch, ELSAA_ERR_CUDA if a launch fails.
+ */
+int elsaa_gates_workspace_size(const elsaa_params *params,
+                               const elsaa_gate_mlp *mlp, size_t *bytes);
+int elsaa_gates(const elsaa_params *params, const elsaa_gate_mlp *mlp,
+                const void *q, float *gates, float *lambda_tok,
+                void *workspace, size_t workspace_bytes, void *stream);
+
+/*
  * Synchronises `stream` and reads the in-band status word that the kernels
  * of the last elsaa_forward on this workspace wrote (bounded waits that ran
  * out, inconsistent sort counts). Returns ELSAA_OK, ELSAA_ERR_DEVICE (with

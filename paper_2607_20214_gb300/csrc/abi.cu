@@ -552,6 +552,91 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
     return ELSAA_OK;
 }
 
+namespace {
+
+// Validates the gate MLP description for the (already planned) shapes.
+int check_gate_mlp(const elsaa_gate_mlp *m, const char **msg) {
+    if (!m) {
+        *msg = "mlp is NULL";
+        return ELSAA_ERR_INVALID_ARG;
+    }
+    if (m->hidden < 16 || m->hidden > 128 || m->hidden % 16) {
+        *msg = "mlp->hidden must be a multiple of 16 in [16, 128]";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
+    if (!m->w1 || !m->b1 || !m->w2 || !m->b2) {
+        *msg = "mlp->w1, b1, w2 and b2 must be non-NULL";
+        return ELSAA_ERR_INVALID_ARG;
+    }
+    if (m->w_lambda && (!m->b_lambda || !m->c_lambda)) {
+        *msg = "mlp->b_lambda and c_lambda are required with w_lambda";
+        return ELSAA_ERR_INVALID_ARG;
+    }
+    if (m->w_lambda && !(m->lambda_min > 0.0f)) {
+        *msg = "mlp->lambda_min must be > 0";
+        return ELSAA_ERR_INVALID_ARG;
+    }
+    return ELSAA_OK;
+}
+
+}  // namespace
+
+extern "C" int elsaa_gates_workspace_size(const elsaa_params *params,
+                                          const elsaa_gate_mlp *mlp,
+                                          size_t *bytes) {
+    g_err[0] = 0;
+    if (!bytes) return fail(ELSAA_ERR_INVALID_ARG, "bytes is NULL");
+    Plan P;
+    const char *msg = "";
+    int rc = make_plan(params, &P, &msg);
+    if (rc == ELSAA_OK) rc = check_gate_mlp(mlp, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    *bytes = gate_workspace_bytes(P, mlp->hidden);
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_gates(const elsaa_params *params,
+                           const elsaa_gate_mlp *mlp, const void *q,
+                           float *gates, float *lambda_tok, void *workspace,
+                           size_t workspace_bytes, void *stream) {
+    g_err[0] = 0;
+    Plan P;
+    const char *msg = "";
+    int rc = make_plan(params, &P, &msg);
+    if (rc == ELSAA_OK) rc = check_gate_mlp(mlp, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    if (!q || !gates)
+        return fail(ELSAA_ERR_INVALID_ARG, "q and gates must be non-NULL");
+    if (mlp->w_lambda && !lambda_tok)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "lambda_tok must be non-NULL when mlp->w_lambda is given");
+    if ((uintptr_t)q % 16 || (uintptr_t)gates % 8)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "q must be 16-byte and gates 8-byte aligned");
+    const size_t need = gate_workspace_bytes(P, mlp->hidden);
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if ((uintptr_t)workspace % 256)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if (workspace_bytes < need)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, need);
+    cudaStream_t st = (cudaStream_t)stream;
+    char *ws = (char *)workspace;
+    DeviceStatus *status = (DeviceStatus *)ws;
+    uint16_t *wbf = (uint16_t *)(ws + 256);
+    ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
+                       "status reset");
+    ELSAA_CHECK_LAUNCH(timed("gate_mlp", st, [&] {
+                           return launch_gates(P, *mlp, q, gates,
+                                               mlp->w_lambda ? lambda_tok
+                                                             : nullptr,
+                                               wbf, status, st);
+                       }),
+                       "gate_mlp");
+    return ELSAA_OK;
+}
+
 extern "C" int elsaa_check_status(const void *workspace, void *stream) {
     g_err[0] = 0;
     if (!workspace) return fail(ELSAA_ERR_INVALID_ARG, "workspace is NULL");

@@ -113,6 +113,15 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
                             const float *gB, float *dk, float *dv,
                             cudaStream_t st);
 
+// Token-wise gate MLP and query-dependent lambda (gates.cu).
+int gate_ng(int hidden);
+bool gate_tc_supported(const Plan &P);
+size_t gate_workspace_bytes(const Plan &P, int hidden);
+cudaError_t launch_gates(const Plan &P, const elsaa_gate_mlp &m,
+                         const void *q, float *gates, float *lam_out,
+                         uint16_t *w_bf16, DeviceStatus *status,
+                         cudaStream_t st);
+
 // Row-major bf16 matrix [rows x cols] as a TMA tensor map with boxes of
 // 64 columns x box_rows rows and 128-byte swizzle (the panel layout).
 // Returns cudaSuccess or an error if the driver entry point is missing or

@@ -28,7 +28,8 @@ ELSAA_IMPL_SIMT = 1
 SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_last_error", "elsaa_abi_version", "elsaa_profile_start",
            "elsaa_profile_stop", "elsaa_forward_noalloc",
-           "elsaa_backward_workspace_size", "elsaa_backward")
+           "elsaa_backward_workspace_size", "elsaa_backward",
+           "elsaa_gates_workspace_size", "elsaa_gates")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -44,6 +45,17 @@ class elsaa_params(ctypes.Structure):
         ("beta", ctypes.c_float), ("eps", ctypes.c_float),
         ("scale", ctypes.c_float), ("lam", ctypes.c_float),
         ("fusion_mode", ctypes.c_int), ("impl", ctypes.c_int),
+    ]
+
+
+class elsaa_gate_mlp(ctypes.Structure):
+    """Mirror of struct elsaa_gate_mlp (device pointers as integers)."""
+    _fields_ = [
+        ("hidden", ctypes.c_int), ("w1", ctypes.c_void_p),
+        ("b1", ctypes.c_void_p), ("w2", ctypes.c_void_p),
+        ("b2", ctypes.c_void_p), ("w_lambda", ctypes.c_void_p),
+        ("b_lambda", ctypes.c_void_p), ("c_lambda", ctypes.c_void_p),
+        ("lambda_min", ctypes.c_float),
     ]
 
 
@@ -99,6 +111,14 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
     L.elsaa_backward.argtypes = [ctypes.POINTER(elsaa_params)] + [vp] * 16 + [
         ctypes.c_size_t, vp]
     L.elsaa_backward.restype = ctypes.c_int
+    L.elsaa_gates_workspace_size.argtypes = [
+        ctypes.POINTER(elsaa_params), ctypes.POINTER(elsaa_gate_mlp),
+        ctypes.POINTER(ctypes.c_size_t)]
+    L.elsaa_gates_workspace_size.restype = ctypes.c_int
+    L.elsaa_gates.argtypes = [ctypes.POINTER(elsaa_params),
+                              ctypes.POINTER(elsaa_gate_mlp)] + [vp] * 4 + [
+        ctypes.c_size_t, vp]
+    L.elsaa_gates.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -272,6 +292,67 @@ def elsaa_backward(params: elsaa_params, q, k, v, w_sort, w_race, d_o,
                             workspace.numel() * workspace.element_size(), sp)
     _check(rc)
     return dq, dk, dv
+
+
+def _gate_struct(params: elsaa_params, mlp: dict, dev) -> elsaa_gate_mlp:
+    H, d, g = params.H, params.d_h, int(mlp["hidden"])
+    has_l = mlp.get("w_lambda") is not None
+    f32 = torch.float32
+    return elsaa_gate_mlp(
+        g, _ptr(mlp["w1"], "w1", f32, H * g * d, dev),
+        _ptr(mlp["b1"], "b1", f32, H * g, dev),
+        _ptr(mlp["w2"], "w2", f32, H * 2 * g, dev),
+        _ptr(mlp["b2"], "b2", f32, H * 2, dev),
+        _ptr(mlp["w_lambda"], "w_lambda", f32, H * d, dev) if has_l else None,
+        _ptr(mlp["b_lambda"], "b_lambda", f32, H, dev) if has_l else None,
+        _ptr(mlp["c_lambda"], "c_lambda", f32, H, dev) if has_l else None,
+        float(mlp.get("lambda_min", 1e-6)))
+
+
+def elsaa_gates_workspace_size(params: elsaa_params, mlp: dict,
+                               device=None) -> int:
+    dev = mlp["w1"].device if device is None else device
+    m = _gate_struct(params, mlp, dev)
+    n = ctypes.c_size_t(0)
+    _check(load_library().elsaa_gates_workspace_size(
+        ctypes.byref(params), ctypes.byref(m), ctypes.byref(n)))
+    return n.value
+
+
+def elsaa_gates(params: elsaa_params, mlp: dict, q, gates=None,
+                lambda_tok=None, workspace=None, stream=None):
+    """Enqueue elsaa_gates on `stream`: per-token (g_sparse, g_lr) and,
+    when mlp["w_lambda"] is given, lambda_i. `mlp` holds device tensors
+    w1, b1, w2, b2 (and w_lambda, b_lambda, c_lambda, lambda_min) as in
+    include/elsaa.h. Returns (gates [B, H, N, 2], lambda_tok [B, H, N] or
+    None), allocated here when not given."""
+    lib = load_library()
+    dev = q.device
+    if dev.type != "cuda":
+        raise ValueError("q must be a CUDA tensor")
+    tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    BHN = params.B * params.H * params.N
+    shape = (params.B, params.H, params.N)
+    m = _gate_struct(params, mlp, dev)
+    if gates is None:
+        gates = torch.empty(shape + (2,), dtype=torch.float32, device=dev)
+    if lambda_tok is None and mlp.get("w_lambda") is not None:
+        lambda_tok = torch.empty(shape, dtype=torch.float32, device=dev)
+    if workspace is None:
+        n = elsaa_gates_workspace_size(params, mlp, dev)
+        workspace = torch.empty(max(n, 256), dtype=torch.uint8, device=dev)
+    if stream is None:
+        stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    rc = lib.elsaa_gates(
+        ctypes.byref(params), ctypes.byref(m),
+        _ptr(q, "q", tdt, BHN * params.d_h, dev),
+        _ptr(gates, "gates", torch.float32, 2 * BHN, dev),
+        _ptr(lambda_tok, "lambda_tok", torch.float32, BHN, dev),
+        _ptr(workspace, "workspace", None, None, dev),
+        workspace.numel() * workspace.element_size(), sp)
+    _check(rc)
+    return gates, lambda_tok
 
 
 def elsaa_check_status(workspace: torch.Tensor, stream=None):

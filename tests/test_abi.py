@@ -133,3 +133,58 @@ def test_missing_library_fails_loudly(tmp_path):
             elsaa.load_library(str(tmp_path / "absent.so"))
     finally:
         elsaa._lib = saved
+
+
+def test_gate_mlp_struct_matches_header():
+    src = open(os.path.join(ROOT, "include", "elsaa.h")).read()
+    body = src[src.index("typedef struct elsaa_gate_mlp"):]
+    body = body[body.index("{") + 1:body.index("} elsaa_gate_mlp;")]
+    body = re.sub(r"/\*.*?\*/", "", body, flags=re.S)
+    names = [re.findall(r"(\w+)\s*$", d.strip())[0]
+             for d in body.split(";") if d.strip()]
+    assert names == [f[0] for f in elsaa.elsaa_gate_mlp._fields_]
+
+
+def test_gates_validation_before_launch(lib):
+    p = elsaa.make_params(B=1, H=2, N=256, d_h=64, block_size=64,
+                          race_tables=4)
+    fake = 1 << 20  # never dereferenced: validation fails first
+    m = elsaa.elsaa_gate_mlp(64, fake, fake, fake, fake, None, None, None,
+                             1e-6)
+    n = ctypes.c_size_t(0)
+    assert lib.elsaa_gates_workspace_size(ctypes.byref(p), ctypes.byref(m),
+                                          ctypes.byref(n)) == elsaa.ELSAA_OK
+    # the bf16 image of [W1; w_lambda; 0] per head after the status word
+    assert n.value == 256 + 2 * (64 + 16) * 64 * 2
+    for hidden, code in ((24, elsaa.ELSAA_ERR_UNSUPPORTED),
+                         (256, elsaa.ELSAA_ERR_UNSUPPORTED),
+                         (0, elsaa.ELSAA_ERR_UNSUPPORTED)):
+        bad = elsaa.elsaa_gate_mlp(hidden, fake, fake, fake, fake, None,
+                                   None, None, 1e-6)
+        assert lib.elsaa_gates_workspace_size(
+            ctypes.byref(p), ctypes.byref(bad), ctypes.byref(n)) == code
+        assert "hidden" in elsaa.elsaa_last_error()
+    # lambda requested without its coefficient arrays / floor
+    bad = elsaa.elsaa_gate_mlp(64, fake, fake, fake, fake, fake, None, None,
+                               1e-6)
+    assert lib.elsaa_gates(ctypes.byref(p), ctypes.byref(bad), fake, fake,
+                           fake, fake, 1 << 30, None) == \
+        elsaa.ELSAA_ERR_INVALID_ARG
+    bad = elsaa.elsaa_gate_mlp(64, fake, fake, fake, fake, fake, fake, fake,
+                               0.0)
+    assert lib.elsaa_gates(ctypes.byref(p), ctypes.byref(bad), fake, fake,
+                           fake, fake, 1 << 30, None) == \
+        elsaa.ELSAA_ERR_INVALID_ARG
+    assert "lambda_min" in elsaa.elsaa_last_error()
+    # lambda output missing, workspace too small, misaligned q
+    lm = elsaa.elsaa_gate_mlp(64, fake, fake, fake, fake, fake, fake, fake,
+                              1e-6)
+    assert lib.elsaa_gates(ctypes.byref(p), ctypes.byref(lm), fake, fake,
+                           None, fake, 1 << 30, None) == \
+        elsaa.ELSAA_ERR_INVALID_ARG
+    assert lib.elsaa_gates(ctypes.byref(p), ctypes.byref(m), fake, fake,
+                           None, fake, 256, None) == elsaa.ELSAA_ERR_WORKSPACE
+    assert lib.elsaa_gates(ctypes.byref(p), ctypes.byref(m), fake + 8, fake,
+                           None, fake, 1 << 30, None) == \
+        elsaa.ELSAA_ERR_INVALID_ARG
+    assert "16-byte" in elsaa.elsaa_last_error()
