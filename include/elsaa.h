@@ -242,7 +242,8 @@ typedef struct elsaa_gate_mlp {
  * workspace   at least elsaa_gates_workspace_size() bytes, 256-byte
  *             aligned (holds the bf16 image of W1 and w_lambda and the
  *             status word that elsaa_check_status reads).
- * All parameter arrays are device pointers. params is validated as for
+ * All parameter arrays are device pointers; b1 and w2 must be 16-byte
+ * aligned (rows are read in 16-byte pieces). params is validated as for
  * elsaa_forward. bf16 inputs with d_h in {64, 128} run on the tensor cores
  * (tcgen05, fp32 accumulation); other shapes and fp32 inputs on CUDA cores
  * in fp32. Errors: ELSAA_ERR_INVALID_ARG / _UNSUPPORTED / _WORKSPACE before

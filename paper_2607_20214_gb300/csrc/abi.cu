@@ -610,9 +610,11 @@ extern "C" int elsaa_gates(const elsaa_params *params,
     if (mlp->w_lambda && !lambda_tok)
         return fail(ELSAA_ERR_INVALID_ARG,
                     "lambda_tok must be non-NULL when mlp->w_lambda is given");
-    if ((uintptr_t)q % 16 || (uintptr_t)gates % 8)
+    if ((uintptr_t)q % 16 || (uintptr_t)gates % 8 ||
+        (uintptr_t)mlp->b1 % 16 || (uintptr_t)mlp->w2 % 16)
         return fail(ELSAA_ERR_INVALID_ARG,
-                    "q must be 16-byte and gates 8-byte aligned");
+                    "q, mlp->b1 and mlp->w2 must be 16-byte and gates 8-byte "
+                    "aligned");
     const size_t need = gate_workspace_bytes(P, mlp->hidden);
     if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
     if ((uintptr_t)workspace % 256)
