@@ -144,7 +144,7 @@ def ncu_traffic(kernel: str, workload: str):
             table = json.load(f)
     except OSError:
         return None
-    ent = table.get(kernel)
+    ent = table.get("%s@%s" % (kernel, workload))
     if not ent or ent.get("workload") != workload:
         return None
     src = os.path.join(ROOT, ent["source"])
@@ -509,6 +509,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override B (smaller cases for profiler captures)")
+    ap.add_argument("--heads", type=int, default=0,
+                    help="override H (smaller cases for profiler captures)")
     ap.add_argument("--no-preroll", action="store_true",
                     help="skip the 1 s loaded pre-roll (profiler captures)")
     ap.add_argument("--gate-mlp", type=int, default=0, metavar="HIDDEN",
@@ -524,6 +526,8 @@ def main():
     wl = WORKLOADS[args.workload]
     if args.batch:
         wl = wl.with_(B=args.batch)
+    if args.heads:
+        wl = wl.with_(H=args.heads)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_ours(args, wl)
