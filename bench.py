@@ -214,10 +214,13 @@ def run_reference(args, wl):
 
 def workload_config(wl):
     return {"workload": "%s: B=%d H=%d N=%d d_h=%d %s b=%d r=%d "
-                        "(L_s=%d, gamma=%d) sort_bits=%d non-causal" % (
+                        "(L_s=%d, gamma=%d) sort_bits=%d non-causal%s" % (
                             wl.name, wl.B, wl.H, wl.N, wl.d_h, wl.dtype,
                             wl.block, wl.r, wl.race_tables, wl.race_bits,
-                            wl.sort_bits),
+                            wl.sort_bits,
+                            (", %d neighbour blocks per side" %
+                             wl.neighbor_blocks) if wl.neighbor_blocks
+                            else ""),
             "B": wl.B, "H": wl.H, "N": wl.N, "d_h": wl.d_h,
             "block": wl.block, "r": wl.r, "global_batch": wl.B,
             "seq_len": wl.N,
@@ -509,6 +512,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--batch", type=int, default=0,
                     help="override B (smaller cases for profiler captures)")
+    ap.add_argument("--neighbors", type=int, default=0, metavar="R",
+                    help="R neighbouring sorted key blocks per side "
+                         "(sparse branch on CUDA cores when R > 0)")
     ap.add_argument("--heads", type=int, default=0,
                     help="override H (smaller cases for profiler captures)")
     ap.add_argument("--no-preroll", action="store_true",
@@ -528,6 +534,8 @@ def main():
         wl = wl.with_(B=args.batch)
     if args.heads:
         wl = wl.with_(H=args.heads)
+    if args.neighbors:
+        wl = wl.with_(neighbor_blocks=args.neighbors)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_ours(args, wl)

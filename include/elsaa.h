@@ -39,7 +39,7 @@
 extern "C" {
 #endif
 
-#define ELSAA_ABI_VERSION 1
+#define ELSAA_ABI_VERSION 2
 
 /* Return codes. */
 #define ELSAA_OK 0
@@ -79,6 +79,13 @@ typedef struct elsaa_params {
     int fusion_mode;    /* 0: ELSAA multiplier of Eq. (5);
                            1: Sort_Lsh_RACE ablation, m := 1 (Section 5)      */
     int impl;           /* ELSAA_IMPL_AUTO or ELSAA_IMPL_SIMT                 */
+    int neighbor_blocks;/* r >= 0: query block t also attends to the r
+                           neighbouring sorted key blocks on each side,
+                           t - r .. t + r clipped to the N / b blocks
+                           (Section 5's cost paragraph: (2r + 1) b keys per
+                           query; the paper's runs use r = 0). r > 0 runs
+                           the sparse branch on CUDA cores (fp32) for both
+                           dtypes; elsaa_backward requires r = 0          */
 } elsaa_params;
 
 /*

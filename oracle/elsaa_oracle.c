@@ -149,21 +149,33 @@ static void block_row(const double *q, const double *K, const double *V,
     free(z);
 }
 
+/* Sorted key blocks that query block blk attends to: blk itself and nb
+ * neighbouring sorted blocks on each side (Section 5's cost paragraph:
+ * r neighbouring blocks give (2r + 1) s keys per query), clipped to the
+ * T = N / b blocks that exist. The blocks are consecutive in perm_k, so the
+ * keys are the sorted positions [lo b, (hi + 1) b). */
+static void key_window(int blk, int nb, int T, int *lo, int *hi) {
+    *lo = blk - nb > 0 ? blk - nb : 0;
+    *hi = blk + nb < T - 1 ? blk + nb : T - 1;
+}
+
 /* Full sortLSH branch for one head, given the sorted orders perm_q, perm_k
  * (sorted position t -> original index). Query block t (positions
- * [t b, (t+1) b)) attends to key block t. Outputs are un-permuted:
- * row perm_q[t] of O receives sorted row t. N % b must be 0. */
+ * [t b, (t+1) b)) attends to key block t and its nb neighbours on each side.
+ * Outputs are un-permuted: row perm_q[t] of O receives sorted row t.
+ * N % b must be 0. */
 void elsaa_oracle_sortlsh(const double *Q, const double *K, const double *V,
                           int N, int d_h, const int32_t *perm_q,
-                          const int32_t *perm_k, int b, double scale,
+                          const int32_t *perm_k, int b, int nb, double scale,
                           double eps, double *O_sparse, double *d_sparse,
                           double *log_d_sparse) {
     for (int t = 0; t < N; ++t) {
-        int blk = t / b;
+        int lo, hi;
+        key_window(t / b, nb, N / b, &lo, &hi);
         int i = perm_q[t];
-        block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)blk * b, b,
-                  scale, eps, O_sparse + (size_t)i * d_h, d_sparse + i,
-                  log_d_sparse + i);
+        block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)lo * b,
+                  (hi - lo + 1) * b, scale, eps, O_sparse + (size_t)i * d_h,
+                  d_sparse + i, log_d_sparse + i);
     }
 }
 
@@ -172,7 +184,7 @@ void elsaa_oracle_sortlsh(const double *Q, const double *K, const double *V,
 void elsaa_oracle_sortlsh_rows(const double *Q, const double *K,
                                const double *V, int N, int d_h,
                                const int32_t *perm_q, const int32_t *perm_k,
-                               int b, double scale, double eps,
+                               int b, int nb, double scale, double eps,
                                const int32_t *rows, int n_rows,
                                double *O_rows, double *d_rows,
                                double *logd_rows) {
@@ -180,10 +192,11 @@ void elsaa_oracle_sortlsh_rows(const double *Q, const double *K,
     for (int t = 0; t < N; ++t) pos[perm_q[t]] = t;
     for (int k = 0; k < n_rows; ++k) {
         int i = rows[k];
-        int blk = pos[i] / b;
-        block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)blk * b, b,
-                  scale, eps, O_rows + (size_t)k * d_h, d_rows + k,
-                  logd_rows + k);
+        int lo, hi;
+        key_window(pos[i] / b, nb, N / b, &lo, &hi);
+        block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)lo * b,
+                  (hi - lo + 1) * b, scale, eps, O_rows + (size_t)k * d_h,
+                  d_rows + k, logd_rows + k);
     }
     free(pos);
 }

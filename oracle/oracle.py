@@ -52,11 +52,11 @@ def configure(L):
     L.elsaa_oracle_stable_argsort.argtypes = [_up, ctypes.c_int, _ip]
     L.elsaa_oracle_sortlsh.argtypes = [
         _dp, _dp, _dp, ctypes.c_int, ctypes.c_int, _ip, _ip, ctypes.c_int,
-        ctypes.c_double, ctypes.c_double, _dp, _dp, _dp]
+        ctypes.c_int, ctypes.c_double, ctypes.c_double, _dp, _dp, _dp]
     L.elsaa_oracle_sortlsh_rows.argtypes = [
         _dp, _dp, _dp, ctypes.c_int, ctypes.c_int, _ip, _ip, ctypes.c_int,
-        ctypes.c_double, ctypes.c_double, _ip, ctypes.c_int, _dp, _dp,
-        _dp]
+        ctypes.c_int, ctypes.c_double, ctypes.c_double, _ip, ctypes.c_int,
+        _dp, _dp, _dp]
     L.elsaa_oracle_race_features.argtypes = [
         _dp, ctypes.c_int, _dp, ctypes.c_int, ctypes.c_int,
         ctypes.c_double, _dp]
@@ -164,7 +164,9 @@ def race_readout_rows(Q, w_race, beta, eps, A, Bs, rows):
     return O, dlr
 
 
-def sortlsh(Q, K, V, perm_q, perm_k, b, scale, eps):
+def sortlsh(Q, K, V, perm_q, perm_k, b, scale, eps, nb=0):
+    """sortLSH branch of one head; query block t attends key blocks
+    t - nb .. t + nb (clipped). Returns O_s, d_s, log d_s (all rows)."""
     Q = _c(Q, np.float64)
     K = _c(K, np.float64)
     V = _c(V, np.float64)
@@ -175,11 +177,11 @@ def sortlsh(Q, K, V, perm_q, perm_k, b, scale, eps):
     lib().elsaa_oracle_sortlsh(
         _ptr(Q, _dp), _ptr(K, _dp), _ptr(V, _dp), N, d,
         _ptr(_c(perm_q, np.int32), _ip), _ptr(_c(perm_k, np.int32), _ip), b,
-        scale, eps, _ptr(O, _dp), _ptr(ds, _dp), _ptr(lds, _dp))
+        nb, scale, eps, _ptr(O, _dp), _ptr(ds, _dp), _ptr(lds, _dp))
     return O, ds, lds
 
 
-def sortlsh_rows(Q, K, V, perm_q, perm_k, b, scale, eps, rows):
+def sortlsh_rows(Q, K, V, perm_q, perm_k, b, scale, eps, rows, nb=0):
     Q = _c(Q, np.float64)
     K = _c(K, np.float64)
     V = _c(V, np.float64)
@@ -192,7 +194,7 @@ def sortlsh_rows(Q, K, V, perm_q, perm_k, b, scale, eps, rows):
     lib().elsaa_oracle_sortlsh_rows(
         _ptr(Q, _dp), _ptr(K, _dp), _ptr(V, _dp), N, d,
         _ptr(_c(perm_q, np.int32), _ip), _ptr(_c(perm_k, np.int32), _ip), b,
-        scale, eps, _ptr(rows, _ip), n, _ptr(O, _dp), _ptr(ds, _dp),
+        nb, scale, eps, _ptr(rows, _ip), n, _ptr(O, _dp), _ptr(ds, _dp),
         _ptr(lds, _dp))
     return O, ds, lds
 
@@ -262,7 +264,8 @@ def forward_head(q32, k32, v32, w_sort, w_race, p: dict, lam=None,
     rows = _c(rows, np.int32)
     # Algorithm sortLSH: block attention, un-permuted to the requested rows.
     O_s, d_s, log_d_s = sortlsh_rows(Q, K, V, perm_q, perm_k, p["block"],
-                                     scale, p["eps"], rows)
+                                     scale, p["eps"], rows,
+                                     nb=p.get("neighbors", 0))
     # Algorithm RACE: key-side summaries over all keys, query readout.
     A, Bs = race_summaries(K, V, w_race, p["beta"])
     O_lr, d_lr = race_readout_rows(Q, w_race, p["beta"], p["eps"], A, Bs,
@@ -291,6 +294,7 @@ def params_from_workload(wl, **over) -> dict:
                        lam=wl.lam, fusion_mode=wl.fusion_mode)
     p["race_tables"] = wl.race_tables
     p["race_bits"] = wl.race_bits
+    p["neighbors"] = getattr(wl, "neighbor_blocks", 0)
     p.update(over)
     return p
 

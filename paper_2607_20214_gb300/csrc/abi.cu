@@ -115,6 +115,8 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
         return bad(ELSAA_ERR_INVALID_ARG, "fusion_mode must be 0 or 1");
     if (p->impl != ELSAA_IMPL_AUTO && p->impl != ELSAA_IMPL_SIMT)
         return bad(ELSAA_ERR_INVALID_ARG, "impl must be AUTO or SIMT");
+    if (p->neighbor_blocks < 0)
+        return bad(ELSAA_ERR_INVALID_ARG, "neighbor_blocks must be >= 0");
     if ((long)p->B * p->H > 65535)
         return bad(ELSAA_ERR_UNSUPPORTED, "B * H must be at most 65535");
     if ((long)p->B * p->H * p->N > (1L << 31) - 1)
@@ -144,6 +146,8 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     Q.scale = p->scale > 0.f ? p->scale : 1.0f / sqrtf((float)p->d_h);
     Q.lambda = p->lambda;
     Q.fusion_mode = p->fusion_mode;
+    // neighbour windows wider than the sequence change nothing: clip
+    Q.nb = p->neighbor_blocks < Q.N / Q.b ? p->neighbor_blocks : Q.N / Q.b;
     Q.impl = 1;
     Q.Lg_pad = (Q.L * Q.gamma + 15) / 16 * 16;
     Q.tiles = (Q.N + kHashTile - 1) / kHashTile;
@@ -357,6 +361,9 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                            return launch_race_reduce(P, part, A, Bm, Bh, st);
                        }),
                        "race_reduce");
+    // neighbouring key blocks (nb > 0) run in the persistent kernel for
+    // b of 128 or 256 and nb = 1, otherwise in the CUDA-core block kernel;
+    // the RACE key side above does not depend on them
     if (P.impl == 2 && ws_supported(P)) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_ws", st, [&] {
                                return launch_block_attn_ws(
@@ -365,7 +372,7 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                    m_sparse, status, st);
                            }),
                            "block_attn_ws");
-    } else if (P.impl == 2) {
+    } else if (P.impl == 2 && P.nb == 0) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_tc", st, [&] {
                                return launch_block_attn_tc(
                                    P, q, k, v, w_race, pq, pk, A, Bh,
@@ -403,6 +410,10 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     q.impl = ELSAA_IMPL_SIMT;  // the backward runs on CUDA cores
     int rc = make_plan(&q, &Bp->P, msg);
     if (rc != ELSAA_OK) return rc;
+    if (Bp->P.nb != 0) {
+        *msg = "elsaa_backward requires neighbor_blocks = 0";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
     rc = make_plan(p, &Bp->Pf, msg);  // A, B as the forward makes them
     if (rc != ELSAA_OK) return rc;
     const Plan &P = Bp->P;

@@ -44,6 +44,7 @@ struct Plan {
     int tiles;       // hash tiles per head
     float beta, eps, scale, lambda;
     int fusion_mode;
+    int nb;          // neighbouring sorted key blocks on each side
     int impl;        // resolved: 1 = SIMT, 2 = tensor core
     int Lg_pad;      // L * gamma rounded up to 16 (projection MMA width)
     size_t off_status, off_keyrank, off_hist, off_perm, off_part, off_A,

@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(kBlkThreads)
                  const float *__restrict__ gates, T *__restrict__ ox,
                  float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
                  float *__restrict__ m_out, int N, int d, int H, int b,
-                 int L, int gamma, int tps, float beta, float eps,
+                 int L, int gamma, int tps, int nb, float beta, float eps,
                  float scale, float lambda, int mode, DeviceStatus *status) {
     extern __shared__ float smem[];
     const int bh = blockIdx.y, h = bh % H;
@@ -207,8 +207,13 @@ __global__ void __launch_bounds__(kBlkThreads)
 #pragma unroll
         for (int c = 0; c < 4; ++c) o_acc[qq][c] = 0.f;
     }
-    const int kbase = blk * b;
-    for (int c0 = 0; c0 < b; c0 += kKC) {
+    // key block blk and its nb neighbouring sorted blocks on each side,
+    // clipped to the N / b blocks: sorted positions [lo b, (hi + 1) b)
+    const int nblk = N / b;
+    const int lo = blk - nb > 0 ? blk - nb : 0;
+    const int hi = blk + nb < nblk - 1 ? blk + nb : nblk - 1;
+    const int kbase = lo * b, nkeys = (hi - lo + 1) * b;
+    for (int c0 = 0; c0 < nkeys; c0 += kKC) {
         __syncthreads();
         for (int i = tid; i < kKC * d; i += kBlkThreads) {
             int row = i / d, col = i - row * d;
@@ -424,8 +429,8 @@ cudaError_t launch_block_attn_simt(
         kern<<<grid, kBlkThreads, smem, st>>>(                                \
             (const T *)q, (const T *)k, (const T *)v, w_race, perm_q, perm_k, \
             A, Bm, lambda_tok, gates, (T *)o, log_d_sparse, d_lr, m_sparse,   \
-            P.N, P.d, P.H, P.b, P.L, P.gamma, P.tables_per_slice, P.beta,     \
-            P.eps, P.scale, P.lambda, P.fusion_mode, status);                 \
+            P.N, P.d, P.H, P.b, P.L, P.gamma, P.tables_per_slice, P.nb,       \
+            P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, status);         \
     } while (0)
     if (P.dtype == ELSAA_FP32)
         ELSAA_LAUNCH_BLK(float);

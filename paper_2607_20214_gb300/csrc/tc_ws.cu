@@ -59,8 +59,9 @@ struct WsBars {
     uint64_t tmem_empty[2];
 };
 
-// NPASS = 2 for key blocks of 256 (two 128-key halves per query tile,
-// online softmax across them), 1 for b <= 128.
+// NPASS 128-key passes per query tile, online softmax across them: 1 for
+// b <= 128; b / 128 for larger blocks; with nb neighbouring sorted key
+// blocks per side (b >= 128), (2 nb + 1) b / 128 passes over the window.
 template <int G, int NPASS>
 __global__ void __launch_bounds__(kWsThreads, 1)
     k_block_attn_ws(const uint16_t *__restrict__ qx,
@@ -75,7 +76,8 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     const float *__restrict__ gates, uint16_t *__restrict__ ox,
                     float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
                     float *__restrict__ m_out, int N, int d, int H, int b,
-                    int L, int Lg_pad, float beta, float eps, float scale,
+                    int nb, int L, int Lg_pad, float beta, float eps,
+                    float scale,
                     float lambda, int mode, int tiles_per_head,
                     long total_tiles, DeviceStatus *status) {
     constexpr int R = 1 << G;
@@ -144,9 +146,21 @@ __global__ void __launch_bounds__(kWsThreads, 1)
         return i == 0 || (tb + i) % tiles_per_head == 0;
     };
     // sorted position of key column 0 of pass p of the tile starting at
-    // query position p0 (key blocks of 256: the block's two 128-key halves)
+    // query position p0: the passes walk the key window of the tile's
+    // query block (the block and nb neighbouring blocks per side) in
+    // 128-key steps. A pass past either end of the sequence holds no keys:
+    // its rows are read from a valid position and its scores are masked.
+    auto key_pos_raw = [=](int p0, int p) {
+        return NPASS == 1 ? p0 : (p0 / b - nb) * b + 128 * p;
+    };
+    auto pass_valid = [=](int p0, int p) {
+        const int k0 = key_pos_raw(p0, p);
+        return k0 >= 0 && k0 < N;
+    };
     auto key_pos = [=](int p0, int p) {
-        return NPASS == 1 ? p0 : (p0 / (128 * NPASS)) * (128 * NPASS) + 128 * p;
+        const int k0 = key_pos_raw(p0, p);
+        if (NPASS == 1) return k0;  // the tile's own keys (ragged end kept)
+        return k0 < 0 ? 0 : (k0 > N - 128 ? N - 128 : k0);
     };
     // global row numbers of the 4 sorted positions pos.. pos + 3 (the
     // ragged end repeats the last row; those rows are never stored)
@@ -351,8 +365,10 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                         ready = (ts < 2 || mbar_test(&bars.tmem_empty[s],
                                                      ((ts >> 1) - 1) & 1)) &&
                                 (!nh || mbar_test(&bars.wb_full, hc & 1));
-                    if (ready && spass > 0)  // S columns hold P of pass 0
-                        ready = mbar_test(&bars.pv0_done[s], (ts >> 1) & 1);
+                    if (ready && spass > 0)  // S columns hold P of pass - 1
+                        ready = mbar_test(&bars.pv0_done[s],
+                                          ((ts >> 1) * (NPASS - 1) + spass -
+                                           1) & 1);
                     if (ready) {
                         if (nh) ++hc;
                         fence_proxy_async_smem();  // cp.async data -> MMA
@@ -497,6 +513,8 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             const int khi = b < 128 ? klo + b : nk;
             float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             const bool masked = b < 128;
+            // pass 0 of a tile whose window starts before the sequence
+            const bool valid0 = NPASS == 1 || pass_valid(p0, 0);
 #pragma unroll
             for (int c = 0; c < nk / 2; c += 16) {
                 uint32_t v[16];
@@ -505,7 +523,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
 #pragma unroll
                 for (int jj = 0; jj < 16; ++jj) {
                     const int key = kbeg + c + jj;
-                    if (!masked || (key >= klo && key < khi))
+                    if (valid0 && (!masked || (key >= klo && key < khi)))
                         mxa[jj & 3] = fmaxf(mxa[jj & 3], __uint_as_float(v[jj]));
                 }
             }
@@ -537,6 +555,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                             a0 = (key >= klo && key < khi) ? a0 : 0.0f;
                             a1 = (key + 1 >= klo && key + 1 < khi) ? a1 : 0.0f;
                         }
+                        if (!valid0) a0 = a1 = 0.0f;
                         ls[(jj >> 1) & 3] += a0 + a1;
                         pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
                     }
@@ -550,34 +569,54 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             named_sync(1 + g, 256);  // every S read of the slot is done
             tc_fence_after();
             lsum = xsum[g][0][row] + xsum[g][1][row];
-            if constexpr (NPASS > 1) {
-                // pass 0's P goes to its P V product; pass 1 scores the
-                // second key half into the same columns
+            bool pass_fail = false;
+#pragma unroll 1
+            for (int ps = 1; ps < NPASS; ++ps) {
+                // the previous pass's P goes to its P V product; this pass
+                // scores the next 128 keys into the same columns
                 tmem_wait_st();
                 tc_fence_before();
                 mbar_arrive(&bars.p_full[g]);
-                if (!wwait(&bars.s_full[g], (k * NPASS + 1) & 1, 56)) break;
+                if (!wwait(&bars.s_full[g], (k * NPASS + ps) & 1, 56)) {
+                    pass_fail = true;
+                    break;
+                }
                 tc_fence_after();
-                if (j + 1 < ntiles && !issue_qk(j + 1)) break;
+                // the K buffer is free again: the next pass's keys, or after
+                // the last pass the next tile's queries and keys
+                if (ps + 1 < NPASS) {
+                    if (!issue_k(j, ps + 1)) {
+                        pass_fail = true;
+                        break;
+                    }
+                } else if (j + 1 < ntiles && !issue_qk(j + 1)) {
+                    pass_fail = true;
+                    break;
+                }
+                const bool pvalid = pass_valid(p0, ps);
                 float mxb[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                if (pvalid) {
 #pragma unroll
-                for (int c = 0; c < nk / 2; c += 16) {
-                    uint32_t v[16];
-                    tmem_ld16(so + kbeg + c, v);
-                    tmem_wait_ld();
+                    for (int c = 0; c < nk / 2; c += 16) {
+                        uint32_t v[16];
+                        tmem_ld16(so + kbeg + c, v);
+                        tmem_wait_ld();
 #pragma unroll
-                    for (int jj = 0; jj < 16; ++jj)
-                        mxb[jj & 3] = fmaxf(mxb[jj & 3], __uint_as_float(v[jj]));
+                        for (int jj = 0; jj < 16; ++jj)
+                            mxb[jj & 3] =
+                                fmaxf(mxb[jj & 3], __uint_as_float(v[jj]));
+                    }
                 }
                 xmax[g][half][row] =
                     fmaxf(fmaxf(mxb[0], mxb[1]), fmaxf(mxb[2], mxb[3]));
                 named_sync(1 + g, 256);
                 const float M2b =
                     fmaxf(xmax[g][0][row], xmax[g][1][row]) * sl2e;
-                // online softmax: keep pass 0's reference unless the row's
-                // max grew by more than 2^8; then rescale the accumulator
-                // (P V of pass 0 is complete: S of pass 1 waited for it)
-                // and the running sum
+                // online softmax: keep the running reference unless the
+                // row's max grew by more than 2^8; then rescale the
+                // accumulator (the previous P V product is complete: these
+                // scores waited for it) and the running sum. From an empty
+                // start (M2 = -inf) the factor is 0.
                 const bool need = M2b > M2 + 8.0f;
                 const float f = need ? ex2_approx(M2 - M2b) : 1.0f;
                 if (__any_sync(0xffffffffu, need)) {
@@ -609,10 +648,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                         tmem_wait_ld();
 #pragma unroll
                         for (int jj = 0; jj < 16; jj += 2) {
-                            const float a0 = ex2_approx(
+                            float a0 = ex2_approx(
                                 fmaf(__uint_as_float(v[jj]), sl2e, -M2));
-                            const float a1 = ex2_approx(
+                            float a1 = ex2_approx(
                                 fmaf(__uint_as_float(v[jj + 1]), sl2e, -M2));
+                            if (!pvalid) a0 = a1 = 0.0f;
                             lb[(jj >> 1) & 3] += a0 + a1;
                             pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
                         }
@@ -625,6 +665,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                 tc_fence_after();
                 lsum += xsum[g][0][row] + xsum[g][1][row];
             }
+            if (pass_fail) break;
             // fusion scalars (Eq. (5) in log-sum-exp form, Eq. (6))
             qi = (qi < 0 || qi >= N) ? 0 : qi;
             const size_t tok = (size_t)bh * N + qi;
@@ -721,13 +762,23 @@ __global__ void __launch_bounds__(kWsThreads, 1)
 
 }  // namespace
 
+// 128-key passes per query tile, or 0 when no instantiation covers it:
+// b <= 128 without neighbours: 1; b = 256: 2; neighbouring blocks (b of
+// 128 or 256, gamma = 4): the (2 nb + 1) b / 128 passes of the window, 3 or
+// 6 for nb = 1.
+static int ws_passes(const Plan &P) {
+    if (P.nb == 0) return P.b <= 128 ? 1 : (P.b == 256 ? 2 : 0);
+    if (P.nb != 1 || P.gamma != 4 || (P.b != 128 && P.b != 256)) return 0;
+    return 3 * (P.b / 128);
+}
+
 bool ws_supported(const Plan &P) {
     // a half's chunks: the first may use up to 32 projection columns, the
     // second (buckets past 128) at most 16, i.e. gamma >= 4 when r > 128;
     // row numbers in int
     const long rows = (long)P.N * P.BH;  // row numbers are int
-    return tc_supported(P) && P.b <= 256 && (P.gamma >= 4 || P.r <= 128) &&
-           rows < (1L << 31);
+    return tc_supported(P) && ws_passes(P) > 0 &&
+           (P.gamma >= 4 || P.r <= 128) && rows < (1L << 31);
 }
 
 cudaError_t launch_block_attn_ws(
@@ -762,11 +813,14 @@ cudaError_t launch_block_attn_ws(
         kern<<<grid, kWsThreads, smem, st>>>(
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
             tmW, tmB, perm_q, perm_k, A, lambda_tok, gates, (uint16_t *)o,
-            log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, P.L, lg, P.beta,
-            P.eps, P.scale, P.lambda, P.fusion_mode, tiles_per_head, total,
-            status);
+            log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, P.nb, P.L, lg,
+            P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, tiles_per_head,
+            total, status);
         return cudaGetLastError();
     };
+    const int passes = ws_passes(P);
+    if (passes == 3) return launch(k_block_attn_ws<4, 3>);
+    if (passes == 6) return launch(k_block_attn_ws<4, 6>);
     switch (P.gamma) {
         case 1: return P.b > 128 ? launch(k_block_attn_ws<1, 2>) : launch(k_block_attn_ws<1, 1>);
         case 2: return P.b > 128 ? launch(k_block_attn_ws<2, 2>) : launch(k_block_attn_ws<2, 1>);

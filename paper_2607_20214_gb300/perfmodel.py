@@ -30,6 +30,7 @@ def flop_model(wl: Workload) -> dict:
     separately.
     """
     N, b, d, r = wl.N, wl.block, wl.d_h, wl.r
+    b = keys_per_query(wl)
     per_head = (4 * N * b * d + 4 * N * r * d + 4 * N * r
                 + 4 * N * d * wl.race_tables * wl.race_bits)
     heads = wl.heads
@@ -46,6 +47,13 @@ def flop_model(wl: Workload) -> dict:
 SIMT_FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
+def keys_per_query(wl: Workload) -> int:
+    """Keys each query attends to in the sparse branch: its block and the
+    neighbouring sorted blocks, (2 r + 1) b (Section 5), at most N (the
+    clipped windows at the two ends are counted as full)."""
+    return min(wl.N, (2 * getattr(wl, "neighbor_blocks", 0) + 1) * wl.block)
+
+
 def kernel_work(wl: Workload, kernel: str) -> dict:
     """Algorithmic work of ONE launch of a kernel over the whole workload.
 
@@ -53,7 +61,7 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
     written once); flops: the kernel's share of the operator's arithmetic;
     unit: which engine runs that arithmetic ("tensor" or "alu").
     """
-    N, b, d, r = wl.N, wl.block, wl.d_h, wl.r
+    N, b, d, r = wl.N, keys_per_query(wl), wl.d_h, wl.r
     H = wl.heads
     Lg = wl.race_tables * wl.race_bits
     e = wl.elt

@@ -40,6 +40,7 @@ class Workload:
     lam: float = 1.0
     fusion_mode: int = 0  # 0: ELSAA multiplier, 1: Sort_Lsh_RACE ablation (m = 1)
     causal: int = 0
+    neighbor_blocks: int = 0  # r neighbouring sorted key blocks per side
     recipe: str = "plain"  # input recipe, see make_inputs
     temperature: float = 1.0
     seed: int = 0

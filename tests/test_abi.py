@@ -58,7 +58,7 @@ def test_params_struct_matches_header():
 
 
 def test_abi_version(lib):
-    assert elsaa.elsaa_abi_version() == 1
+    assert elsaa.elsaa_abi_version() == 2
 
 
 @pytest.mark.parametrize("name", sorted(WORKLOADS))
@@ -83,6 +83,7 @@ BAD = [
     (dict(race_tables=64, race_bits=5), elsaa.ELSAA_ERR_UNSUPPORTED, "1024"),
     (dict(fusion_mode=3), elsaa.ELSAA_ERR_INVALID_ARG, "fusion_mode"),
     (dict(B=0), elsaa.ELSAA_ERR_INVALID_ARG, "positive"),
+    (dict(neighbor_blocks=-1), elsaa.ELSAA_ERR_INVALID_ARG, "neighbor"),
 ]
 
 

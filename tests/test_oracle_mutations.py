@@ -29,11 +29,17 @@ MUTATIONS = [
     ("dropped_eps_sparse", "o[e] /= (den + floor_);", "o[e] /= den;",
      pins.test_zero_sort_bits_is_block_diagonal_local_attention, (16,)),
     ("next_key_block",
-     "block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)blk * b, b,\n"
-     "                  scale, eps, O_rows",
-     "block_row(Q + (size_t)i * d_h, K, V, d_h, perm_k + (size_t)((blk + 1) %"
-     " (N / b)) * b, b,\n                  scale, eps, O_rows",
+     "key_window(pos[i] / b, nb, N / b, &lo, &hi);",
+     "key_window((pos[i] / b + 1) % (N / b), nb, N / b, &lo, &hi);",
      pins.test_query_block_t_attends_exactly_key_block_t, ()),
+    ("neighbour_window_too_wide",
+     "*lo = blk - nb > 0 ? blk - nb : 0;",
+     "*lo = blk - 2 * nb > 0 ? blk - 2 * nb : 0;",
+     pins.test_neighbour_blocks_with_zero_sort_bits_are_banded, (16, 1)),
+    ("upper_neighbours_dropped",
+     "*hi = blk + nb < T - 1 ? blk + nb : T - 1;",
+     "*hi = blk < T - 1 ? blk : T - 1;",
+     pins.test_neighbour_blocks_with_zero_sort_bits_are_banded, (8, 2)),
     ("dropped_table_average", "den /= (double)L;", "",
      pins.test_race_beta_zero_closed_form, ()),
     ("phi_from_values", "race_phi(K + (size_t)j * d_h, d_h, w_l, gamma",

@@ -161,6 +161,46 @@ def test_zero_sort_bits_is_block_diagonal_local_attention(b):
     np.testing.assert_allclose(res["d_sparse"], den, rtol=1e-12)
 
 
+@pytest.mark.parametrize("b,nb", [(16, 1), (8, 2), (32, 1)])
+def test_neighbour_blocks_with_zero_sort_bits_are_banded(b, nb):
+    """n_s = 0 and nb neighbouring blocks: query i attends to the keys of
+    blocks i // b - nb .. i // b + nb (clipped at the ends), brute force."""
+    N, d = 96, 16
+    q, k, v = rand_head(N, d, b + nb, temp=1.5)
+    _, w_race = planes(d, 0, 2, 2, b)
+    p = orc.default_params(block=b, sort_bits=0, eps=1e-6, neighbors=nb)
+    res = orc.forward_head(q, k, v, np.zeros((0, d), np.float32), w_race, p)
+    z = (q.astype(np.float64) @ k.astype(np.float64).T) / np.sqrt(d)
+    blk = np.arange(N) // b
+    band = np.abs(blk[:, None] - blk[None, :]) <= nb
+    e = np.exp(np.where(band, z, -np.inf))
+    den = e.sum(axis=1)
+    o_ref = (e @ v.astype(np.float64)) / (den + 1e-6)[:, None]
+    np.testing.assert_allclose(res["O_sparse"], o_ref, rtol=1e-11,
+                               atol=1e-12)
+    np.testing.assert_allclose(res["d_sparse"], den, rtol=1e-12)
+    # the first and last blocks see nb fewer blocks than the middle ones
+    assert band[0].sum() == (nb + 1) * b
+    assert band[N // 2].sum() == min(N, (2 * nb + 1) * b)
+
+
+def test_neighbour_blocks_covering_all_blocks_give_dense_attention():
+    """nb >= N / b - 1: every query attends to all N keys, whatever the
+    hash and the sort (dense softmax attention, scipy)."""
+    N, d, b = 64, 16, 16
+    q, k, v = rand_head(N, d, 9, temp=2.0)
+    w_sort, w_race = planes(d, 5, 2, 2, 9)
+    p = orc.default_params(block=b, sort_bits=5, eps=0.0,
+                           neighbors=N // b - 1)
+    res = orc.forward_head(q, k, v, w_sort, w_race, p)
+    z = (q.astype(np.float64) @ k.astype(np.float64).T) / np.sqrt(d)
+    np.testing.assert_allclose(res["O_sparse"],
+                               softmax(z, axis=1) @ v.astype(np.float64),
+                               rtol=1e-11, atol=1e-12)
+    np.testing.assert_allclose(np.log(res["d_sparse"]),
+                               logsumexp(z, axis=1), rtol=1e-12)
+
+
 def test_query_block_t_attends_exactly_key_block_t():
     """V = identity: sparse weights of query i are nonzero exactly on the
     keys of its block (query block t <-> key block t of the sorted orders)."""

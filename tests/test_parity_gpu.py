@@ -145,6 +145,24 @@ def test_bf16_hash_variants(over):
     compare(wl, run_gpu(wl, x), run_oracle(wl, x), label=str(over))
 
 
+@pytest.mark.parametrize("dtype,b,nb,N,d_h", [("fp32", 32, 1, 1184, 64),
+                                              ("bf16", 64, 2, 1024, 64),
+                                              ("bf16", 128, 1, 1152, 64),
+                                              ("bf16", 128, 1, 512, 128),
+                                              ("bf16", 256, 1, 1536, 64),
+                                              ("bf16", 256, 1, 512, 128),
+                                              ("bf16", 32, 9, 256, 64)])
+def test_neighbour_blocks(dtype, b, nb, N, d_h):
+    """r = nb neighbouring sorted key blocks per side (Section 5's cost
+    paragraph), clipped at the ends; the last case covers every block.
+    b of 128 / 256 with nb = 1 run in the persistent tensor-core kernel
+    (3 / 6 key passes per query tile, the passes past either end masked);
+    the others on CUDA cores."""
+    wl = small(dtype, H=2, N=N, block=b, d_h=d_h).with_(neighbor_blocks=nb)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="nb%d" % nb)
+
+
 def test_single_block_and_minimum_size():
     wl = small("fp32", N=32, block=32, B=3, H=1)
     x = make_inputs(wl)
@@ -188,13 +206,16 @@ def test_c2_full_size_subset_of_heads():
     compare(wl, run_gpu(wl, x), run_oracle(wl, x, heads=heads), label="c2")
 
 
-@pytest.mark.parametrize("name,heads", [("c3", [(0, 0), (1, 15)]),
-                                        ("c4", [(0, 0), (0, 31)]),
-                                        ("c5", [(0, 0), (7, 11)])])
-def test_full_size_sampled_rows(name, heads):
+@pytest.mark.parametrize("name,heads,nb", [("c3", [(0, 0), (1, 15)], 0),
+                                           ("c4", [(0, 0), (0, 31)], 0),
+                                           ("c5", [(0, 0), (7, 11)], 0),
+                                           ("c3", [(1, 3)], 1),
+                                           ("c4", [(0, 7)], 1)])
+def test_full_size_sampled_rows(name, heads, nb):
     """Full-size launch; exact perms of sampled heads; outputs on 512
-    sampled rows per head (plus the duplicated-key rows for c4)."""
-    wl = WORKLOADS[name]
+    sampled rows per head (plus the duplicated-key rows for c4). nb = 1:
+    the same workloads with one neighbouring sorted block per side."""
+    wl = WORKLOADS[name].with_(neighbor_blocks=nb)
     x = make_inputs(wl, device="cuda")
     g = run_gpu(wl, x)
     rng = np.random.default_rng(0)
