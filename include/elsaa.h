@@ -83,9 +83,11 @@ typedef struct elsaa_params {
                            neighbouring sorted key blocks on each side,
                            t - r .. t + r clipped to the N / b blocks
                            (Section 5's cost paragraph: (2r + 1) b keys per
-                           query; the paper's runs use r = 0). r > 0 runs
-                           the sparse branch on CUDA cores (fp32) for both
-                           dtypes; elsaa_backward requires r = 0          */
+                           query; the paper's runs use r = 0). bf16 with
+                           b of 128 or 256, r = 1 and race_bits = 4 runs on
+                           the tensor cores; other r > 0 shapes run the
+                           sparse branch on CUDA cores (fp32).
+                           elsaa_backward requires r = 0                  */
 } elsaa_params;
 
 /*

@@ -62,7 +62,9 @@ struct WsBars {
 // NPASS 128-key passes per query tile, online softmax across them: 1 for
 // b <= 128; b / 128 for larger blocks; with nb neighbouring sorted key
 // blocks per side (b >= 128), (2 nb + 1) b / 128 passes over the window.
-template <int G, int NPASS>
+// WIN: the passes walk a neighbour window (nb > 0), whose passes past
+// either end of the sequence are masked; false compiles those checks out.
+template <int G, int NPASS, bool WIN>
 __global__ void __launch_bounds__(kWsThreads, 1)
     k_block_attn_ws(const uint16_t *__restrict__ qx,
                     const uint16_t *__restrict__ kx,
@@ -151,9 +153,10 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     // 128-key steps. A pass past either end of the sequence holds no keys:
     // its rows are read from a valid position and its scores are masked.
     auto key_pos_raw = [=](int p0, int p) {
-        return NPASS == 1 ? p0 : (p0 / b - nb) * b + 128 * p;
+        return NPASS == 1 ? p0 : (p0 / b - (WIN ? nb : 0)) * b + 128 * p;
     };
     auto pass_valid = [=](int p0, int p) {
+        if (!WIN) return true;
         const int k0 = key_pos_raw(p0, p);
         return k0 >= 0 && k0 < N;
     };
@@ -514,7 +517,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             float mxa[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
             const bool masked = b < 128;
             // pass 0 of a tile whose window starts before the sequence
-            const bool valid0 = NPASS == 1 || pass_valid(p0, 0);
+            const bool valid0 = !WIN || pass_valid(p0, 0);
 #pragma unroll
             for (int c = 0; c < nk / 2; c += 16) {
                 uint32_t v[16];
@@ -523,7 +526,8 @@ __global__ void __launch_bounds__(kWsThreads, 1)
 #pragma unroll
                 for (int jj = 0; jj < 16; ++jj) {
                     const int key = kbeg + c + jj;
-                    if (valid0 && (!masked || (key >= klo && key < khi)))
+                    if ((!WIN || valid0) &&
+                        (!masked || (key >= klo && key < khi)))
                         mxa[jj & 3] = fmaxf(mxa[jj & 3], __uint_as_float(v[jj]));
                 }
             }
@@ -555,7 +559,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                             a0 = (key >= klo && key < khi) ? a0 : 0.0f;
                             a1 = (key + 1 >= klo && key + 1 < khi) ? a1 : 0.0f;
                         }
-                        if (!valid0) a0 = a1 = 0.0f;
+                        if (WIN && !valid0) a0 = a1 = 0.0f;
                         ls[(jj >> 1) & 3] += a0 + a1;
                         pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
                     }
@@ -570,7 +574,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             tc_fence_after();
             lsum = xsum[g][0][row] + xsum[g][1][row];
             bool pass_fail = false;
-#pragma unroll 1
+#pragma unroll
             for (int ps = 1; ps < NPASS; ++ps) {
                 // the previous pass's P goes to its P V product; this pass
                 // scores the next 128 keys into the same columns
@@ -593,9 +597,9 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     pass_fail = true;
                     break;
                 }
-                const bool pvalid = pass_valid(p0, ps);
+                const bool pvalid = !WIN || pass_valid(p0, ps);
                 float mxb[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                if (pvalid) {
+                if (!WIN || pvalid) {
 #pragma unroll
                     for (int c = 0; c < nk / 2; c += 16) {
                         uint32_t v[16];
@@ -652,7 +656,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                                 fmaf(__uint_as_float(v[jj]), sl2e, -M2));
                             float a1 = ex2_approx(
                                 fmaf(__uint_as_float(v[jj + 1]), sl2e, -M2));
-                            if (!pvalid) a0 = a1 = 0.0f;
+                            if (WIN && !pvalid) a0 = a1 = 0.0f;
                             lb[(jj >> 1) & 3] += a0 + a1;
                             pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
                         }
@@ -819,15 +823,15 @@ cudaError_t launch_block_attn_ws(
         return cudaGetLastError();
     };
     const int passes = ws_passes(P);
-    if (passes == 3) return launch(k_block_attn_ws<4, 3>);
-    if (passes == 6) return launch(k_block_attn_ws<4, 6>);
+    if (passes == 3) return launch(k_block_attn_ws<4, 3, true>);
+    if (passes == 6) return launch(k_block_attn_ws<4, 6, true>);
     switch (P.gamma) {
-        case 1: return P.b > 128 ? launch(k_block_attn_ws<1, 2>) : launch(k_block_attn_ws<1, 1>);
-        case 2: return P.b > 128 ? launch(k_block_attn_ws<2, 2>) : launch(k_block_attn_ws<2, 1>);
-        case 3: return P.b > 128 ? launch(k_block_attn_ws<3, 2>) : launch(k_block_attn_ws<3, 1>);
-        case 4: return P.b > 128 ? launch(k_block_attn_ws<4, 2>) : launch(k_block_attn_ws<4, 1>);
-        case 5: return P.b > 128 ? launch(k_block_attn_ws<5, 2>) : launch(k_block_attn_ws<5, 1>);
-        case 6: return P.b > 128 ? launch(k_block_attn_ws<6, 2>) : launch(k_block_attn_ws<6, 1>);
+        case 1: return P.b > 128 ? launch(k_block_attn_ws<1, 2, false>) : launch(k_block_attn_ws<1, 1, false>);
+        case 2: return P.b > 128 ? launch(k_block_attn_ws<2, 2, false>) : launch(k_block_attn_ws<2, 1, false>);
+        case 3: return P.b > 128 ? launch(k_block_attn_ws<3, 2, false>) : launch(k_block_attn_ws<3, 1, false>);
+        case 4: return P.b > 128 ? launch(k_block_attn_ws<4, 2, false>) : launch(k_block_attn_ws<4, 1, false>);
+        case 5: return P.b > 128 ? launch(k_block_attn_ws<5, 2, false>) : launch(k_block_attn_ws<5, 1, false>);
+        case 6: return P.b > 128 ? launch(k_block_attn_ws<6, 2, false>) : launch(k_block_attn_ws<6, 1, false>);
         default: return cudaErrorInvalidValue;
     }
 }
