@@ -23,6 +23,12 @@
  *     the workspace argument, sized by elsaa_workspace_size().
  *   - Calls are asynchronous on the caller's CUDA stream (cudaStream_t passed
  *     as void*; NULL = the legacy default stream) and never synchronise.
+ *     elsaa_forward also runs the RACE key side, which needs no sort, on a
+ *     library-owned stream (one per host thread and device, created on first
+ *     use, non-blocking), forked from the caller's stream after the call's
+ *     first operation and joined back into it with events before the block
+ *     kernel: the call's work stays ordered on the caller's stream as a unit
+ *     and can be captured into a CUDA graph.
  *   - Arguments are validated on the host before any launch. The return value
  *     is ELSAA_OK or one of the ELSAA_ERR_* codes; elsaa_last_error() then
  *     holds a one-line description (thread-local).

@@ -62,6 +62,39 @@ cudaError_t timed(const char *name, cudaStream_t st, F fn) {
     return e;
 }
 
+// A second stream per host thread and device for the RACE key side, which
+// needs no sort: forked from the caller's stream after the status reset and
+// joined back before the block kernel, so it overlaps the hash, scan and
+// scatter. Created on first use, kept for the life of the process.
+struct SideStream {
+    int dev = -1;
+    cudaStream_t s = nullptr;
+    cudaEvent_t fork = nullptr, join = nullptr;
+};
+
+cudaError_t side_stream(SideStream **out) {
+    thread_local std::vector<SideStream> ss;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    for (auto &x : ss)
+        if (x.dev == dev) {
+            *out = &x;
+            return cudaSuccess;
+        }
+    SideStream x;
+    x.dev = dev;
+    e = cudaStreamCreateWithFlags(&x.s, cudaStreamNonBlocking);
+    if (e == cudaSuccess)
+        e = cudaEventCreateWithFlags(&x.fork, cudaEventDisableTiming);
+    if (e == cudaSuccess)
+        e = cudaEventCreateWithFlags(&x.join, cudaEventDisableTiming);
+    if (e != cudaSuccess) return e;
+    ss.push_back(x);
+    *out = &ss.back();
+    return cudaSuccess;
+}
+
 // RACE key-chunk CTAs aimed for: about two per SM of a 152-SM GB300. A
 // constant (not a device query) keeps the workspace size device-independent.
 constexpr long kRaceTargetCtas = 304;
@@ -327,6 +360,35 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
 
     ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
                        "status reset");
+    // RACE key side (no sort needed) on the side stream, launched first so
+    // that its CTAs are placed before the hash kernel's
+    SideStream *side = nullptr;
+    ELSAA_CHECK_LAUNCH(side_stream(&side), "side stream");
+    cudaStream_t ks = side->s;
+    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->fork, st), "fork");
+    ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(ks, side->fork, 0), "fork wait");
+    if (P.impl == 2) {
+        ELSAA_CHECK_LAUNCH(timed("prep_planes", ks, [&] {
+                               return launch_prep_planes(P, w_race, Wbf, ks);
+                           }),
+                           "prep_planes");
+        ELSAA_CHECK_LAUNCH(timed("race_keys_ws", ks, [&] {
+                               return launch_race_keys_ws(P, k, v, Wbf, part,
+                                                          status, ks);
+                           }),
+                           "race_keys_ws");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("race_partial_simt", ks, [&] {
+                               return launch_race_partial_simt(P, k, v, w_race,
+                                                               part, ks);
+                           }),
+                           "race_partial_simt");
+    }
+    ELSAA_CHECK_LAUNCH(timed("race_reduce", ks, [&] {
+                           return launch_race_reduce(P, part, A, Bm, Bh, ks);
+                       }),
+                       "race_reduce");
+    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->join, ks), "join");
     ELSAA_CHECK_LAUNCH(timed("sort_hash", st, [&] {
                            return launch_sort_hash(P, q, k, w_sort, keyrank,
                                                    hist, status, st);
@@ -340,27 +402,7 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                                       pk, status, st);
                        }),
                        "sort_scatter");
-    if (P.impl == 2) {
-        ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
-                               return launch_prep_planes(P, w_race, Wbf, st);
-                           }),
-                           "prep_planes");
-        ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
-                               return launch_race_keys_ws(P, k, v, Wbf, part,
-                                                          status, st);
-                           }),
-                           "race_keys_ws");
-    } else {
-        ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
-                               return launch_race_partial_simt(P, k, v, w_race,
-                                                               part, st);
-                           }),
-                           "race_partial_simt");
-    }
-    ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
-                           return launch_race_reduce(P, part, A, Bm, Bh, st);
-                       }),
-                       "race_reduce");
+    ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(st, side->join, 0), "join wait");
     // neighbouring key blocks (nb > 0) run in the persistent kernel for
     // b of 128 or 256 and nb = 1, otherwise in the CUDA-core block kernel;
     // the RACE key side above does not depend on them
