@@ -296,6 +296,20 @@ int elsaa_profile_start(void);
 int elsaa_profile_stop(elsaa_kernel_stat *out, int max_entries,
                        int *n_entries);
 
+/*
+ * Self-test of the in-band failure path, for tests. Every wait inside the
+ * kernels is bounded; one that runs out records {code 3 (wait timeout),
+ * site, CTA} in the workspace status word and lets its kernel return, and
+ * elsaa_check_status reports it. This call enqueues one CTA whose bounded
+ * mbarrier wait can never complete (nothing arrives): after limit_ms
+ * milliseconds (1..2000) it records the timeout at site 0x7e57 and returns.
+ * Nothing faults or hangs; the context stays usable and the next
+ * elsaa_forward on the workspace clears the word. workspace: 256-byte
+ * aligned, at least 16 bytes.
+ */
+int elsaa_selftest_wait_timeout(void *workspace, size_t workspace_bytes,
+                                int limit_ms, void *stream);
+
 /* One-line description of the last error on this thread ("" if none). */
 const char *elsaa_last_error(void);
 

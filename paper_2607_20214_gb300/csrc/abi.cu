@@ -692,6 +692,25 @@ extern "C" int elsaa_gates(const elsaa_params *params,
     return ELSAA_OK;
 }
 
+extern "C" int elsaa_selftest_wait_timeout(void *workspace,
+                                           size_t workspace_bytes,
+                                           int limit_ms, void *stream) {
+    g_err[0] = 0;
+    if (!workspace || workspace_bytes < sizeof(DeviceStatus))
+        return fail(ELSAA_ERR_WORKSPACE, "workspace missing or too small");
+    if ((uintptr_t)workspace % 256)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if (limit_ms < 1 || limit_ms > 2000)
+        return fail(ELSAA_ERR_INVALID_ARG, "limit_ms must be in [1, 2000]");
+    cudaStream_t st = (cudaStream_t)stream;
+    DeviceStatus *status = (DeviceStatus *)workspace;
+    ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
+                       "status reset");
+    ELSAA_CHECK_LAUNCH(launch_selftest_wait(status, limit_ms, st),
+                       "selftest_wait");
+    return ELSAA_OK;
+}
+
 extern "C" int elsaa_check_status(const void *workspace, void *stream) {
     g_err[0] = 0;
     if (!workspace) return fail(ELSAA_ERR_INVALID_ARG, "workspace is NULL");

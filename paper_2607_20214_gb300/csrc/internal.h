@@ -114,6 +114,10 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
                             const float *gB, float *dk, float *dv,
                             cudaStream_t st);
 
+// One bounded mbarrier wait that can never complete (selftest.cu).
+cudaError_t launch_selftest_wait(DeviceStatus *status, int limit_ms,
+                                 cudaStream_t st);
+
 // Token-wise gate MLP and query-dependent lambda (gates.cu).
 int gate_ng(int hidden);
 bool gate_tc_supported(const Plan &P);

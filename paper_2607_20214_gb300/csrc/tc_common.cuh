@@ -90,18 +90,28 @@ __device__ __forceinline__ void record_timeout(DeviceStatus *st, int site) {
     }
 }
 
-// Bounded wait; returns false (and records the site) if it ran out.
-__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
-                                          DeviceStatus *st, int site) {
+// Bounded wait with an explicit limit; returns false (and records the
+// site) if it ran out.
+__device__ __forceinline__ bool mbar_wait_limit(uint64_t *bar,
+                                                uint32_t parity,
+                                                DeviceStatus *st, int site,
+                                                unsigned long long limit_ns) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     while (!mbar_try_wait(bar, parity)) {
-        if (global_ns() - t0 > kWaitLimitNs) {
+        if (global_ns() - t0 > limit_ns) {
             record_timeout(st, site);
             return false;
         }
     }
     return true;
+}
+
+// Bounded wait (kWaitLimitNs); returns false (and records the site) if it
+// ran out.
+__device__ __forceinline__ bool mbar_wait(uint64_t *bar, uint32_t parity,
+                                          DeviceStatus *st, int site) {
+    return mbar_wait_limit(bar, parity, st, site, kWaitLimitNs);
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t *bar) {

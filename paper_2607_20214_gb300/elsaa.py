@@ -29,7 +29,8 @@ SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_last_error", "elsaa_abi_version", "elsaa_profile_start",
            "elsaa_profile_stop", "elsaa_forward_noalloc",
            "elsaa_backward_workspace_size", "elsaa_backward",
-           "elsaa_gates_workspace_size", "elsaa_gates")
+           "elsaa_gates_workspace_size", "elsaa_gates",
+           "elsaa_selftest_wait_timeout")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -120,6 +121,9 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
                               ctypes.POINTER(elsaa_gate_mlp)] + [vp] * 4 + [
         ctypes.c_size_t, vp]
     L.elsaa_gates.restype = ctypes.c_int
+    L.elsaa_selftest_wait_timeout.argtypes = [vp, ctypes.c_size_t,
+                                              ctypes.c_int, vp]
+    L.elsaa_selftest_wait_timeout.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -355,6 +359,19 @@ def elsaa_gates(params: elsaa_params, mlp: dict, q, gates=None,
         workspace.numel() * workspace.element_size(), sp)
     _check(rc)
     return gates, lambda_tok
+
+
+def elsaa_selftest_wait_timeout(workspace: torch.Tensor, limit_ms=100,
+                                stream=None):
+    """Enqueue the bounded-wait self-test: one wait that nothing satisfies
+    runs out after limit_ms and records a timeout in the status word."""
+    lib = load_library()
+    if stream is None:
+        stream = torch.cuda.current_stream(workspace.device)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    _check(lib.elsaa_selftest_wait_timeout(
+        workspace.data_ptr(), workspace.numel() * workspace.element_size(),
+        int(limit_ms), sp))
 
 
 def elsaa_check_status(workspace: torch.Tensor, stream=None):

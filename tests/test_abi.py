@@ -189,3 +189,15 @@ def test_gates_validation_before_launch(lib):
                            None, fake, 1 << 30, None) == \
         elsaa.ELSAA_ERR_INVALID_ARG
     assert "16-byte" in elsaa.elsaa_last_error()
+
+
+def test_selftest_arguments_checked_before_launch(lib):
+    fake = 1 << 20  # never dereferenced: validation fails first
+    assert lib.elsaa_selftest_wait_timeout(None, 256, 100, None) == \
+        elsaa.ELSAA_ERR_WORKSPACE
+    assert lib.elsaa_selftest_wait_timeout(fake + 16, 256, 100, None) == \
+        elsaa.ELSAA_ERR_WORKSPACE
+    for bad in (0, 5000):
+        assert lib.elsaa_selftest_wait_timeout(fake, 256, bad, None) == \
+            elsaa.ELSAA_ERR_INVALID_ARG
+        assert "limit_ms" in elsaa.elsaa_last_error()
