@@ -444,7 +444,8 @@ struct BwdPlan {
     Plan P;    // forward geometry with CUDA-core RACE chunking
     Plan Pf;   // the forward's own plan (tensor-core key summaries if bf16)
     size_t off_status, off_part, off_A, off_B, off_gA, off_gB, off_gnum,
-        off_gden, off_W, total;
+        off_gden, off_W, off_Bh, total;
+    bool tc;   // tensor-core block kernel (bf16 operands)
 };
 
 int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
@@ -486,6 +487,13 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     off = align_up(off + BHN * sizeof(float), 256);
     Bp->off_W = off;
     off = align_up(off + (size_t)P.H * P.Lg_pad * P.d * sizeof(uint16_t), 256);
+    // the tensor-core block kernel reads B as bf16
+    Bp->tc = p->impl == ELSAA_IMPL_AUTO && Bp->Pf.impl == 2 &&
+             bwd_tc_supported(Bp->Pf);
+    Bp->off_Bh = off;
+    if (Bp->tc)
+        off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(uint16_t),
+                       256);
     Bp->total = off;
     return ELSAA_OK;
 }
@@ -575,18 +583,31 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                            }),
                            "race_partial_simt");
     }
+    uint16_t *Bhw = Bp.tc ? (uint16_t *)(ws + Bp.off_Bh) : nullptr;
     ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
-                           return launch_race_reduce(Pf, part, A, Bm, nullptr,
+                           return launch_race_reduce(Pf, part, A, Bm, Bhw,
                                                      st);
                        }),
                        "race_reduce");
-    ELSAA_CHECK_LAUNCH(timed("bwd_block", st, [&] {
-                           return launch_bwd_block(
-                               P, q, k, v, d_o, w_race, A, Bm, perm_q, perm_k,
-                               lambda_tok, gates, dq, dk, dv, d_gates,
-                               d_lambda, gnum, gden, st);
-                       }),
-                       "bwd_block");
+    if (Bp.tc) {
+        ELSAA_CHECK_LAUNCH(timed("bwd_block_tc", st, [&] {
+                               return launch_bwd_block_tc(
+                                   Pf, q, k, v, d_o,
+                                   (const uint16_t *)(ws + Bp.off_W), Bhw, A,
+                                   perm_q, perm_k, lambda_tok, gates, dq, dk,
+                                   dv, d_gates, d_lambda, gnum, gden, status,
+                                   st);
+                           }),
+                           "bwd_block_tc");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("bwd_block", st, [&] {
+                               return launch_bwd_block(
+                                   P, q, k, v, d_o, w_race, A, Bm, perm_q,
+                                   perm_k, lambda_tok, gates, dq, dk, dv,
+                                   d_gates, d_lambda, gnum, gden, st);
+                           }),
+                           "bwd_block");
+    }
     ELSAA_CHECK_LAUNCH(timed("bwd_race_sums", st, [&] {
                            return launch_race_partial_weighted(
                                P, q, gnum, gden, w_race, part, st);

@@ -1,0 +1,561 @@
+// Tensor-core backward of the sparse branch and of the RACE query side
+// (bf16 inputs, b = 64, d_h = 64, gamma = 4, L_s in {4, 8}): the derivative
+// of Algorithm "sortLSH Sparse Exact Attention Branch" (block step), of the
+// RACE readout (Algorithm "RACE Low-Rank Attention Branch", steps 9-10) and
+// of the fusion, Eq. (5)-(6), the same quantities as k_bwd_block.
+//
+// One persistent CTA per SM walks 128-query tiles (two sorted blocks of 64)
+// ordered by head. Per tile, with operands in shared memory (bf16, 128-byte
+// swizzled panels; transposes are MN-major views of the same bytes) and
+// accumulators in tensor memory:
+//   MMA  [Z | U]  = Q [K ; W]^T          scores and RACE projections
+//   CUDA E = exp(scale Z - M) on each query's own block (the other block's
+//        keys are zero), l, features phi(Q) and Den
+//   MMA  Y = E V,  Num = phi B
+//   CUDA per-query scalars (Eq. (5)-(6) backward), X = gN_s e^M = c_x G,
+//        gNum = G g_lr / (Den + eps)
+//   MMA  dV = E^T X,  P = X V^T,  Gphi = gNum B^T
+//   CUDA dZ = scale E (P + e^M dL/dd_s), dL/dphi = (Gphi + A dL/dDen) / L,
+//        back through the corner softmax and tanh -> dL/d(W q)
+//   MMA  dQ = dZ K + dL/d(W q) W,  dK = dZ^T Q
+// Every key belongs to exactly one block, so dV, dK (sparse part) are
+// plain stores; the RACE key side adds to them afterwards.
+// Operands in bf16 (relative rounding 2^-9), accumulation in fp32.
+#include "device_common.cuh"
+#include "tc_common.cuh"
+#include "tc_race.cuh"
+
+namespace elsaa {
+
+namespace {
+
+using namespace tc;
+
+constexpr int kBtThreads = 256;
+constexpr int kBtT = 128;  // queries (and keys) of a tile: two blocks of 64
+constexpr int kBtD = 64;   // d_h
+// TMEM columns (512 allocated)
+constexpr uint32_t kCS = 0;      // scores [0, 128), projections [128, 160)
+constexpr uint32_t kCO = 160;    // E V, then dQ
+constexpr uint32_t kCN = 224;    // phi B, then dK
+constexpr uint32_t kCdV = 288;   // E^T X
+constexpr uint32_t kCG = 352;    // gNum B^T (r <= 128 columns)
+
+__device__ __forceinline__ void unpack_bf16x8(const uint4 &u, float *x) {
+    const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        x[2 * i] = __uint_as_float(w[i] << 16);
+        x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+
+__device__ __forceinline__ float lse2f(float a, float b) {
+    const float mx = fmaxf(a, b);
+    if (mx == -INFINITY) return -INFINITY;
+    return mx + __logf(__expf(a - mx) + __expf(b - mx));
+}
+
+template <int L>
+__global__ void __launch_bounds__(kBtThreads, 1)
+    k_bwd_block_tc(const uint16_t *__restrict__ qx,
+                   const uint16_t *__restrict__ kx,
+                   const uint16_t *__restrict__ vx,
+                   const uint16_t *__restrict__ gx,
+                   const uint16_t *__restrict__ w_bf16,
+                   const uint16_t *__restrict__ Bh,
+                   const float *__restrict__ Ag,
+                   const int32_t *__restrict__ perm_q,
+                   const int32_t *__restrict__ perm_k,
+                   const float *__restrict__ lambda_tok,
+                   const float *__restrict__ gates, int N, int H,
+                   float beta, float eps, float scale, float lambda, int mode,
+                   int tiles_per_head, long total_tiles,
+                   float *__restrict__ dq, float *__restrict__ dk,
+                   float *__restrict__ dv, float *__restrict__ d_gates,
+                   float *__restrict__ d_lambda, float *__restrict__ gnum,
+                   float *__restrict__ gden, DeviceStatus *status) {
+    constexpr int R = 16, G = 4;
+    constexpr int r = L * R, Lg = L * G;
+    constexpr int Lg_pad = (Lg + 15) / 16 * 16;
+    constexpr int NR = kBtT + Lg_pad;  // key rows + plane rows
+    constexpr int TL = L / 2;          // tables per row half
+    constexpr int d = kBtD;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tbase;
+    __shared__ int abort_flag;
+    __shared__ float xa[2][kBtT], xb[2][kBtT], xc[2][kBtT];
+    __shared__ int qrow_s[kBtT], krow_s[kBtT];
+    volatile int *abort = &abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
+    const int half = warp >> 2;
+    const int row = (warp & 3) * 32 + lane_id;  // TMEM lane
+    const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t sQ = base;                       // [128 x 64]
+    const uint32_t sG = sQ + 16384;                 // dO rows
+    const uint32_t sKW = sG + 16384;                // [NR x 64]: K, then W
+    const uint32_t sV = sKW + align1k(NR * 128);    // [128 x 64]
+    const uint32_t sE = sV + 16384;                 // [128 x 128]: E, dZ
+    const uint32_t sPhi = sE + 32768;               // [128 x r]
+    const uint32_t sB = sPhi + align1k(kBtT * r * 2);  // [r x 64]
+    const uint32_t sX = sB + align1k(r * 128);      // [128 x 64]
+    const uint32_t sGN = sX + 16384;                // [128 x 64]
+    const uint32_t sDU = sGN + 16384;               // [128 x 64] (Lg_pad used)
+    const uint32_t sAo = sDU + 16384;               // fp32 [r]
+    const float *Asm =
+        reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
+
+    const long t_begin = total_tiles * blockIdx.x / gridDim.x;
+    const long t_end = total_tiles * (blockIdx.x + 1) / gridDim.x;
+
+    if (warp == 0) tmem_alloc(&tbase, 512);
+    if (tid == 0) {
+        mbar_init(&mma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = tbase;
+    uint32_t mph = 0;  // MMA barrier phases completed
+    // thread 0 issues, everyone waits for the commit
+    auto mma_done = [&](int site) -> bool {
+        if (tid == 0) mma_commit(&mma_bar);
+        const bool ok = mbar_wait_or_abort(&mma_bar, mph & 1, abort, status,
+                                           site);
+        ++mph;
+        tc_fence_after();
+        return __syncthreads_and(ok);
+    };
+    // 16-byte chunk (8 bf16) at (row, chunk) of a panel region of `rows`
+    auto st8 = [&](uint32_t region, int rr, int chunk, int rows,
+                   const float *v) {
+        st_shared_bf16x8(region + panel_offset(rr, chunk, rows), v);
+    };
+    auto ld8 = [&](uint32_t region, int rr, int chunk, int rows, float *v) {
+        unpack_bf16x8(ld_shared_v4(region + panel_offset(rr, chunk, rows)),
+                      v);
+    };
+
+    int cur_bh = -1;
+    bool ok = true;
+    for (long tt = t_begin; tt < t_end && ok; ++tt) {
+        const int bh = (int)(tt / tiles_per_head);
+        const int p0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
+        const int h = bh % H;
+        const size_t hb = (size_t)bh * N;
+        // ---------------------------------------------------- phase 0: load
+        if (tid < kBtT) {
+            int qi = perm_q[hb + p0 + tid], ki = perm_k[hb + p0 + tid];
+            qi = (qi < 0 || qi >= N) ? 0 : qi;
+            ki = (ki < 0 || ki >= N) ? 0 : ki;
+            qrow_s[tid] = (int)(hb + qi);
+            krow_s[tid] = (int)(hb + ki);
+        }
+        __syncthreads();
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            const size_t qo = (size_t)qrow_s[rr] * d + c * 8;
+            const size_t ko = (size_t)krow_s[rr] * d + c * 8;
+            cp_async16(sQ + panel_offset(rr, c, kBtT), qx + qo);
+            cp_async16(sG + panel_offset(rr, c, kBtT), gx + qo);
+            cp_async16(sKW + panel_offset(rr, c, NR), kx + ko);
+            cp_async16(sV + panel_offset(rr, c, kBtT), vx + ko);
+        }
+        if (bh != cur_bh) {  // the head's planes, B summary (bf16) and A
+            for (int i = tid; i < Lg_pad * 8; i += kBtThreads) {
+                const int rr = i >> 3, c = i & 7;
+                cp_async16(sKW + panel_offset(kBtT + rr, c, NR),
+                           w_bf16 + ((size_t)h * Lg_pad + rr) * d + c * 8);
+            }
+            for (int i = tid; i < r * 8; i += kBtThreads) {
+                const int rr = i >> 3, c = i & 7;
+                cp_async16(sB + panel_offset(rr, c, r),
+                           Bh + ((size_t)bh * r + rr) * d + c * 8);
+            }
+            for (int i = tid; i < r / 4; i += kBtThreads)
+                cp_async16(sAo + 16 * i, Ag + (size_t)bh * r + 4 * i);
+            cur_bh = bh;
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        __syncthreads();
+
+        // ------------------------------------- phase 1: scores, projections
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, NR, false, false);
+#pragma unroll
+            for (int k = 0; k < d / 16; ++k)
+                mma_ss(tm + kCS, smem_desc(sQ + k * 32, 16, 1024),
+                       smem_desc(sKW + k * 32, 16, 1024), id, k > 0);
+        }
+        if (!(ok = mma_done(80))) break;
+
+        // ---------------------- phase 2: E on the query's own block, phi, Den
+        const int blk = row >> 6;
+        const int c0 = 64 * blk + 32 * half;  // this thread's 32 key columns
+        float e[32];
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCS + c0, v);
+            tmem_wait_ld();
+            float mx = -INFINITY;
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                e[j] = __uint_as_float(v[j]) * scale;
+                mx = fmaxf(mx, e[j]);
+            }
+            xa[half][row] = mx;
+        }
+        __syncthreads();
+        const float M = fmaxf(xa[0][row], xa[1][row]);
+        float lp = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            e[j] = __expf(e[j] - M);
+            lp += e[j];
+        }
+        xb[half][row] = lp;
+        // E rows (bf16), zeros on the other block's keys
+#pragma unroll
+        for (int q = 0; q < 4; ++q) st8(sE, row, (c0 >> 3) + q, kBtT, e + 8 * q);
+        {
+            const float z[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+            const int cz = 64 * (1 - blk) + 32 * half;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) st8(sE, row, (cz >> 3) + q, kBtT, z);
+        }
+        // RACE features of this half's tables
+        float u[2 * L > 16 ? 16 : 2 * L];  // projections of TL tables
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCS + kBtT, v);  // all Lg_pad projections
+            tmem_wait_ld();
+#pragma unroll
+            for (int b = 0; b < TL * G; ++b)
+                u[b] = __uint_as_float(v[half * TL * G + b]);
+        }
+        float denp = 0.0f;
+#pragma unroll
+        for (int t = 0; t < TL; ++t) {
+            float sp[G], sn[G], phi[R];
+#pragma unroll
+            for (int b = 0; b < G; ++b)
+                race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
+#pragma unroll
+            for (int rr = 0; rr < R; ++rr) {
+                float p = 1.0f;
+#pragma unroll
+                for (int b = 0; b < G; ++b) p *= ((rr >> b) & 1) ? sp[b] : sn[b];
+                phi[rr] = p;
+            }
+            const int tg = half * TL + t;
+#pragma unroll
+            for (int rr = 0; rr < R; ++rr)
+                denp = fmaf(phi[rr], Asm[tg * R + rr], denp);
+            st8(sPhi, row, tg * 2, kBtT, phi);
+            st8(sPhi, row, tg * 2 + 1, kBtT, phi + 8);
+        }
+        xc[half][row] = denp;
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        const float lsum = xb[0][row] + xb[1][row];
+        const float Den = (xc[0][row] + xc[1][row]) * (1.0f / (float)L);
+
+        // ------------------------------------------- phase 3: E V and phi B
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, d, false, true);
+#pragma unroll
+            for (int k = 0; k < kBtT / 16; ++k)
+                mma_ss(tm + kCO,
+                       smem_desc(sE + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                 1024),
+                       smem_desc(sV + k * 2048, 16384, 1024), id, k > 0);
+#pragma unroll
+            for (int k = 0; k < r / 16; ++k)
+                mma_ss(tm + kCN,
+                       smem_desc(sPhi + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                 1024),
+                       smem_desc(sB + k * 2048, (uint32_t)r * 128, 1024), id,
+                       k > 0);
+        }
+        if (!(ok = mma_done(81))) break;
+
+        // ------------------------------------- phase 4: per-query scalars
+        const int qrow = qrow_s[row];
+        float gv[32], Y[32], Nm[32];
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCO + 32 * half, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) Y[j] = __uint_as_float(v[j]);
+            tmem_ld32(tm + lane + kCN + 32 * half, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) Nm[j] = __uint_as_float(v[j]);
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) ld8(sG, row, 4 * half + q, kBtT, gv + 8 * q);
+        float go = 0.0f, gn = 0.0f;
+#pragma unroll
+        for (int j = 0; j < 32; ++j) {
+            go = fmaf(gv[j], Y[j], go);
+            gn = fmaf(gv[j], Nm[j], gn);
+        }
+        // the two halves' partial dot products (xa is free again: M was
+        // read before the last barrier)
+        xa[half][row] = go;
+        xc[half][row] = gn;
+        __syncthreads();
+        const float lsE = lsum + eps * __expf(-M);  // (d_s + eps) e^-M
+        const float GOs = (xa[0][row] + xa[1][row]) / lsE;
+        // G . O_lr with O_lr = (phi B / L) / (Den + eps)
+        const float GOlr = (xc[0][row] + xc[1][row]) /
+                           ((float)L * (Den + eps));
+        const size_t tok = (size_t)qrow;
+        const float lam = lambda_tok ? lambda_tok[tok] : lambda;
+        const float gs = gates ? gates[2 * tok] : 1.0f;
+        const float gl = gates ? gates[2 * tok + 1] : 1.0f;
+        const float logds = M + __logf(lsum);
+        const float cc = lam * Den + eps;
+        const float logD = lse2f(logds, __logf(cc));
+        const float m = mode == 1 ? 1.0f : __expf(logds - logD);
+        const float invD = __expf(-logD);
+        const float dm = mode == 1 ? 0.0f : gs * GOs;
+        const float cx = gs * m / lsE;
+        const float gdsE = -(gs * m * GOs) / lsE + dm * (cc * invD) * (m / lsum);
+        const float cn = gl / (Den + eps);
+        const float gDen = -(gl * GOlr) / (Den + eps) - dm * lam * m * invD;
+        if (half == 0) {
+            if (d_gates) {
+                d_gates[2 * tok] = m * GOs;
+                d_gates[2 * tok + 1] = GOlr;
+            }
+            if (d_lambda) d_lambda[tok] = -dm * m * Den * invD;
+            gden[tok] = gDen * (1.0f / (float)L);
+        }
+        {
+            float xv[32], nv[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j) {
+                xv[j] = cx * gv[j];
+                nv[j] = cn * gv[j];
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                st8(sX, row, 4 * half + q, kBtT, xv + 8 * q);
+                st8(sGN, row, 4 * half + q, kBtT, nv + 8 * q);
+            }
+            float4 *go4 = reinterpret_cast<float4 *>(gnum + tok * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                go4[q] = make_float4(nv[4 * q] / L, nv[4 * q + 1] / L,
+                                     nv[4 * q + 2] / L, nv[4 * q + 3] / L);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+
+        // --------------------------- phase 5: E^T X, X V^T, gNum B^T
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id_v = idesc_bf16(128, d, true, true);
+#pragma unroll
+            for (int k = 0; k < kBtT / 16; ++k)  // dV = E^T X (K = queries)
+                mma_ss(tm + kCdV, smem_desc(sE + k * 2048, 16384, 1024),
+                       smem_desc(sX + k * 2048, 16384, 1024), id_v, k > 0);
+            const uint32_t id_p = idesc_bf16(128, kBtT, false, false);
+#pragma unroll
+            for (int k = 0; k < d / 16; ++k)  // P = X V^T (K = d)
+                mma_ss(tm + kCS, smem_desc(sX + k * 32, 16, 1024),
+                       smem_desc(sV + k * 32, 16, 1024), id_p, k > 0);
+            const uint32_t id_g = idesc_bf16(128, r, false, false);
+#pragma unroll
+            for (int k = 0; k < d / 16; ++k)  // Gphi = gNum B^T (K = d)
+                mma_ss(tm + kCG, smem_desc(sGN + k * 32, 16, 1024),
+                       smem_desc(sB + k * 32, 16, 1024), id_g, k > 0);
+        }
+        if (!(ok = mma_done(82))) break;
+
+        // ------------- phase 6: dZ, back through the features, dV stores
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCS + c0, v);
+            tmem_wait_ld();
+            float dz[32];
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                dz[j] = scale * e[j] * (__uint_as_float(v[j]) + gdsE);
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+                st8(sE, row, (c0 >> 3) + q, kBtT, dz + 8 * q);
+        }
+        {
+            float du[2 * L > 16 ? 16 : 2 * L];
+#pragma unroll
+            for (int t = 0; t < TL; ++t) {
+                const int tg = half * TL + t;
+                uint32_t v[16];
+                tmem_ld16(tm + lane + kCG + tg * R, v);
+                tmem_wait_ld();
+                float sp[G], sn[G], uu[G], phi[R], gp[R];
+#pragma unroll
+                for (int b = 0; b < G; ++b) {
+                    race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
+                    uu[b] = tanhf(u[t * G + b]);
+                }
+                float s = 0.0f;
+#pragma unroll
+                for (int rr = 0; rr < R; ++rr) {
+                    float p = 1.0f;
+#pragma unroll
+                    for (int b = 0; b < G; ++b)
+                        p *= ((rr >> b) & 1) ? sp[b] : sn[b];
+                    phi[rr] = p;
+                    gp[rr] = (__uint_as_float(v[rr]) + Asm[tg * R + rr] * gDen) *
+                             (1.0f / (float)L);
+                    s = fmaf(p, gp[rr], s);
+                }
+#pragma unroll
+                for (int b = 0; b < G; ++b) {
+                    float g = 0.0f;
+#pragma unroll
+                    for (int rr = 0; rr < R; ++rr) {
+                        const float ga = phi[rr] * (gp[rr] - s);
+                        g += ((rr >> b) & 1) ? ga : -ga;
+                    }
+                    du[t * G + b] = (1.0f - uu[b] * uu[b]) * beta * g;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < TL * G / 8; ++q)
+                st8(sDU, row, (half * TL * G) / 8 + q, kBtT, du + 8 * q);
+        }
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCdV + 32 * half, v);
+            tmem_wait_ld();
+            float4 *o4 =
+                reinterpret_cast<float4 *>(dv + (size_t)krow_s[row] * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                o4[q] = make_float4(__uint_as_float(v[4 * q]),
+                                    __uint_as_float(v[4 * q + 1]),
+                                    __uint_as_float(v[4 * q + 2]),
+                                    __uint_as_float(v[4 * q + 3]));
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+
+        // -------------------------- phase 7: dQ = dZ K + dU W, dK = dZ^T Q
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id_q = idesc_bf16(128, d, false, true);
+#pragma unroll
+            for (int k = 0; k < kBtT / 16; ++k)  // K = keys
+                mma_ss(tm + kCO,
+                       smem_desc(sE + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                 1024),
+                       smem_desc(sKW + k * 2048, (uint32_t)NR * 128, 1024),
+                       id_q, k > 0);
+#pragma unroll
+            for (int k = 0; k < Lg_pad / 16; ++k)  // K = projections
+                mma_ss(tm + kCO, smem_desc(sDU + k * 32, 16, 1024),
+                       smem_desc(sKW + kBtT * 128 + k * 2048,
+                                 (uint32_t)NR * 128, 1024),
+                       id_q, 1);
+            const uint32_t id_k = idesc_bf16(128, d, true, true);
+#pragma unroll
+            for (int k = 0; k < kBtT / 16; ++k)  // K = queries
+                mma_ss(tm + kCN, smem_desc(sE + k * 2048, 16384, 1024),
+                       smem_desc(sQ + k * 2048, 16384, 1024), id_k, k > 0);
+        }
+        if (!(ok = mma_done(83))) break;
+
+        // ------------------------------------------- phase 8: dQ, dK stores
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCO + 32 * half, v);
+            tmem_wait_ld();
+            float4 *q4 = reinterpret_cast<float4 *>(dq + (size_t)qrow * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                q4[q] = make_float4(__uint_as_float(v[4 * q]),
+                                    __uint_as_float(v[4 * q + 1]),
+                                    __uint_as_float(v[4 * q + 2]),
+                                    __uint_as_float(v[4 * q + 3]));
+            tmem_ld32(tm + lane + kCN + 32 * half, v);
+            tmem_wait_ld();
+            float4 *k4 = reinterpret_cast<float4 *>(dk + (size_t)krow_s[row] * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                k4[q] = make_float4(__uint_as_float(v[4 * q]),
+                                    __uint_as_float(v[4 * q + 1]),
+                                    __uint_as_float(v[4 * q + 2]),
+                                    __uint_as_float(v[4 * q + 3]));
+        }
+        tc_fence_before();
+        __syncthreads();  // TMEM and shared memory are reused by the next tile
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+}  // namespace
+
+bool bwd_tc_supported(const Plan &P) {
+    return P.dtype == ELSAA_BF16 && P.d == kBtD && P.b == 64 &&
+           P.gamma == 4 && (P.L == 4 || P.L == 8) && P.N % kBtT == 0 &&
+           P.nb == 0 && (long)P.BH * P.N < (1l << 31);
+}
+
+size_t bwd_tc_smem(const Plan &P) {
+    const size_t r = (size_t)P.L * 16;
+    const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
+    auto a1k = [](size_t x) { return (x + 1023) / 1024 * 1024; };
+    return 1024 + 16384 * 2 + a1k((kBtT + lg_pad) * 128) + 16384 + 32768 +
+           a1k(kBtT * r * 2) + a1k(r * 128) + 16384 * 3 + r * 4;
+}
+
+cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
+                                const void *v, const void *d_o,
+                                const uint16_t *w_bf16, const uint16_t *Bh,
+                                const float *A, const int32_t *perm_q,
+                                const int32_t *perm_k, const float *lambda_tok,
+                                const float *gates, float *dq, float *dk,
+                                float *dv, float *d_gates, float *d_lambda,
+                                float *gnum, float *gden, DeviceStatus *status,
+                                cudaStream_t st) {
+    const int tiles_per_head = P.N / kBtT;
+    const long total = (long)tiles_per_head * P.BH;
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess)
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = (int)(total < sms ? total : sms);
+    const size_t smem = bwd_tc_smem(P);
+    auto launch = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<grid, kBtThreads, smem, st>>>(
+            (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
+            (const uint16_t *)d_o, w_bf16, Bh, A, perm_q, perm_k, lambda_tok,
+            gates, P.N, P.H, P.beta, P.eps, P.scale, P.lambda, P.fusion_mode,
+            tiles_per_head, total, dq, dk, dv, d_gates, d_lambda, gnum, gden,
+            status);
+        return cudaGetLastError();
+    };
+    return P.L == 8 ? launch(k_bwd_block_tc<8>) : launch(k_bwd_block_tc<4>);
+}
+
+}  // namespace elsaa

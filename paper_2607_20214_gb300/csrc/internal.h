@@ -114,6 +114,19 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
                             const float *gB, float *dk, float *dv,
                             cudaStream_t st);
 
+// Tensor-core backward block kernel (bwd_tc.cu).
+bool bwd_tc_supported(const Plan &P);
+size_t bwd_tc_smem(const Plan &P);
+cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
+                                const void *v, const void *d_o,
+                                const uint16_t *w_bf16, const uint16_t *Bh,
+                                const float *A, const int32_t *perm_q,
+                                const int32_t *perm_k, const float *lambda_tok,
+                                const float *gates, float *dq, float *dk,
+                                float *dv, float *d_gates, float *d_lambda,
+                                float *gnum, float *gden, DeviceStatus *status,
+                                cudaStream_t st);
+
 // One bounded mbarrier wait that can never complete (selftest.cu).
 cudaError_t launch_selftest_wait(DeviceStatus *status, int limit_ms,
                                  cudaStream_t st);
