@@ -444,7 +444,7 @@ struct BwdPlan {
     Plan P;    // forward geometry with CUDA-core RACE chunking
     Plan Pf;   // the forward's own plan (tensor-core key summaries if bf16)
     size_t off_status, off_part, off_A, off_B, off_gA, off_gB, off_gnum,
-        off_gden, off_W, off_Bh, total;
+        off_gden, off_W, off_Bh, off_gBh, total;
     bool tc;   // tensor-core block kernel (bf16 operands)
 };
 
@@ -491,6 +491,10 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     Bp->tc = p->impl == ELSAA_IMPL_AUTO && Bp->Pf.impl == 2 &&
              bwd_tc_supported(Bp->Pf);
     Bp->off_Bh = off;
+    if (Bp->tc)
+        off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(uint16_t),
+                       256);
+    Bp->off_gBh = off;
     if (Bp->tc)
         off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(uint16_t),
                        256);
@@ -613,16 +617,27 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                                P, q, gnum, gden, w_race, part, st);
                        }),
                        "bwd_race_sums");
+    uint16_t *gBhw = Bp.tc ? (uint16_t *)(ws + Bp.off_gBh) : nullptr;
     ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
-                           return launch_race_reduce(P, part, gA, gB, nullptr,
+                           return launch_race_reduce(P, part, gA, gB, gBhw,
                                                      st);
                        }),
                        "race_reduce");
-    ELSAA_CHECK_LAUNCH(timed("bwd_keys", st, [&] {
-                           return launch_bwd_keys(P, k, v, w_race, gA, gB, dk,
-                                                  dv, st);
-                       }),
-                       "bwd_keys");
+    if (Bp.tc) {
+        ELSAA_CHECK_LAUNCH(timed("bwd_keys_tc", st, [&] {
+                               return launch_bwd_keys_tc(
+                                   Pf, k, v,
+                                   (const uint16_t *)(ws + Bp.off_W), gBhw, gA,
+                                   dk, dv, status, st);
+                           }),
+                           "bwd_keys_tc");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("bwd_keys", st, [&] {
+                               return launch_bwd_keys(P, k, v, w_race, gA, gB,
+                                                      dk, dv, st);
+                           }),
+                           "bwd_keys");
+    }
     return ELSAA_OK;
 }
 

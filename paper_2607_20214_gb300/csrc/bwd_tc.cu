@@ -512,6 +512,275 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     if (warp == 0) tmem_dealloc(tm, 512);
 }
 
+// RACE key side of the backward on tensor cores, per 128-key tile (keys in
+// their original order): with gB = sum_i phi(Q_i) gNum_i^T / L and
+// gA = sum_i phi(Q_i) dL/dDen_i / L (bf16 / fp32, per head),
+//   MMA  U = K W^T                         projections
+//   CUDA phi(K)
+//   MMA  dV_k = phi gB,  Gphi = V gB^T
+//   CUDA dV += dV_k; dL/dphi = Gphi + gA, back through the corner softmax
+//        and tanh -> dL/d(W k)
+//   MMA  dK_k = dL/d(W k) W
+//   CUDA dK += dK_k
+// Each key belongs to one tile: plain read-modify-write of dV and dK (the
+// sparse parts were stored by the block kernel before).
+constexpr uint32_t kKU = 0;     // projections [0, 32)
+constexpr uint32_t kKdV = 32;   // phi gB
+constexpr uint32_t kKG = 96;    // V gB^T (r <= 128)
+constexpr uint32_t kKdK = 224;  // dL/du W
+
+template <int L>
+__global__ void __launch_bounds__(kBtThreads, 1)
+    k_bwd_keys_tc(const uint16_t *__restrict__ kx,
+                  const uint16_t *__restrict__ vx,
+                  const uint16_t *__restrict__ w_bf16,
+                  const uint16_t *__restrict__ gBh,
+                  const float *__restrict__ gAg, int N, int H, float beta,
+                  int tiles_per_head, long total_tiles,
+                  float *__restrict__ dk, float *__restrict__ dv,
+                  DeviceStatus *status) {
+    constexpr int R = 16, G = 4;
+    constexpr int r = L * R, Lg = L * G;
+    constexpr int Lg_pad = (Lg + 15) / 16 * 16;
+    constexpr int NR = kBtT + Lg_pad;
+    constexpr int TL = L / 2;
+    constexpr int d = kBtD;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tbase;
+    __shared__ int abort_flag;
+    volatile int *abort = &abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
+    const int half = warp >> 2;
+    const int row = (warp & 3) * 32 + lane_id;  // key of the tile = lane
+    const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t sKW = base;                        // [NR x 64]: K, W
+    const uint32_t sV = sKW + align1k(NR * 128);      // [128 x 64]
+    const uint32_t sPhi = sV + 16384;                 // [128 x r]
+    const uint32_t sgB = sPhi + align1k(kBtT * r * 2);  // [r x 64]
+    const uint32_t sDU = sgB + align1k(r * 128);      // [128 x 64]
+    const uint32_t sAo = sDU + 16384;                 // fp32 gA [r]
+    const float *gAs =
+        reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
+
+    const long t_begin = total_tiles * blockIdx.x / gridDim.x;
+    const long t_end = total_tiles * (blockIdx.x + 1) / gridDim.x;
+    if (warp == 0) tmem_alloc(&tbase, 512);
+    if (tid == 0) {
+        mbar_init(&mma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = tbase;
+    uint32_t mph = 0;
+    auto mma_done = [&](int site) -> bool {
+        if (tid == 0) mma_commit(&mma_bar);
+        const bool ok = mbar_wait_or_abort(&mma_bar, mph & 1, abort, status,
+                                           site);
+        ++mph;
+        tc_fence_after();
+        return __syncthreads_and(ok);
+    };
+    auto st8 = [&](uint32_t region, int rr, int chunk, int rows,
+                   const float *v) {
+        st_shared_bf16x8(region + panel_offset(rr, chunk, rows), v);
+    };
+
+    int cur_bh = -1;
+    bool ok = true;
+    for (long tt = t_begin; tt < t_end && ok; ++tt) {
+        const int bh = (int)(tt / tiles_per_head);
+        const int k0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
+        const int h = bh % H;
+        const size_t row0 = (size_t)bh * N + k0;
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            const size_t o = (row0 + rr) * d + c * 8;
+            cp_async16(sKW + panel_offset(rr, c, NR), kx + o);
+            cp_async16(sV + panel_offset(rr, c, kBtT), vx + o);
+        }
+        if (bh != cur_bh) {  // the head's planes, gB (bf16) and gA
+            for (int i = tid; i < Lg_pad * 8; i += kBtThreads) {
+                const int rr = i >> 3, c = i & 7;
+                cp_async16(sKW + panel_offset(kBtT + rr, c, NR),
+                           w_bf16 + ((size_t)h * Lg_pad + rr) * d + c * 8);
+            }
+            for (int i = tid; i < r * 8; i += kBtThreads) {
+                const int rr = i >> 3, c = i & 7;
+                cp_async16(sgB + panel_offset(rr, c, r),
+                           gBh + ((size_t)bh * r + rr) * d + c * 8);
+            }
+            for (int i = tid; i < r / 4; i += kBtThreads)
+                cp_async16(sAo + 16 * i, gAg + (size_t)bh * r + 4 * i);
+            cur_bh = bh;
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        __syncthreads();
+
+        // projections U = K W^T
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, Lg_pad, false, false);
+#pragma unroll
+            for (int k = 0; k < d / 16; ++k)
+                mma_ss(tm + kKU, smem_desc(sKW + k * 32, 16, 1024),
+                       smem_desc(sKW + kBtT * 128 + k * 32, 16, 1024), id,
+                       k > 0);
+        }
+        if (!(ok = mma_done(90))) break;
+
+        // features of this half's tables
+        float u[2 * L > 16 ? 16 : 2 * L];
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kKU, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int b = 0; b < TL * G; ++b)
+                u[b] = __uint_as_float(v[half * TL * G + b]);
+        }
+#pragma unroll
+        for (int t = 0; t < TL; ++t) {
+            float sp[G], sn[G], phi[R];
+#pragma unroll
+            for (int b = 0; b < G; ++b)
+                race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
+#pragma unroll
+            for (int rr = 0; rr < R; ++rr) {
+                float p = 1.0f;
+#pragma unroll
+                for (int b = 0; b < G; ++b) p *= ((rr >> b) & 1) ? sp[b] : sn[b];
+                phi[rr] = p;
+            }
+            const int tg = half * TL + t;
+            st8(sPhi, row, tg * 2, kBtT, phi);
+            st8(sPhi, row, tg * 2 + 1, kBtT, phi + 8);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+
+        // dV_k = phi gB, Gphi = V gB^T
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id_v = idesc_bf16(128, d, false, true);
+#pragma unroll
+            for (int k = 0; k < r / 16; ++k)
+                mma_ss(tm + kKdV,
+                       smem_desc(sPhi + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                 1024),
+                       smem_desc(sgB + k * 2048, (uint32_t)r * 128, 1024),
+                       id_v, k > 0);
+            const uint32_t id_g = idesc_bf16(128, r, false, false);
+#pragma unroll
+            for (int k = 0; k < d / 16; ++k)
+                mma_ss(tm + kKG, smem_desc(sV + k * 32, 16, 1024),
+                       smem_desc(sgB + k * 32, 16, 1024), id_g, k > 0);
+        }
+        if (!(ok = mma_done(91))) break;
+
+        const size_t key = row0 + row;
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kKdV + 32 * half, v);
+            tmem_wait_ld();
+            float4 *o4 = reinterpret_cast<float4 *>(dv + key * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float4 a = o4[q];
+                a.x += __uint_as_float(v[4 * q]);
+                a.y += __uint_as_float(v[4 * q + 1]);
+                a.z += __uint_as_float(v[4 * q + 2]);
+                a.w += __uint_as_float(v[4 * q + 3]);
+                o4[q] = a;
+            }
+        }
+        {
+            float du[2 * L > 16 ? 16 : 2 * L];
+#pragma unroll
+            for (int t = 0; t < TL; ++t) {
+                const int tg = half * TL + t;
+                uint32_t v[16];
+                tmem_ld16(tm + lane + kKG + tg * R, v);
+                tmem_wait_ld();
+                float sp[G], sn[G], uu[G], phi[R], gp[R];
+#pragma unroll
+                for (int b = 0; b < G; ++b) {
+                    race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
+                    uu[b] = tanhf(u[t * G + b]);
+                }
+                float s = 0.0f;
+#pragma unroll
+                for (int rr = 0; rr < R; ++rr) {
+                    float p = 1.0f;
+#pragma unroll
+                    for (int b = 0; b < G; ++b)
+                        p *= ((rr >> b) & 1) ? sp[b] : sn[b];
+                    phi[rr] = p;
+                    gp[rr] = __uint_as_float(v[rr]) + gAs[tg * R + rr];
+                    s = fmaf(p, gp[rr], s);
+                }
+#pragma unroll
+                for (int b = 0; b < G; ++b) {
+                    float g = 0.0f;
+#pragma unroll
+                    for (int rr = 0; rr < R; ++rr) {
+                        const float ga = phi[rr] * (gp[rr] - s);
+                        g += ((rr >> b) & 1) ? ga : -ga;
+                    }
+                    du[t * G + b] = (1.0f - uu[b] * uu[b]) * beta * g;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < TL * G / 8; ++q)
+                st8(sDU, row, (half * TL * G) / 8 + q, kBtT, du + 8 * q);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+
+        // dK_k = dL/du W
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id_q = idesc_bf16(128, d, false, true);
+#pragma unroll
+            for (int k = 0; k < Lg_pad / 16; ++k)
+                mma_ss(tm + kKdK, smem_desc(sDU + k * 32, 16, 1024),
+                       smem_desc(sKW + kBtT * 128 + k * 2048,
+                                 (uint32_t)NR * 128, 1024),
+                       id_q, k > 0);
+        }
+        if (!(ok = mma_done(92))) break;
+        {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kKdK + 32 * half, v);
+            tmem_wait_ld();
+            float4 *o4 = reinterpret_cast<float4 *>(dk + key * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q) {
+                float4 a = o4[q];
+                a.x += __uint_as_float(v[4 * q]);
+                a.y += __uint_as_float(v[4 * q + 1]);
+                a.z += __uint_as_float(v[4 * q + 2]);
+                a.w += __uint_as_float(v[4 * q + 3]);
+                o4[q] = a;
+            }
+        }
+        tc_fence_before();
+        __syncthreads();
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tm, 512);
+}
+
 }  // namespace
 
 bool bwd_tc_supported(const Plan &P) {
@@ -556,6 +825,40 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
         return cudaGetLastError();
     };
     return P.L == 8 ? launch(k_bwd_block_tc<8>) : launch(k_bwd_block_tc<4>);
+}
+
+}  // namespace elsaa
+
+namespace elsaa {
+
+size_t bwd_keys_tc_smem(const Plan &P) {
+    const size_t r = (size_t)P.L * 16;
+    const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
+    auto a1k = [](size_t x) { return (x + 1023) / 1024 * 1024; };
+    return 1024 + a1k((kBtT + lg_pad) * 128) + 16384 + a1k(kBtT * r * 2) +
+           a1k(r * 128) + 16384 + r * 4;
+}
+
+cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
+                               const uint16_t *w_bf16, const uint16_t *gBh,
+                               const float *gA, float *dk, float *dv,
+                               DeviceStatus *status, cudaStream_t st) {
+    const int tiles_per_head = P.N / kBtT;
+    const long total = (long)tiles_per_head * P.BH;
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess)
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int grid = (int)(total < sms ? total : sms);
+    const size_t smem = bwd_keys_tc_smem(P);
+    auto launch = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<grid, kBtThreads, smem, st>>>(
+            (const uint16_t *)k, (const uint16_t *)v, w_bf16, gBh, gA, P.N,
+            P.H, P.beta, tiles_per_head, total, dk, dv, status);
+        return cudaGetLastError();
+    };
+    return P.L == 8 ? launch(k_bwd_keys_tc<8>) : launch(k_bwd_keys_tc<4>);
 }
 
 }  // namespace elsaa

@@ -127,6 +127,12 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 float *gnum, float *gden, DeviceStatus *status,
                                 cudaStream_t st);
 
+size_t bwd_keys_tc_smem(const Plan &P);
+cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
+                               const uint16_t *w_bf16, const uint16_t *gBh,
+                               const float *gA, float *dk, float *dv,
+                               DeviceStatus *status, cudaStream_t st);
+
 // One bounded mbarrier wait that can never complete (selftest.cu).
 cudaError_t launch_selftest_wait(DeviceStatus *status, int limit_ms,
                                  cudaStream_t st);
