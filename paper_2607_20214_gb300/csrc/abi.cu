@@ -439,7 +439,9 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
 namespace {
 
 // Backward workspace: status | RACE chunk partials (A, B, then gA, gB) |
-// A | B | gA | gB | gNum / L [B*H][N][d_h] | gDen / L [B*H][N].
+// A | B | gA | gB | gNum / L [B*H][N][d_h] | gDen / L [B*H][N] | bf16
+// planes | bf16 B | bf16 gB. The tensor-core path sums gA, gB inside the
+// block kernel: it has no gNum / gDen arrays.
 struct BwdPlan {
     Plan P;    // forward geometry with CUDA-core RACE chunking
     Plan Pf;   // the forward's own plan (tensor-core key summaries if bf16)
@@ -460,7 +462,11 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     rc = make_plan(p, &Bp->Pf, msg);  // A, B as the forward makes them
     if (rc != ELSAA_OK) return rc;
     const Plan &P = Bp->P;
-    const int S = P.S > Bp->Pf.S ? P.S : Bp->Pf.S;
+    // the tensor-core kernels read B and write gB as bf16
+    Bp->tc = p->impl == ELSAA_IMPL_AUTO && Bp->Pf.impl == 2 &&
+             bwd_tc_supported(Bp->Pf);
+    int S = P.S > Bp->Pf.S ? P.S : Bp->Pf.S;
+    if (Bp->tc && bwd_tc_segments(Bp->Pf) > S) S = bwd_tc_segments(Bp->Pf);
     if (!bwd_supported(P)) {
         *msg = "backward: this block size, d_h and r need more shared "
                "memory than an SM has";
@@ -482,14 +488,11 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     Bp->off_gB = off;
     off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(float), 256);
     Bp->off_gnum = off;
-    off = align_up(off + BHN * P.d * sizeof(float), 256);
+    if (!Bp->tc) off = align_up(off + BHN * P.d * sizeof(float), 256);
     Bp->off_gden = off;
-    off = align_up(off + BHN * sizeof(float), 256);
+    if (!Bp->tc) off = align_up(off + BHN * sizeof(float), 256);
     Bp->off_W = off;
     off = align_up(off + (size_t)P.H * P.Lg_pad * P.d * sizeof(uint16_t), 256);
-    // the tensor-core block kernel reads B as bf16
-    Bp->tc = p->impl == ELSAA_IMPL_AUTO && Bp->Pf.impl == 2 &&
-             bwd_tc_supported(Bp->Pf);
     Bp->off_Bh = off;
     if (Bp->tc)
         off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(uint16_t),
@@ -599,8 +602,7 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                                    Pf, q, k, v, d_o,
                                    (const uint16_t *)(ws + Bp.off_W), Bhw, A,
                                    perm_q, perm_k, lambda_tok, gates, dq, dk,
-                                   dv, d_gates, d_lambda, gnum, gden, status,
-                                   st);
+                                   dv, d_gates, d_lambda, part, status, st);
                            }),
                            "bwd_block_tc");
     } else {
@@ -612,17 +614,25 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                            }),
                            "bwd_block");
     }
-    ELSAA_CHECK_LAUNCH(timed("bwd_race_sums", st, [&] {
-                           return launch_race_partial_weighted(
-                               P, q, gnum, gden, w_race, part, st);
-                       }),
-                       "bwd_race_sums");
     uint16_t *gBhw = Bp.tc ? (uint16_t *)(ws + Bp.off_gBh) : nullptr;
-    ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
-                           return launch_race_reduce(P, part, gA, gB, gBhw,
-                                                     st);
-                       }),
-                       "race_reduce");
+    if (Bp.tc) {
+        ELSAA_CHECK_LAUNCH(timed("bwd_sums_reduce", st, [&] {
+                               return launch_bwd_sums_reduce(Pf, part, gBhw,
+                                                             gA, st);
+                           }),
+                           "bwd_sums_reduce");
+    } else {
+        ELSAA_CHECK_LAUNCH(timed("bwd_race_sums", st, [&] {
+                               return launch_race_partial_weighted(
+                                   P, q, gnum, gden, w_race, part, st);
+                           }),
+                           "bwd_race_sums");
+        ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
+                               return launch_race_reduce(P, part, gA, gB,
+                                                         nullptr, st);
+                           }),
+                           "race_reduce");
+    }
     if (Bp.tc) {
         ELSAA_CHECK_LAUNCH(timed("bwd_keys_tc", st, [&] {
                                return launch_bwd_keys_tc(

@@ -14,12 +14,17 @@
 //   MMA  Y = E V,  Num = phi B
 //   CUDA per-query scalars (Eq. (5)-(6) backward), X = gN_s e^M = c_x G,
 //        gNum = G g_lr / (Den + eps)
-//   MMA  dV = E^T X,  P = X V^T,  Gphi = gNum B^T
+//   MMA  dV = E^T X,  P = X V^T,  Gphi = gNum B^T,
+//        [gB | gA] += phi^T [gNum | dL/dDen]  (summed over the CTA's tiles
+//        of one head in tensor memory)
 //   CUDA dZ = scale E (P + e^M dL/dd_s), dL/dphi = (Gphi + A dL/dDen) / L,
 //        back through the corner softmax and tanh -> dL/d(W q)
 //   MMA  dQ = dZ K + dL/d(W q) W,  dK = dZ^T Q
 // Every key belongs to exactly one block, so dV, dK (sparse part) are
-// plain stores; the RACE key side adds to them afterwards.
+// plain stores; the RACE key side adds to them afterwards. The per-head
+// sums gB, gA that the key side needs leave the kernel as one partial per
+// (head, CTA that worked on the head), summed in a fixed order by
+// k_bwd_sums_reduce.
 // Operands in bf16 (relative rounding 2^-9), accumulation in fp32.
 #include "device_common.cuh"
 #include "tc_common.cuh"
@@ -34,12 +39,23 @@ using namespace tc;
 constexpr int kBtThreads = 256;
 constexpr int kBtT = 128;  // queries (and keys) of a tile: two blocks of 64
 constexpr int kBtD = 64;   // d_h
+// persistent CTAs of the block kernel: one per SM of a GB300 (fixed, so the
+// workspace size does not depend on the device the plan is made on)
+constexpr int kBtGrid = 152;
 // TMEM columns (512 allocated)
 constexpr uint32_t kCS = 0;      // scores [0, 128), projections [128, 160)
 constexpr uint32_t kCO = 160;    // E V, then dQ
 constexpr uint32_t kCN = 224;    // phi B, then dK
+constexpr uint32_t kCG = 160;    // gNum B^T (r <= 128 columns) between them
 constexpr uint32_t kCdV = 288;   // E^T X
-constexpr uint32_t kCG = 352;    // gNum B^T (r <= 128 columns)
+constexpr uint32_t kCAcc = 352;  // [gB | gA] of the current head, d + 16
+
+// The CTA (of `grid` over `total` tiles, CTA c taking tiles
+// [total c / grid, total (c + 1) / grid)) that works on tile t.
+__host__ __device__ __forceinline__ long tile_owner(long t, long total,
+                                                    long grid) {
+    return ((t + 1) * grid + total - 1) / total - 1;
+}
 
 __device__ __forceinline__ void unpack_bf16x8(const uint4 &u, float *x) {
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
@@ -73,8 +89,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                    int tiles_per_head, long total_tiles,
                    float *__restrict__ dq, float *__restrict__ dk,
                    float *__restrict__ dv, float *__restrict__ d_gates,
-                   float *__restrict__ d_lambda, float *__restrict__ gnum,
-                   float *__restrict__ gden, DeviceStatus *status) {
+                   float *__restrict__ d_lambda, float *__restrict__ part,
+                   int S_seg, DeviceStatus *status) {
     constexpr int R = 16, G = 4;
     constexpr int r = L * R, Lg = L * G;
     constexpr int Lg_pad = (Lg + 15) / 16 * 16;
@@ -341,7 +357,12 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 d_gates[2 * tok + 1] = GOlr;
             }
             if (d_lambda) d_lambda[tok] = -dm * m * Den * invD;
-            gden[tok] = gDen * (1.0f / (float)L);
+        }
+        {  // dL/dDen repeated over the 16 columns after gNum
+            float gd[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) gd[j] = gDen;
+            st8(sDU, row, half, kBtT, gd);
         }
         {
             float xv[32], nv[32];
@@ -355,17 +376,15 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 st8(sX, row, 4 * half + q, kBtT, xv + 8 * q);
                 st8(sGN, row, 4 * half + q, kBtT, nv + 8 * q);
             }
-            float4 *go4 = reinterpret_cast<float4 *>(gnum + tok * d + 32 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                go4[q] = make_float4(nv[4 * q] / L, nv[4 * q + 1] / L,
-                                     nv[4 * q + 2] / L, nv[4 * q + 3] / L);
         }
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
 
-        // --------------------------- phase 5: E^T X, X V^T, gNum B^T
+        // ------------- phase 5: E^T X, X V^T, gNum B^T, phi^T [gNum | gDen]
+        const bool seg_first = tt == t_begin || (tt % tiles_per_head) == 0;
+        const bool seg_last =
+            tt + 1 == t_end || ((tt + 1) % tiles_per_head) == 0;
         if (tid == 0) {
             tc_fence_after();
             const uint32_t id_v = idesc_bf16(128, d, true, true);
@@ -383,8 +402,40 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             for (int k = 0; k < d / 16; ++k)  // Gphi = gNum B^T (K = d)
                 mma_ss(tm + kCG, smem_desc(sGN + k * 32, 16, 1024),
                        smem_desc(sB + k * 32, 16, 1024), id_g, k > 0);
+            // bucket sums (K = queries; M = 128 buckets, rows past r unused;
+            // the B operand is gNum followed by the dL/dDen panel)
+            const uint32_t id_s = idesc_bf16(128, d + 16, true, true);
+#pragma unroll
+            for (int k = 0; k < kBtT / 16; ++k)
+                mma_ss(tm + kCAcc, smem_desc(sPhi + k * 2048, 16384, 1024),
+                       smem_desc(sGN + k * 2048, 16384, 1024), id_s,
+                       (k > 0 || !seg_first) ? 1u : 0u);
         }
         if (!(ok = mma_done(82))) break;
+        if (seg_last && row < r) {  // this CTA's share of the head's sums
+            const long j = (long)blockIdx.x -
+                           tile_owner((long)bh * tiles_per_head, total_tiles,
+                                      gridDim.x);
+            float *out =
+                part + ((size_t)bh * S_seg + j) * ((size_t)r * d + r);
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCAcc + 32 * half, v);
+            tmem_wait_ld();
+            float4 *o4 =
+                reinterpret_cast<float4 *>(out + (size_t)row * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                o4[q] = make_float4(__uint_as_float(v[4 * q]),
+                                    __uint_as_float(v[4 * q + 1]),
+                                    __uint_as_float(v[4 * q + 2]),
+                                    __uint_as_float(v[4 * q + 3]));
+            if (half == 0) {
+                uint32_t a16[16];
+                tmem_ld16(tm + lane + kCAcc + d, a16);
+                tmem_wait_ld();
+                out[(size_t)r * d + row] = __uint_as_float(a16[0]);
+            }
+        }
 
         // ------------- phase 6: dZ, back through the features, dV stores
         {
@@ -510,6 +561,35 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+// gB, gA of each head: the partials of the CTAs that worked on the head,
+// summed in CTA order, times 1 / L; gB leaves as bf16 (the key side's MMA
+// operand), gA as fp32. Grid (ceil((r d + r) / 256), B*H).
+__global__ void k_bwd_sums_reduce(const float *__restrict__ part, int S_seg,
+                                  int r, int d, int L, int tiles_per_head,
+                                  long total, int grid,
+                                  uint16_t *__restrict__ gBh,
+                                  float *__restrict__ gA) {
+    const int bh = blockIdx.y;
+    const size_t per = (size_t)r * d + r;
+    const long c0 = tile_owner((long)bh * tiles_per_head, total, grid);
+    const long c1 =
+        tile_owner((long)(bh + 1) * tiles_per_head - 1, total, grid);
+    const float inv = 1.0f / (float)L;
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < per;
+         i += (size_t)gridDim.x * blockDim.x) {
+        const float *p = part + (size_t)bh * S_seg * per + i;
+        float s = 0.f;
+        for (long c = 0; c <= c1 - c0; ++c) s += p[(size_t)c * per];
+        s *= inv;
+        if (i < (size_t)r * d) {
+            const __nv_bfloat16 hb = __float2bfloat16_rn(s);
+            gBh[(size_t)bh * r * d + i] = *reinterpret_cast<const uint16_t *>(&hb);
+        } else {
+            gA[(size_t)bh * r + (i - (size_t)r * d)] = s;
+        }
+    }
 }
 
 // RACE key side of the backward on tensor cores, per 128-key tile (keys in
@@ -797,6 +877,24 @@ size_t bwd_tc_smem(const Plan &P) {
            a1k(kBtT * r * 2) + a1k(r * 128) + 16384 * 3 + r * 4;
 }
 
+int bwd_tc_grid(const Plan &P) {
+    const long total = (long)(P.N / kBtT) * P.BH;
+    return (int)(total < kBtGrid ? total : kBtGrid);
+}
+
+int bwd_tc_segments(const Plan &P) {
+    const int T = P.N / kBtT;
+    const long total = (long)T * P.BH;
+    const long grid = bwd_tc_grid(P);
+    long most = 1;
+    for (long bh = 0; bh < P.BH; ++bh) {
+        const long n = tile_owner((bh + 1) * T - 1, total, grid) -
+                       tile_owner(bh * T, total, grid) + 1;
+        if (n > most) most = n;
+    }
+    return (int)most;
+}
+
 cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 const void *v, const void *d_o,
                                 const uint16_t *w_bf16, const uint16_t *Bh,
@@ -804,14 +902,12 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 const int32_t *perm_k, const float *lambda_tok,
                                 const float *gates, float *dq, float *dk,
                                 float *dv, float *d_gates, float *d_lambda,
-                                float *gnum, float *gden, DeviceStatus *status,
+                                float *part, DeviceStatus *status,
                                 cudaStream_t st) {
     const int tiles_per_head = P.N / kBtT;
     const long total = (long)tiles_per_head * P.BH;
-    int dev = 0, sms = 148;
-    if (cudaGetDevice(&dev) == cudaSuccess)
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int grid = (int)(total < sms ? total : sms);
+    const int grid = bwd_tc_grid(P);
+    const int S_seg = bwd_tc_segments(P);
     const size_t smem = bwd_tc_smem(P);
     auto launch = [&](auto kern) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -820,11 +916,23 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
             (const uint16_t *)d_o, w_bf16, Bh, A, perm_q, perm_k, lambda_tok,
             gates, P.N, P.H, P.beta, P.eps, P.scale, P.lambda, P.fusion_mode,
-            tiles_per_head, total, dq, dk, dv, d_gates, d_lambda, gnum, gden,
+            tiles_per_head, total, dq, dk, dv, d_gates, d_lambda, part, S_seg,
             status);
         return cudaGetLastError();
     };
     return P.L == 8 ? launch(k_bwd_block_tc<8>) : launch(k_bwd_block_tc<4>);
+}
+
+cudaError_t launch_bwd_sums_reduce(const Plan &P, const float *part,
+                                   uint16_t *gBh, float *gA, cudaStream_t st) {
+    const int tiles_per_head = P.N / kBtT;
+    const long total = (long)tiles_per_head * P.BH;
+    const int per = P.r * P.d + P.r;
+    dim3 grid((per + 255) / 256, P.BH);
+    k_bwd_sums_reduce<<<grid, 256, 0, st>>>(part, bwd_tc_segments(P), P.r,
+                                            P.d, P.L, tiles_per_head, total,
+                                            bwd_tc_grid(P), gBh, gA);
+    return cudaGetLastError();
 }
 
 }  // namespace elsaa

@@ -114,9 +114,15 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
                             const float *gB, float *dk, float *dv,
                             cudaStream_t st);
 
-// Tensor-core backward block kernel (bwd_tc.cu).
+// Tensor-core backward (bwd_tc.cu): the block kernel also sums gB, gA per
+// head into bwd_tc_segments(P) partials per head (layout of the RACE chunk
+// partials), which launch_bwd_sums_reduce folds into bf16 gB and fp32 gA.
 bool bwd_tc_supported(const Plan &P);
 size_t bwd_tc_smem(const Plan &P);
+int bwd_tc_grid(const Plan &P);
+int bwd_tc_segments(const Plan &P);
+cudaError_t launch_bwd_sums_reduce(const Plan &P, const float *part,
+                                   uint16_t *gBh, float *gA, cudaStream_t st);
 cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 const void *v, const void *d_o,
                                 const uint16_t *w_bf16, const uint16_t *Bh,
@@ -124,7 +130,7 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 const int32_t *perm_k, const float *lambda_tok,
                                 const float *gates, float *dq, float *dk,
                                 float *dv, float *d_gates, float *d_lambda,
-                                float *gnum, float *gden, DeviceStatus *status,
+                                float *part, DeviceStatus *status,
                                 cudaStream_t st);
 
 size_t bwd_keys_tc_smem(const Plan &P);

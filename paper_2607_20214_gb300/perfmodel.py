@@ -75,13 +75,22 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
     elif kernel.startswith("bwd_block"):
         # recompute scores and O_s, dZ, dV, dK, dQ (12 N b d) and the query
         # side of RACE (4 N r d + 4 N d Lg); reads Q, K, V, dO, writes dQ,
-        # dK, dV and gNum in fp32
-        by = H * (4 * N * d * e + 4 * N * d * 4)
-        fl = H * (12 * N * b * d + 4 * N * r * d + 4 * N * d * Lg)
-        simt = True
+        # dK, dV in fp32. The CUDA-core kernel also writes gNum (fp32) for
+        # a separate pass; the tensor-core kernel sums gB, gA itself
+        # (2 N r (d + 1)) on the tensor cores.
+        tc = kernel.endswith("_tc")
+        by = H * (4 * N * d * e + (3 if tc else 4) * N * d * 4)
+        fl = H * (12 * N * b * d + 4 * N * r * d + 4 * N * d * Lg +
+                  (2 * N * r * (d + 1) if tc else 0))
+        simt = not tc
     elif kernel.startswith("bwd_keys"):
+        # reads K, V, adds into dK, dV (fp32 read + write)
         by = H * (2 * N * d * e + 4 * N * d * 4)
         fl = H * (4 * N * r * d + 4 * N * d * Lg)
+        simt = not kernel.endswith("_tc")
+    elif kernel.startswith("bwd_sums_reduce"):
+        by = H * r * (d + 1) * 4
+        fl = 0
         simt = True
     elif kernel.startswith("bwd_race_sums"):
         by = H * (N * d * e + N * d * 4)
