@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define ELSAA_ABI_VERSION 2
+#define ELSAA_ABI_VERSION 3
 
 /* Return codes. */
 #define ELSAA_OK 0
@@ -66,8 +66,17 @@ extern "C" {
 typedef struct elsaa_params {
     int B, H, N, d_h;   /* Q, K, V are [B, H, N, d_h] (Section 3)            */
     int dtype;          /* ELSAA_BF16 or ELSAA_FP32                           */
-    int causal;         /* must be 0: the causal variant (Algorithm "Causal
-                           ELSAA") is not built; 1 -> ELSAA_ERR_UNSUPPORTED   */
+    int causal;         /* 0: Algorithm 1 (non-causal); 1: Algorithm "Causal
+                           ELSAA": the recursive causal sortLSH branch
+                           (CausalSparse with SortLSH blocks and MergeLSE)
+                           and the chunked causal RACE branch, fused with the
+                           log-domain multiplier. Built for bf16, impl AUTO,
+                           d_h 64 or 128, race_bits 4 with race_tables 4, 8
+                           or 16, block_size 32/64/128/256, neighbor_blocks
+                           0, and N = n_leaf 2^k where the recursion stops at
+                           segments of n_leaf <= causal_base_len rows, a
+                           multiple of 128 and of block_size (no odd-length
+                           padding); ELSAA_ERR_UNSUPPORTED otherwise.        */
     int block_size;     /* b, keys per query (sortLSH block size; Table 7 "s").
                            Requires N % b == 0 and b % 32 == 0, b <= 1024.    */
     int sort_bits;      /* sortLSH hash bits n_s in [0, 8] (Table 7: 4-5);
@@ -94,6 +103,13 @@ typedef struct elsaa_params {
                            the tensor cores; other r > 0 shapes run the
                            sparse branch on CUDA cores (fp32).
                            elsaa_backward requires r = 0                  */
+    int causal_chunk;   /* C >= 1, chunk length of causal RACE (Algorithm
+                           "Causal RACE"). The result does not depend on C
+                           (the prefix-state form is exact); the device
+                           uses 128-token chunks. Ignored when causal = 0  */
+    int causal_base_len;/* N_0 >= 1, segment length at which CausalSparse
+                           switches to exact causal attention (Table 7,
+                           "Sort_LSH min length"). Ignored when causal = 0 */
 } elsaa_params;
 
 /*
@@ -134,6 +150,11 @@ int elsaa_workspace_size(const elsaa_params *params, size_t *bytes);
  * workspace    device scratch of at least elsaa_workspace_size() bytes,
  *              256-byte aligned. Its contents need no initialisation.
  * stream       cudaStream_t (as void*) on which all work is enqueued.
+ *
+ * With params->causal = 1 the same call runs Algorithm "Causal ELSAA":
+ * o, log_d_sparse (log of the merged CausalSparse denominator), d_lr (the
+ * causal Den) and m_sparse keep their meanings; perm_q and perm_k are not
+ * written (each level of the recursion sorts its own halves).
  *
  * Errors: ELSAA_ERR_INVALID_ARG / _UNSUPPORTED / _WORKSPACE before any
  * launch; ELSAA_ERR_CUDA if a launch fails (the message names the kernel).

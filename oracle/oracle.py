@@ -295,6 +295,8 @@ def params_from_workload(wl, **over) -> dict:
     p["race_tables"] = wl.race_tables
     p["race_bits"] = wl.race_bits
     p["neighbors"] = getattr(wl, "neighbor_blocks", 0)
+    p["causal_chunk"] = getattr(wl, "causal_chunk", 128)
+    p["causal_base_len"] = getattr(wl, "causal_base_len", 4096)
     p.update(over)
     return p
 

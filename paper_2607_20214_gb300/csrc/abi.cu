@@ -113,9 +113,6 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
         return bad(ELSAA_ERR_INVALID_ARG, "dtype must be ELSAA_BF16 or ELSAA_FP32");
     if (p->causal != 0 && p->causal != 1)
         return bad(ELSAA_ERR_INVALID_ARG, "causal must be 0 or 1");
-    if (p->causal)
-        return bad(ELSAA_ERR_UNSUPPORTED,
-                   "the causal variant is not built (causal must be 0)");
     if (p->block_size <= 0)
         return bad(ELSAA_ERR_INVALID_ARG, "block_size must be positive");
     if (p->N % p->block_size != 0)
@@ -286,6 +283,191 @@ int set_last_error(int code, const char *fmt, ...) {
 
 using namespace elsaa;
 
+#define ELSAA_CHECK_LAUNCH(expr, name)                                       \
+    do {                                                                     \
+        cudaError_t e_ = (expr);                                             \
+        if (e_ != cudaSuccess)                                               \
+            return fail(ELSAA_ERR_CUDA, "%s: %s", name,                      \
+                        cudaGetErrorString(e_));                             \
+    } while (0)
+
+namespace {
+
+// Causal forward (Algorithm "Causal ELSAA"). Workspace: status | codes
+// (sort hash, [2][B*H][N]) | tile histograms of the hash | per level and
+// side the sorted halves [Lv][2][B*H][N / 2] | running sparse result O
+// [B*H][N][d_h] fp32 and log d [B*H][N] | RACE chunk summaries
+// [B*H][N / 128][r d_h + r] | prefix states sB (bf16) and sA | bf16 planes.
+struct CausalPlan {
+    Plan P;   // geometry and the forward's hash / RACE settings
+    Plan Pc;  // P with RACE chunks of 128 keys
+    int Lv, n_leaf;
+    size_t off_status, off_keyrank, off_hist, off_perms, off_RO, off_RL,
+        off_part, off_sB, off_sA, off_W, total;
+};
+
+int make_causal_plan(const elsaa_params *p, CausalPlan *C, const char **msg) {
+    if (p->causal_chunk < 1 || p->causal_base_len < 1) {
+        *msg = "causal_chunk and causal_base_len must be >= 1";
+        return ELSAA_ERR_INVALID_ARG;
+    }
+    int rc = make_plan(p, &C->P, msg);
+    if (rc != ELSAA_OK) return rc;
+    const Plan &P = C->P;
+    if (P.nb != 0) {
+        *msg = "the causal variant requires neighbor_blocks = 0";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
+    // unrolled recursion: halve until a segment fits the base length
+    int n = P.N, Lv = 0;
+    while (n > p->causal_base_len) {
+        if (n % 2) {
+            *msg = "causal: this N and causal_base_len make the recursion pad "
+                   "an odd-length segment (built: N = n_leaf 2^k with "
+                   "n_leaf <= causal_base_len)";
+            return ELSAA_ERR_UNSUPPORTED;
+        }
+        n /= 2;
+        ++Lv;
+    }
+    C->Lv = Lv;
+    C->n_leaf = n;
+    if (!causal_tc_supported(P, n)) {
+        *msg = "causal: built for bf16 with impl AUTO, d_h of 64 or 128, "
+               "race_bits 4 with race_tables 4, 8 or 16, block_size 32, 64, "
+               "128 or 256 dividing the base segments, base segments a "
+               "multiple of 128 rows";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
+    C->Pc = P;
+    C->Pc.S = P.N / 128;
+    C->Pc.chunk = 128;
+    const size_t BHN = (size_t)P.BH * P.N;
+    const size_t nc = (size_t)P.N / 128;
+    size_t off = 0;
+    C->off_status = off;
+    off = align_up(off + sizeof(DeviceStatus), 256);
+    C->off_keyrank = off;
+    off = align_up(off + 2 * BHN * sizeof(uint32_t), 256);
+    C->off_hist = off;
+    off = align_up(off + (size_t)2 * P.BH * P.tiles * P.bins * sizeof(int),
+                   256);
+    C->off_perms = off;
+    off = align_up(off + (size_t)Lv * BHN * sizeof(int32_t), 256);
+    C->off_RO = off;
+    off = align_up(off + BHN * P.d * sizeof(float), 256);
+    C->off_RL = off;
+    off = align_up(off + BHN * sizeof(float), 256);
+    C->off_part = off;
+    off = align_up(off + (size_t)P.BH * nc * ((size_t)P.r * P.d + P.r) *
+                             sizeof(float), 256);
+    C->off_sB = off;
+    off = align_up(off + (size_t)P.BH * nc * P.r * P.d * sizeof(uint16_t),
+                   256);
+    C->off_sA = off;
+    off = align_up(off + (size_t)P.BH * nc * P.r * sizeof(float), 256);
+    C->off_W = off;
+    off = align_up(off + (size_t)P.H * P.Lg_pad * P.d * sizeof(uint16_t), 256);
+    C->total = off;
+    return ELSAA_OK;
+}
+
+int causal_forward(const elsaa_params *params, const void *q, const void *k,
+                   const void *v, const float *w_sort, const float *w_race,
+                   const float *lambda_tok, const float *gates, void *o,
+                   float *log_d_sparse, float *d_lr, float *m_sparse,
+                   void *workspace, size_t workspace_bytes, void *stream) {
+    CausalPlan C;
+    const char *msg = "";
+    int rc = make_causal_plan(params, &C, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    const Plan &P = C.P;
+    if (!q || !k || !v || !o)
+        return fail(ELSAA_ERR_INVALID_ARG, "q, k, v and o must be non-NULL");
+    if (!w_race) return fail(ELSAA_ERR_INVALID_ARG, "w_race must be non-NULL");
+    if (P.n_s > 0 && !w_sort)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "w_sort must be non-NULL when sort_bits > 0");
+    const void *ptrs[] = {q, k, v, o, w_race};
+    for (const void *p : ptrs)
+        if ((uintptr_t)p % 16)
+            return fail(ELSAA_ERR_INVALID_ARG,
+                        "q, k, v, o and w_race must be 16-byte aligned");
+    if (gates && (uintptr_t)gates % 8)
+        return fail(ELSAA_ERR_INVALID_ARG, "gates must be 8-byte aligned");
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if ((uintptr_t)workspace % 256)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if (workspace_bytes < C.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, C.total);
+    cudaStream_t st = (cudaStream_t)stream;
+    char *ws = (char *)workspace;
+    DeviceStatus *status = (DeviceStatus *)(ws + C.off_status);
+    uint32_t *keyrank = (uint32_t *)(ws + C.off_keyrank);
+    int *hist = (int *)(ws + C.off_hist);
+    int32_t *perms = (int32_t *)(ws + C.off_perms);
+    float *RO = (float *)(ws + C.off_RO);
+    float *RL = (float *)(ws + C.off_RL);
+    float *part = (float *)(ws + C.off_part);
+    uint16_t *sB = (uint16_t *)(ws + C.off_sB);
+    float *sA = (float *)(ws + C.off_sA);
+    uint16_t *Wbf = (uint16_t *)(ws + C.off_W);
+
+    ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
+                       "status reset");
+    // sparse branch: codes, sorted halves, base segments, then the levels
+    ELSAA_CHECK_LAUNCH(timed("sort_hash", st, [&] {
+                           return launch_sort_hash(P, q, k, w_sort, keyrank,
+                                                   hist, status, st);
+                       }),
+                       "sort_hash");
+    ELSAA_CHECK_LAUNCH(timed("seg_sort", st, [&] {
+                           return launch_seg_sort(P, C.Lv, keyrank, perms,
+                                                  st);
+                       }),
+                       "seg_sort");
+    ELSAA_CHECK_LAUNCH(timed("causal_attn_base", st, [&] {
+                           return launch_causal_attn(P, 0, C.n_leaf, 0, q, k,
+                                                     v, perms, RO, RL, status,
+                                                     st);
+                       }),
+                       "causal_attn_base");
+    for (int level = C.Lv; level >= 1; --level)
+        ELSAA_CHECK_LAUNCH(timed("causal_attn_merge", st, [&] {
+                               return launch_causal_attn(P, 1, C.n_leaf,
+                                                         level, q, k, v,
+                                                         perms, RO, RL,
+                                                         status, st);
+                           }),
+                           "causal_attn_merge");
+    // low-rank branch: chunk summaries, prefix states, readout + fusion
+    ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
+                           return launch_prep_planes(P, w_race, Wbf, st);
+                       }),
+                       "prep_planes");
+    ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
+                           return launch_race_keys_ws(C.Pc, k, v, Wbf, part,
+                                                      status, st);
+                       }),
+                       "race_keys_ws");
+    ELSAA_CHECK_LAUNCH(timed("causal_prefix", st, [&] {
+                           return launch_causal_prefix(P, part, sB, sA, st);
+                       }),
+                       "causal_prefix");
+    ELSAA_CHECK_LAUNCH(timed("causal_race", st, [&] {
+                           return launch_causal_race(
+                               P, q, k, v, Wbf, sB, sA, RO, RL, lambda_tok,
+                               gates, o, log_d_sparse, d_lr, m_sparse, status,
+                               st);
+                       }),
+                       "causal_race");
+    return ELSAA_OK;
+}
+
+}  // namespace
+
 extern "C" int elsaa_abi_version(void) { return ELSAA_ABI_VERSION; }
 
 extern "C" const char *elsaa_last_error(void) { return g_err; }
@@ -294,6 +476,14 @@ extern "C" int elsaa_workspace_size(const elsaa_params *params,
                                     size_t *bytes) {
     g_err[0] = 0;
     if (!bytes) return fail(ELSAA_ERR_INVALID_ARG, "bytes is NULL");
+    if (params && params->causal == 1) {
+        CausalPlan C;
+        const char *msg = "";
+        int rc = make_causal_plan(params, &C, &msg);
+        if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+        *bytes = C.total;
+        return ELSAA_OK;
+    }
     Plan P;
     const char *msg = "";
     int rc = make_plan(params, &P, &msg);
@@ -302,13 +492,6 @@ extern "C" int elsaa_workspace_size(const elsaa_params *params,
     return ELSAA_OK;
 }
 
-#define ELSAA_CHECK_LAUNCH(expr, name)                                       \
-    do {                                                                     \
-        cudaError_t e_ = (expr);                                             \
-        if (e_ != cudaSuccess)                                               \
-            return fail(ELSAA_ERR_CUDA, "%s: %s", name,                      \
-                        cudaGetErrorString(e_));                             \
-    } while (0)
 
 extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                              const void *k, const void *v,
@@ -319,6 +502,10 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                              int32_t *perm_k, void *workspace,
                              size_t workspace_bytes, void *stream) {
     g_err[0] = 0;
+    if (params && params->causal == 1)
+        return causal_forward(params, q, k, v, w_sort, w_race, lambda_tok,
+                              gates, o, log_d_sparse, d_lr, m_sparse,
+                              workspace, workspace_bytes, stream);
     Plan P;
     const char *msg = "";
     int rc = make_plan(params, &P, &msg);
@@ -451,6 +638,10 @@ struct BwdPlan {
 };
 
 int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
+    if (p && p->causal) {
+        *msg = "elsaa_backward: the causal variant has no backward pass here";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
     elsaa_params q = *p;
     q.impl = ELSAA_IMPL_SIMT;  // the backward runs on CUDA cores
     int rc = make_plan(&q, &Bp->P, msg);

@@ -1,0 +1,787 @@
+// Causal ELSAA (Algorithm "Causal ELSAA"): the recursive causal sortLSH
+// branch (Algorithm "Causal sortLSH Sparse Exact Attention Branch":
+// CausalSparse, SortLSH, MergeLSE) and the chunked causal RACE branch
+// (Algorithm "Causal RACE Low-Rank Attention Branch"), bf16 inputs on the
+// tensor cores.
+//
+// The recursion is unrolled. For N = n_leaf 2^Lv (n_leaf <= N0 < 2 n_leaf)
+// a row's result is its base segment's exact causal attention, then, from
+// the deepest level to the top, MergeLSE with the SortLSH attention of its
+// node's future half against the node's past half wherever the row lies in
+// a future half. So:
+//   k_seg_sort       stable counting sort of each node's future-half query
+//                    codes and past-half key codes (codes from the sort hash)
+//   k_causal_attn_tc base segments (exact causal attention, 128-row tiles
+//                    over 128-key tiles with an online softmax), then one
+//                    launch per level, deepest first, for the SortLSH blocks,
+//                    merged into the running (O, log d) with MergeLSE
+//   race_keys_ws     per-chunk summaries A_n, B_n (chunks of 128 keys)
+//   k_causal_prefix  strict prefix states sA_n, sB_n (cumulative sum shifted
+//                    by one chunk; sB_n leaves as bf16)
+//   k_causal_race_tc per chunk: inter-chunk readout phi_Q sB_n, intra-chunk
+//                    masked products tril(phi_Q phi_K^T) V, then the fusion
+//                    of Eq. (5)-(6) with the sparse result.
+// The causal RACE result does not depend on the chunk size (exact
+// arithmetic); the device uses chunks of 128.
+#include "device_common.cuh"
+#include "tc_common.cuh"
+#include "tc_race.cuh"
+
+namespace elsaa {
+
+namespace {
+
+using namespace tc;
+
+constexpr int kSegThreads = 512;
+constexpr int kSegWarps = kSegThreads / 32;
+constexpr int kCaThreads = 256;
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr size_t kSmemPerSM = 233472;  // 228 KB of shared memory per SM
+
+// -------------------------------------------------------------- seg sort
+
+// One CTA sorts one segment of m codes stably (equal codes keep increasing
+// token order). Segment s of the launch: level l = floor(log2(s + 1)) + 1,
+// node j = s + 1 - 2^(l-1); node size n_l = N / 2^(l-1), half m = n_l / 2.
+// which 0: the future half's queries (codes of Q), 1: the past half's keys.
+// out[l - 1][which][bh][j m + pos] = token index within the head.
+__global__ void __launch_bounds__(kSegThreads)
+    k_seg_sort(const uint32_t *__restrict__ keyrank, int N, int bins,
+               int32_t *__restrict__ perms) {
+    __shared__ int cnt[256];
+    __shared__ int wc[kSegWarps][256];
+    const int s = blockIdx.x, bh = blockIdx.y, which = blockIdx.z;
+    const int BH = gridDim.y;
+    int l = 1;
+    while ((2 << (l - 1)) <= s + 1) ++l;
+    const int j = s + 1 - (1 << (l - 1));
+    const int n_l = N >> (l - 1), m = n_l >> 1;
+    const int base = j * n_l + (which == 0 ? m : 0);
+    const uint32_t *codes = keyrank + ((size_t)which * BH + bh) * N + base;
+    int32_t *out = perms + (((size_t)(l - 1) * 2 + which) * BH + bh) *
+                               (size_t)(N >> 1) +
+                   (size_t)j * m;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < bins; i += kSegThreads) cnt[i] = 0;
+    for (int i = tid; i < kSegWarps * 256; i += kSegThreads)
+        (&wc[0][0])[i] = 0;
+    __syncthreads();
+    for (int i = tid; i < m; i += kSegThreads)
+        atomicAdd(&cnt[codes[i] & 0xffffu], 1);
+    __syncthreads();
+    if (tid == 0) {  // exclusive scan of the histogram
+        int run = 0;
+        for (int b = 0; b < bins; ++b) {
+            const int c = cnt[b];
+            cnt[b] = run;
+            run += c;
+        }
+    }
+    __syncthreads();
+    for (int c0 = 0; c0 < m; c0 += kSegThreads) {
+        const int i = c0 + tid;
+        const bool in = i < m;
+        const int key = in ? (int)(codes[i] & 0xffffu) : -1;
+        const unsigned act = __ballot_sync(0xffffffffu, in);
+        const unsigned peers = __match_any_sync(0xffffffffu, key) & act;
+        const int rank_w = __popc(peers & ((1u << lane) - 1u));
+        if (in && rank_w == 0) wc[warp][key] = __popc(peers);
+        __syncthreads();
+        if (in) {
+            int rank = rank_w;
+            for (int w = 0; w < warp; ++w) rank += wc[w][key];
+            const int pos = cnt[key] + rank;
+            if (pos >= 0 && pos < m) out[pos] = base + i;
+        }
+        __syncthreads();
+        for (int b = tid; b < bins; b += kSegThreads) {
+            int t = 0;
+            for (int w = 0; w < kSegWarps; ++w) {
+                t += wc[w][b];
+                wc[w][b] = 0;
+            }
+            cnt[b] += t;
+        }
+        __syncthreads();
+    }
+}
+
+// ------------------------------------------------------- attention tiles
+
+// One CTA = one tile of 128 query rows and its key tiles, online softmax:
+//   mode 0 (base segments): rows leaf n_leaf + 128 qt + [0, 128), key tiles
+//          kt = 0..qt of the same segment, the last one masked j <= i;
+//          writes (O, log d) of exact causal attention.
+//   mode 1 (SortLSH of one level): rows = sorted future-half queries
+//          128 qt.. of node j, keys = the node's sorted past-half keys of
+//          the same block (b >= 128: b / 128 key tiles; b < 128: one tile,
+//          rows and keys paired by block, r / b == c / b); MergeLSE into
+//          the running (O, log d).
+// Per key tile: MMA S = Q K^T (TMEM [0, 128)); CUDA scale, mask, running
+// max, P = exp(S - max) as bf16 over the consumed K tile; MMA P V (TMEM
+// [128, 128 + D)); CUDA O = O alpha + P V. Two threads per row (TMEM lane
+// = row; each takes half of the key columns and half of the output).
+template <int D>
+__global__ void __launch_bounds__(kCaThreads, 2)
+    k_causal_attn_tc(const uint16_t *__restrict__ qx,
+                     const uint16_t *__restrict__ kx,
+                     const uint16_t *__restrict__ vx,
+                     const int32_t *__restrict__ permq,
+                     const int32_t *__restrict__ permk, int N, int mode,
+                     int n_leaf, int m, int b, float scale, float eps,
+                     float *__restrict__ RO, float *__restrict__ RL,
+                     DeviceStatus *status) {
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tbase;
+    __shared__ int abort_flag;
+    __shared__ float xm[2][128], xl[2][128];
+    __shared__ int qrow_s[128], krow_s[128];
+    volatile int *abort = &abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
+    const int half = warp >> 2;
+    const int row = (warp & 3) * 32 + lane_id;
+    const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
+    constexpr int DH = D / 2;  // output columns per thread
+    constexpr uint32_t kTileB = 128 * D * 2;
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t sQ = base;
+    const uint32_t sKP = sQ + kTileB;                       // K, then P
+    const uint32_t sV = sKP + (kTileB > 32768 ? kTileB : 32768);
+
+    // ---- work item
+    int bh, qt, nkt, kt0;
+    size_t qbase = 0, kbase = 0;  // mode 0: first row of the segment
+    const int32_t *ql = nullptr, *kl = nullptr;
+    if (mode == 0) {
+        const int nq = n_leaf / 128, nleaves = N / n_leaf;
+        const int item = blockIdx.x;
+        qt = nq - 1 - item % nq;  // longest rows first
+        const int rest = item / nq;
+        const int leaf = rest % nleaves;
+        bh = rest / nleaves;
+        qbase = (size_t)bh * N + (size_t)leaf * n_leaf + (size_t)qt * 128;
+        kbase = (size_t)bh * N + (size_t)leaf * n_leaf;
+        kt0 = 0;
+        nkt = qt + 1;
+    } else {
+        const int tpn = m / 128, nodes = N / (2 * m);
+        const int item = blockIdx.x;
+        qt = item % tpn;
+        const int rest = item / tpn;
+        const int j = rest % nodes;
+        bh = rest / nodes;
+        ql = permq + (size_t)bh * (N >> 1) + (size_t)j * m;
+        kl = permk + (size_t)bh * (N >> 1) + (size_t)j * m;
+        if (b >= 128) {
+            kt0 = (qt * 128 / b) * (b / 128);
+            nkt = b / 128;
+        } else {
+            kt0 = qt;
+            nkt = 1;
+        }
+    }
+
+    if (warp == 0) tmem_alloc(&tbase, 256);
+    if (tid == 0) {
+        mbar_init(&mma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    if (tid < 128) {
+        int t;
+        if (mode == 0) {
+            t = (int)(qbase - (size_t)bh * N) + tid;
+        } else {
+            t = ql[qt * 128 + tid];
+            t = (t < 0 || t >= N) ? 0 : t;
+        }
+        qrow_s[tid] = t;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = tbase;
+    uint32_t mph = 0;
+    auto mma_done = [&](int site) -> bool {
+        if (tid == 0) mma_commit(&mma_bar);
+        const bool ok =
+            mbar_wait_or_abort(&mma_bar, mph & 1, abort, status, site);
+        ++mph;
+        tc_fence_after();
+        return __syncthreads_and(ok);
+    };
+    const size_t hN = (size_t)bh * N;
+    // key rows of tile kt into krow_s (tokens within the head)
+    auto key_rows = [&](int kt) {
+        if (tid < 128) {
+            int t;
+            if (mode == 0) {
+                t = (int)(kbase - hN) + kt * 128 + tid;
+            } else {
+                t = kl[kt * 128 + tid];
+                t = (t < 0 || t >= N) ? 0 : t;
+            }
+            krow_s[tid] = t;
+        }
+    };
+    auto load_kv = [&]() {
+        for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+            const int rr = i / (D / 8), c = i % (D / 8);
+            const size_t o = (hN + krow_s[rr]) * D + c * 8;
+            cp_async16(sKP + panel_offset(rr, c, 128), kx + o);
+            cp_async16(sV + panel_offset(rr, c, 128), vx + o);
+        }
+        cp_async_commit();
+    };
+    key_rows(kt0);
+    __syncthreads();
+    for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+        const int rr = i / (D / 8), c = i % (D / 8);
+        cp_async16(sQ + panel_offset(rr, c, 128),
+                   qx + (hN + qrow_s[rr]) * D + c * 8);
+    }
+    load_kv();
+
+    float o_acc[DH];
+#pragma unroll
+    for (int j = 0; j < DH; ++j) o_acc[j] = 0.0f;
+    float mrun = -INFINITY, lrun = 0.0f;  // log2 domain running max, sum
+    const float sl2 = scale * kLog2e;
+    bool ok = true;
+    for (int it = 0; it < nkt && ok; ++it) {
+        const int kt = kt0 + it;
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, 128, false, false);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)
+                mma_ss(tm, smem_desc(sQ + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                     1024),
+                       smem_desc(sKP + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                 1024),
+                       id, k > 0);
+        }
+        if (!(ok = mma_done(120))) break;
+
+        // ---- scale, mask, running max, P (each thread's 64 key columns
+        // in two 32-column passes over TMEM: max first, then exp)
+        const bool diag = mode == 0 && kt == qt;
+        auto masked = [&](const uint32_t(&v)[32], int j0, int j) -> float {
+            const int c = 64 * half + j0 + j;
+            bool keep = true;
+            if (diag) keep = c <= row;
+            if (mode == 1 && b < 128) keep = (c / b) == (row / b);
+            return keep ? __uint_as_float(v[j]) * sl2 : -INFINITY;
+        };
+        float mx = -INFINITY;
+#pragma unroll
+        for (int j0 = 0; j0 < 64; j0 += 32) {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + 64 * half + j0, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j) mx = fmaxf(mx, masked(v, j0, j));
+        }
+        xm[half][row] = mx;
+        __syncthreads();
+        const float mnew = fmaxf(mrun, fmaxf(xm[0][row], xm[1][row]));
+        const float alpha = exp2f(mrun - mnew);  // 0 on the first tile
+        float ls = 0.0f;
+#pragma unroll
+        for (int j0 = 0; j0 < 64; j0 += 32) {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + 64 * half + j0, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                float p[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    p[e] = exp2f(masked(v, j0, 8 * q + e) - mnew);
+                    ls += p[e];
+                }
+                st_shared_bf16x8(
+                    sKP + panel_offset(row, 8 * half + j0 / 8 + q, 128), p);
+            }
+        }
+        xl[half][row] = ls;
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        lrun = lrun * alpha + xl[0][row] + xl[1][row];
+        mrun = mnew;
+
+        // ---- P V
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, D, false, true);
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                mma_ss(tm + 128,
+                       smem_desc(sKP + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                 1024),
+                       smem_desc(sV + k * 2048, 16384, 1024), id, k > 0);
+        }
+        if (!(ok = mma_done(121))) break;
+        if (it + 1 < nkt) {  // next key tile (K and V buffers are free)
+            key_rows(kt + 1);
+            __syncthreads();
+            load_kv();
+        }
+#pragma unroll
+        for (int c = 0; c < DH; c += 32) {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + 128 + half * DH + c, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                o_acc[c + j] = o_acc[c + j] * alpha + __uint_as_float(v[j]);
+        }
+        tc_fence_before();
+    }
+    cp_async_wait<0>();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tm, 256);
+    if (!ok) return;
+
+    // ---- O = sum e^z V / (sum e^z + eps), log d (natural log)
+    const float logd = (mrun + log2f(lrun)) * kLn2;
+    const float inv = 1.0f / (lrun + eps * exp2f(-mrun));
+    const size_t tok = hN + qrow_s[row];
+    float *o = RO + tok * D + half * DH;
+    if (mode == 0) {
+#pragma unroll
+        for (int j = 0; j < DH; j += 4)
+            *reinterpret_cast<float4 *>(o + j) =
+                make_float4(o_acc[j] * inv, o_acc[j + 1] * inv,
+                            o_acc[j + 2] * inv, o_acc[j + 3] * inv);
+        if (half == 0) RL[tok] = logd;
+    } else {
+        // MergeLSE(running = diag, this = off)
+        const float ld1 = RL[tok];
+        const float mu = fmaxf(ld1, logd);
+        const float w1 = __expf(ld1 - mu), w2 = __expf(logd - mu);
+        const float ssum = w1 + w2;
+        const float r = 1.0f / (ssum + eps);
+        const float c1 = w1 * r, c2 = w2 * inv * r;
+#pragma unroll
+        for (int j = 0; j < DH; j += 4) {
+            float4 a = *reinterpret_cast<float4 *>(o + j);
+            a.x = c1 * a.x + c2 * o_acc[j];
+            a.y = c1 * a.y + c2 * o_acc[j + 1];
+            a.z = c1 * a.z + c2 * o_acc[j + 2];
+            a.w = c1 * a.w + c2 * o_acc[j + 3];
+            *reinterpret_cast<float4 *>(o + j) = a;
+        }
+        __syncthreads();  // both halves read RL before it changes
+        if (half == 0) RL[tok] = mu + __logf(ssum + eps);
+    }
+}
+
+// ---------------------------------------------------- RACE prefix states
+
+// part[bh][n] = (B_n [r][d], A_n [r]) of chunk n; writes the strict prefix
+// sums sB_n (bf16, [bh][n][r][d]) and sA_n (fp32, [bh][n][r]).
+__global__ void k_causal_prefix(const float *__restrict__ part, int nc,
+                                int r, int d, uint16_t *__restrict__ sBh,
+                                float *__restrict__ sA) {
+    const int bh = blockIdx.y;
+    const size_t per = (size_t)r * d + r;
+    const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= per) return;
+    const float *p = part + (size_t)bh * nc * per + i;
+    float run = 0.0f;
+    for (int n = 0; n < nc; ++n) {
+        const size_t c = (size_t)bh * nc + n;
+        if (i < (size_t)r * d) {
+            const __nv_bfloat16 h = __float2bfloat16_rn(run);
+            sBh[c * r * d + i] = *reinterpret_cast<const uint16_t *>(&h);
+        } else {
+            sA[c * r + (i - (size_t)r * d)] = run;
+        }
+        run += p[(size_t)n * per];
+    }
+}
+
+// ----------------------------------------------- causal RACE + fusion
+
+// One CTA = one chunk of 128 tokens of one head (original order):
+//   MMA  U_Q = Q W^T, U_K = K W^T
+//   per 128-bucket group h: CUDA phi_Q, phi_K of the group's tables and
+//        phi_Q . sA_n; MMA S += phi_Q phi_K^T, Num += phi_Q sB_n
+//   CUDA P = tril(S) (bf16), row sums
+//   MMA  Num += P V
+//   CUDA O_lr = Num / L / (Den / L + eps), then Eq. (5)-(6) with the
+//        sparse branch's (O_s, log d_s).
+// TMEM: U_Q [0, 64), U_K [64, 128), S [128, 256), Num [256, 256 + D).
+template <int D, int L>
+__global__ void __launch_bounds__(kCaThreads, 1)
+    k_causal_race_tc(const uint16_t *__restrict__ qx,
+                     const uint16_t *__restrict__ kx,
+                     const uint16_t *__restrict__ vx,
+                     const uint16_t *__restrict__ w_bf16,
+                     const uint16_t *__restrict__ sBh,
+                     const float *__restrict__ sAg, const float *__restrict__ RO,
+                     const float *__restrict__ RL,
+                     const float *__restrict__ lambda_tok,
+                     const float *__restrict__ gates, int N, int H, float beta,
+                     float eps, float lambda, int mode,
+                     uint16_t *__restrict__ ox, float *__restrict__ log_ds_out,
+                     float *__restrict__ dlr_out, float *__restrict__ m_out,
+                     DeviceStatus *status) {
+    constexpr int R = 16, G = 4;
+    constexpr int r = L * R, Lg = L * G;
+    constexpr int Lg_pad = (Lg + 15) / 16 * 16;
+    constexpr int RB = r < 128 ? r : 128;  // buckets per group
+    constexpr int NG = r / RB;             // groups
+    constexpr int TPT = RB / R / 2;        // tables per thread and group
+    constexpr int DH = D / 2;
+    constexpr uint32_t kTileB = 128 * D * 2;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tbase;
+    __shared__ int abort_flag;
+    __shared__ float xd[2][128];
+    volatile int *abort = &abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
+    const int half = warp >> 2;
+    const int row = (warp & 3) * 32 + lane_id;
+    const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t sQ = base;            // Q, then phi_Q of a group, then P
+    const uint32_t sK = sQ + 32768;      // K, then phi_K of a group
+    const uint32_t sB = sK + 32768;      // sB_n [r x D]
+    const uint32_t sV = sB + (uint32_t)r * D * 2;
+    const uint32_t sW = sV + kTileB;     // [Lg_pad x D]
+    const uint32_t sAo = sW + (uint32_t)Lg_pad * D * 2;  // fp32 sA_n [r]
+    const float *sAf =
+        reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
+
+    const int nc = N / 128;
+    const int bh = blockIdx.x / nc, n = blockIdx.x % nc;
+    const int h = bh % H;
+    const size_t row0 = (size_t)bh * N + (size_t)n * 128;
+
+    if (warp == 0) tmem_alloc(&tbase, 512);
+    if (tid == 0) {
+        mbar_init(&mma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+        const int rr = i / (D / 8), c = i % (D / 8);
+        const size_t o = (row0 + rr) * D + c * 8;
+        cp_async16(sQ + panel_offset(rr, c, 128), qx + o);
+        cp_async16(sK + panel_offset(rr, c, 128), kx + o);
+        cp_async16(sV + panel_offset(rr, c, 128), vx + o);
+    }
+    for (int i = tid; i < Lg_pad * (D / 8); i += kCaThreads) {
+        const int rr = i / (D / 8), c = i % (D / 8);
+        cp_async16(sW + panel_offset(rr, c, Lg_pad),
+                   w_bf16 + ((size_t)h * Lg_pad + rr) * D + c * 8);
+    }
+    const size_t cidx = (size_t)bh * nc + n;
+    for (int i = tid; i < r * (D / 8); i += kCaThreads) {
+        const int rr = i / (D / 8), c = i % (D / 8);
+        cp_async16(sB + panel_offset(rr, c, r),
+                   sBh + (cidx * r + rr) * D + c * 8);
+    }
+    for (int i = tid; i < r / 4; i += kCaThreads)
+        cp_async16(sAo + 16 * i, sAg + cidx * r + 4 * i);
+    cp_async_commit();
+    cp_async_wait<0>();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = tbase;
+    uint32_t mph = 0;
+    auto mma_done = [&](int site) -> bool {
+        if (tid == 0) mma_commit(&mma_bar);
+        const bool ok =
+            mbar_wait_or_abort(&mma_bar, mph & 1, abort, status, site);
+        ++mph;
+        tc_fence_after();
+        return __syncthreads_and(ok);
+    };
+
+    bool ok = true;
+    // ---- projections
+    if (tid == 0) {
+        const uint32_t id = idesc_bf16(128, Lg_pad, false, false);
+#pragma unroll
+        for (int k = 0; k < D / 16; ++k) {
+            const uint32_t oa = (k >> 2) * 16384 + (k & 3) * 32;
+            const uint64_t bw =
+                smem_desc(sW + (k >> 2) * Lg_pad * 128 + (k & 3) * 32, 16,
+                          1024);
+            mma_ss(tm, smem_desc(sQ + oa, 16, 1024), bw, id, k > 0);
+            mma_ss(tm + 64, smem_desc(sK + oa, 16, 1024), bw, id, k > 0);
+        }
+    }
+    ok = mma_done(130);
+
+    float den_inter = 0.0f;
+    for (int g = 0; g < NG && ok; ++g) {
+        // features of this thread's tables in group g (the group's
+        // projections are TMEM columns [32 g, 32 g + RB / 4); with 128
+        // buckets per group each half's 16 columns load alone, with 64 the
+        // two halves share one 16-column load)
+        uint32_t uq[16], uk[16];
+        const uint32_t c0 = 32 * g + (RB == 128 ? 16 * half : 0);
+        tmem_ld16(tm + lane + c0, uq);
+        tmem_ld16(tm + lane + 64 + c0, uk);
+        tmem_wait_ld();
+        auto pick = [&](const uint32_t(&u)[16], int i) -> float {
+            if (RB == 128) return __uint_as_float(u[i]);
+            return __uint_as_float(half ? u[(8 + i) & 15] : u[i]);
+        };
+#pragma unroll
+        for (int t = 0; t < TPT; ++t) {
+            const int tl = half * TPT + t;       // table within the group
+            const int tbl = g * (RB / R) + tl;  // table
+            float spq[G], snq[G], spk[G], snk[G];
+#pragma unroll
+            for (int bb = 0; bb < G; ++bb) {
+                race_bit_factors(pick(uq, t * G + bb), beta, spq[bb],
+                                 snq[bb]);
+                race_bit_factors(pick(uk, t * G + bb), beta, spk[bb],
+                                 snk[bb]);
+            }
+            float pq[R], pk[R];
+#pragma unroll
+            for (int rr = 0; rr < R; ++rr) {
+                float a = 1.0f, c = 1.0f;
+#pragma unroll
+                for (int bb = 0; bb < G; ++bb) {
+                    const bool on = (rr >> bb) & 1;
+                    a *= on ? spq[bb] : snq[bb];
+                    c *= on ? spk[bb] : snk[bb];
+                }
+                pq[rr] = a;
+                pk[rr] = c;
+                den_inter = fmaf(a, sAf[tbl * R + rr], den_inter);
+            }
+            const int col = tl * R;  // bucket within the group
+            st_shared_bf16x8(sQ + panel_offset(row, col / 8, 128), pq);
+            st_shared_bf16x8(sQ + panel_offset(row, col / 8 + 1, 128), pq + 8);
+            st_shared_bf16x8(sK + panel_offset(row, col / 8, 128), pk);
+            st_shared_bf16x8(sK + panel_offset(row, col / 8 + 1, 128), pk + 8);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {
+            tc_fence_after();
+            const uint32_t id_s = idesc_bf16(128, 128, false, false);
+            const uint32_t id_n = idesc_bf16(128, D, false, true);
+#pragma unroll
+            for (int k = 0; k < RB / 16; ++k) {
+                const uint32_t oa = (k >> 2) * 16384 + (k & 3) * 32;
+                mma_ss(tm + 128, smem_desc(sQ + oa, 16, 1024),
+                       smem_desc(sK + oa, 16, 1024), id_s, (g > 0 || k > 0));
+                mma_ss(tm + 256, smem_desc(sQ + oa, 16, 1024),
+                       smem_desc(sB + (uint32_t)(g * RB + 16 * k) * 128,
+                                 (uint32_t)r * 128, 1024),
+                       id_n, (g > 0 || k > 0));
+            }
+        }
+        ok = mma_done(131);
+    }
+
+    // ---- P = tril(S): row i keeps keys j <= i of the chunk
+    float dintra = 0.0f;
+    if (ok) {
+        float s[64];
+        uint32_t v[32];
+        tmem_ld32(tm + lane + 128 + 64 * half, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) s[j] = __uint_as_float(v[j]);
+        tmem_ld32(tm + lane + 128 + 64 * half + 32, v);
+        tmem_wait_ld();
+#pragma unroll
+        for (int j = 0; j < 32; ++j) s[32 + j] = __uint_as_float(v[j]);
+#pragma unroll
+        for (int j = 0; j < 64; ++j) {
+            s[j] = (64 * half + j <= row) ? s[j] : 0.0f;
+            dintra += s[j];
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            st_shared_bf16x8(sQ + panel_offset(row, 8 * half + q, 128),
+                             s + 8 * q);
+        fence_proxy_async_smem();
+        tc_fence_before();
+    }
+    xd[half][row] = den_inter + dintra;
+    __syncthreads();
+    if (ok && tid == 0) {
+        tc_fence_after();
+        const uint32_t id = idesc_bf16(128, D, false, true);
+#pragma unroll
+        for (int k = 0; k < 8; ++k)
+            mma_ss(tm + 256,
+                   smem_desc(sQ + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024),
+                   smem_desc(sV + k * 2048, 16384, 1024), id, 1u);
+    }
+    if (ok) ok = mma_done(132);
+
+    if (ok) {
+        const float invL = 1.0f / (float)L;
+        const float den = (xd[0][row] + xd[1][row]) * invL;
+        const float rl = 1.0f / (den + eps);
+        const size_t tok = row0 + row;
+        const float log_ds = RL[tok];
+        const float lam = lambda_tok ? lambda_tok[tok] : lambda;
+        const float gs = gates ? gates[2 * tok] : 1.0f;
+        const float gl = gates ? gates[2 * tok + 1] : 1.0f;
+        const float mm = fusion_multiplier(log_ds, lam, den, eps, mode);
+        const float cs = gs * mm, cl = gl * invL * rl;
+        const float *os = RO + tok * D + half * DH;
+        uint16_t *o = ox + tok * D + half * DH;
+#pragma unroll
+        for (int c = 0; c < DH; c += 32) {
+            uint32_t v[32];
+            tmem_ld32(tm + lane + 256 + half * DH + c, v);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; j += 8) {
+                float y[8];
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    y[e] = cs * os[c + j + e] +
+                           cl * __uint_as_float(v[j + e]);
+                uint4 pk;
+                pk.x = pack_bf16x2(y[0], y[1]);
+                pk.y = pack_bf16x2(y[2], y[3]);
+                pk.z = pack_bf16x2(y[4], y[5]);
+                pk.w = pack_bf16x2(y[6], y[7]);
+                *reinterpret_cast<uint4 *>(o + c + j) = pk;
+            }
+        }
+        if (half == 0) {
+            if (log_ds_out) log_ds_out[tok] = log_ds;
+            if (dlr_out) dlr_out[tok] = den;
+            if (m_out) m_out[tok] = mm;
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tm, 512);
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ host
+
+bool causal_tc_supported(const Plan &P, int n_leaf) {
+    if (P.dtype != ELSAA_BF16 || P.impl != 2) return false;
+    if (P.d != 64 && P.d != 128) return false;
+    if (P.gamma != 4 || !(P.L == 4 || P.L == 8 || P.L == 16)) return false;
+    if (n_leaf % 128 != 0 || P.N % 128 != 0) return false;
+    if (!(P.b == 32 || P.b == 64 || P.b == 128 || P.b == 256)) return false;
+    if (n_leaf != P.N && n_leaf % P.b != 0) return false;
+    return true;
+}
+
+size_t causal_attn_smem(int d) {
+    const size_t tile = (size_t)128 * d * 2;
+    return 1024 + tile + (tile > 32768 ? tile : 32768) + tile;
+}
+
+size_t causal_race_smem(const Plan &P) {
+    const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
+    return 1024 + 65536 + (size_t)P.r * P.d * 2 + (size_t)128 * P.d * 2 +
+           lg_pad * P.d * 2 + (size_t)P.r * 4;
+}
+
+cudaError_t launch_seg_sort(const Plan &P, int Lv, const uint32_t *keyrank,
+                            int32_t *perms, cudaStream_t st) {
+    if (Lv == 0) return cudaSuccess;
+    dim3 grid((1u << Lv) - 1, P.BH, 2);
+    k_seg_sort<<<grid, kSegThreads, 0, st>>>(keyrank, P.N, P.bins, perms);
+    return cudaGetLastError();
+}
+
+// mode 0: base segments of n_leaf rows; mode 1: SortLSH blocks of level
+// `level` (1 = top) whose halves hold m = N / 2^level rows.
+cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
+                               const void *q, const void *k, const void *v,
+                               const int32_t *perms, float *RO, float *RL,
+                               DeviceStatus *status, cudaStream_t st) {
+    int items, m = 0;
+    const int32_t *pq = nullptr, *pk = nullptr;
+    if (mode == 0) {
+        items = P.BH * (P.N / n_leaf) * (n_leaf / 128);
+    } else {
+        m = P.N >> level;
+        items = P.BH * (P.N / (2 * m)) * (m / 128);
+        const size_t lvl = (size_t)(level - 1) * 2 * P.BH * (P.N / 2);
+        pq = perms + lvl;
+        pk = perms + lvl + (size_t)P.BH * (P.N / 2);
+    }
+    // at most two CTAs per SM (each holds 256 TMEM columns)
+    size_t smem = causal_attn_smem(P.d);
+    if (smem < kSmemPerSM / 3 + 1024) smem = kSmemPerSM / 3 + 1024;
+    auto launch = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<items, kCaThreads, smem, st>>>(
+            (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v, pq,
+            pk, P.N, mode, n_leaf, m, P.b, P.scale, P.eps, RO, RL, status);
+        return cudaGetLastError();
+    };
+    return P.d == 128 ? launch(k_causal_attn_tc<128>)
+                      : launch(k_causal_attn_tc<64>);
+}
+
+cudaError_t launch_causal_prefix(const Plan &P, const float *part,
+                                 uint16_t *sBh, float *sA, cudaStream_t st) {
+    const int per = P.r * P.d + P.r;
+    dim3 grid((per + 255) / 256, P.BH);
+    k_causal_prefix<<<grid, 256, 0, st>>>(part, P.N / 128, P.r, P.d, sBh, sA);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_causal_race(const Plan &P, const void *q, const void *k,
+                               const void *v, const uint16_t *w_bf16,
+                               const uint16_t *sBh, const float *sA,
+                               const float *RO, const float *RL,
+                               const float *lambda_tok, const float *gates,
+                               void *o, float *log_ds, float *dlr, float *m,
+                               DeviceStatus *status, cudaStream_t st) {
+    const int blocks = P.BH * (P.N / 128);
+    // one CTA per SM (it holds all 512 TMEM columns)
+    size_t smem = causal_race_smem(P);
+    if (smem < kSmemPerSM / 2 + 1024) smem = kSmemPerSM / 2 + 1024;
+    auto launch = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<blocks, kCaThreads, smem, st>>>(
+            (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
+            w_bf16, sBh, sA, RO, RL, lambda_tok, gates, P.N, P.H, P.beta,
+            P.eps, P.lambda, P.fusion_mode, (uint16_t *)o, log_ds, dlr, m,
+            status);
+        return cudaGetLastError();
+    };
+    if (P.d == 128) {
+        if (P.L == 16) return launch(k_causal_race_tc<128, 16>);
+        if (P.L == 8) return launch(k_causal_race_tc<128, 8>);
+        return launch(k_causal_race_tc<128, 4>);
+    }
+    if (P.L == 16) return launch(k_causal_race_tc<64, 16>);
+    if (P.L == 8) return launch(k_causal_race_tc<64, 8>);
+    return launch(k_causal_race_tc<64, 4>);
+}
+
+}  // namespace elsaa

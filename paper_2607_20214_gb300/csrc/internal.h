@@ -139,6 +139,24 @@ cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
                                const float *gA, float *dk, float *dv,
                                DeviceStatus *status, cudaStream_t st);
 
+// Causal variant (causal.cu).
+bool causal_tc_supported(const Plan &P, int n_leaf);
+cudaError_t launch_seg_sort(const Plan &P, int Lv, const uint32_t *keyrank,
+                            int32_t *perms, cudaStream_t st);
+cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
+                               const void *q, const void *k, const void *v,
+                               const int32_t *perms, float *RO, float *RL,
+                               DeviceStatus *status, cudaStream_t st);
+cudaError_t launch_causal_prefix(const Plan &P, const float *part,
+                                 uint16_t *sBh, float *sA, cudaStream_t st);
+cudaError_t launch_causal_race(const Plan &P, const void *q, const void *k,
+                               const void *v, const uint16_t *w_bf16,
+                               const uint16_t *sBh, const float *sA,
+                               const float *RO, const float *RL,
+                               const float *lambda_tok, const float *gates,
+                               void *o, float *log_ds, float *dlr, float *m,
+                               DeviceStatus *status, cudaStream_t st);
+
 // One bounded mbarrier wait that can never complete (selftest.cu).
 cudaError_t launch_selftest_wait(DeviceStatus *status, int limit_ms,
                                  cudaStream_t st);

@@ -46,7 +46,8 @@ class elsaa_params(ctypes.Structure):
         ("beta", ctypes.c_float), ("eps", ctypes.c_float),
         ("scale", ctypes.c_float), ("lam", ctypes.c_float),
         ("fusion_mode", ctypes.c_int), ("impl", ctypes.c_int),
-        ("neighbor_blocks", ctypes.c_int),
+        ("neighbor_blocks", ctypes.c_int), ("causal_chunk", ctypes.c_int),
+        ("causal_base_len", ctypes.c_int),
     ]
 
 
@@ -144,12 +145,14 @@ def _check(rc: int):
 def make_params(B, H, N, d_h, dtype="bf16", block_size=64, sort_bits=5,
                 gray_order=1, race_tables=4, race_bits=4, beta=1.0, eps=1e-6,
                 scale=0.0, lam=1.0, fusion_mode=0, causal=0,
-                impl=ELSAA_IMPL_AUTO, neighbor_blocks=0) -> elsaa_params:
+                impl=ELSAA_IMPL_AUTO, neighbor_blocks=0, causal_chunk=128,
+                causal_base_len=4096) -> elsaa_params:
     dt = {"bf16": ELSAA_BF16, "fp32": ELSAA_FP32}[dtype] if isinstance(
         dtype, str) else int(dtype)
     return elsaa_params(B, H, N, d_h, dt, causal, block_size, sort_bits,
                         gray_order, race_tables, race_bits, beta, eps, scale,
-                        lam, fusion_mode, impl, neighbor_blocks)
+                        lam, fusion_mode, impl, neighbor_blocks, causal_chunk,
+                        causal_base_len)
 
 
 def params_for(wl, **over) -> elsaa_params:
@@ -159,7 +162,9 @@ def params_for(wl, **over) -> elsaa_params:
               gray_order=wl.gray_order, race_tables=wl.race_tables,
               race_bits=wl.race_bits, beta=wl.beta, eps=wl.eps,
               lam=wl.lam, fusion_mode=wl.fusion_mode, causal=wl.causal,
-              neighbor_blocks=wl.neighbor_blocks)
+              neighbor_blocks=wl.neighbor_blocks,
+              causal_chunk=wl.causal_chunk,
+              causal_base_len=wl.causal_base_len)
     kw.update(over)
     return make_params(**kw)
 

@@ -39,7 +39,9 @@ class Workload:
     eps: float = 1e-6
     lam: float = 1.0
     fusion_mode: int = 0  # 0: ELSAA multiplier, 1: Sort_Lsh_RACE ablation (m = 1)
-    causal: int = 0
+    causal: int = 0  # 1: Algorithm "Causal ELSAA"
+    causal_chunk: int = 128  # C of causal RACE
+    causal_base_len: int = 4096  # N_0 of CausalSparse (Table 7, text: 4096)
     neighbor_blocks: int = 0  # r neighbouring sorted key blocks per side
     recipe: str = "plain"  # input recipe, see make_inputs
     temperature: float = 1.0
@@ -86,6 +88,12 @@ WORKLOADS = {
                    plane_seed=1003),
     "c4": Workload("c4", B=1, H=32, N=65536, d_h=128, dtype="bf16", block=256,
                    race_tables=16, recipe="dup_keys", seed=3, plane_seed=1004),
+    # c3 through Algorithm "Causal ELSAA": C = 128, N_0 = 4096 (Table 7's
+    # text setting), so CausalSparse has two levels above 4096-row segments
+    "c3c": Workload("c3c", B=2, H=16, N=16384, d_h=128, dtype="bf16",
+                    block=128, race_tables=16, recipe="uniform_temp", seed=2,
+                    plane_seed=1003, causal=1, causal_chunk=128,
+                    causal_base_len=4096),
     "c5": Workload("c5", B=8, H=12, N=8192, d_h=64, dtype="bf16", block=64,
                    race_tables=8, recipe="plain", temperature=2.0, seed=4,
                    plane_seed=1005, backward=True),

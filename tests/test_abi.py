@@ -58,7 +58,7 @@ def test_params_struct_matches_header():
 
 
 def test_abi_version(lib):
-    assert elsaa.elsaa_abi_version() == 2
+    assert elsaa.elsaa_abi_version() == 3
 
 
 @pytest.mark.parametrize("name", sorted(WORKLOADS))
@@ -71,7 +71,18 @@ def test_workspace_size_is_positive_and_deterministic(lib, name):
 
 BAD = [
     (dict(N=1000, block_size=64), elsaa.ELSAA_ERR_INVALID_ARG, "multiple"),
-    (dict(causal=1), elsaa.ELSAA_ERR_UNSUPPORTED, "causal"),
+    (dict(causal=2), elsaa.ELSAA_ERR_INVALID_ARG, "causal"),
+    (dict(causal=1, dtype="fp32"), elsaa.ELSAA_ERR_UNSUPPORTED, "causal"),
+    (dict(causal=1, causal_base_len=0), elsaa.ELSAA_ERR_INVALID_ARG,
+     "causal_base_len"),
+    (dict(causal=1, causal_chunk=0), elsaa.ELSAA_ERR_INVALID_ARG,
+     "causal_chunk"),
+    (dict(causal=1, N=192, causal_base_len=2), elsaa.ELSAA_ERR_UNSUPPORTED,
+     "odd"),
+    (dict(causal=1, N=384, causal_base_len=100), elsaa.ELSAA_ERR_UNSUPPORTED,
+     "multiple of 128"),
+    (dict(causal=1, neighbor_blocks=1), elsaa.ELSAA_ERR_UNSUPPORTED,
+     "neighbor_blocks"),
     (dict(d_h=96), elsaa.ELSAA_ERR_UNSUPPORTED, "d_h"),
     (dict(eps=0.0), elsaa.ELSAA_ERR_INVALID_ARG, "eps"),
     (dict(lam=-1.0), elsaa.ELSAA_ERR_INVALID_ARG, "lambda"),

@@ -1,0 +1,126 @@
+"""GPU causal path (elsaa_forward with causal = 1, through the C ABI) versus
+the fp64 causal oracle (oracle/causal.py) on the same seeded inputs.
+
+Tolerances as for the non-causal bf16 path: O within 2e-2 absolute (bf16
+inputs and output; the kernels round the softmax weights, the RACE features,
+the masked intra-chunk products and the prefix states sB_n to bf16 before
+their tensor-core products, relative 2^-9 each, and accumulate in fp32),
+log d_sparse within 2e-2 absolute (fp32 running maximum and sum), d_lr
+within 1e-2 relative, m within 1e-2 absolute.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import causal as oc
+from oracle import oracle as orc
+from paper_2607_20214_gb300 import build, elsaa
+from paper_2607_20214_gb300.workloads import (WORKLOADS, Workload,
+                                              make_gates_lambda, make_inputs)
+
+pytestmark = pytest.mark.gpu
+
+TOL_O, TOL_LOGD, TOL_DLR_REL, TOL_M = 2e-2, 2e-2, 1e-2, 1e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    build.build()
+    elsaa.load_library()
+
+
+def run_gpu(wl, x, gates=None, lam=None):
+    dev = torch.device("cuda:0")
+    p = elsaa.params_for(wl)
+    xd = {k: v.to(dev) for k, v in x.items()}
+    BHN = (wl.B, wl.H, wl.N)
+    out = dict(log_d_sparse=torch.full(BHN, float("nan"), device=dev),
+               d_lr=torch.full(BHN, float("nan"), device=dev),
+               m_sparse=torch.full(BHN, float("nan"), device=dev))
+    ws = elsaa.new_workspace(p, dev)
+    o = elsaa.elsaa_forward(
+        p, xd["q"], xd["k"], xd["v"], xd["w_sort"], xd["w_race"],
+        lambda_tok=None if lam is None else lam.to(dev),
+        gates=None if gates is None else gates.to(dev), workspace=ws, **out)
+    elsaa.elsaa_check_status(ws)
+    torch.cuda.synchronize()
+    res = {k: v.cpu() for k, v in out.items()}
+    res["O"] = o.float().cpu()
+    return res
+
+
+def compare(g, ref, label=""):
+    for (b, h), r in ref.items():
+        e = np.abs(g["O"][b, h].numpy() - r["O"]).max()
+        assert e <= TOL_O, (label, b, h, "O", e)
+        e = np.abs(g["log_d_sparse"][b, h].numpy() - r["log_d_sparse"]).max()
+        assert e <= TOL_LOGD, (label, b, h, "log d_s", e)
+        dl = g["d_lr"][b, h].numpy()
+        e = (np.abs(dl - r["d_lr"]) / np.abs(r["d_lr"])).max()
+        assert e <= TOL_DLR_REL, (label, b, h, "d_lr", e)
+        e = np.abs(g["m_sparse"][b, h].numpy() - r["m_log"]).max()
+        assert e <= TOL_M, (label, b, h, "m", e)
+
+
+def small(**kw):
+    base = dict(name="causal", B=1, H=2, N=1024, d_h=64, dtype="bf16",
+                block=64, race_tables=8, recipe="plain", temperature=2.0,
+                seed=21, plane_seed=1021, causal=1, causal_chunk=128,
+                causal_base_len=256)
+    base.update(kw)
+    return Workload(**base)
+
+
+@pytest.mark.parametrize("d_h,b,L,N,N0", [
+    (64, 64, 8, 1024, 256),      # two levels above 256-row segments
+    (128, 128, 16, 1024, 256),
+    (128, 256, 16, 2048, 512),   # blocks of two key tiles
+    (64, 32, 4, 512, 128),       # four blocks per 128-row tile
+    (64, 64, 8, 512, 4096),      # one segment: exact causal attention
+    (128, 128, 8, 2048, 300),    # three levels, segments of 256 rows
+])
+def test_causal_matches_oracle(d_h, b, L, N, N0):
+    wl = small(d_h=d_h, block=b, race_tables=L, N=N, causal_base_len=N0)
+    x = make_inputs(wl)
+    ref = oc.forward(x, orc.params_from_workload(wl))
+    compare(run_gpu(wl, x), ref, label=(d_h, b, L, N, N0))
+
+
+def test_causal_gates_lambda_and_ablation():
+    wl = small(H=3)
+    x = make_inputs(wl)
+    gates, lam = make_gates_lambda(wl, seed=5)
+    ref = oc.forward(x, orc.params_from_workload(wl), lam=lam, gates=gates)
+    compare(run_gpu(wl, x, gates=gates, lam=lam), ref, label="gates")
+    wl1 = wl.with_(fusion_mode=1)
+    ref = oc.forward(x, orc.params_from_workload(wl1))
+    g = run_gpu(wl1, x)
+    for (b, h), r in ref.items():
+        assert np.abs(g["O"][b, h].numpy() - r["O"]).max() <= TOL_O
+        assert (g["m_sparse"][b, h].numpy() == 1.0).all()
+
+
+def test_causal_prefix_rows_ignore_later_keys():
+    """Rows before t do not change when keys and values after t change
+    (the device path keeps the causal structure)."""
+    wl = small(N=1024)
+    x = make_inputs(wl)
+    a = run_gpu(wl, x)
+    y = {k: v.clone() for k, v in x.items()}
+    y["k"][:, :, 700:] = -y["k"][:, :, 700:]
+    y["v"][:, :, 700:] = 3.0
+    c = run_gpu(wl, y)
+    assert torch.equal(a["O"][:, :, :700], c["O"][:, :, :700])
+    assert (a["O"][:, :, 700:] - c["O"][:, :, 700:]).abs().max() > 0.1
+
+
+def test_c3_causal_full_size_heads():
+    """The c3 causal workload (B=2 H=16 N=16384 d_h=128, b=128, r=256,
+    C=128, N_0=4096) in the benchmark's launch configuration; every row of
+    two heads against the oracle."""
+    wl = WORKLOADS["c3c"]
+    x = make_inputs(wl)
+    g = run_gpu(wl, x)
+    ref = oc.forward(x, orc.params_from_workload(wl), heads=[(0, 3), (1, 12)])
+    compare(g, ref, label="c3c")
+    assert torch.isfinite(g["O"]).all()
