@@ -161,7 +161,12 @@ def cpu_oracle_time(wl, x_cpu, heads, threads):
     from oracle import oracle
     p = oracle.params_from_workload(wl)
     t0 = time.perf_counter()
-    res = oracle.forward(x_cpu, p, heads=heads, threads=threads)
+    if wl.causal:
+        # numpy fp64 (one head after another; its BLAS may use every core)
+        from oracle import causal
+        res = causal.forward(x_cpu, p, heads=heads)
+    else:
+        res = oracle.forward(x_cpu, p, heads=heads, threads=threads)
     return time.perf_counter() - t0, res
 
 
@@ -183,7 +188,9 @@ def run_reference(args, wl):
     from oracle import oracle
     oracle.build()
     cores = os.cpu_count() or 1
-    per_step = max(1, min(wl.heads, cores))
+    # the causal oracle runs one head at a time (numpy, about 3 s per c3
+    # causal head): two heads per step
+    per_step = 2 if wl.causal else max(1, min(wl.heads, cores))
     x = make_inputs(wl.with_(B=1, H=min(wl.H, per_step)))
     heads = [(0, h) for h in range(min(wl.H, per_step))]
     times = []
@@ -214,10 +221,13 @@ def run_reference(args, wl):
 
 def workload_config(wl):
     return {"workload": "%s: B=%d H=%d N=%d d_h=%d %s b=%d r=%d "
-                        "(L_s=%d, gamma=%d) sort_bits=%d non-causal%s" % (
+                        "(L_s=%d, gamma=%d) sort_bits=%d %s%s" % (
                             wl.name, wl.B, wl.H, wl.N, wl.d_h, wl.dtype,
                             wl.block, wl.r, wl.race_tables, wl.race_bits,
                             wl.sort_bits,
+                            ("causal (C=%d, N_0=%d)" % (
+                                wl.causal_chunk, wl.causal_base_len))
+                            if wl.causal else "non-causal",
                             (", %d neighbour blocks per side" %
                              wl.neighbor_blocks) if wl.neighbor_blocks
                             else ""),
@@ -485,17 +495,23 @@ def run_ours(args, wl):
     if rank == 0 and world == 1 and not args.no_cpu_baseline and \
             not args.backward and not args.gate_mlp:
         cores = os.cpu_count() or 1
-        n_heads = min(wl.heads, 2 * cores)
+        n_heads = 2 if wl.causal else min(wl.heads, 2 * cores)
         heads = [(i // wl.H, i % wl.H) for i in range(n_heads)]
         xc = heads_to_cpu(x, heads)
         t_cpu, res = cpu_oracle_time(wl, xc, [(0, j) for j in range(n_heads)],
                                      threads=min(cores, n_heads))
         cpu = {"value": wl.tokens * (n_heads / wl.heads) / t_cpu,
-               "unit": "tokens/s", "cores": min(cores, n_heads),
+               "unit": "tokens/s",
+               "cores": cores if wl.causal else min(cores, n_heads),
                "kind": "oracle",
-               "sample": "%d of %d heads of one step (fp64 C oracle, "
-                         "threads over heads), %.1f s wall" % (
-                             n_heads, wl.heads, t_cpu)}
+               "sample": ("%d of %d heads of one step (fp64 numpy causal "
+                          "oracle, one head at a time, BLAS threads up to "
+                          "%d cores), %.1f s wall" % (n_heads, wl.heads,
+                                                      cores, t_cpu))
+               if wl.causal else
+               "%d of %d heads of one step (fp64 C oracle, "
+               "threads over heads), %.1f s wall" % (
+                   n_heads, wl.heads, t_cpu)}
         of = o.float()
         err = 0.0
         for j, (b, h) in enumerate(heads):

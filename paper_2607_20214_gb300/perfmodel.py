@@ -30,6 +30,8 @@ def flop_model(wl: Workload) -> dict:
     separately.
     """
     N, b, d, r = wl.N, wl.block, wl.d_h, wl.r
+    if getattr(wl, "causal", 0):
+        return causal_flop_model(wl)
     b = keys_per_query(wl)
     per_head = (4 * N * b * d + 4 * N * r * d + 4 * N * r
                 + 4 * N * d * wl.race_tables * wl.race_bits)
@@ -45,6 +47,37 @@ def flop_model(wl: Workload) -> dict:
 # CUDA-core fp32 peak of a 152-SM GB300 at its 2070 MHz maximum clock:
 # 152 SMs x 128 FP32 lanes x 2 FLOP per FMA x 2.07e9 / s.
 SIMT_FP32_PEAK_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def causal_levels(wl: Workload):
+    """(levels, base segment length) of the unrolled CausalSparse
+    recursion: halve N until a segment fits the base length N_0."""
+    n, lv = wl.N, 0
+    while n > wl.causal_base_len:
+        n //= 2
+        lv += 1
+    return lv, n
+
+
+def causal_flop_model(wl: Workload) -> dict:
+    """Useful tensor FLOPs of Algorithm "Causal ELSAA", per head:
+    base segments 4 d_h sum_i (i + 1) over each segment (exact causal
+    attention, ~2 N n_leaf d_h); each level's SortLSH blocks 4 (N / 2) b d_h;
+    causal RACE: chunk summaries 2 N r d_h + 2 N r, inter-chunk readout
+    2 N r d_h + 2 N r, intra-chunk masked products (C + 1) / 2 keys per row
+    of 2 (r + d_h) each (C = 128 on the device), projections 4 N d_h L_s
+    gamma. Bytes: Q, K, V read once and O written once."""
+    N, b, d, r = wl.N, wl.block, wl.d_h, wl.r
+    lv, n_leaf = causal_levels(wl)
+    C = 128
+    sparse = 2 * d * N * (n_leaf + 1) + lv * 4 * (N // 2) * b * d
+    race = (4 * N * r * d + 4 * N * r + N * (C + 1) * (r + d)
+            + 4 * N * d * wl.race_tables * wl.race_bits)
+    heads = wl.heads
+    return {"tensor_flops": (sparse + race) * heads,
+            "sparse_flops": sparse * heads,
+            "hash_flops": 4 * N * d * wl.sort_bits * heads,
+            "bytes": 4 * N * d * wl.elt * heads}
 
 
 def keys_per_query(wl: Workload) -> int:
@@ -88,6 +121,33 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
         by = H * (2 * N * d * e + 4 * N * d * 4)
         fl = H * (4 * N * r * d + 4 * N * d * Lg)
         simt = not kernel.endswith("_tc")
+    elif kernel.startswith("causal_attn_base"):
+        # exact causal attention of the base segments: reads Q, K, V once,
+        # writes the running O (fp32) and log d
+        _, n_leaf = causal_levels(wl)
+        by = H * (3 * N * d * e + N * d * 4 + N * 4)
+        fl = H * 2 * d * N * (n_leaf + 1)
+        simt = False
+    elif kernel.startswith("causal_attn_merge"):
+        # one level's SortLSH blocks: half the rows as queries, half as
+        # keys and values; the running O and log d read and written
+        by = H * (3 * (N // 2) * d * e + (N // 2) * (d + 1) * 4 * 2)
+        fl = H * 4 * (N // 2) * wl.block * d
+        simt = False
+    elif kernel.startswith("causal_race"):
+        # reads Q, K, V, the chunk's prefix state sB (bf16) and the sparse
+        # result, writes O; inter + intra products and projections
+        nc = N // 128
+        by = H * (3 * N * d * e + nc * r * d * 2 + N * (d + 1) * 4 +
+                  N * d * e)
+        fl = H * (2 * N * r * d + N * 129 * (r + d) +
+                  4 * N * d * Lg)
+        simt = False
+    elif kernel.startswith("causal_prefix"):
+        nc = N // 128
+        by = H * nc * (r * (d + 1) * 4 + r * d * 2 + r * 4)
+        fl = 0
+        simt = True
     elif kernel.startswith("bwd_sums_reduce"):
         by = H * r * (d + 1) * 4
         fl = 0
