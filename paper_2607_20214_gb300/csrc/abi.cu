@@ -417,6 +417,27 @@ int causal_forward(const elsaa_params *params, const void *q, const void *k,
 
     ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
                        "status reset");
+    // the low-rank branch needs no sort: chunk summaries and prefix states
+    // on the side stream, joined back before the readout
+    SideStream *side = nullptr;
+    ELSAA_CHECK_LAUNCH(side_stream(&side), "side stream");
+    cudaStream_t ks = side->s;
+    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->fork, st), "fork");
+    ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(ks, side->fork, 0), "fork wait");
+    ELSAA_CHECK_LAUNCH(timed("prep_planes", ks, [&] {
+                           return launch_prep_planes(P, w_race, Wbf, ks);
+                       }),
+                       "prep_planes");
+    ELSAA_CHECK_LAUNCH(timed("race_keys_ws", ks, [&] {
+                           return launch_race_keys_ws(C.Pc, k, v, Wbf, part,
+                                                      status, ks);
+                       }),
+                       "race_keys_ws");
+    ELSAA_CHECK_LAUNCH(timed("causal_prefix", ks, [&] {
+                           return launch_causal_prefix(P, part, sB, sA, ks);
+                       }),
+                       "causal_prefix");
+    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->join, ks), "join");
     // sparse branch: codes, sorted halves, base segments, then the levels
     ELSAA_CHECK_LAUNCH(timed("sort_hash", st, [&] {
                            return launch_sort_hash(P, q, k, w_sort, keyrank,
@@ -442,20 +463,7 @@ int causal_forward(const elsaa_params *params, const void *q, const void *k,
                                                          status, st);
                            }),
                            "causal_attn_merge");
-    // low-rank branch: chunk summaries, prefix states, readout + fusion
-    ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
-                           return launch_prep_planes(P, w_race, Wbf, st);
-                       }),
-                       "prep_planes");
-    ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
-                           return launch_race_keys_ws(C.Pc, k, v, Wbf, part,
-                                                      status, st);
-                       }),
-                       "race_keys_ws");
-    ELSAA_CHECK_LAUNCH(timed("causal_prefix", st, [&] {
-                           return launch_causal_prefix(P, part, sB, sA, st);
-                       }),
-                       "causal_prefix");
+    ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(st, side->join, 0), "join wait");
     ELSAA_CHECK_LAUNCH(timed("causal_race", st, [&] {
                            return launch_causal_race(
                                P, q, k, v, Wbf, sB, sA, RO, RL, lambda_tok,

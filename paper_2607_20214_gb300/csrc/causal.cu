@@ -119,10 +119,16 @@ __global__ void __launch_bounds__(kSegThreads)
 //          the same block (b >= 128: b / 128 key tiles; b < 128: one tile,
 //          rows and keys paired by block, r / b == c / b); MergeLSE into
 //          the running (O, log d).
-// Per key tile: MMA S = Q K^T (TMEM [0, 128)); CUDA scale, mask, running
-// max, P = exp(S - max) as bf16 over the consumed K tile; MMA P V (TMEM
-// [128, 128 + D)); CUDA O = O alpha + P V. Two threads per row (TMEM lane
-// = row; each takes half of the key columns and half of the output).
+// Per key tile: MMA S = Q K^T (TMEM [0, 128)); the next K tile's copies
+// start at once (K is consumed); CUDA scale, mask, running max and
+// P = exp(S - max), packed as bf16 pairs into TMEM over the scores already
+// read (keys [64h, 64h + 64) of row half h in columns [64h, 64h + 32));
+// MMA P V with P from TMEM (TMEM [128, 128 + D)); the next V tile's copies
+// start; CUDA O = O alpha + P V in registers. Two threads per row (TMEM
+// lane = row; each takes half of the key columns and half of the output).
+// cp.async groups are committed in a fixed order (Q and K0, V0, then per
+// tile: next K, next V; empty groups past the last tile), so "all but the
+// newest group done" always means the operand about to be used has landed.
 template <int D>
 __global__ void __launch_bounds__(kCaThreads, 2)
     k_causal_attn_tc(const uint16_t *__restrict__ qx,
@@ -138,7 +144,8 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     __shared__ uint32_t tbase;
     __shared__ int abort_flag;
     __shared__ float xm[2][128], xl[2][128];
-    __shared__ int qrow_s[128], krow_s[128];
+    __shared__ int qrow_s[128];
+    __shared__ int krow_s[2][128];  // mode 1: key rows of the next tiles
     volatile int *abort = &abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
     const int half = warp >> 2;
@@ -149,12 +156,12 @@ __global__ void __launch_bounds__(kCaThreads, 2)
 
     const uint32_t base = align1k(smem_u32(smem_raw));
     const uint32_t sQ = base;
-    const uint32_t sKP = sQ + kTileB;                       // K, then P
-    const uint32_t sV = sKP + (kTileB > 32768 ? kTileB : 32768);
+    const uint32_t sK = sQ + kTileB;
+    const uint32_t sV = sK + kTileB;
 
     // ---- work item
     int bh, qt, nkt, kt0;
-    size_t qbase = 0, kbase = 0;  // mode 0: first row of the segment
+    int seg0 = 0;  // mode 0: first row of the segment (within the head)
     const int32_t *ql = nullptr, *kl = nullptr;
     if (mode == 0) {
         const int nq = n_leaf / 128, nleaves = N / n_leaf;
@@ -163,8 +170,7 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         const int rest = item / nq;
         const int leaf = rest % nleaves;
         bh = rest / nleaves;
-        qbase = (size_t)bh * N + (size_t)leaf * n_leaf + (size_t)qt * 128;
-        kbase = (size_t)bh * N + (size_t)leaf * n_leaf;
+        seg0 = leaf * n_leaf;
         kt0 = 0;
         nkt = qt + 1;
     } else {
@@ -184,6 +190,13 @@ __global__ void __launch_bounds__(kCaThreads, 2)
             nkt = 1;
         }
     }
+    const size_t hN = (size_t)bh * N;
+    auto stage_rows = [&](int kt) {
+        if (mode == 1 && tid < 128) {
+            const int t = kl[kt * 128 + tid];
+            krow_s[kt & 1][tid] = (t < 0 || t >= N) ? 0 : t;
+        }
+    };
 
     if (warp == 0) tmem_alloc(&tbase, 256);
     if (tid == 0) {
@@ -194,13 +207,14 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     if (tid < 128) {
         int t;
         if (mode == 0) {
-            t = (int)(qbase - (size_t)bh * N) + tid;
+            t = seg0 + qt * 128 + tid;
         } else {
             t = ql[qt * 128 + tid];
             t = (t < 0 || t >= N) ? 0 : t;
         }
         qrow_s[tid] = t;
     }
+    stage_rows(kt0);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -214,37 +228,31 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         tc_fence_after();
         return __syncthreads_and(ok);
     };
-    const size_t hN = (size_t)bh * N;
-    // key rows of tile kt into krow_s (tokens within the head)
-    auto key_rows = [&](int kt) {
-        if (tid < 128) {
-            int t;
-            if (mode == 0) {
-                t = (int)(kbase - hN) + kt * 128 + tid;
-            } else {
-                t = kl[kt * 128 + tid];
-                t = (t < 0 || t >= N) ? 0 : t;
-            }
-            krow_s[tid] = t;
-        }
-    };
-    auto load_kv = [&]() {
+    // key rows of tile kt (tokens within the head); mode 1 reads them from
+    // the level's index list into krow_s[kt & 1] (then a barrier)
+    auto load_tile = [&](uint32_t dst, const uint16_t *src, int kt) {
         for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
             const int rr = i / (D / 8), c = i % (D / 8);
-            const size_t o = (hN + krow_s[rr]) * D + c * 8;
-            cp_async16(sKP + panel_offset(rr, c, 128), kx + o);
-            cp_async16(sV + panel_offset(rr, c, 128), vx + o);
+            const int t =
+                mode == 0 ? seg0 + kt * 128 + rr : krow_s[kt & 1][rr];
+            cp_async16(dst + panel_offset(rr, c, 128),
+                       src + (hN + t) * D + c * 8);
         }
-        cp_async_commit();
     };
-    key_rows(kt0);
-    __syncthreads();
+    auto wait_older = [&]() {  // all groups but the newest have landed
+        cp_async_wait<1>();
+        fence_proxy_async_smem();
+        __syncthreads();
+    };
     for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
         const int rr = i / (D / 8), c = i % (D / 8);
         cp_async16(sQ + panel_offset(rr, c, 128),
                    qx + (hN + qrow_s[rr]) * D + c * 8);
     }
-    load_kv();
+    load_tile(sK, kx, kt0);
+    cp_async_commit();
+    load_tile(sV, vx, kt0);
+    cp_async_commit();
 
     float o_acc[DH];
 #pragma unroll
@@ -254,9 +262,7 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     bool ok = true;
     for (int it = 0; it < nkt && ok; ++it) {
         const int kt = kt0 + it;
-        cp_async_wait<0>();
-        fence_proxy_async_smem();
-        __syncthreads();
+        wait_older();  // K of this tile
         if (tid == 0) {
             tc_fence_after();
             const uint32_t id = idesc_bf16(128, 128, false, false);
@@ -264,21 +270,29 @@ __global__ void __launch_bounds__(kCaThreads, 2)
             for (int k = 0; k < D / 16; ++k)
                 mma_ss(tm, smem_desc(sQ + (k >> 2) * 16384 + (k & 3) * 32, 16,
                                      1024),
-                       smem_desc(sKP + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                       smem_desc(sK + (k >> 2) * 16384 + (k & 3) * 32, 16,
                                  1024),
                        id, k > 0);
         }
         if (!(ok = mma_done(120))) break;
+        if (it + 1 < nkt) {
+            if (mode == 1) {
+                stage_rows(kt + 1);
+                __syncthreads();
+            }
+            load_tile(sK, kx, kt + 1);
+        }
+        cp_async_commit();
 
-        // ---- scale, mask, running max, P (each thread's 64 key columns
-        // in two 32-column passes over TMEM: max first, then exp)
+        // ---- running max (two 32-column passes over the raw scores; the
+        // scale is positive), then P = 2^(scale log2e S - max) packed over
+        // the scores already read. Masks only on the diagonal tile (mode 0)
+        // or with several blocks per tile (mode 1, b < 128).
         const bool diag = mode == 0 && kt == qt;
-        auto masked = [&](const uint32_t(&v)[32], int j0, int j) -> float {
-            const int c = 64 * half + j0 + j;
-            bool keep = true;
-            if (diag) keep = c <= row;
-            if (mode == 1 && b < 128) keep = (c / b) == (row / b);
-            return keep ? __uint_as_float(v[j]) * sl2 : -INFINITY;
+        const bool blockmask = mode == 1 && b < 128;
+        const bool any_mask = diag || blockmask;
+        auto keep = [&](int c) -> bool {
+            return diag ? c <= row : (c / b) == (row / b);
         };
         float mx = -INFINITY;
 #pragma unroll
@@ -286,55 +300,64 @@ __global__ void __launch_bounds__(kCaThreads, 2)
             uint32_t v[32];
             tmem_ld32(tm + lane + 64 * half + j0, v);
             tmem_wait_ld();
+            if (any_mask) {
 #pragma unroll
-            for (int j = 0; j < 32; ++j) mx = fmaxf(mx, masked(v, j0, j));
+                for (int j = 0; j < 32; ++j)
+                    if (keep(64 * half + j0 + j))
+                        mx = fmaxf(mx, __uint_as_float(v[j]));
+            } else {
+#pragma unroll
+                for (int j = 0; j < 32; ++j)
+                    mx = fmaxf(mx, __uint_as_float(v[j]));
+            }
         }
-        xm[half][row] = mx;
+        xm[half][row] = mx * sl2;  // -inf stays -inf
         __syncthreads();
         const float mnew = fmaxf(mrun, fmaxf(xm[0][row], xm[1][row]));
-        const float alpha = exp2f(mrun - mnew);  // 0 on the first tile
+        const float alpha = ex2_approx(mrun - mnew);  // 0 on the first tile
         float ls = 0.0f;
 #pragma unroll
         for (int j0 = 0; j0 < 64; j0 += 32) {
             uint32_t v[32];
             tmem_ld32(tm + lane + 64 * half + j0, v);
             tmem_wait_ld();
+            uint32_t pk[16];
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                float p[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    p[e] = exp2f(masked(v, j0, 8 * q + e) - mnew);
-                    ls += p[e];
+            for (int j = 0; j < 32; j += 2) {
+                float a0 = ex2_approx(fmaf(__uint_as_float(v[j]), sl2, -mnew));
+                float a1 =
+                    ex2_approx(fmaf(__uint_as_float(v[j + 1]), sl2, -mnew));
+                if (any_mask) {
+                    a0 = keep(64 * half + j0 + j) ? a0 : 0.0f;
+                    a1 = keep(64 * half + j0 + j + 1) ? a1 : 0.0f;
                 }
-                st_shared_bf16x8(
-                    sKP + panel_offset(row, 8 * half + j0 / 8 + q, 128), p);
+                ls += a0 + a1;
+                pk[j >> 1] = pack_bf16x2(a0, a1);
             }
+            // over scores of this thread's half already read
+            tmem_st16(tm + lane + 64 * half + j0 / 2, pk);
         }
+        tmem_wait_st();
         xl[half][row] = ls;
-        fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
         lrun = lrun * alpha + xl[0][row] + xl[1][row];
         mrun = mnew;
 
-        // ---- P V
+        // ---- P V (P from TMEM: keys 16 k.. of half k / 4 sit at columns
+        // 64 (k / 4) + 8 (k % 4))
+        wait_older();  // V of this tile
         if (tid == 0) {
             tc_fence_after();
             const uint32_t id = idesc_bf16(128, D, false, true);
 #pragma unroll
             for (int k = 0; k < 8; ++k)
-                mma_ss(tm + 128,
-                       smem_desc(sKP + (k >> 2) * 16384 + (k & 3) * 32, 16,
-                                 1024),
+                mma_ts(tm + 128, tm + (uint32_t)(64 * (k >> 2) + 8 * (k & 3)),
                        smem_desc(sV + k * 2048, 16384, 1024), id, k > 0);
         }
         if (!(ok = mma_done(121))) break;
-        if (it + 1 < nkt) {  // next key tile (K and V buffers are free)
-            key_rows(kt + 1);
-            __syncthreads();
-            load_kv();
-        }
+        if (it + 1 < nkt) load_tile(sV, vx, kt + 1);
+        cp_async_commit();
 #pragma unroll
         for (int c = 0; c < DH; c += 32) {
             uint32_t v[32];
@@ -354,7 +377,7 @@ __global__ void __launch_bounds__(kCaThreads, 2)
 
     // ---- O = sum e^z V / (sum e^z + eps), log d (natural log)
     const float logd = (mrun + log2f(lrun)) * kLn2;
-    const float inv = 1.0f / (lrun + eps * exp2f(-mrun));
+    const float inv = 1.0f / (lrun + eps * ex2_approx(-mrun));
     const size_t tok = hN + qrow_s[row];
     float *o = RO + tok * D + half * DH;
     if (mode == 0) {
@@ -549,28 +572,25 @@ __global__ void __launch_bounds__(kCaThreads, 1)
         for (int t = 0; t < TPT; ++t) {
             const int tl = half * TPT + t;       // table within the group
             const int tbl = g * (RB / R) + tl;  // table
-            float spq[G], snq[G], spk[G], snk[G];
+            // per-bit factors sigma(2 beta tanh u) = 1/2 + tanh(beta tanh u)/2
+            float spq[G], spk[G];
 #pragma unroll
             for (int bb = 0; bb < G; ++bb) {
-                race_bit_factors(pick(uq, t * G + bb), beta, spq[bb],
-                                 snq[bb]);
-                race_bit_factors(pick(uk, t * G + bb), beta, spk[bb],
-                                 snk[bb]);
+                spq[bb] = fmaf(0.5f,
+                               tanh_approx(beta * tanh_approx(
+                                                      pick(uq, t * G + bb))),
+                               0.5f);
+                spk[bb] = fmaf(0.5f,
+                               tanh_approx(beta * tanh_approx(
+                                                      pick(uk, t * G + bb))),
+                               0.5f);
             }
             float pq[R], pk[R];
+            table_phi<G>(spq, pq);
+            table_phi<G>(spk, pk);
 #pragma unroll
-            for (int rr = 0; rr < R; ++rr) {
-                float a = 1.0f, c = 1.0f;
-#pragma unroll
-                for (int bb = 0; bb < G; ++bb) {
-                    const bool on = (rr >> bb) & 1;
-                    a *= on ? spq[bb] : snq[bb];
-                    c *= on ? spk[bb] : snk[bb];
-                }
-                pq[rr] = a;
-                pk[rr] = c;
-                den_inter = fmaf(a, sAf[tbl * R + rr], den_inter);
-            }
+            for (int rr = 0; rr < R; ++rr)
+                den_inter = fmaf(pq[rr], sAf[tbl * R + rr], den_inter);
             const int col = tl * R;  // bucket within the group
             st_shared_bf16x8(sQ + panel_offset(row, col / 8, 128), pq);
             st_shared_bf16x8(sQ + panel_offset(row, col / 8 + 1, 128), pq + 8);
@@ -647,7 +667,8 @@ __global__ void __launch_bounds__(kCaThreads, 1)
         const float gl = gates ? gates[2 * tok + 1] : 1.0f;
         const float mm = fusion_multiplier(log_ds, lam, den, eps, mode);
         const float cs = gs * mm, cl = gl * invL * rl;
-        const float *os = RO + tok * D + half * DH;
+        const float4 *os =
+            reinterpret_cast<const float4 *>(RO + tok * D + half * DH);
         uint16_t *o = ox + tok * D + half * DH;
 #pragma unroll
         for (int c = 0; c < DH; c += 32) {
@@ -656,11 +677,13 @@ __global__ void __launch_bounds__(kCaThreads, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int j = 0; j < 32; j += 8) {
+                const float4 s0 = os[(c + j) / 4], s1 = os[(c + j) / 4 + 1];
+                const float sv[8] = {s0.x, s0.y, s0.z, s0.w,
+                                     s1.x, s1.y, s1.z, s1.w};
                 float y[8];
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
-                    y[e] = cs * os[c + j + e] +
-                           cl * __uint_as_float(v[j + e]);
+                    y[e] = cs * sv[e] + cl * __uint_as_float(v[j + e]);
                 uint4 pk;
                 pk.x = pack_bf16x2(y[0], y[1]);
                 pk.y = pack_bf16x2(y[2], y[3]);
@@ -694,10 +717,7 @@ bool causal_tc_supported(const Plan &P, int n_leaf) {
     return true;
 }
 
-size_t causal_attn_smem(int d) {
-    const size_t tile = (size_t)128 * d * 2;
-    return 1024 + tile + (tile > 32768 ? tile : 32768) + tile;
-}
+size_t causal_attn_smem(int d) { return 1024 + (size_t)3 * 128 * d * 2; }
 
 size_t causal_race_smem(const Plan &P) {
     const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
