@@ -608,6 +608,7 @@ constexpr uint32_t kKU = 0;     // projections [0, 32)
 constexpr uint32_t kKdV = 32;   // phi gB
 constexpr uint32_t kKG = 96;    // V gB^T (r <= 128)
 constexpr uint32_t kKdK = 224;  // dL/du W
+constexpr uint32_t kOldRow = 272; // bytes per staged fp32 dV / dK row
 
 template <int L>
 __global__ void __launch_bounds__(kBtThreads, 1)
@@ -642,6 +643,11 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     const uint32_t sgB = sPhi + align1k(kBtT * r * 2);  // [r x 64]
     const uint32_t sDU = sgB + align1k(r * 128);      // [128 x 64]
     const uint32_t sAo = sDU + 16384;                 // fp32 gA [r]
+    // fp32 dV, dK rows of the tile as the block kernel left them, rows of
+    // 272 bytes (16-byte pad: a warp's 16-byte reads of 8 rows hit distinct
+    // bank groups)
+    const uint32_t sDVo = sAo + (uint32_t)r * 4;
+    const uint32_t sDKo = sDVo + kBtT * kOldRow;
     const float *gAs =
         reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
 
@@ -671,20 +677,45 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         st_shared_bf16x8(region + panel_offset(rr, chunk, rows), v);
     };
 
+    // cp.async groups, in commit order: K and V of the first tile; then per
+    // tile t: [planes, gB, gA on a head change,] old dV, dK of t; K of
+    // t + 1; V of t + 1 (empty past the last tile). "All but the newest
+    // group" is then always the operand about to be used.
+    auto tile_row0 = [&](long tt) {
+        const int bh = (int)(tt / tiles_per_head);
+        return (size_t)bh * N +
+               (size_t)(tt - (long)bh * tiles_per_head) * kBtT;
+    };
+    auto load_k = [&](long tt) {
+        const size_t r0 = tile_row0(tt);
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            cp_async16(sKW + panel_offset(rr, c, NR),
+                       kx + (r0 + rr) * d + c * 8);
+        }
+    };
+    auto load_v = [&](long tt) {
+        const size_t r0 = tile_row0(tt);
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            cp_async16(sV + panel_offset(rr, c, kBtT),
+                       vx + (r0 + rr) * d + c * 8);
+        }
+    };
+    if (t_begin < t_end) {
+        load_k(t_begin);
+        load_v(t_begin);
+    }
+    cp_async_commit();
+
     int cur_bh = -1;
     bool ok = true;
     for (long tt = t_begin; tt < t_end && ok; ++tt) {
         const int bh = (int)(tt / tiles_per_head);
-        const int k0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
         const int h = bh % H;
-        const size_t row0 = (size_t)bh * N + k0;
-        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
-            const int rr = i >> 3, c = i & 7;
-            const size_t o = (row0 + rr) * d + c * 8;
-            cp_async16(sKW + panel_offset(rr, c, NR), kx + o);
-            cp_async16(sV + panel_offset(rr, c, kBtT), vx + o);
-        }
-        if (bh != cur_bh) {  // the head's planes, gB (bf16) and gA
+        const size_t row0 = tile_row0(tt);
+        const bool new_head = bh != cur_bh;
+        if (new_head) {  // the head's planes, gB (bf16) and gA
             for (int i = tid; i < Lg_pad * 8; i += kBtThreads) {
                 const int rr = i >> 3, c = i & 7;
                 cp_async16(sKW + panel_offset(kBtT + rr, c, NR),
@@ -697,10 +728,22 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             }
             for (int i = tid; i < r / 4; i += kBtThreads)
                 cp_async16(sAo + 16 * i, gAg + (size_t)bh * r + 4 * i);
+            cp_async_commit();
             cur_bh = bh;
         }
+        // old dV, dK rows of this tile (read back in the epilogues)
+        for (int i = tid; i < kBtT * 16; i += kBtThreads) {
+            const int rr = i >> 4, c = i & 15;
+            cp_async16(sDVo + rr * kOldRow + c * 16,
+                       dv + (row0 + rr) * d + c * 4);
+            cp_async16(sDKo + rr * kOldRow + c * 16,
+                       dk + (row0 + rr) * d + c * 4);
+        }
         cp_async_commit();
-        cp_async_wait<0>();
+        if (new_head)
+            cp_async_wait<0>();
+        else
+            cp_async_wait<1>();  // K and V of this tile
         fence_proxy_async_smem();
         __syncthreads();
 
@@ -715,6 +758,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        k > 0);
         }
         if (!(ok = mma_done(90))) break;
+        if (tt + 1 < t_end) load_k(tt + 1);  // this tile's K is consumed
+        cp_async_commit();
 
         // features of this half's tables
         float u[2 * L > 16 ? 16 : 2 * L];
@@ -765,6 +810,10 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        smem_desc(sgB + k * 32, 16, 1024), id_g, k > 0);
         }
         if (!(ok = mma_done(91))) break;
+        cp_async_wait<1>();  // old dV, dK rows of this tile
+        __syncthreads();
+        if (tt + 1 < t_end) load_v(tt + 1);  // this tile's V is consumed
+        cp_async_commit();
 
         const size_t key = row0 + row;
         {
@@ -772,9 +821,12 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             tmem_ld32(tm + lane + kKdV + 32 * half, v);
             tmem_wait_ld();
             float4 *o4 = reinterpret_cast<float4 *>(dv + key * d + 32 * half);
+            const float4 *p4 = reinterpret_cast<const float4 *>(
+                smem_raw + (sDVo - smem_u32(smem_raw)) + row * kOldRow +
+                128 * half);
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
-                float4 a = o4[q];
+                float4 a = p4[q];
                 a.x += __uint_as_float(v[4 * q]);
                 a.y += __uint_as_float(v[4 * q + 1]);
                 a.z += __uint_as_float(v[4 * q + 2]);
@@ -843,9 +895,12 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             tmem_ld32(tm + lane + kKdK + 32 * half, v);
             tmem_wait_ld();
             float4 *o4 = reinterpret_cast<float4 *>(dk + key * d + 32 * half);
+            const float4 *p4 = reinterpret_cast<const float4 *>(
+                smem_raw + (sDKo - smem_u32(smem_raw)) + row * kOldRow +
+                128 * half);
 #pragma unroll
             for (int q = 0; q < 8; ++q) {
-                float4 a = o4[q];
+                float4 a = p4[q];
                 a.x += __uint_as_float(v[4 * q]);
                 a.y += __uint_as_float(v[4 * q + 1]);
                 a.z += __uint_as_float(v[4 * q + 2]);
@@ -856,6 +911,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         tc_fence_before();
         __syncthreads();
     }
+    cp_async_wait<0>();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tm, 512);
@@ -944,7 +1000,7 @@ size_t bwd_keys_tc_smem(const Plan &P) {
     const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
     auto a1k = [](size_t x) { return (x + 1023) / 1024 * 1024; };
     return 1024 + a1k((kBtT + lg_pad) * 128) + 16384 + a1k(kBtT * r * 2) +
-           a1k(r * 128) + 16384 + r * 4;
+           a1k(r * 128) + 16384 + r * 4 + 2 * kBtT * kOldRow;
 }
 
 cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
