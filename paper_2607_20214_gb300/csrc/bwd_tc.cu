@@ -102,7 +102,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     __shared__ uint32_t tbase;
     __shared__ int abort_flag;
     __shared__ float xa[2][kBtT], xb[2][kBtT], xc[2][kBtT];
-    __shared__ int qrow_s[kBtT], krow_s[kBtT];
+    __shared__ int qrow2[2][kBtT], krow2[2][kBtT];  // by tile parity
     volatile int *abort = &abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
     const int half = warp >> 2;
@@ -157,31 +157,65 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                       v);
     };
 
+    // Rows of tile tt (sorted positions -> original rows) into the index
+    // arrays of parity tt & 1. The next tile's copies start as soon as
+    // their buffers are free: dO after phase 4, V after phase 5, Q and K
+    // after phase 7; the top of each tile waits for every copy.
+    auto stage_rows = [&](long tt) {
+        if (tid < kBtT) {
+            const int bh = (int)(tt / tiles_per_head);
+            const size_t hb = (size_t)bh * N;
+            const int p0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
+            int qi = perm_q[hb + p0 + tid], ki = perm_k[hb + p0 + tid];
+            qi = (qi < 0 || qi >= N) ? 0 : qi;
+            ki = (ki < 0 || ki >= N) ? 0 : ki;
+            qrow2[tt & 1][tid] = (int)(hb + qi);
+            krow2[tt & 1][tid] = (int)(hb + ki);
+        }
+    };
+    auto load_qk = [&](long tt) {
+        const int *qr = qrow2[tt & 1], *kr = krow2[tt & 1];
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            cp_async16(sQ + panel_offset(rr, c, kBtT),
+                       qx + (size_t)qr[rr] * d + c * 8);
+            cp_async16(sKW + panel_offset(rr, c, NR),
+                       kx + (size_t)kr[rr] * d + c * 8);
+        }
+    };
+    auto load_g = [&](long tt) {
+        const int *qr = qrow2[tt & 1];
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            cp_async16(sG + panel_offset(rr, c, kBtT),
+                       gx + (size_t)qr[rr] * d + c * 8);
+        }
+    };
+    auto load_v = [&](long tt) {
+        const int *kr = krow2[tt & 1];
+        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            cp_async16(sV + panel_offset(rr, c, kBtT),
+                       vx + (size_t)kr[rr] * d + c * 8);
+        }
+    };
+    if (t_begin < t_end) {
+        stage_rows(t_begin);
+        __syncthreads();
+        load_qk(t_begin);
+        load_g(t_begin);
+        load_v(t_begin);
+        cp_async_commit();
+    }
+
     int cur_bh = -1;
     bool ok = true;
     for (long tt = t_begin; tt < t_end && ok; ++tt) {
         const int bh = (int)(tt / tiles_per_head);
-        const int p0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
         const int h = bh % H;
-        const size_t hb = (size_t)bh * N;
+        const int *qrow_s = qrow2[tt & 1], *krow_s = krow2[tt & 1];
+        const bool more = tt + 1 < t_end;
         // ---------------------------------------------------- phase 0: load
-        if (tid < kBtT) {
-            int qi = perm_q[hb + p0 + tid], ki = perm_k[hb + p0 + tid];
-            qi = (qi < 0 || qi >= N) ? 0 : qi;
-            ki = (ki < 0 || ki >= N) ? 0 : ki;
-            qrow_s[tid] = (int)(hb + qi);
-            krow_s[tid] = (int)(hb + ki);
-        }
-        __syncthreads();
-        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
-            const int rr = i >> 3, c = i & 7;
-            const size_t qo = (size_t)qrow_s[rr] * d + c * 8;
-            const size_t ko = (size_t)krow_s[rr] * d + c * 8;
-            cp_async16(sQ + panel_offset(rr, c, kBtT), qx + qo);
-            cp_async16(sG + panel_offset(rr, c, kBtT), gx + qo);
-            cp_async16(sKW + panel_offset(rr, c, NR), kx + ko);
-            cp_async16(sV + panel_offset(rr, c, kBtT), vx + ko);
-        }
         if (bh != cur_bh) {  // the head's planes, B summary (bf16) and A
             for (int i = tid; i < Lg_pad * 8; i += kBtThreads) {
                 const int rr = i >> 3, c = i & 7;
@@ -199,6 +233,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         }
         cp_async_commit();
         cp_async_wait<0>();
+        if (more) stage_rows(tt + 1);  // the next tile's rows, parity flips
         fence_proxy_async_smem();
         __syncthreads();
 
@@ -380,6 +415,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
+        if (more) load_g(tt + 1);  // dO of this tile was read in phase 4
+        cp_async_commit();
 
         // ------------- phase 5: E^T X, X V^T, gNum B^T, phi^T [gNum | gDen]
         const bool seg_first = tt == t_begin || (tt % tiles_per_head) == 0;
@@ -412,6 +449,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        (k > 0 || !seg_first) ? 1u : 0u);
         }
         if (!(ok = mma_done(82))) break;
+        if (more) load_v(tt + 1);  // V's last reader (P = X V^T) is done
+        cp_async_commit();
         if (seg_last && row < r) {  // this CTA's share of the head's sums
             const long j = (long)blockIdx.x -
                            tile_owner((long)bh * tiles_per_head, total_tiles,
@@ -532,6 +571,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        smem_desc(sQ + k * 2048, 16384, 1024), id_k, k > 0);
         }
         if (!(ok = mma_done(83))) break;
+        if (more) load_qk(tt + 1);  // Q and K's last readers are done
+        cp_async_commit();
 
         // ------------------------------------------- phase 8: dQ, dK stores
         {
@@ -558,6 +599,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         tc_fence_before();
         __syncthreads();  // TMEM and shared memory are reused by the next tile
     }
+    cp_async_wait<0>();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tm, 512);
