@@ -129,14 +129,14 @@ __global__ void __launch_bounds__(kSegThreads)
 // cp.async groups are committed in a fixed order (Q and K0, V0, then per
 // tile: next K, next V; empty groups past the last tile), so "all but the
 // newest group done" always means the operand about to be used has landed.
-template <int D>
+template <int D, int MODE>
 __global__ void __launch_bounds__(kCaThreads, 2)
     k_causal_attn_tc(const uint16_t *__restrict__ qx,
                      const uint16_t *__restrict__ kx,
                      const uint16_t *__restrict__ vx,
                      const int32_t *__restrict__ permq,
-                     const int32_t *__restrict__ permk, int N, int mode,
-                     int n_leaf, int m, int b, float scale, float eps,
+                     const int32_t *__restrict__ permk, int N, int n_leaf,
+                     int m, int b, int items, float scale, float eps,
                      float *__restrict__ RO, float *__restrict__ RL,
                      DeviceStatus *status) {
     extern __shared__ unsigned char smem_raw[];
@@ -145,7 +145,7 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     __shared__ int abort_flag;
     __shared__ float xm[2][128], xl[2][128];
     __shared__ int qrow_s[128];
-    __shared__ int krow_s[2][128];  // mode 1: key rows of the next tiles
+    __shared__ int krow_s[2][128];  // MODE 1: key rows of the next tiles
     volatile int *abort = &abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
     const int half = warp >> 2;
@@ -159,62 +159,12 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     const uint32_t sK = sQ + kTileB;
     const uint32_t sV = sK + kTileB;
 
-    // ---- work item
-    int bh, qt, nkt, kt0;
-    int seg0 = 0;  // mode 0: first row of the segment (within the head)
-    const int32_t *ql = nullptr, *kl = nullptr;
-    if (mode == 0) {
-        const int nq = n_leaf / 128, nleaves = N / n_leaf;
-        const int item = blockIdx.x;
-        qt = nq - 1 - item % nq;  // longest rows first
-        const int rest = item / nq;
-        const int leaf = rest % nleaves;
-        bh = rest / nleaves;
-        seg0 = leaf * n_leaf;
-        kt0 = 0;
-        nkt = qt + 1;
-    } else {
-        const int tpn = m / 128, nodes = N / (2 * m);
-        const int item = blockIdx.x;
-        qt = item % tpn;
-        const int rest = item / tpn;
-        const int j = rest % nodes;
-        bh = rest / nodes;
-        ql = permq + (size_t)bh * (N >> 1) + (size_t)j * m;
-        kl = permk + (size_t)bh * (N >> 1) + (size_t)j * m;
-        if (b >= 128) {
-            kt0 = (qt * 128 / b) * (b / 128);
-            nkt = b / 128;
-        } else {
-            kt0 = qt;
-            nkt = 1;
-        }
-    }
-    const size_t hN = (size_t)bh * N;
-    auto stage_rows = [&](int kt) {
-        if (mode == 1 && tid < 128) {
-            const int t = kl[kt * 128 + tid];
-            krow_s[kt & 1][tid] = (t < 0 || t >= N) ? 0 : t;
-        }
-    };
-
     if (warp == 0) tmem_alloc(&tbase, 256);
     if (tid == 0) {
         mbar_init(&mma_bar, 1);
         abort_flag = 0;
         fence_mbar_init();
     }
-    if (tid < 128) {
-        int t;
-        if (mode == 0) {
-            t = seg0 + qt * 128 + tid;
-        } else {
-            t = ql[qt * 128 + tid];
-            t = (t < 0 || t >= N) ? 0 : t;
-        }
-        qrow_s[tid] = t;
-    }
-    stage_rows(kt0);
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -228,185 +178,246 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         tc_fence_after();
         return __syncthreads_and(ok);
     };
-    // key rows of tile kt (tokens within the head); mode 1 reads them from
-    // the level's index list into krow_s[kt & 1] (then a barrier)
-    auto load_tile = [&](uint32_t dst, const uint16_t *src, int kt) {
-        for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
-            const int rr = i / (D / 8), c = i % (D / 8);
-            const int t =
-                mode == 0 ? seg0 + kt * 128 + rr : krow_s[kt & 1][rr];
-            cp_async16(dst + panel_offset(rr, c, 128),
-                       src + (hN + t) * D + c * 8);
-        }
-    };
-    auto wait_older = [&]() {  // all groups but the newest have landed
-        cp_async_wait<1>();
-        fence_proxy_async_smem();
-        __syncthreads();
-    };
-    for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
-        const int rr = i / (D / 8), c = i % (D / 8);
-        cp_async16(sQ + panel_offset(rr, c, 128),
-                   qx + (hN + qrow_s[rr]) * D + c * 8);
-    }
-    load_tile(sK, kx, kt0);
-    cp_async_commit();
-    load_tile(sV, vx, kt0);
-    cp_async_commit();
-
-    float o_acc[DH];
-#pragma unroll
-    for (int j = 0; j < DH; ++j) o_acc[j] = 0.0f;
-    float mrun = -INFINITY, lrun = 0.0f;  // log2 domain running max, sum
     const float sl2 = scale * kLog2e;
     bool ok = true;
-    for (int it = 0; it < nkt && ok; ++it) {
-        const int kt = kt0 + it;
-        wait_older();  // K of this tile
-        if (tid == 0) {
-            tc_fence_after();
-            const uint32_t id = idesc_bf16(128, 128, false, false);
-#pragma unroll
-            for (int k = 0; k < D / 16; ++k)
-                mma_ss(tm, smem_desc(sQ + (k >> 2) * 16384 + (k & 3) * 32, 16,
-                                     1024),
-                       smem_desc(sK + (k >> 2) * 16384 + (k & 3) * 32, 16,
-                                 1024),
-                       id, k > 0);
-        }
-        if (!(ok = mma_done(120))) break;
-        if (it + 1 < nkt) {
-            if (mode == 1) {
-                stage_rows(kt + 1);
-                __syncthreads();
-            }
-            load_tile(sK, kx, kt + 1);
-        }
-        cp_async_commit();
 
-        // ---- running max (two 32-column passes over the raw scores; the
-        // scale is positive), then P = 2^(scale log2e S - max) packed over
-        // the scores already read. Masks only on the diagonal tile (mode 0)
-        // or with several blocks per tile (mode 1, b < 128).
-        const bool diag = mode == 0 && kt == qt;
-        const bool blockmask = mode == 1 && b < 128;
-        const bool any_mask = diag || blockmask;
-        auto keep = [&](int c) -> bool {
-            return diag ? c <= row : (c / b) == (row / b);
-        };
-        float mx = -INFINITY;
-#pragma unroll
-        for (int j0 = 0; j0 < 64; j0 += 32) {
-            uint32_t v[32];
-            tmem_ld32(tm + lane + 64 * half + j0, v);
-            tmem_wait_ld();
-            if (any_mask) {
-#pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    if (keep(64 * half + j0 + j))
-                        mx = fmaxf(mx, __uint_as_float(v[j]));
+    // persistent CTAs: items blockIdx.x, + gridDim.x, ...
+    for (int item = blockIdx.x; item < items && ok; item += gridDim.x) {
+        // ---- work item
+        int bh, qt, nkt, kt0;
+        int seg0 = 0;  // MODE 0: first row of the segment (within the head)
+        const int32_t *ql = nullptr, *kl = nullptr;
+        if (MODE == 0) {
+            const int nq = n_leaf / 128, nleaves = N / n_leaf;
+            qt = nq - 1 - item % nq;  // longest rows first
+            const int rest = item / nq;
+            const int leaf = rest % nleaves;
+            bh = rest / nleaves;
+            seg0 = leaf * n_leaf;
+            kt0 = 0;
+            nkt = qt + 1;
+        } else {
+            const int tpn = m / 128, nodes = N / (2 * m);
+            qt = item % tpn;
+            const int rest = item / tpn;
+            const int j = rest % nodes;
+            bh = rest / nodes;
+            ql = permq + (size_t)bh * (N >> 1) + (size_t)j * m;
+            kl = permk + (size_t)bh * (N >> 1) + (size_t)j * m;
+            if (b >= 128) {
+                kt0 = (qt * 128 / b) * (b / 128);
+                nkt = b / 128;
             } else {
+                kt0 = qt;
+                nkt = 1;
+            }
+        }
+        const size_t hN = (size_t)bh * N;
+        // key rows of tile kt (tokens within the head); MODE 1 reads them
+        // from the level's index list into krow_s[kt & 1] (then a barrier)
+        auto stage_rows = [&](int kt) {
+            if (MODE == 1 && tid < 128) {
+                const int t = kl[kt * 128 + tid];
+                krow_s[kt & 1][tid] = (t < 0 || t >= N) ? 0 : t;
+            }
+        };
+        auto load_tile = [&](uint32_t dst, const uint16_t *src, int kt) {
+            for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+                const int rr = i / (D / 8), c = i % (D / 8);
+                const int t =
+                    MODE == 0 ? seg0 + kt * 128 + rr : krow_s[kt & 1][rr];
+                cp_async16(dst + panel_offset(rr, c, 128),
+                           src + (hN + t) * D + c * 8);
+            }
+        };
+        auto wait_older = [&]() {  // all groups but the newest have landed
+            cp_async_wait<1>();
+            fence_proxy_async_smem();
+            __syncthreads();
+        };
+        if (tid < 128) {
+            int t;
+            if (MODE == 0) {
+                t = seg0 + qt * 128 + tid;
+            } else {
+                t = ql[qt * 128 + tid];
+                t = (t < 0 || t >= N) ? 0 : t;
+            }
+            qrow_s[tid] = t;
+        }
+        stage_rows(kt0);
+        __syncthreads();
+        for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+            const int rr = i / (D / 8), c = i % (D / 8);
+            cp_async16(sQ + panel_offset(rr, c, 128),
+                       qx + (hN + qrow_s[rr]) * D + c * 8);
+        }
+        load_tile(sK, kx, kt0);
+        cp_async_commit();
+        load_tile(sV, vx, kt0);
+        cp_async_commit();
+
+        float o_acc[DH];
+#pragma unroll
+        for (int j = 0; j < DH; ++j) o_acc[j] = 0.0f;
+        float mrun = -INFINITY, lrun = 0.0f;  // log2 domain max, sum
+        for (int it = 0; it < nkt && ok; ++it) {
+            const int kt = kt0 + it;
+            wait_older();  // K of this tile
+            if (tid == 0) {
+                tc_fence_after();
+                const uint32_t id = idesc_bf16(128, 128, false, false);
+#pragma unroll
+                for (int k = 0; k < D / 16; ++k)
+                    mma_ss(tm,
+                           smem_desc(sQ + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                     1024),
+                           smem_desc(sK + (k >> 2) * 16384 + (k & 3) * 32, 16,
+                                     1024),
+                           id, k > 0);
+            }
+            if (!(ok = mma_done(120))) break;
+            if (it + 1 < nkt) {
+                if (MODE == 1) {
+                    stage_rows(kt + 1);
+                    __syncthreads();
+                }
+                load_tile(sK, kx, kt + 1);
+            }
+            cp_async_commit();
+
+            // ---- running max (two 32-column passes over the raw scores;
+            // the scale is positive), then P = 2^(scale log2e S - max)
+            // packed over the scores already read. Masks only on the
+            // diagonal tile (MODE 0) or with several blocks per tile
+            // (MODE 1, b < 128).
+            const bool any_mask = MODE == 0 ? kt == qt : b < 128;
+            // kept key columns [klo, khi) of this row: the causal prefix of
+            // the diagonal tile, or the row's own block
+            const int klo = MODE == 0 ? 0 : (row / b) * b;
+            const int khi = MODE == 0 ? row + 1 : klo + b;
+            auto keep = [&](int c) -> bool { return c >= klo && c < khi; };
+            float mx = -INFINITY;
+#pragma unroll
+            for (int j0 = 0; j0 < 64; j0 += 32) {
+                uint32_t v[32];
+                tmem_ld32(tm + lane + 64 * half + j0, v);
+                tmem_wait_ld();
+                if (any_mask) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (keep(64 * half + j0 + j))
+                            mx = fmaxf(mx, __uint_as_float(v[j]));
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        mx = fmaxf(mx, __uint_as_float(v[j]));
+                }
+            }
+            xm[half][row] = mx * sl2;  // -inf stays -inf
+            __syncthreads();
+            const float mnew = fmaxf(mrun, fmaxf(xm[0][row], xm[1][row]));
+            const float alpha = ex2_approx(mrun - mnew);  // 0 on tile 0
+            float ls = 0.0f;
+#pragma unroll
+            for (int j0 = 0; j0 < 64; j0 += 32) {
+                uint32_t v[32];
+                tmem_ld32(tm + lane + 64 * half + j0, v);
+                tmem_wait_ld();
+                uint32_t pk[16];
+#pragma unroll
+                for (int j = 0; j < 32; j += 2) {
+                    float a0 =
+                        ex2_approx(fmaf(__uint_as_float(v[j]), sl2, -mnew));
+                    float a1 = ex2_approx(
+                        fmaf(__uint_as_float(v[j + 1]), sl2, -mnew));
+                    if (any_mask) {
+                        a0 = keep(64 * half + j0 + j) ? a0 : 0.0f;
+                        a1 = keep(64 * half + j0 + j + 1) ? a1 : 0.0f;
+                    }
+                    ls += a0 + a1;
+                    pk[j >> 1] = pack_bf16x2(a0, a1);
+                }
+                // over scores of this thread's half already read
+                tmem_st16(tm + lane + 64 * half + j0 / 2, pk);
+            }
+            tmem_wait_st();
+            xl[half][row] = ls;
+            tc_fence_before();
+            __syncthreads();
+            lrun = lrun * alpha + xl[0][row] + xl[1][row];
+            mrun = mnew;
+
+            // ---- P V (P from TMEM: keys 16 k.. of half k / 4 sit at
+            // columns 64 (k / 4) + 8 (k % 4))
+            wait_older();  // V of this tile
+            if (tid == 0) {
+                tc_fence_after();
+                const uint32_t id = idesc_bf16(128, D, false, true);
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_ts(tm + 128,
+                           tm + (uint32_t)(64 * (k >> 2) + 8 * (k & 3)),
+                           smem_desc(sV + k * 2048, 16384, 1024), id, k > 0);
+            }
+            if (!(ok = mma_done(121))) break;
+            if (it + 1 < nkt) load_tile(sV, vx, kt + 1);
+            cp_async_commit();
+#pragma unroll
+            for (int c = 0; c < DH; c += 32) {
+                uint32_t v[32];
+                tmem_ld32(tm + lane + 128 + half * DH + c, v);
+                tmem_wait_ld();
 #pragma unroll
                 for (int j = 0; j < 32; ++j)
-                    mx = fmaxf(mx, __uint_as_float(v[j]));
+                    o_acc[c + j] = o_acc[c + j] * alpha + __uint_as_float(v[j]);
             }
+            tc_fence_before();
         }
-        xm[half][row] = mx * sl2;  // -inf stays -inf
-        __syncthreads();
-        const float mnew = fmaxf(mrun, fmaxf(xm[0][row], xm[1][row]));
-        const float alpha = ex2_approx(mrun - mnew);  // 0 on the first tile
-        float ls = 0.0f;
-#pragma unroll
-        for (int j0 = 0; j0 < 64; j0 += 32) {
-            uint32_t v[32];
-            tmem_ld32(tm + lane + 64 * half + j0, v);
-            tmem_wait_ld();
-            uint32_t pk[16];
-#pragma unroll
-            for (int j = 0; j < 32; j += 2) {
-                float a0 = ex2_approx(fmaf(__uint_as_float(v[j]), sl2, -mnew));
-                float a1 =
-                    ex2_approx(fmaf(__uint_as_float(v[j + 1]), sl2, -mnew));
-                if (any_mask) {
-                    a0 = keep(64 * half + j0 + j) ? a0 : 0.0f;
-                    a1 = keep(64 * half + j0 + j + 1) ? a1 : 0.0f;
-                }
-                ls += a0 + a1;
-                pk[j >> 1] = pack_bf16x2(a0, a1);
-            }
-            // over scores of this thread's half already read
-            tmem_st16(tm + lane + 64 * half + j0 / 2, pk);
-        }
-        tmem_wait_st();
-        xl[half][row] = ls;
-        tc_fence_before();
-        __syncthreads();
-        lrun = lrun * alpha + xl[0][row] + xl[1][row];
-        mrun = mnew;
+        cp_async_wait<0>();
+        __syncthreads();  // the next item's copies reuse every buffer
+        if (!ok) break;
 
-        // ---- P V (P from TMEM: keys 16 k.. of half k / 4 sit at columns
-        // 64 (k / 4) + 8 (k % 4))
-        wait_older();  // V of this tile
-        if (tid == 0) {
-            tc_fence_after();
-            const uint32_t id = idesc_bf16(128, D, false, true);
+        // ---- O = sum e^z V / (sum e^z + eps), log d (natural log)
+        const float logd = (mrun + log2f(lrun)) * kLn2;
+        const float inv = 1.0f / (lrun + eps * ex2_approx(-mrun));
+        const size_t tok = hN + qrow_s[row];
+        float *o = RO + tok * D + half * DH;
+        float ld_new = logd;
+        if (MODE == 0) {
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-                mma_ts(tm + 128, tm + (uint32_t)(64 * (k >> 2) + 8 * (k & 3)),
-                       smem_desc(sV + k * 2048, 16384, 1024), id, k > 0);
+            for (int j = 0; j < DH; j += 4)
+                *reinterpret_cast<float4 *>(o + j) =
+                    make_float4(o_acc[j] * inv, o_acc[j + 1] * inv,
+                                o_acc[j + 2] * inv, o_acc[j + 3] * inv);
+            if (half == 0) RL[tok] = logd;
+        } else {
+            // MergeLSE(running = diag, this = off)
+            const float ld1 = RL[tok];
+            const float mu = fmaxf(ld1, logd);
+            const float w1 = __expf(ld1 - mu), w2 = __expf(logd - mu);
+            const float ssum = w1 + w2;
+            const float r = 1.0f / (ssum + eps);
+            const float c1 = w1 * r, c2 = w2 * inv * r;
+#pragma unroll
+            for (int j = 0; j < DH; j += 4) {
+                float4 a = *reinterpret_cast<float4 *>(o + j);
+                a.x = c1 * a.x + c2 * o_acc[j];
+                a.y = c1 * a.y + c2 * o_acc[j + 1];
+                a.z = c1 * a.z + c2 * o_acc[j + 2];
+                a.w = c1 * a.w + c2 * o_acc[j + 3];
+                *reinterpret_cast<float4 *>(o + j) = a;
+            }
+            ld_new = mu + __logf(ssum + eps);
         }
-        if (!(ok = mma_done(121))) break;
-        if (it + 1 < nkt) load_tile(sV, vx, kt + 1);
-        cp_async_commit();
-#pragma unroll
-        for (int c = 0; c < DH; c += 32) {
-            uint32_t v[32];
-            tmem_ld32(tm + lane + 128 + half * DH + c, v);
-            tmem_wait_ld();
-#pragma unroll
-            for (int j = 0; j < 32; ++j)
-                o_acc[c + j] = o_acc[c + j] * alpha + __uint_as_float(v[j]);
-        }
-        tc_fence_before();
+        __syncthreads();  // qrow_s is rewritten by the next item; both
+                          // halves read RL before it changes
+        if (MODE == 1 && half == 0) RL[tok] = ld_new;
     }
     cp_async_wait<0>();
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tm, 256);
-    if (!ok) return;
-
-    // ---- O = sum e^z V / (sum e^z + eps), log d (natural log)
-    const float logd = (mrun + log2f(lrun)) * kLn2;
-    const float inv = 1.0f / (lrun + eps * ex2_approx(-mrun));
-    const size_t tok = hN + qrow_s[row];
-    float *o = RO + tok * D + half * DH;
-    if (mode == 0) {
-#pragma unroll
-        for (int j = 0; j < DH; j += 4)
-            *reinterpret_cast<float4 *>(o + j) =
-                make_float4(o_acc[j] * inv, o_acc[j + 1] * inv,
-                            o_acc[j + 2] * inv, o_acc[j + 3] * inv);
-        if (half == 0) RL[tok] = logd;
-    } else {
-        // MergeLSE(running = diag, this = off)
-        const float ld1 = RL[tok];
-        const float mu = fmaxf(ld1, logd);
-        const float w1 = __expf(ld1 - mu), w2 = __expf(logd - mu);
-        const float ssum = w1 + w2;
-        const float r = 1.0f / (ssum + eps);
-        const float c1 = w1 * r, c2 = w2 * inv * r;
-#pragma unroll
-        for (int j = 0; j < DH; j += 4) {
-            float4 a = *reinterpret_cast<float4 *>(o + j);
-            a.x = c1 * a.x + c2 * o_acc[j];
-            a.y = c1 * a.y + c2 * o_acc[j + 1];
-            a.z = c1 * a.z + c2 * o_acc[j + 2];
-            a.w = c1 * a.w + c2 * o_acc[j + 3];
-            *reinterpret_cast<float4 *>(o + j) = a;
-        }
-        __syncthreads();  // both halves read RL before it changes
-        if (half == 0) RL[tok] = mu + __logf(ssum + eps);
-    }
 }
 
 // ---------------------------------------------------- RACE prefix states
@@ -750,19 +761,24 @@ cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
         pq = perms + lvl;
         pk = perms + lvl + (size_t)P.BH * (P.N / 2);
     }
-    // at most two CTAs per SM (each holds 256 TMEM columns)
+    // at most two CTAs per SM (each holds 256 TMEM columns); persistent
+    // CTAs, two per SM of a 152-SM GB300
     size_t smem = causal_attn_smem(P.d);
     if (smem < kSmemPerSM / 3 + 1024) smem = kSmemPerSM / 3 + 1024;
+    const int grid = items < 2 * 152 ? items : 2 * 152;
     auto launch = [&](auto kern) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-        kern<<<items, kCaThreads, smem, st>>>(
+        kern<<<grid, kCaThreads, smem, st>>>(
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v, pq,
-            pk, P.N, mode, n_leaf, m, P.b, P.scale, P.eps, RO, RL, status);
+            pk, P.N, n_leaf, m, P.b, items, P.scale, P.eps, RO, RL, status);
         return cudaGetLastError();
     };
-    return P.d == 128 ? launch(k_causal_attn_tc<128>)
-                      : launch(k_causal_attn_tc<64>);
+    if (P.d == 128)
+        return mode == 0 ? launch(k_causal_attn_tc<128, 0>)
+                         : launch(k_causal_attn_tc<128, 1>);
+    return mode == 0 ? launch(k_causal_attn_tc<64, 0>)
+                     : launch(k_causal_attn_tc<64, 1>);
 }
 
 cudaError_t launch_causal_prefix(const Plan &P, const float *part,
