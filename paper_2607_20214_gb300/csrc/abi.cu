@@ -303,7 +303,7 @@ struct CausalPlan {
     Plan Pc;  // P with RACE chunks of 128 keys
     int Lv, n_leaf;
     size_t off_status, off_keyrank, off_hist, off_perms, off_RO, off_RL,
-        off_part, off_sB, off_sA, off_W, total;
+        off_part, off_sB, off_sA, off_W, off_ctr, total;
 };
 
 int make_causal_plan(const elsaa_params *p, CausalPlan *C, const char **msg) {
@@ -368,6 +368,8 @@ int make_causal_plan(const elsaa_params *p, CausalPlan *C, const char **msg) {
     off = align_up(off + (size_t)P.BH * nc * P.r * sizeof(float), 256);
     C->off_W = off;
     off = align_up(off + (size_t)P.H * P.Lg_pad * P.d * sizeof(uint16_t), 256);
+    C->off_ctr = off;  // work counters of the attention launches
+    off = align_up(off + (size_t)(Lv + 1) * sizeof(int), 256);
     C->total = off;
     return ELSAA_OK;
 }
@@ -414,9 +416,13 @@ int causal_forward(const elsaa_params *params, const void *q, const void *k,
     uint16_t *sB = (uint16_t *)(ws + C.off_sB);
     float *sA = (float *)(ws + C.off_sA);
     uint16_t *Wbf = (uint16_t *)(ws + C.off_W);
+    int *ctr = (int *)(ws + C.off_ctr);
 
     ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
                        "status reset");
+    ELSAA_CHECK_LAUNCH(
+        cudaMemsetAsync(ctr, 0, (size_t)(C.Lv + 1) * sizeof(int), st),
+        "counter reset");
     // the low-rank branch needs no sort: chunk summaries and prefix states
     // on the side stream, joined back before the readout
     SideStream *side = nullptr;
@@ -451,16 +457,16 @@ int causal_forward(const elsaa_params *params, const void *q, const void *k,
                        "seg_sort");
     ELSAA_CHECK_LAUNCH(timed("causal_attn_base", st, [&] {
                            return launch_causal_attn(P, 0, C.n_leaf, 0, q, k,
-                                                     v, perms, RO, RL, status,
-                                                     st);
+                                                     v, perms, ctr, RO, RL,
+                                                     status, st);
                        }),
                        "causal_attn_base");
     for (int level = C.Lv; level >= 1; --level)
         ELSAA_CHECK_LAUNCH(timed("causal_attn_merge", st, [&] {
                                return launch_causal_attn(P, 1, C.n_leaf,
                                                          level, q, k, v,
-                                                         perms, RO, RL,
-                                                         status, st);
+                                                         perms, ctr + level,
+                                                         RO, RL, status, st);
                            }),
                            "causal_attn_merge");
     ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(st, side->join, 0), "join wait");

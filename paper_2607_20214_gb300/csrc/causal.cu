@@ -136,9 +136,9 @@ __global__ void __launch_bounds__(kCaThreads, 2)
                      const uint16_t *__restrict__ vx,
                      const int32_t *__restrict__ permq,
                      const int32_t *__restrict__ permk, int N, int n_leaf,
-                     int m, int b, int items, float scale, float eps,
-                     float *__restrict__ RO, float *__restrict__ RL,
-                     DeviceStatus *status) {
+                     int m, int b, int items, int *__restrict__ next_item,
+                     float scale, float eps, float *__restrict__ RO,
+                     float *__restrict__ RL, DeviceStatus *status) {
     extern __shared__ unsigned char smem_raw[];
     __shared__ uint64_t mma_bar;
     __shared__ uint32_t tbase;
@@ -146,6 +146,7 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     __shared__ float xm[2][128], xl[2][128];
     __shared__ int qrow_s[128];
     __shared__ int krow_s[2][128];  // MODE 1: key rows of the next tiles
+    __shared__ int item_s;
     volatile int *abort = &abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
     const int half = warp >> 2;
@@ -181,16 +182,24 @@ __global__ void __launch_bounds__(kCaThreads, 2)
     const float sl2 = scale * kLog2e;
     bool ok = true;
 
-    // persistent CTAs: items blockIdx.x, + gridDim.x, ...
-    for (int item = blockIdx.x; item < items && ok; item += gridDim.x) {
+    // persistent CTAs take items from a counter (items are numbered longest
+    // first, so the take order balances the CTAs)
+    while (ok) {
+        if (tid == 0) item_s = atomicAdd(next_item, 1);
+        __syncthreads();
+        const int item = item_s;
+        if (item >= items) break;
         // ---- work item
         int bh, qt, nkt, kt0;
         int seg0 = 0;  // MODE 0: first row of the segment (within the head)
         const int32_t *ql = nullptr, *kl = nullptr;
         if (MODE == 0) {
+            // item -> (row tile, segment, head), row tiles with the most key
+            // tiles first across all segments and heads
             const int nq = n_leaf / 128, nleaves = N / n_leaf;
-            qt = nq - 1 - item % nq;  // longest rows first
-            const int rest = item / nq;
+            const int per = items / nq;  // segments x heads
+            qt = nq - 1 - item / per;
+            const int rest = item % per;
             const int leaf = rest % nleaves;
             bh = rest / nleaves;
             seg0 = leaf * n_leaf;
@@ -748,8 +757,9 @@ cudaError_t launch_seg_sort(const Plan &P, int Lv, const uint32_t *keyrank,
 // `level` (1 = top) whose halves hold m = N / 2^level rows.
 cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
                                const void *q, const void *k, const void *v,
-                               const int32_t *perms, float *RO, float *RL,
-                               DeviceStatus *status, cudaStream_t st) {
+                               const int32_t *perms, int *next_item, float *RO,
+                               float *RL, DeviceStatus *status,
+                               cudaStream_t st) {
     int items, m = 0;
     const int32_t *pq = nullptr, *pk = nullptr;
     if (mode == 0) {
@@ -771,7 +781,8 @@ cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
                              (int)smem);
         kern<<<grid, kCaThreads, smem, st>>>(
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v, pq,
-            pk, P.N, n_leaf, m, P.b, items, P.scale, P.eps, RO, RL, status);
+            pk, P.N, n_leaf, m, P.b, items, next_item, P.scale, P.eps, RO, RL,
+            status);
         return cudaGetLastError();
     };
     if (P.d == 128)

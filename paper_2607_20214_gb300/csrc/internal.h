@@ -145,8 +145,9 @@ cudaError_t launch_seg_sort(const Plan &P, int Lv, const uint32_t *keyrank,
                             int32_t *perms, cudaStream_t st);
 cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
                                const void *q, const void *k, const void *v,
-                               const int32_t *perms, float *RO, float *RL,
-                               DeviceStatus *status, cudaStream_t st);
+                               const int32_t *perms, int *next_item, float *RO,
+                               float *RL, DeviceStatus *status,
+                               cudaStream_t st);
 cudaError_t launch_causal_prefix(const Plan &P, const float *part,
                                  uint16_t *sBh, float *sA, cudaStream_t st);
 cudaError_t launch_causal_race(const Plan &P, const void *q, const void *k,
