@@ -296,8 +296,9 @@ namespace {
 // Causal forward (Algorithm "Causal ELSAA"). Workspace: status | codes
 // (sort hash, [2][B*H][N]) | tile histograms of the hash | per level and
 // side the sorted halves [Lv][2][B*H][N / 2] | running sparse result O
-// [B*H][N][d_h] fp32 and log d [B*H][N] | RACE chunk summaries
-// [B*H][N / 128][r d_h + r] | prefix states sB (bf16) and sA | bf16 planes.
+// [B*H][N][d_h] fp32 and log d [B*H][N] | RACE segment summaries, then
+// offsets [B*H][segments][r d_h + r] | prefix states sB (bf16) and sA of
+// every 128-key chunk | bf16 planes | work counters.
 struct CausalPlan {
     Plan P;   // geometry and the forward's hash / RACE settings
     Plan Pc;  // P with RACE chunks of 128 keys
@@ -339,9 +340,11 @@ int make_causal_plan(const elsaa_params *p, CausalPlan *C, const char **msg) {
                "multiple of 128 rows";
         return ELSAA_ERR_UNSUPPORTED;
     }
+    // RACE key summaries of segments of whole 128-key chunks
+    const int nseg = causal_segments(P);
     C->Pc = P;
-    C->Pc.S = P.N / 128;
-    C->Pc.chunk = 128;
+    C->Pc.S = nseg;
+    C->Pc.chunk = P.N / nseg;
     const size_t BHN = (size_t)P.BH * P.N;
     const size_t nc = (size_t)P.N / 128;
     size_t off = 0;
@@ -359,7 +362,7 @@ int make_causal_plan(const elsaa_params *p, CausalPlan *C, const char **msg) {
     C->off_RL = off;
     off = align_up(off + BHN * sizeof(float), 256);
     C->off_part = off;
-    off = align_up(off + (size_t)P.BH * nc * ((size_t)P.r * P.d + P.r) *
+    off = align_up(off + (size_t)P.BH * nseg * ((size_t)P.r * P.d + P.r) *
                              sizeof(float), 256);
     C->off_sB = off;
     off = align_up(off + (size_t)P.BH * nc * P.r * P.d * sizeof(uint16_t),
@@ -423,27 +426,6 @@ int causal_forward(const elsaa_params *params, const void *q, const void *k,
     ELSAA_CHECK_LAUNCH(
         cudaMemsetAsync(ctr, 0, (size_t)(C.Lv + 1) * sizeof(int), st),
         "counter reset");
-    // the low-rank branch needs no sort: chunk summaries and prefix states
-    // on the side stream, joined back before the readout
-    SideStream *side = nullptr;
-    ELSAA_CHECK_LAUNCH(side_stream(&side), "side stream");
-    cudaStream_t ks = side->s;
-    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->fork, st), "fork");
-    ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(ks, side->fork, 0), "fork wait");
-    ELSAA_CHECK_LAUNCH(timed("prep_planes", ks, [&] {
-                           return launch_prep_planes(P, w_race, Wbf, ks);
-                       }),
-                       "prep_planes");
-    ELSAA_CHECK_LAUNCH(timed("race_keys_ws", ks, [&] {
-                           return launch_race_keys_ws(C.Pc, k, v, Wbf, part,
-                                                      status, ks);
-                       }),
-                       "race_keys_ws");
-    ELSAA_CHECK_LAUNCH(timed("causal_prefix", ks, [&] {
-                           return launch_causal_prefix(P, part, sB, sA, ks);
-                       }),
-                       "causal_prefix");
-    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->join, ks), "join");
     // sparse branch: codes, sorted halves, base segments, then the levels
     ELSAA_CHECK_LAUNCH(timed("sort_hash", st, [&] {
                            return launch_sort_hash(P, q, k, w_sort, keyrank,
@@ -461,6 +443,30 @@ int causal_forward(const elsaa_params *params, const void *q, const void *k,
                                                      status, st);
                        }),
                        "causal_attn_base");
+    // the low-rank branch (chunk summaries, prefix states) on the side
+    // stream from here: the base segments' persistent CTAs fill every SM
+    // (all of TMEM), so these run beside the SortLSH levels instead of
+    // delaying the sorts and the base segments
+    SideStream *side = nullptr;
+    ELSAA_CHECK_LAUNCH(side_stream(&side), "side stream");
+    cudaStream_t ks = side->s;
+    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->fork, st), "fork");
+    ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(ks, side->fork, 0), "fork wait");
+    ELSAA_CHECK_LAUNCH(timed("prep_planes", ks, [&] {
+                           return launch_prep_planes(P, w_race, Wbf, ks);
+                       }),
+                       "prep_planes");
+    ELSAA_CHECK_LAUNCH(timed("race_keys_ws", ks, [&] {
+                           return launch_race_keys_ws(C.Pc, k, v, Wbf, part,
+                                                      status, ks);
+                       }),
+                       "race_keys_ws");
+    ELSAA_CHECK_LAUNCH(timed("causal_scan", ks, [&] {
+                           return launch_causal_scan(P, k, v, Wbf, part, sB,
+                                                     sA, status, ks);
+                       }),
+                       "causal_scan");
+    ELSAA_CHECK_LAUNCH(cudaEventRecord(side->join, ks), "join");
     for (int level = C.Lv; level >= 1; --level)
         ELSAA_CHECK_LAUNCH(timed("causal_attn_merge", st, [&] {
                                return launch_causal_attn(P, 1, C.n_leaf,

@@ -15,9 +15,11 @@
 //                    over 128-key tiles with an online softmax), then one
 //                    launch per level, deepest first, for the SortLSH blocks,
 //                    merged into the running (O, log d) with MergeLSE
-//   race_keys_ws     per-chunk summaries A_n, B_n (chunks of 128 keys)
-//   k_causal_prefix  strict prefix states sA_n, sB_n (cumulative sum shifted
-//                    by one chunk; sB_n leaves as bf16)
+//   race_keys_ws     summaries of segments of G chunks of 128 keys
+//   k_seg_offsets    their exclusive prefix over the segments of a head
+//   k_causal_scan    per segment, chunk after chunk: the strict prefix
+//                    states sA_n, sB_n (offset + the segment's earlier
+//                    chunks, accumulated in TMEM; sB_n leaves as bf16)
 //   k_causal_race_tc per chunk: inter-chunk readout phi_Q sB_n, intra-chunk
 //                    masked products tril(phi_Q phi_K^T) V, then the fusion
 //                    of Eq. (5)-(6) with the sparse result.
@@ -431,27 +433,256 @@ __global__ void __launch_bounds__(kCaThreads, 2)
 
 // ---------------------------------------------------- RACE prefix states
 
-// part[bh][n] = (B_n [r][d], A_n [r]) of chunk n; writes the strict prefix
-// sums sB_n (bf16, [bh][n][r][d]) and sA_n (fp32, [bh][n][r]).
-__global__ void k_causal_prefix(const float *__restrict__ part, int nc,
-                                int r, int d, uint16_t *__restrict__ sBh,
-                                float *__restrict__ sA) {
+// Segment offsets in place: part[bh][s] (segment totals B, A) becomes the
+// sum over the segments before s (fp32).
+__global__ void k_seg_offsets(float *__restrict__ part, int nseg, int r,
+                              int d) {
     const int bh = blockIdx.y;
     const size_t per = (size_t)r * d + r;
     const size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= per) return;
-    const float *p = part + (size_t)bh * nc * per + i;
+    float *p = part + (size_t)bh * nseg * per + i;
     float run = 0.0f;
-    for (int n = 0; n < nc; ++n) {
-        const size_t c = (size_t)bh * nc + n;
-        if (i < (size_t)r * d) {
-            const __nv_bfloat16 h = __float2bfloat16_rn(run);
-            sBh[c * r * d + i] = *reinterpret_cast<const uint16_t *>(&h);
-        } else {
-            sA[c * r + (i - (size_t)r * d)] = run;
-        }
-        run += p[(size_t)n * per];
+    for (int s = 0; s < nseg; ++s) {
+        const float v = p[(size_t)s * per];
+        p[(size_t)s * per] = run;
+        run += v;
     }
+}
+
+// Prefix states of one segment of G chunks (128 keys each), in order: the
+// state starts at the segment's offset (the sum over earlier segments) and
+// grows by each chunk's [B_n | A_n] = phi(K_n)^T [V_n | 1]; before chunk n
+// is added, sB_n (bf16) and sA_n (fp32) are written. One CTA per (head,
+// segment), 256 threads, TMEM: accumulator M-tile m at m (D + 16) (B in the
+// first D columns, A repeated in the next 16), projections after them.
+template <int D, int L>
+__global__ void __launch_bounds__(kCaThreads, 1)
+    k_causal_scan(const uint16_t *__restrict__ kx,
+                  const uint16_t *__restrict__ vx,
+                  const uint16_t *__restrict__ w_bf16,
+                  const float *__restrict__ offs, int N, int H, int nseg,
+                  int G, float beta, uint16_t *__restrict__ sBh,
+                  float *__restrict__ sA, DeviceStatus *status) {
+    constexpr int R = 16, Gb = 4;
+    constexpr int r = L * R, Lg = L * Gb;
+    constexpr int Lg_pad = (Lg + 15) / 16 * 16;
+    constexpr int r_pad = r < 128 ? 128 : r;
+    constexpr int nM = r_pad / 128;
+    constexpr int TPT = L / 2;  // tables per thread (two threads per key)
+    constexpr uint32_t kAccN = D + 16;
+    constexpr uint32_t kColP = nM * kAccN;  // projections
+    constexpr uint32_t kTileB = 128 * D * 2;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ uint64_t mma_bar;
+    __shared__ uint32_t tbase;
+    __shared__ int abort_flag;
+    volatile int *abort = &abort_flag;
+    const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
+    const int half = warp >> 2;
+    const int row = (warp & 3) * 32 + lane_id;
+    const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
+
+    const uint32_t base = align1k(smem_u32(smem_raw));
+    const uint32_t sK = base;                    // [128 x D]
+    const uint32_t sV = sK + kTileB;             // [128 x D], then ones
+    const uint32_t sW = sV + kTileB + 16384;     // [Lg_pad x D]
+    const uint32_t sPhi = sW + align1k((uint32_t)Lg_pad * D * 2);  // [128 x r_pad]
+
+    const int seg = blockIdx.x % nseg, bh = blockIdx.x / nseg;
+    const int h = bh % H;
+    const int nc = N / 128;
+    const size_t per = (size_t)r * D + r;
+    const float *off = offs + ((size_t)bh * nseg + seg) * per;
+
+    if (warp == 0) tmem_alloc(&tbase, 512);
+    if (tid == 0) {
+        mbar_init(&mma_bar, 1);
+        abort_flag = 0;
+        fence_mbar_init();
+    }
+    for (int i = tid; i < 16384 / 16; i += kCaThreads)  // bf16 ones
+        asm volatile("st.shared.v4.b32 [%0], {%1, %1, %1, %1};" ::"r"(
+                         sV + kTileB + i * 16),
+                     "r"(0x3F803F80u)
+                     : "memory");
+    if (r < r_pad)  // buckets past r stay zero
+        for (int i = tid; i < 128 * (r_pad - r) / 8; i += kCaThreads) {
+            const int rr = i / ((r_pad - r) / 8), c = i % ((r_pad - r) / 8);
+            st_shared_zero16(sPhi + panel_offset(rr, r / 8 + c, 128));
+        }
+    for (int i = tid; i < Lg_pad * (D / 8); i += kCaThreads) {
+        const int rr = i / (D / 8), c = i % (D / 8);
+        cp_async16(sW + panel_offset(rr, c, Lg_pad),
+                   w_bf16 + ((size_t)h * Lg_pad + rr) * D + c * 8);
+    }
+    auto load_k = [&](int n) {
+        const size_t r0 = (size_t)bh * N + (size_t)n * 128;
+        for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+            const int rr = i / (D / 8), c = i % (D / 8);
+            cp_async16(sK + panel_offset(rr, c, 128), kx + (r0 + rr) * D + c * 8);
+        }
+    };
+    auto load_v = [&](int n) {
+        const size_t r0 = (size_t)bh * N + (size_t)n * 128;
+        for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+            const int rr = i / (D / 8), c = i % (D / 8);
+            cp_async16(sV + panel_offset(rr, c, 128), vx + (r0 + rr) * D + c * 8);
+        }
+    };
+    const int n0 = seg * G;
+    load_k(n0);
+    load_v(n0);
+    cp_async_commit();
+    fence_proxy_async_smem();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tm = tbase;
+    uint32_t mph = 0;
+    auto mma_done = [&](int site) -> bool {
+        if (tid == 0) mma_commit(&mma_bar);
+        const bool ok =
+            mbar_wait_or_abort(&mma_bar, mph & 1, abort, status, site);
+        ++mph;
+        tc_fence_after();
+        return __syncthreads_and(ok);
+    };
+    // The accumulator starts at the segment's offset (written into TMEM by
+    // the lanes that own the buckets), so every state is read from TMEM:
+    // thread (lane, half) owns buckets m 128 + lane of M-tiles m = half,
+    // half + 2, ...
+    for (int m = half; m < nM; m += 2) {
+        const int bk = m * 128 + row;
+        const float *ob = off + (size_t)(bk < r ? bk : 0) * D;
+#pragma unroll
+        for (int c = 0; c < D; c += 32) {
+            uint32_t v[32];
+#pragma unroll
+            for (int j = 0; j < 32; j += 4) {
+                const float4 a = *reinterpret_cast<const float4 *>(ob + c + j);
+                v[j] = __float_as_uint(bk < r ? a.x : 0.0f);
+                v[j + 1] = __float_as_uint(bk < r ? a.y : 0.0f);
+                v[j + 2] = __float_as_uint(bk < r ? a.z : 0.0f);
+                v[j + 3] = __float_as_uint(bk < r ? a.w : 0.0f);
+            }
+            tmem_st32(tm + lane + m * kAccN + c, v);
+        }
+        uint32_t a16[16];
+        const float av = bk < r ? off[(size_t)r * D + bk] : 0.0f;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) a16[j] = __float_as_uint(av);
+        tmem_st16(tm + lane + m * kAccN + D, a16);
+    }
+    tmem_wait_st();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    // sB_n (bf16), sA_n = the accumulated state
+    auto write_state = [&](int n) {
+        const size_t cidx = (size_t)bh * nc + n;
+        for (int m = half; m < nM; m += 2) {
+            const int bk = m * 128 + row;
+            uint16_t *out = sBh + (cidx * r + (bk < r ? bk : 0)) * D;
+#pragma unroll
+            for (int c = 0; c < D; c += 32) {
+                uint32_t v[32];
+                tmem_ld32(tm + lane + m * kAccN + c, v);
+                tmem_wait_ld();
+                if (bk < r) {
+#pragma unroll
+                    for (int j = 0; j < 32; j += 8) {
+                        uint4 pk;
+                        pk.x = pack_bf16x2(__uint_as_float(v[j]),
+                                           __uint_as_float(v[j + 1]));
+                        pk.y = pack_bf16x2(__uint_as_float(v[j + 2]),
+                                           __uint_as_float(v[j + 3]));
+                        pk.z = pack_bf16x2(__uint_as_float(v[j + 4]),
+                                           __uint_as_float(v[j + 5]));
+                        pk.w = pack_bf16x2(__uint_as_float(v[j + 6]),
+                                           __uint_as_float(v[j + 7]));
+                        *reinterpret_cast<uint4 *>(out + c + j) = pk;
+                    }
+                }
+            }
+            uint32_t v16[16];
+            tmem_ld16(tm + lane + m * kAccN + D, v16);
+            tmem_wait_ld();
+            if (bk < r) sA[cidx * r + bk] = __uint_as_float(v16[0]);
+        }
+    };
+    write_state(n0);
+
+    bool ok = true;
+    for (int c = 0; c < G && ok; ++c) {
+        const int n = n0 + c;
+        cp_async_wait<0>();
+        fence_proxy_async_smem();
+        __syncthreads();
+        if (tid == 0) {  // projections U = K W^T
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, Lg_pad, false, false);
+#pragma unroll
+            for (int k = 0; k < D / 16; ++k)
+                mma_ss(tm + kColP,
+                       smem_desc(sK + (k >> 2) * 16384 + (k & 3) * 32, 16, 1024),
+                       smem_desc(sW + (k >> 2) * Lg_pad * 128 + (k & 3) * 32,
+                                 16, 1024),
+                       id, k > 0);
+        }
+        if (!(ok = mma_done(140))) break;
+        if (c + 1 < G) load_k(n + 1);  // this chunk's K is consumed
+        // features of this thread's tables
+#pragma unroll
+        for (int t = 0; t < TPT; ++t) {
+            const int tbl = half * TPT + t;
+            uint32_t u4[16];
+            tmem_ld16(tm + lane + kColP + (tbl * Gb) / 16 * 16, u4);
+            tmem_wait_ld();
+            float sp[Gb];
+#pragma unroll
+            for (int bb = 0; bb < Gb; ++bb) {
+                // column of bit bb of table tbl within the 16 loaded; the
+                // half-dependent part is 0 or 8 (no dynamic indexing)
+                const int i0 = (t * Gb) % 16 + bb;
+                const uint32_t u =
+                    (TPT * Gb) % 16 == 0 ? u4[i0]
+                                         : (half ? u4[(i0 + 8) & 15] : u4[i0]);
+                sp[bb] = fmaf(0.5f,
+                              tanh_approx(beta * tanh_approx(__uint_as_float(u))),
+                              0.5f);
+            }
+            float phi[R];
+            table_phi<Gb>(sp, phi);
+            st_shared_bf16x8(sPhi + panel_offset(row, tbl * 2, 128), phi);
+            st_shared_bf16x8(sPhi + panel_offset(row, tbl * 2 + 1, 128), phi + 8);
+        }
+        fence_proxy_async_smem();
+        tc_fence_before();
+        __syncthreads();
+        if (tid == 0) {  // state += phi^T [V | 1]
+            tc_fence_after();
+            const uint32_t id = idesc_bf16(128, D + 16, true, true);
+            for (int m = 0; m < nM; ++m)
+#pragma unroll
+                for (int k = 0; k < 8; ++k)
+                    mma_ss(tm + m * kAccN,
+                           smem_desc(sPhi + 2 * m * 16384 + k * 2048, 16384, 1024),
+                           smem_desc(sV + k * 2048, 16384, 1024), id, 1u);
+        }
+        if (!(ok = mma_done(141))) break;
+        if (c + 1 < G) {
+            load_v(n + 1);  // this chunk's V is consumed
+            cp_async_commit();
+            write_state(n + 1);
+        }
+        tc_fence_before();
+        __syncthreads();
+    }
+    cp_async_wait<0>();
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(tm, 512);
 }
 
 // ----------------------------------------------- causal RACE + fusion
@@ -792,12 +1023,52 @@ cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
                      : launch(k_causal_attn_tc<64, 1>);
 }
 
-cudaError_t launch_causal_prefix(const Plan &P, const float *part,
-                                 uint16_t *sBh, float *sA, cudaStream_t st) {
+int causal_segments(const Plan &P) {
+    const int nc = P.N / 128;
+    int nseg = 1;
+    while (nseg * 2 <= nc && nc % (nseg * 2) == 0 &&
+           (long)P.BH * nseg * 2 <= 304)
+        nseg *= 2;
+    return nseg;
+}
+
+size_t causal_scan_smem(const Plan &P) {
+    const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
+    const size_t r_pad = P.r < 128 ? 128 : P.r;
+    return 1024 + (size_t)2 * 128 * P.d * 2 + 16384 +
+           (lg_pad * P.d * 2 + 1023) / 1024 * 1024 + 128 * r_pad * 2;
+}
+
+cudaError_t launch_causal_scan(const Plan &P, const void *k, const void *v,
+                               const uint16_t *w_bf16, float *part,
+                               uint16_t *sBh, float *sA, DeviceStatus *status,
+                               cudaStream_t st) {
+    const int nseg = causal_segments(P);
     const int per = P.r * P.d + P.r;
-    dim3 grid((per + 255) / 256, P.BH);
-    k_causal_prefix<<<grid, 256, 0, st>>>(part, P.N / 128, P.r, P.d, sBh, sA);
-    return cudaGetLastError();
+    dim3 g1((per + 255) / 256, P.BH);
+    k_seg_offsets<<<g1, 256, 0, st>>>(part, nseg, P.r, P.d);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int G = (P.N / 128) / nseg;
+    // one CTA per SM (it holds all 512 TMEM columns)
+    size_t smem = causal_scan_smem(P);
+    if (smem < kSmemPerSM / 2 + 1024) smem = kSmemPerSM / 2 + 1024;
+    auto launch = [&](auto kern) {
+        cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+        kern<<<P.BH * nseg, kCaThreads, smem, st>>>(
+            (const uint16_t *)k, (const uint16_t *)v, w_bf16, part, P.N, P.H,
+            nseg, G, P.beta, sBh, sA, status);
+        return cudaGetLastError();
+    };
+    if (P.d == 128) {
+        if (P.L == 16) return launch(k_causal_scan<128, 16>);
+        if (P.L == 8) return launch(k_causal_scan<128, 8>);
+        return launch(k_causal_scan<128, 4>);
+    }
+    if (P.L == 16) return launch(k_causal_scan<64, 16>);
+    if (P.L == 8) return launch(k_causal_scan<64, 8>);
+    return launch(k_causal_scan<64, 4>);
 }
 
 cudaError_t launch_causal_race(const Plan &P, const void *q, const void *k,

@@ -148,8 +148,11 @@ cudaError_t launch_causal_attn(const Plan &P, int mode, int n_leaf, int level,
                                const int32_t *perms, int *next_item, float *RO,
                                float *RL, DeviceStatus *status,
                                cudaStream_t st);
-cudaError_t launch_causal_prefix(const Plan &P, const float *part,
-                                 uint16_t *sBh, float *sA, cudaStream_t st);
+int causal_segments(const Plan &P);
+cudaError_t launch_causal_scan(const Plan &P, const void *k, const void *v,
+                               const uint16_t *w_bf16, float *part,
+                               uint16_t *sBh, float *sA, DeviceStatus *status,
+                               cudaStream_t st);
 cudaError_t launch_causal_race(const Plan &P, const void *q, const void *k,
                                const void *v, const uint16_t *w_bf16,
                                const uint16_t *sBh, const float *sA,
