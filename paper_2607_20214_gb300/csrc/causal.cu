@@ -443,10 +443,17 @@ __global__ void k_seg_offsets(float *__restrict__ part, int nseg, int r,
     if (i >= per) return;
     float *p = part + (size_t)bh * nseg * per + i;
     float run = 0.0f;
-    for (int s = 0; s < nseg; ++s) {
-        const float v = p[(size_t)s * per];
-        p[(size_t)s * per] = run;
-        run += v;
+    for (int s0 = 0; s0 < nseg; s0 += 8) {  // eight loads in flight
+        float v[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            v[j] = s0 + j < nseg ? p[(size_t)(s0 + j) * per] : 0.0f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+            if (s0 + j < nseg) {
+                p[(size_t)(s0 + j) * per] = run;
+                run += v[j];
+            }
     }
 }
 
