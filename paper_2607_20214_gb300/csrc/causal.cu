@@ -758,12 +758,13 @@ __global__ void __launch_bounds__(kCaThreads, 1)
         abort_flag = 0;
         fence_mbar_init();
     }
+    // two copy groups: what the projections and features need (Q, K,
+    // planes, sA_n), then what the products after them need (V, sB_n)
     for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
         const int rr = i / (D / 8), c = i % (D / 8);
         const size_t o = (row0 + rr) * D + c * 8;
         cp_async16(sQ + panel_offset(rr, c, 128), qx + o);
         cp_async16(sK + panel_offset(rr, c, 128), kx + o);
-        cp_async16(sV + panel_offset(rr, c, 128), vx + o);
     }
     for (int i = tid; i < Lg_pad * (D / 8); i += kCaThreads) {
         const int rr = i / (D / 8), c = i % (D / 8);
@@ -771,15 +772,20 @@ __global__ void __launch_bounds__(kCaThreads, 1)
                    w_bf16 + ((size_t)h * Lg_pad + rr) * D + c * 8);
     }
     const size_t cidx = (size_t)bh * nc + n;
+    for (int i = tid; i < r / 4; i += kCaThreads)
+        cp_async16(sAo + 16 * i, sAg + cidx * r + 4 * i);
+    cp_async_commit();
+    for (int i = tid; i < 128 * (D / 8); i += kCaThreads) {
+        const int rr = i / (D / 8), c = i % (D / 8);
+        cp_async16(sV + panel_offset(rr, c, 128), vx + (row0 + rr) * D + c * 8);
+    }
     for (int i = tid; i < r * (D / 8); i += kCaThreads) {
         const int rr = i / (D / 8), c = i % (D / 8);
         cp_async16(sB + panel_offset(rr, c, r),
                    sBh + (cidx * r + rr) * D + c * 8);
     }
-    for (int i = tid; i < r / 4; i += kCaThreads)
-        cp_async16(sAo + 16 * i, sAg + cidx * r + 4 * i);
     cp_async_commit();
-    cp_async_wait<0>();
+    cp_async_wait<1>();
     fence_proxy_async_smem();
     tc_fence_before();
     __syncthreads();
@@ -855,6 +861,7 @@ __global__ void __launch_bounds__(kCaThreads, 1)
             st_shared_bf16x8(sK + panel_offset(row, col / 8, 128), pk);
             st_shared_bf16x8(sK + panel_offset(row, col / 8 + 1, 128), pk + 8);
         }
+        if (g == 0) cp_async_wait<0>();  // V and sB_n
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
@@ -874,6 +881,19 @@ __global__ void __launch_bounds__(kCaThreads, 1)
             }
         }
         ok = mma_done(131);
+    }
+
+    // the sparse result of the chunk's rows into the consumed sB_n space
+    // (fp32 rows, 16-byte chunk c of row i at c ^ (i & 7)), read back by
+    // the epilogue; with r < 256 the epilogue reads it from global memory
+    constexpr bool kStageRO = r >= 256;
+    if (kStageRO && ok) {
+        for (int i = tid; i < 128 * (D / 4); i += kCaThreads) {
+            const int rr = i / (D / 4), c = i % (D / 4);
+            cp_async16(sB + rr * (D * 4) + ((c ^ (rr & 7)) << 4),
+                       RO + (row0 + rr) * D + c * 4);
+        }
+        cp_async_commit();
     }
 
     // ---- P = tril(S): row i keeps keys j <= i of the chunk
@@ -913,6 +933,10 @@ __global__ void __launch_bounds__(kCaThreads, 1)
                    smem_desc(sV + k * 2048, 16384, 1024), id, 1u);
     }
     if (ok) ok = mma_done(132);
+    if (kStageRO) {
+        cp_async_wait<0>();
+        __syncthreads();
+    }
 
     if (ok) {
         const float invL = 1.0f / (float)L;
@@ -935,7 +959,19 @@ __global__ void __launch_bounds__(kCaThreads, 1)
             tmem_wait_ld();
 #pragma unroll
             for (int j = 0; j < 32; j += 8) {
-                const float4 s0 = os[(c + j) / 4], s1 = os[(c + j) / 4 + 1];
+                float4 s0, s1;
+                if (kStageRO) {
+                    const int c0 = (half * DH + c + j) / 4;  // 16-byte chunk
+                    const unsigned char *rb =
+                        smem_raw + (sB - smem_u32(smem_raw)) + row * (D * 4);
+                    s0 = *reinterpret_cast<const float4 *>(
+                        rb + ((c0 ^ (row & 7)) << 4));
+                    s1 = *reinterpret_cast<const float4 *>(
+                        rb + (((c0 + 1) ^ (row & 7)) << 4));
+                } else {
+                    s0 = os[(c + j) / 4];
+                    s1 = os[(c + j) / 4 + 1];
+                }
                 const float sv[8] = {s0.x, s0.y, s0.z, s0.w,
                                      s1.x, s1.y, s1.z, s1.w};
                 float y[8];
