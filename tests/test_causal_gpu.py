@@ -78,6 +78,8 @@ def small(**kw):
     (64, 32, 4, 512, 128),       # four blocks per 128-row tile
     (64, 64, 8, 512, 4096),      # one segment: exact causal attention
     (128, 128, 8, 2048, 300),    # three levels, segments of 256 rows
+    (128, 64, 4, 1024, 256),     # r = 64 (one half-filled bucket group)
+    (64, 128, 16, 1024, 512),    # r = 256 at d_h = 64 (staged sparse rows)
 ])
 def test_causal_matches_oracle(d_h, b, L, N, N0):
     wl = small(d_h=d_h, block=b, race_tables=L, N=N, causal_base_len=N0)
