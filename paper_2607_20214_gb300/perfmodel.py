@@ -143,11 +143,14 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
         fl = H * (2 * N * r * d + N * 129 * (r + d) +
                   4 * N * d * Lg)
         simt = False
-    elif kernel.startswith("causal_prefix"):
+    elif kernel.startswith("causal_scan"):
+        # prefix states chunk after chunk: reads K, V again, writes sB_n
+        # (bf16) and sA_n of every 128-key chunk; the chunk summaries
+        # phi^T [V | 1] and the projections on the tensor cores
         nc = N // 128
-        by = H * nc * (r * (d + 1) * 4 + r * d * 2 + r * 4)
-        fl = 0
-        simt = True
+        by = H * (2 * N * d * e + nc * r * (d * 2 + 4))
+        fl = H * (2 * N * r * (d + 16) + 2 * N * d * Lg)
+        simt = False
     elif kernel.startswith("bwd_sums_reduce"):
         by = H * r * (d + 1) * 4
         fl = 0
