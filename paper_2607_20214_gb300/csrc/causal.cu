@@ -110,6 +110,24 @@ __global__ void __launch_bounds__(kSegThreads)
     }
 }
 
+// Two fp32 lanes per instruction (fma.rn.f32x2): d = a * b + c lane by lane.
+__device__ __forceinline__ unsigned long long ffma2(unsigned long long a,
+                                                    unsigned long long b,
+                                                    unsigned long long c) {
+    unsigned long long d;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+    return d;
+}
+__device__ __forceinline__ unsigned long long f2pack(float lo, float hi) {
+    unsigned long long d;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(lo), "f"(hi));
+    return d;
+}
+__device__ __forceinline__ void f2unpack(unsigned long long d, float &lo,
+                                         float &hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(d));
+}
+
 // ------------------------------------------------------- attention tiles
 
 // One CTA = one tile of 128 query rows and its key tiles, online softmax:
@@ -268,9 +286,9 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         load_tile(sV, vx, kt0);
         cp_async_commit();
 
-        float o_acc[DH];
+        unsigned long long o_acc[DH / 2];  // output pairs (f32x2)
 #pragma unroll
-        for (int j = 0; j < DH; ++j) o_acc[j] = 0.0f;
+        for (int j = 0; j < DH / 2; ++j) o_acc[j] = 0ull;
         float mrun = -INFINITY, lrun = 0.0f;  // log2 domain max, sum
         for (int it = 0; it < nkt && ok; ++it) {
             const int kt = kt0 + it;
@@ -329,7 +347,10 @@ __global__ void __launch_bounds__(kCaThreads, 2)
             __syncthreads();
             const float mnew = fmaxf(mrun, fmaxf(xm[0][row], xm[1][row]));
             const float alpha = ex2_approx(mrun - mnew);  // 0 on tile 0
-            float ls = 0.0f;
+            const unsigned long long sl2x2 = f2pack(sl2, sl2);
+            const unsigned long long nm2 = f2pack(-mnew, -mnew);
+            const unsigned long long one2 = f2pack(1.0f, 1.0f);
+            unsigned long long ls2 = 0ull;
 #pragma unroll
             for (int j0 = 0; j0 < 64; j0 += 32) {
                 uint32_t v[32];
@@ -338,22 +359,27 @@ __global__ void __launch_bounds__(kCaThreads, 2)
                 uint32_t pk[16];
 #pragma unroll
                 for (int j = 0; j < 32; j += 2) {
-                    float a0 =
-                        ex2_approx(fmaf(__uint_as_float(v[j]), sl2, -mnew));
-                    float a1 = ex2_approx(
-                        fmaf(__uint_as_float(v[j + 1]), sl2, -mnew));
+                    float x0, x1;
+                    f2unpack(ffma2(f2pack(__uint_as_float(v[j]),
+                                          __uint_as_float(v[j + 1])),
+                                   sl2x2, nm2),
+                             x0, x1);
+                    float a0 = ex2_approx(x0);
+                    float a1 = ex2_approx(x1);
                     if (any_mask) {
                         a0 = keep(64 * half + j0 + j) ? a0 : 0.0f;
                         a1 = keep(64 * half + j0 + j + 1) ? a1 : 0.0f;
                     }
-                    ls += a0 + a1;
+                    ls2 = ffma2(f2pack(a0, a1), one2, ls2);
                     pk[j >> 1] = pack_bf16x2(a0, a1);
                 }
                 // over scores of this thread's half already read
                 tmem_st16(tm + lane + 64 * half + j0 / 2, pk);
             }
             tmem_wait_st();
-            xl[half][row] = ls;
+            float lsa, lsb;
+            f2unpack(ls2, lsa, lsb);
+            xl[half][row] = lsa + lsb;
             tc_fence_before();
             __syncthreads();
             lrun = lrun * alpha + xl[0][row] + xl[1][row];
@@ -374,14 +400,18 @@ __global__ void __launch_bounds__(kCaThreads, 2)
             if (!(ok = mma_done(121))) break;
             if (it + 1 < nkt) load_tile(sV, vx, kt + 1);
             cp_async_commit();
+            const unsigned long long al2 = f2pack(alpha, alpha);
 #pragma unroll
             for (int c = 0; c < DH; c += 32) {
                 uint32_t v[32];
                 tmem_ld32(tm + lane + 128 + half * DH + c, v);
                 tmem_wait_ld();
 #pragma unroll
-                for (int j = 0; j < 32; ++j)
-                    o_acc[c + j] = o_acc[c + j] * alpha + __uint_as_float(v[j]);
+                for (int j = 0; j < 32; j += 2)
+                    o_acc[(c + j) / 2] =
+                        ffma2(o_acc[(c + j) / 2], al2,
+                              f2pack(__uint_as_float(v[j]),
+                                     __uint_as_float(v[j + 1])));
             }
             tc_fence_before();
         }
@@ -395,12 +425,15 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         const size_t tok = hN + qrow_s[row];
         float *o = RO + tok * D + half * DH;
         float ld_new = logd;
+        float of[DH];
+#pragma unroll
+        for (int j = 0; j < DH / 2; ++j) f2unpack(o_acc[j], of[2 * j], of[2 * j + 1]);
         if (MODE == 0) {
 #pragma unroll
             for (int j = 0; j < DH; j += 4)
                 *reinterpret_cast<float4 *>(o + j) =
-                    make_float4(o_acc[j] * inv, o_acc[j + 1] * inv,
-                                o_acc[j + 2] * inv, o_acc[j + 3] * inv);
+                    make_float4(of[j] * inv, of[j + 1] * inv,
+                                of[j + 2] * inv, of[j + 3] * inv);
             if (half == 0) RL[tok] = logd;
         } else {
             // MergeLSE(running = diag, this = off)
@@ -413,10 +446,10 @@ __global__ void __launch_bounds__(kCaThreads, 2)
 #pragma unroll
             for (int j = 0; j < DH; j += 4) {
                 float4 a = *reinterpret_cast<float4 *>(o + j);
-                a.x = c1 * a.x + c2 * o_acc[j];
-                a.y = c1 * a.y + c2 * o_acc[j + 1];
-                a.z = c1 * a.z + c2 * o_acc[j + 2];
-                a.w = c1 * a.w + c2 * o_acc[j + 3];
+                a.x = c1 * a.x + c2 * of[j];
+                a.y = c1 * a.y + c2 * of[j + 1];
+                a.z = c1 * a.z + c2 * of[j + 2];
+                a.w = c1 * a.w + c2 * of[j + 3];
                 *reinterpret_cast<float4 *>(o + j) = a;
             }
             ld_new = mu + __logf(ssum + eps);
