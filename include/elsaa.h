@@ -224,10 +224,14 @@ int elsaa_forward_noalloc(const elsaa_params *params, const void *q,
  * workspace    at least elsaa_backward_workspace_size() bytes, 256-byte
  *              aligned (a different size from the forward workspace).
  *
- * Computed on CUDA cores in fp32 (all dtypes). Supported: the forward's
- * shapes with b * (4 d_h + b + r + 2) * 4 bytes of block state <= 200 KiB
- * (e.g. b = 64, d_h = 64, r = 128); ELSAA_ERR_UNSUPPORTED otherwise.
- * Errors as for elsaa_forward.
+ * Paths: with impl AUTO, bf16, b = 64, d_h = 64, race_bits 4 with
+ * race_tables 4 or 8 and N a multiple of 128, the products run on the
+ * tensor cores (bf16 operands, fp32 accumulation; gradients within about
+ * 1e-2 of the largest gradient magnitude); otherwise on CUDA cores in fp32
+ * (all dtypes) for the forward's shapes with b * (4 d_h + b + r + 2) * 4
+ * bytes of block state <= 200 KiB (e.g. b = 64, d_h = 64, r = 128);
+ * ELSAA_ERR_UNSUPPORTED otherwise and for causal = 1. Errors as for
+ * elsaa_forward.
  */
 int elsaa_backward_workspace_size(const elsaa_params *params, size_t *bytes);
 int elsaa_backward(const elsaa_params *params, const void *q, const void *k,
