@@ -285,14 +285,17 @@ def run_ours(args, wl):
                                 workspace=ws, stream=stream)
 
     if args.backward:
-        # the backward pass of the same inputs: permutations from one
-        # forward (outside the timed region), then elsaa_backward per step
+        # the backward pass of the same inputs: permutations and the RACE
+        # summaries A, B saved from one forward (outside the timed region,
+        # as a training step keeps them), then elsaa_backward per step
         BHN = (wl.B, wl.H, wl.N)
         perm_q = torch.empty(BHN, dtype=torch.int32, device=dev)
         perm_k = torch.empty(BHN, dtype=torch.int32, device=dev)
         elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
                             x["w_race"], o=o, perm_q=perm_q, perm_k=perm_k,
                             workspace=ws, stream=stream)
+        race_A, race_B = elsaa.elsaa_forward_race_summaries(p, ws,
+                                                            stream=stream)
         wsb = torch.empty(max(elsaa.elsaa_backward_workspace_size(p), 256),
                           dtype=torch.uint8, device=dev)
         grads = [torch.empty(x["q"].shape, dtype=torch.float32, device=dev)
@@ -302,6 +305,7 @@ def run_ours(args, wl):
             elsaa.elsaa_backward(p, x["q"], x["k"], x["v"], x["w_sort"],
                                  x["w_race"], x["do"], perm_q, perm_k,
                                  dq=grads[0], dk=grads[1], dv=grads[2],
+                                 race_A=race_A, race_B=race_B,
                                  workspace=wsb, stream=stream)
 
     barrier = multirank.barrier
@@ -367,9 +371,11 @@ def run_ours(args, wl):
     if args.backward and not args.no_e2e:
         names = ("q", "k", "v", "w_race", "do")
         hx = {k: x[k].cpu().pin_memory() for k in names}
-        hp = [perm_q.cpu().pin_memory(), perm_k.cpu().pin_memory()]
+        hp = [perm_q.cpu().pin_memory(), perm_k.cpu().pin_memory(),
+              race_A.cpu().pin_memory(), race_B.cpu().pin_memory()]
         dx = {k: torch.empty_like(x[k]) for k in hx}
-        dp = [torch.empty_like(perm_q), torch.empty_like(perm_k)]
+        dp = [torch.empty_like(perm_q), torch.empty_like(perm_k),
+              torch.empty_like(race_A), torch.empty_like(race_B)]
         hg = [torch.empty(g.shape, dtype=g.dtype).pin_memory() for g in grads]
         h2d = sum(t.numel() * t.element_size() for t in hx.values()) + sum(
             t.numel() * t.element_size() for t in hp)
@@ -383,6 +389,7 @@ def run_ours(args, wl):
             elsaa.elsaa_backward(p, dx["q"], dx["k"], dx["v"], None,
                                  dx["w_race"], dx["do"], dp[0], dp[1],
                                  dq=grads[0], dk=grads[1], dv=grads[2],
+                                 race_A=dp[2], race_B=dp[3],
                                  workspace=wsb, stream=stream)
             for hh, g in zip(hg, grads):
                 hh.copy_(g, non_blocking=True)

@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define ELSAA_ABI_VERSION 3
+#define ELSAA_ABI_VERSION 4
 
 /* Return codes. */
 #define ELSAA_OK 0
@@ -212,7 +212,9 @@ int elsaa_forward_noalloc(const elsaa_params *params, const void *q,
  * Branch", Eq. (5)-(6)). The hash and the sort are piecewise constant and
  * carry no gradient: the caller passes the permutations perm_q, perm_k that
  * elsaa_forward returned for the same inputs (required, not recomputed).
- * Everything else (block scores, features, A and B) is recomputed.
+ * The RACE summaries A and B are taken from race_A, race_B when given
+ * (saved from the forward with elsaa_forward_race_summaries) and
+ * recomputed otherwise; block scores and features are always recomputed.
  *
  * params, q, k, v, w_sort, w_race, lambda_tok, gates: as for elsaa_forward
  *              (w_sort is not read).
@@ -221,6 +223,9 @@ int elsaa_forward_noalloc(const elsaa_params *params, const void *q,
  * dq, dk, dv   [B, H, N, d_h] fp32 (device, written).
  * d_gates      [B, H, N, 2] fp32 dL/d(g_sparse, g_lr), or NULL.
  * d_lambda     [B, H, N] fp32 dL/dlambda_i, or NULL.
+ * race_A       [B, H, r] fp32 and race_B [B, H, r, d_h] fp32: the forward's
+ *              summaries (device, read only), both or neither (NULL, NULL:
+ *              recomputed); 16-byte aligned.
  * workspace    at least elsaa_backward_workspace_size() bytes, 256-byte
  *              aligned (a different size from the forward workspace).
  *
@@ -239,8 +244,24 @@ int elsaa_backward(const elsaa_params *params, const void *q, const void *k,
                    const float *lambda_tok, const float *gates,
                    const void *d_o, const int32_t *perm_q,
                    const int32_t *perm_k, float *dq, float *dk, float *dv,
-                   float *d_gates, float *d_lambda, void *workspace,
+                   float *d_gates, float *d_lambda, const float *race_A,
+                   const float *race_B, void *workspace,
                    size_t workspace_bytes, void *stream);
+
+/*
+ * Copies the RACE summaries of the last elsaa_forward enqueued with this
+ * `params` and `workspace` (Algorithm "RACE Low-Rank Attention Branch",
+ * steps 5-7: A = Phi_K^T 1, B = Phi_K^T V, per table and bucket, summed over
+ * all keys) into race_A [B, H, r] and race_B [B, H, r, d_h] (fp32, device,
+ * written), stream-ordered after that forward on `stream`: the saved
+ * activations elsaa_backward can take instead of recomputing them.
+ * ELSAA_ERR_UNSUPPORTED for causal = 1 (its RACE branch keeps per-chunk
+ * prefix states instead); other errors as for elsaa_forward.
+ */
+int elsaa_forward_race_summaries(const elsaa_params *params,
+                                 const void *workspace,
+                                 size_t workspace_bytes, float *race_A,
+                                 float *race_B, void *stream);
 
 /*
  * Token-wise gates and query-dependent lambda, the learned inputs of the

@@ -718,6 +718,42 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
 
 }  // namespace
 
+extern "C" int elsaa_forward_race_summaries(const elsaa_params *params,
+                                            const void *workspace,
+                                            size_t workspace_bytes,
+                                            float *race_A, float *race_B,
+                                            void *stream) {
+    g_err[0] = 0;
+    if (params && params->causal == 1)
+        return fail(ELSAA_ERR_UNSUPPORTED,
+                    "the causal forward keeps per-chunk prefix states, not "
+                    "whole-sequence summaries");
+    Plan P;
+    const char *msg = "";
+    int rc = make_plan(params, &P, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    if (!race_A || !race_B)
+        return fail(ELSAA_ERR_INVALID_ARG, "race_A and race_B must be non-NULL");
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if (workspace_bytes < P.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, P.total);
+    cudaStream_t st = (cudaStream_t)stream;
+    const char *ws = (const char *)workspace;
+    ELSAA_CHECK_LAUNCH(
+        cudaMemcpyAsync(race_A, ws + P.off_A,
+                        (size_t)P.BH * P.r * sizeof(float),
+                        cudaMemcpyDeviceToDevice, st),
+        "copy of A");
+    ELSAA_CHECK_LAUNCH(
+        cudaMemcpyAsync(race_B, ws + P.off_B,
+                        (size_t)P.BH * P.r * P.d * sizeof(float),
+                        cudaMemcpyDeviceToDevice, st),
+        "copy of B");
+    return ELSAA_OK;
+}
+
 extern "C" int elsaa_backward_workspace_size(const elsaa_params *params,
                                              size_t *bytes) {
     g_err[0] = 0;
@@ -737,6 +773,7 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                               const void *d_o, const int32_t *perm_q,
                               const int32_t *perm_k, float *dq, float *dk,
                               float *dv, float *d_gates, float *d_lambda,
+                              const float *race_A, const float *race_B,
                               void *workspace, size_t workspace_bytes,
                               void *stream) {
     (void)w_sort;  // the permutations are given
@@ -759,6 +796,12 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
             return fail(ELSAA_ERR_INVALID_ARG,
                         "q, k, v, d_o, w_race, dq, dk and dv must be 16-byte "
                         "aligned");
+    if ((race_A == nullptr) != (race_B == nullptr))
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "race_A and race_B must be given together");
+    if ((uintptr_t)race_A % 16 || (uintptr_t)race_B % 16)
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "race_A and race_B must be 16-byte aligned");
     if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
     if ((uintptr_t)workspace % 256)
         return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
@@ -780,33 +823,46 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
 
     ELSAA_CHECK_LAUNCH(cudaMemsetAsync(status, 0, sizeof(DeviceStatus), st),
                        "status reset");
-    // A, B exactly as the forward made them
+    // A, B: the forward's saved summaries, or recomputed exactly as the
+    // forward made them
     const Plan &Pf = Bp.Pf;
-    if (Pf.impl == 2) {
-        uint16_t *Wbf = (uint16_t *)(ws + Bp.off_W);
+    uint16_t *Wbf = (uint16_t *)(ws + Bp.off_W);
+    uint16_t *Bhw = Bp.tc ? (uint16_t *)(ws + Bp.off_Bh) : nullptr;
+    if (Pf.impl == 2)
         ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
                                return launch_prep_planes(Pf, w_race, Wbf, st);
                            }),
                            "prep_planes");
-        ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
-                               return launch_race_keys_ws(Pf, k, v, Wbf, part,
-                                                          status, st);
-                           }),
-                           "race_keys_ws");
+    if (race_A) {
+        A = const_cast<float *>(race_A);
+        Bm = const_cast<float *>(race_B);
+        if (Bhw)
+            ELSAA_CHECK_LAUNCH(timed("bf16_image", st, [&] {
+                                   return launch_bf16_image(
+                                       race_B, Bhw,
+                                       (size_t)P.BH * P.r * P.d, st);
+                               }),
+                               "bf16_image");
     } else {
-        ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
-                               return launch_race_partial_simt(Pf, k, v,
-                                                               w_race, part,
-                                                               st);
+        if (Pf.impl == 2) {
+            ELSAA_CHECK_LAUNCH(timed("race_keys_ws", st, [&] {
+                                   return launch_race_keys_ws(
+                                       Pf, k, v, Wbf, part, status, st);
+                               }),
+                               "race_keys_ws");
+        } else {
+            ELSAA_CHECK_LAUNCH(timed("race_partial_simt", st, [&] {
+                                   return launch_race_partial_simt(
+                                       Pf, k, v, w_race, part, st);
+                               }),
+                               "race_partial_simt");
+        }
+        ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
+                               return launch_race_reduce(Pf, part, A, Bm,
+                                                         Bhw, st);
                            }),
-                           "race_partial_simt");
+                           "race_reduce");
     }
-    uint16_t *Bhw = Bp.tc ? (uint16_t *)(ws + Bp.off_Bh) : nullptr;
-    ELSAA_CHECK_LAUNCH(timed("race_reduce", st, [&] {
-                           return launch_race_reduce(Pf, part, A, Bm, Bhw,
-                                                     st);
-                       }),
-                       "race_reduce");
     if (Bp.tc) {
         ELSAA_CHECK_LAUNCH(timed("bwd_block_tc", st, [&] {
                                return launch_bwd_block_tc(

@@ -120,6 +120,9 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
 bool bwd_tc_supported(const Plan &P);
 size_t bwd_tc_smem(const Plan &P);
 int bwd_tc_grid(const Plan &P);
+// bf16 copy (round to nearest even) of n fp32 values.
+cudaError_t launch_bf16_image(const float *x, uint16_t *y, size_t n,
+                              cudaStream_t st);
 int bwd_tc_segments(const Plan &P);
 cudaError_t launch_bwd_sums_reduce(const Plan &P, const float *part,
                                    uint16_t *gBh, float *gA, cudaStream_t st);

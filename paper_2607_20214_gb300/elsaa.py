@@ -30,7 +30,7 @@ SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_profile_stop", "elsaa_forward_noalloc",
            "elsaa_backward_workspace_size", "elsaa_backward",
            "elsaa_gates_workspace_size", "elsaa_gates",
-           "elsaa_selftest_wait_timeout")
+           "elsaa_selftest_wait_timeout", "elsaa_forward_race_summaries")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -111,8 +111,11 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
     L.elsaa_backward_workspace_size.argtypes = [
         ctypes.POINTER(elsaa_params), ctypes.POINTER(ctypes.c_size_t)]
     L.elsaa_backward_workspace_size.restype = ctypes.c_int
-    L.elsaa_backward.argtypes = [ctypes.POINTER(elsaa_params)] + [vp] * 16 + [
+    L.elsaa_backward.argtypes = [ctypes.POINTER(elsaa_params)] + [vp] * 18 + [
         ctypes.c_size_t, vp]
+    L.elsaa_forward_race_summaries.argtypes = [
+        ctypes.POINTER(elsaa_params), vp, ctypes.c_size_t, vp, vp, vp]
+    L.elsaa_forward_race_summaries.restype = ctypes.c_int
     L.elsaa_backward.restype = ctypes.c_int
     L.elsaa_gates_workspace_size.argtypes = [
         ctypes.POINTER(elsaa_params), ctypes.POINTER(elsaa_gate_mlp),
@@ -255,13 +258,41 @@ def elsaa_backward_workspace_size(params: elsaa_params) -> int:
     return n.value
 
 
+def elsaa_forward_race_summaries(params: elsaa_params, workspace,
+                                 race_A=None, race_B=None, stream=None):
+    """Copy the RACE summaries A [B, H, r], B [B, H, r, d_h] (fp32) of the
+    last elsaa_forward on `workspace` into race_A, race_B (allocated here
+    when not given); returns (race_A, race_B)."""
+    lib = load_library()
+    dev = workspace.device
+    r = params.race_tables << params.race_bits
+    BH = params.B * params.H
+    if race_A is None:
+        race_A = torch.empty((params.B, params.H, r), dtype=torch.float32,
+                             device=dev)
+    if race_B is None:
+        race_B = torch.empty((params.B, params.H, r, params.d_h),
+                             dtype=torch.float32, device=dev)
+    if stream is None:
+        stream = torch.cuda.current_stream(dev)
+    sp = stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+    rc = lib.elsaa_forward_race_summaries(
+        ctypes.byref(params), _ptr(workspace, "workspace", None, None, dev),
+        workspace.numel() * workspace.element_size(),
+        _ptr(race_A, "race_A", torch.float32, BH * r, dev),
+        _ptr(race_B, "race_B", torch.float32, BH * r * params.d_h, dev), sp)
+    _check(rc)
+    return race_A, race_B
+
+
 def elsaa_backward(params: elsaa_params, q, k, v, w_sort, w_race, d_o,
                    perm_q, perm_k, lambda_tok=None, gates=None, dq=None,
                    dk=None, dv=None, d_gates=None, d_lambda=None,
-                   workspace=None, stream=None):
+                   race_A=None, race_B=None, workspace=None, stream=None):
     """Enqueue elsaa_backward on `stream`; returns (dq, dk, dv) (fp32,
     allocated here when not given). perm_q, perm_k come from elsaa_forward
-    on the same inputs."""
+    on the same inputs; race_A, race_B (optional) from
+    elsaa_forward_race_summaries."""
     lib = load_library()
     dev = q.device
     if dev.type != "cuda":
@@ -269,6 +300,7 @@ def elsaa_backward(params: elsaa_params, q, k, v, w_sort, w_race, d_o,
     tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
     BHN = params.B * params.H * params.N
     nqkv = BHN * params.d_h
+    r = params.race_tables << params.race_bits
     shape = tuple(q.shape)
     dq = torch.empty(shape, dtype=torch.float32, device=dev) if dq is None else dq
     dk = torch.empty(shape, dtype=torch.float32, device=dev) if dk is None else dk
@@ -297,6 +329,9 @@ def elsaa_backward(params: elsaa_params, q, k, v, w_sort, w_race, d_o,
         _ptr(dv, "dv", torch.float32, nqkv, dev),
         _ptr(d_gates, "d_gates", torch.float32, 2 * BHN, dev),
         _ptr(d_lambda, "d_lambda", torch.float32, BHN, dev),
+        _ptr(race_A, "race_A", torch.float32, params.B * params.H * r, dev),
+        _ptr(race_B, "race_B", torch.float32,
+             params.B * params.H * r * params.d_h, dev),
         _ptr(workspace, "workspace", None, None, dev),
     ]
     rc = lib.elsaa_backward(ctypes.byref(params), *args,

@@ -58,7 +58,7 @@ def test_params_struct_matches_header():
 
 
 def test_abi_version(lib):
-    assert elsaa.elsaa_abi_version() == 3
+    assert elsaa.elsaa_abi_version() == 4
 
 
 @pytest.mark.parametrize("name", sorted(WORKLOADS))

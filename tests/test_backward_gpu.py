@@ -62,6 +62,44 @@ def run_gpu(wl, x, gates=None, lam=None, impl=elsaa.ELSAA_IMPL_AUTO):
                 tc="bwd_block_tc" in prof)
 
 
+@pytest.mark.parametrize("impl,dtype", [(elsaa.ELSAA_IMPL_AUTO, "bf16"),
+                                        (elsaa.ELSAA_IMPL_SIMT, "fp32")])
+def test_saved_race_summaries_match_recompute(impl, dtype):
+    """elsaa_backward with the forward's A, B (elsaa_forward_race_summaries)
+    gives the same gradients, bit for bit, as with A, B recomputed; and the
+    saved summaries equal the oracle's to rounding."""
+    wl = small(dtype, N=1024, race_tables=8)
+    x = make_inputs(wl)
+    dev = torch.device("cuda:0")
+    p = elsaa.params_for(wl, impl=impl)
+    xd = {k: v.to(dev) for k, v in x.items()}
+    BHN = (wl.B, wl.H, wl.N)
+    perm_q = torch.empty(BHN, dtype=torch.int32, device=dev)
+    perm_k = torch.empty(BHN, dtype=torch.int32, device=dev)
+    ws = elsaa.new_workspace(p, dev)
+    elsaa.elsaa_forward(p, xd["q"], xd["k"], xd["v"], xd["w_sort"],
+                        xd["w_race"], perm_q=perm_q, perm_k=perm_k,
+                        workspace=ws)
+    A, B = elsaa.elsaa_forward_race_summaries(p, ws)
+    args = (p, xd["q"], xd["k"], xd["v"], xd["w_sort"], xd["w_race"],
+            xd["do"], perm_q, perm_k)
+    g0 = elsaa.elsaa_backward(*args)
+    g1 = elsaa.elsaa_backward(*args, race_A=A, race_B=B)
+    torch.cuda.synchronize()
+    for a, c in zip(g0, g1):
+        assert torch.equal(a, c)
+    # the saved summaries are the forward's A, B (Algorithm RACE steps 5-7)
+    for h in range(wl.H):
+        Ar, Br = orc.race_summaries(x["k"][0, h].double().numpy(),
+                                    x["v"][0, h].double().numpy(),
+                                    x["w_race"][h].double().numpy(), wl.beta)
+        Ag = A[0, h].cpu().double().numpy().reshape(Ar.shape)
+        Bg = B[0, h].cpu().double().numpy().reshape(Br.shape)
+        tol = 1e-2 if dtype == "bf16" else 1e-4
+        assert np.abs(Ag - Ar).max() <= tol * np.abs(Ar).max()
+        assert np.abs(Bg - Br).max() <= tol * np.abs(Br).max()
+
+
 def oracle_head(wl, x, b, h, gates=None, lam=None):
     f32 = lambda t: t[b, h].float().cpu().numpy()
     p = orc.params_from_workload(wl)
