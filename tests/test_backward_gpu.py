@@ -188,3 +188,48 @@ def test_c5_full_size_sampled_heads():
     assert g["tc"]
     xc = {k: v.cpu() for k, v in x.items()}
     compare(wl, g, xc, [(0, 0), (7, 11)])
+
+
+def test_backward_cuda_graph_with_saved_summaries():
+    """elsaa_backward with saved A, B captured into a CUDA graph and
+    replayed: bit-identical to an eager call."""
+    wl = small("bf16", N=1024, race_tables=8)
+    x = make_inputs(wl)
+    dev = torch.device("cuda:0")
+    p = elsaa.params_for(wl)
+    xd = {k: v.to(dev) for k, v in x.items()}
+    BHN = (wl.B, wl.H, wl.N)
+    perm_q = torch.empty(BHN, dtype=torch.int32, device=dev)
+    perm_k = torch.empty(BHN, dtype=torch.int32, device=dev)
+    ws = elsaa.new_workspace(p, dev)
+    st = torch.cuda.Stream(dev)
+    with torch.cuda.stream(st):
+        elsaa.elsaa_forward(p, xd["q"], xd["k"], xd["v"], xd["w_sort"],
+                            xd["w_race"], perm_q=perm_q, perm_k=perm_k,
+                            workspace=ws, stream=st)
+        A, B = elsaa.elsaa_forward_race_summaries(p, ws, stream=st)
+    wsb = torch.empty(elsaa.elsaa_backward_workspace_size(p),
+                      dtype=torch.uint8, device=dev)
+    grads = [torch.empty(xd["q"].shape, dtype=torch.float32, device=dev)
+             for _ in range(3)]
+
+    def call():
+        elsaa.elsaa_backward(p, xd["q"], xd["k"], xd["v"], xd["w_sort"],
+                             xd["w_race"], xd["do"], perm_q, perm_k,
+                             dq=grads[0], dk=grads[1], dv=grads[2],
+                             race_A=A, race_B=B, workspace=wsb, stream=st)
+
+    with torch.cuda.stream(st):
+        call()
+    st.synchronize()
+    eager = [g.clone() for g in grads]
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=st):
+        call()
+    for g in grads:
+        g.zero_()
+    graph.replay()
+    torch.cuda.synchronize()
+    elsaa.elsaa_check_status(wsb)
+    for a, b in zip(eager, grads):
+        assert torch.equal(a, b)

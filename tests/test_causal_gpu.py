@@ -1,12 +1,15 @@
 """GPU causal path (elsaa_forward with causal = 1, through the C ABI) versus
 the fp64 causal oracle (oracle/causal.py) on the same seeded inputs.
 
-Tolerances as for the non-causal bf16 path: O within 2e-2 absolute (bf16
-inputs and output; the kernels round the softmax weights, the RACE features,
-the masked intra-chunk products and the prefix states sB_n to bf16 before
-their tensor-core products, relative 2^-9 each, and accumulate in fp32),
-log d_sparse within 2e-2 absolute (fp32 running maximum and sum), d_lr
-within 1e-2 relative, m within 1e-2 absolute.
+Tolerances: O within 2e-2 + 2^-8 |O_ref| elementwise: the non-causal bf16
+bound (the kernels round the softmax weights, the RACE features, the masked
+intra-chunk products and the prefix states sB_n to bf16 before their
+tensor-core products and accumulate in fp32) plus half a bf16 ulp of the
+output itself. Causal rows near the start average over a handful of keys,
+so |O| reaches 5-8 there, where rounding the exact result to bf16 alone
+moves it by up to 0.016-0.03: an absolute 2e-2 would fail on exact
+arithmetic. log d_sparse within 2e-2 absolute (fp32 running maximum and
+sum), d_lr within 1e-2 relative, m within 1e-2 absolute.
 """
 import numpy as np
 import pytest
@@ -21,6 +24,12 @@ from paper_2607_20214_gb300.workloads import (WORKLOADS, Workload,
 pytestmark = pytest.mark.gpu
 
 TOL_O, TOL_LOGD, TOL_DLR_REL, TOL_M = 2e-2, 2e-2, 1e-2, 1e-2
+HALF_ULP_BF16 = 2.0 ** -8  # relative
+
+
+def o_err(got, ref):
+    """Largest error of O in units of its bound 2e-2 + 2^-8 |O_ref|."""
+    return (np.abs(got - ref) / (TOL_O + HALF_ULP_BF16 * np.abs(ref))).max()
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -51,8 +60,8 @@ def run_gpu(wl, x, gates=None, lam=None):
 
 def compare(g, ref, label=""):
     for (b, h), r in ref.items():
-        e = np.abs(g["O"][b, h].numpy() - r["O"]).max()
-        assert e <= TOL_O, (label, b, h, "O", e)
+        e = o_err(g["O"][b, h].numpy(), r["O"])
+        assert e <= 1.0, (label, b, h, "O (in units of its bound)", e)
         e = np.abs(g["log_d_sparse"][b, h].numpy() - r["log_d_sparse"]).max()
         assert e <= TOL_LOGD, (label, b, h, "log d_s", e)
         dl = g["d_lr"][b, h].numpy()
@@ -98,7 +107,7 @@ def test_causal_gates_lambda_and_ablation():
     ref = oc.forward(x, orc.params_from_workload(wl1))
     g = run_gpu(wl1, x)
     for (b, h), r in ref.items():
-        assert np.abs(g["O"][b, h].numpy() - r["O"]).max() <= TOL_O
+        assert o_err(g["O"][b, h].numpy(), r["O"]) <= 1.0
         assert (g["m_sparse"][b, h].numpy() == 1.0).all()
 
 
@@ -126,3 +135,44 @@ def test_c3_causal_full_size_heads():
     ref = oc.forward(x, orc.params_from_workload(wl), heads=[(0, 3), (1, 12)])
     compare(g, ref, label="c3c")
     assert torch.isfinite(g["O"]).all()
+
+
+def test_causal_cuda_graph_capture_and_replay():
+    """The causal forward (work counters reset, side-stream fork and join)
+    captured into a CUDA graph and replayed on new inputs in the same
+    buffers: bit-identical to an eager call, and to the oracle."""
+    wl = small(H=2, N=1024, d_h=128, block=128, race_tables=16)
+    dev = torch.device("cuda:0")
+    p = elsaa.params_for(wl)
+    x1 = make_inputs(wl)
+    x2 = make_inputs(wl.with_(seed=wl.seed + 1))
+    xd = {k: v.to(dev) for k, v in x1.items()}
+    o = torch.empty_like(xd["q"])
+    ws = elsaa.new_workspace(p, dev)
+    st = torch.cuda.Stream(dev)
+
+    def call():
+        elsaa.elsaa_forward(p, xd["q"], xd["k"], xd["v"], xd["w_sort"],
+                            xd["w_race"], o=o, workspace=ws, stream=st)
+
+    with torch.cuda.stream(st):
+        call()
+    st.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=st):
+        call()
+    for k in xd:
+        xd[k].copy_(x2[k].to(dev))
+    o.zero_()
+    graph.replay()
+    graph.replay()  # counters are reset inside the graph
+    torch.cuda.synchronize()
+    elsaa.elsaa_check_status(ws)
+    replay = o.clone()
+    with torch.cuda.stream(st):
+        call()
+    st.synchronize()
+    assert torch.equal(replay, o)
+    ref = oc.forward(x2, orc.params_from_workload(wl))
+    for (b, h), r in ref.items():
+        assert o_err(replay[b, h].float().cpu().numpy(), r["O"]) <= 1.0
