@@ -66,6 +66,18 @@ __device__ __forceinline__ void unpack_bf16x8(const uint4 &u, float *x) {
     }
 }
 
+// Per-bit factors of a table with the tanh approximation (as the forward's
+// tensor-core kernels): sp = sigma(2 beta tanh u) = 1/2 + tanh(beta tanh u)/2,
+// sn = 1 - sp; tu = tanh u (for the derivative of the projection).
+__device__ __forceinline__ void bit_factors_fast(float u, float beta,
+                                                 float &sp, float &sn,
+                                                 float &tu) {
+    tu = tanh_approx(u);
+    const float t = tanh_approx(beta * tu);
+    sp = fmaf(0.5f, t, 0.5f);
+    sn = fmaf(-0.5f, t, 0.5f);
+}
+
 __device__ __forceinline__ float lse2f(float a, float b) {
     const float mx = fmaxf(a, b);
     if (mx == -INFINITY) return -INFINITY;
@@ -297,8 +309,10 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         for (int t = 0; t < TL; ++t) {
             float sp[G], sn[G], phi[R];
 #pragma unroll
-            for (int b = 0; b < G; ++b)
-                race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
+            for (int b = 0; b < G; ++b) {
+                float tu;
+                bit_factors_fast(u[t * G + b], beta, sp[b], sn[b], tu);
+            }
 #pragma unroll
             for (int rr = 0; rr < R; ++rr) {
                 float p = 1.0f;
@@ -500,8 +514,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 float sp[G], sn[G], uu[G], phi[R], gp[R];
 #pragma unroll
                 for (int b = 0; b < G; ++b) {
-                    race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
-                    uu[b] = tanhf(u[t * G + b]);
+                    bit_factors_fast(u[t * G + b], beta, sp[b], sn[b],
+                                     uu[b]);
                 }
                 float s = 0.0f;
 #pragma unroll
@@ -817,8 +831,10 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         for (int t = 0; t < TL; ++t) {
             float sp[G], sn[G], phi[R];
 #pragma unroll
-            for (int b = 0; b < G; ++b)
-                race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
+            for (int b = 0; b < G; ++b) {
+                float tu;
+                bit_factors_fast(u[t * G + b], beta, sp[b], sn[b], tu);
+            }
 #pragma unroll
             for (int rr = 0; rr < R; ++rr) {
                 float p = 1.0f;
@@ -887,8 +903,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 float sp[G], sn[G], uu[G], phi[R], gp[R];
 #pragma unroll
                 for (int b = 0; b < G; ++b) {
-                    race_bit_factors(u[t * G + b], beta, sp[b], sn[b]);
-                    uu[b] = tanhf(u[t * G + b]);
+                    bit_factors_fast(u[t * G + b], beta, sp[b], sn[b],
+                                     uu[b]);
                 }
                 float s = 0.0f;
 #pragma unroll
