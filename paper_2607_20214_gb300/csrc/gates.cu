@@ -192,7 +192,7 @@ __global__ void __launch_bounds__(kGateWsThreads, 1)
             for (int s = 0; s < S; ++s) {
                 const int last = i - 1 - (((i - 1 - s) % S) + S) % S;
                 if (last >= 0 && last < i)
-                    mbar_wait(&full[s], (last / S) & 1, nullptr, 0);
+                    mbar_wait(&full[s], (last / S) & 1, status, 0x6107);
             }
         }
     } else if (warp == 1) {
@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(kGateWsThreads, 1)
             // no MMA may still be writing tensor memory or reading the
             // image when the CTA ends
             mma_commit(&drain);
-            mbar_wait(&drain, drains & 1, nullptr, 0);
+            mbar_wait(&drain, drains & 1, status, 0x6108);
         }
         __syncwarp();
     } else {

@@ -270,7 +270,8 @@ __global__ void __launch_bounds__(kHashThreads, 2)
                 int last = issued - 1 - ((issued - 1 - s) % kHashStages +
                                          kHashStages) % kHashStages;
                 if (last >= 0 && last < issued)
-                    mbar_wait(&full[s], (last / kHashStages) & 1, nullptr, 0);
+                    mbar_wait(&full[s], (last / kHashStages) & 1, status,
+                              0x5003);
             }
         }
         return;
