@@ -238,6 +238,185 @@ def workload_config(wl):
                 3 * wl.heads * wl.N * wl.d_h * wl.elt / 1e6)}
 
 
+def measure(step, steps, warmup, dev, stream):
+    """Mean device milliseconds of one step over `steps` timed steps (CUDA
+    events on the launching stream, after `warmup` untimed steps) and the
+    library's per-kernel event times over the same region."""
+    from paper_2607_20214_gb300 import elsaa
+    for _ in range(warmup):
+        step()
+    torch.cuda.synchronize(dev)
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    elsaa.elsaa_profile_start()
+    ev0.record(stream)
+    for _ in range(steps):
+        step()
+    ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    prof = elsaa.elsaa_profile_stop()
+    return ev0.elapsed_time(ev1) / steps, prof
+
+
+def dominant_roofline(wl, prof, peaks, ms_step, steps):
+    """Roofline of the kernel with the largest share of the device time."""
+    dom = max(prof, key=lambda k: prof[k][1])
+    n_dom, ms_dom = prof[dom]
+    work = perfmodel.kernel_work(wl, dom)
+    roof = perfmodel.roofline(work, ms_dom / n_dom / 1e3, peaks)
+    roof["kernel"] = dom
+    roof["share_of_step"] = ms_dom / steps / ms_step
+    roof["peak_source"] = peaks.get("source", "measured")
+    roof["traffic"] = ncu_traffic(dom, wl.name)
+    roof["algorithmic"] = work["bytes"] if roof["bound"] == "hbm" else \
+        work["flops"]
+    return roof
+
+
+def output_errors(got, ref):
+    """max-abs, relative l2 (||got - ref|| / ||ref||) and max-abs over
+    max |ref| of arrays of the same shape."""
+    import numpy as np
+    d = got - ref
+    return {"max_abs": float(np.abs(d).max()),
+            "rel_l2": float(np.linalg.norm(d) / np.linalg.norm(ref)),
+            "max_abs_over_max_ref": float(np.abs(d).max() /
+                                          np.abs(ref).max())}
+
+
+def forward_errors(wl, x, o, heads, rows=None):
+    """The oracle on the listed heads (rows: a sample of query rows, None =
+    all) against the device output o; the errors over all of them."""
+    import numpy as np
+    from oracle import oracle as orc
+    xc = heads_to_cpu(x, heads)
+    res = orc.forward(xc, orc.params_from_workload(wl),
+                      heads=[(0, j) for j in range(len(heads))], rows=rows,
+                      threads=len(heads))
+    got, ref = [], []
+    for j, (b, h) in enumerate(heads):
+        r = res[(0, j)]
+        got.append(o[b, h].float().cpu().numpy()[r["rows"]])
+        ref.append(r["O"])
+    return output_errors(np.concatenate(got), np.concatenate(ref))
+
+
+def extra_workloads(args, dev, stream, peaks):
+    """The long-context forward (c4: B=1 H=32 N=65536 d_h=128, b=256,
+    r=256) and the training step (c5: forward + backward, B=8 H=12 N=8192
+    d_h=64, b=64, r=128), timed in the same run as the headline workload,
+    each with its dominant kernel's roofline, the step's roofline fraction
+    and errors against the oracle on sampled heads and rows."""
+    import numpy as np
+    from oracle import backward as obwd
+    from oracle import oracle as orc
+    from paper_2607_20214_gb300 import elsaa
+    out = {}
+    # -- c4: forward
+    wl = WORKLOADS["c4"]
+    x = make_inputs(wl, device=dev)
+    p = elsaa.params_for(wl)
+    ws = elsaa.new_workspace(p, dev)
+    o = torch.empty_like(x["q"])
+
+    def step():
+        elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                            x["w_race"], o=o, workspace=ws, stream=stream)
+
+    ms, prof = measure(step, args.steps, args.warmup, dev, stream)
+    elsaa.elsaa_check_status(ws)
+    fm = perfmodel.flop_model(wl)
+    rows = np.random.default_rng(4).choice(wl.N, 512, replace=False)
+    rows.sort()
+    out["c4"] = {
+        "config": workload_config(wl), "ms_per_step": ms,
+        "value": wl.tokens / (ms / 1e3), "unit": "tokens/s",
+        "tflops": fm["tensor_flops"] / (ms / 1e3) / 1e12,
+        "step_roofline_frac": max(
+            fm["tensor_flops"] / (peaks["bf16_tflops"] * 1e12),
+            fm["bytes"] / (peaks["hbm_gbs"] * 1e9)) / (ms / 1e3),
+        "roofline": dominant_roofline(wl, prof, peaks, ms, args.steps),
+        "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n}
+                    for k, (n, t) in sorted(prof.items())},
+        "gpu_launches": sum(n for n, _ in prof.values()),
+        "err_vs_oracle": dict(forward_errors(wl, x, o, [(0, 0), (0, 31)],
+                                             rows=rows),
+                              sample="512 rows of heads (0, 0), (0, 31)"),
+    }
+    del x, o, ws
+    # -- c5: training step, forward + backward
+    wl = WORKLOADS["c5"]
+    x = make_inputs(wl.with_(backward=True), device=dev)
+    p = elsaa.params_for(wl)
+    ws = elsaa.new_workspace(p, dev)
+    wsb = torch.empty(max(elsaa.elsaa_backward_workspace_size(p), 256),
+                      dtype=torch.uint8, device=dev)
+    BHN = (wl.B, wl.H, wl.N)
+    o = torch.empty_like(x["q"])
+    pq = torch.empty(BHN, dtype=torch.int32, device=dev)
+    pk = torch.empty(BHN, dtype=torch.int32, device=dev)
+    r = wl.r
+    rA = torch.empty((wl.B, wl.H, r), dtype=torch.float32, device=dev)
+    rB = torch.empty((wl.B, wl.H, r, wl.d_h), dtype=torch.float32,
+                     device=dev)
+    grads = [torch.empty(x["q"].shape, dtype=torch.float32, device=dev)
+             for _ in range(3)]
+
+    def step():
+        elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                            x["w_race"], o=o, perm_q=pq, perm_k=pk,
+                            workspace=ws, stream=stream)
+        elsaa.elsaa_forward_race_summaries(p, ws, rA, rB, stream=stream)
+        elsaa.elsaa_backward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                             x["w_race"], x["do"], pq, pk, dq=grads[0],
+                             dk=grads[1], dv=grads[2], race_A=rA, race_B=rB,
+                             workspace=wsb, stream=stream)
+
+    ms, prof = measure(step, args.steps, args.warmup, dev, stream)
+    elsaa.elsaa_check_status(ws)
+    elsaa.elsaa_check_status(wsb)
+    ff = perfmodel.flop_model(wl)
+    fb = perfmodel.backward_flop_model(wl)
+    flops = ff["tensor_flops"] + fb["tensor_flops"]
+    nbytes = ff["bytes"] + fb["bytes"]
+    rows = np.random.default_rng(5).choice(wl.N, 512, replace=False)
+    rows.sort()
+    fwd_err = forward_errors(wl, x, o, [(0, 0), (wl.B - 1, wl.H - 1)],
+                             rows=rows)
+    # the oracle's fp64 analytic gradient of one whole head
+    b, h = wl.B - 1, wl.H - 1
+    f32 = lambda t: t[b, h].float().cpu().numpy()  # noqa: E731
+    t0 = time.perf_counter()
+    ref = obwd.backward_head(
+        f32(x["q"]), f32(x["k"]), f32(x["v"]),
+        x["w_sort"][h].float().cpu().numpy(),
+        x["w_race"][h].double().cpu().numpy(), f32(x["do"]),
+        orc.params_from_workload(wl), lam=np.full(wl.N, wl.lam))
+    t_cpu = time.perf_counter() - t0
+    grad_err = {}
+    for name, g in zip(("dQ", "dK", "dV"), grads):
+        grad_err[name] = output_errors(g[b, h].cpu().numpy(), ref[name])
+    out["c5_train"] = {
+        "config": workload_config(wl),
+        "step": "elsaa_forward (perms saved) + RACE summaries saved + "
+                "elsaa_backward (dQ, dK, dV fp32)",
+        "ms_per_step": ms, "value": wl.tokens / (ms / 1e3),
+        "unit": "tokens/s", "tflops": flops / (ms / 1e3) / 1e12,
+        "step_roofline_frac": max(
+            flops / (peaks["bf16_tflops"] * 1e12),
+            nbytes / (peaks["hbm_gbs"] * 1e9)) / (ms / 1e3),
+        "roofline": dominant_roofline(wl, prof, peaks, ms, args.steps),
+        "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n}
+                    for k, (n, t) in sorted(prof.items())},
+        "gpu_launches": sum(n for n, _ in prof.values()),
+        "fwd_err_vs_oracle": dict(fwd_err, sample="512 rows of two heads"),
+        "grad_err_vs_oracle": dict(grad_err, sample=(
+            "head (%d, %d), every row; fp64 analytic gradient, %.1f s on "
+            "one host thread" % (b, h, t_cpu))),
+    }
+    return out
+
+
 def run_ours(args, wl):
     from paper_2607_20214_gb300 import build as nvbuild
     from paper_2607_20214_gb300 import elsaa
@@ -472,6 +651,7 @@ def run_ours(args, wl):
     # fits in the sample budget, also used as a parity spot check
     cpu = None
     err = None
+    errs = None
     if args.backward and rank == 0 and world == 1 and \
             not args.no_cpu_baseline:
         # the oracle's fp64 gradient of whole heads on one host core, also a
@@ -519,12 +699,20 @@ def run_ours(args, wl):
                "%d of %d heads of one step (fp64 C oracle, "
                "threads over heads), %.1f s wall" % (
                    n_heads, wl.heads, t_cpu)}
+        import numpy as np
         of = o.float()
-        err = 0.0
-        for j, (b, h) in enumerate(heads):
-            import numpy as np
-            err = max(err, float(np.abs(of[b, h].cpu().numpy() -
-                                        res[(0, j)]["O"]).max()))
+        errs = output_errors(
+            np.concatenate([of[b, h].cpu().numpy()
+                            for b, h in heads]),
+            np.concatenate([res[(0, j)]["O"] for j in range(len(heads))]))
+        err = errs["max_abs"]
+
+    extra = None
+    if rank == 0 and world == 1 and not args.no_extra and \
+            args.workload == "c3" and not (args.backward or args.gate_mlp or
+                                           args.batch or args.heads or
+                                           args.neighbors):
+        extra = extra_workloads(args, dev, stream, peaks)
 
     if rank != 0:
         return 0
@@ -547,6 +735,11 @@ def run_ours(args, wl):
         ("max_rel_grad_err_vs_oracle" if args.backward else
          "max_abs_err_vs_oracle"): err,
     }
+    if errs is not None:
+        line["rel_l2_err_vs_oracle"] = errs["rel_l2"]
+        line["max_abs_over_max_ref_vs_oracle"] = errs["max_abs_over_max_ref"]
+    if extra is not None:
+        line["extra_workloads"] = extra
     print(json.dumps(line))
     if world > 1:
         torch.distributed.destroy_process_group()
@@ -562,6 +755,9 @@ def main():
     ap.add_argument("--workload", default="c3", choices=sorted(WORKLOADS))
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extra", action="store_true",
+                    help="skip the c4 forward and c5 training-step lines "
+                         "that the default c3 run adds")
     ap.add_argument("--batch", type=int, default=0,
                     help="override B (smaller cases for profiler captures)")
     ap.add_argument("--neighbors", type=int, default=0, metavar="R",

@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define ELSAA_ABI_VERSION 4
+#define ELSAA_ABI_VERSION 5
 
 /* Return codes. */
 #define ELSAA_OK 0
@@ -110,6 +110,11 @@ typedef struct elsaa_params {
     int causal_base_len;/* N_0 >= 1, segment length at which CausalSparse
                            switches to exact causal attention (Table 7,
                            "Sort_LSH min length"). Ignored when causal = 0 */
+    int out_fp32;       /* 0: O has the element type dtype; 1: O is fp32
+                           [B, H, N, d_h] whatever dtype is: the result is
+                           not rounded to bf16 (the same arithmetic, with
+                           the final rounding of a bf16 O left out). Not
+                           used by elsaa_backward or elsaa_gates          */
 } elsaa_params;
 
 /*
@@ -141,7 +146,8 @@ int elsaa_workspace_size(const elsaa_params *params, size_t *bytes);
  * gates        [B, H, N, 2] fp32 (g_sparse, g_lr) per token, or NULL for
  *              (1, 1). The paper's gates are sigma(G_theta(q_i)); the gate
  *              network itself runs outside the operator.
- * o            [B, H, N, d_h] of params->dtype (device, written).
+ * o            [B, H, N, d_h] of params->dtype, or fp32 with
+ *              params->out_fp32 = 1 (device, written).
  * log_d_sparse [B, H, N] fp32 log of the sparse denominator, or NULL.
  * d_lr         [B, H, N] fp32 low-rank denominator Den, or NULL.
  * m_sparse     [B, H, N] fp32 multiplier of Eq. (5), or NULL.
@@ -154,7 +160,8 @@ int elsaa_workspace_size(const elsaa_params *params, size_t *bytes);
  * With params->causal = 1 the same call runs Algorithm "Causal ELSAA":
  * o, log_d_sparse (log of the merged CausalSparse denominator), d_lr (the
  * causal Den) and m_sparse keep their meanings; perm_q and perm_k are not
- * written (each level of the recursion sorts its own halves).
+ * written (each level of the recursion sorts its own halves: see
+ * elsaa_causal_index_lists).
  *
  * Errors: ELSAA_ERR_INVALID_ARG / _UNSUPPORTED / _WORKSPACE before any
  * launch; ELSAA_ERR_CUDA if a launch fails (the message names the kernel).
@@ -180,9 +187,10 @@ int elsaa_forward(const elsaa_params *params, const void *q, const void *k,
  * Scratch comes from one fixed array of ELSAA_STATIC_WORKSPACE_BYTES inside
  * the library's device image. Every GPU on which the library's kernels are
  * loaded reserves that memory until the process exits.
- *  - The first call on each device looks up the array's device address
- *    (with that device current) and caches it; make that first call before
- *    any stream capture.
+ *  - Every call looks up the array's device address on the current device
+ *    (cudaGetSymbolAddress: a query, not an allocation), so a device reset
+ *    leaves no stale address behind. The first call on a device may load
+ *    the library's module there; make it before any stream capture.
  *  - Problems whose elsaa_workspace_size() exceeds the array are rejected
  *    with ELSAA_ERR_WORKSPACE (the message gives both sizes); nothing is
  *    launched.
@@ -201,6 +209,22 @@ int elsaa_forward_noalloc(const elsaa_params *params, const void *q,
                           const float *gates, void *o, float *log_d_sparse,
                           float *d_lr, float *m_sparse, int32_t *perm_q,
                           int32_t *perm_k, void *stream);
+
+/*
+ * elsaa_check_status for elsaa_forward_noalloc, whose callers never see the
+ * static array's address: synchronises `stream` and reads the status word
+ * that the last elsaa_forward_noalloc wrote at the start of the array
+ * (bounded waits that ran out, inconsistent sort counts). Returns as
+ * elsaa_check_status. Read it before the next call overwrites the word.
+ */
+int elsaa_check_status_noalloc(void *stream);
+
+/*
+ * elsaa_selftest_wait_timeout on the static array (see that function): lets
+ * a test see elsaa_check_status_noalloc report a timed-out wait without any
+ * fault. The next elsaa_forward_noalloc clears the word.
+ */
+int elsaa_selftest_wait_timeout_noalloc(int limit_ms, void *stream);
 
 /*
  * Backward pass: gradients of a loss L with respect to Q, K, V (and
@@ -262,6 +286,35 @@ int elsaa_forward_race_summaries(const elsaa_params *params,
                                  const void *workspace,
                                  size_t workspace_bytes, float *race_A,
                                  float *race_B, void *stream);
+
+/*
+ * The selection of the causal sparse branch (Algorithm "Causal sortLSH
+ * Sparse Exact Attention Branch"): every node of the recursion above the
+ * base segments calls SortLSH on its future half's queries and its past
+ * half's keys, each stably sorted by sort code; sorted query block t of the
+ * node attends exactly to sorted key block t.
+ *
+ * elsaa_causal_levels writes the number Lv of halving levels for params
+ * (N = n_leaf 2^Lv, n_leaf <= causal_base_len; 0 when N fits one segment).
+ *
+ * elsaa_causal_index_lists copies the sorted orders of the last causal
+ * elsaa_forward enqueued with this `params` and `workspace` into `lists`
+ * (device, written, stream-ordered after that forward on `stream`):
+ *     lists[l - 1][w][b][h][j m + p],  l = 1..Lv (1 = the top level),
+ *     m = N / 2^l rows per half, node j in [0, 2^(l-1)), p in [0, m),
+ * w = 0: the token index (within the head) of the future-half query at
+ * sorted position p of node j, whose half is rows [(2j+1) m, (2j+2) m);
+ * w = 1: the same for the past-half keys, rows [2j m, (2j+1) m). Equal codes
+ * keep increasing token order. Query at sorted position p attends to the
+ * keys at sorted positions [floor(p / b) b, floor(p / b) b + b) of the same
+ * node. Lv * 2 * B * H * N / 2 int32 values; nothing is copied when Lv = 0.
+ * Errors as for elsaa_forward_race_summaries; ELSAA_ERR_INVALID_ARG unless
+ * params->causal = 1.
+ */
+int elsaa_causal_levels(const elsaa_params *params, int *levels);
+int elsaa_causal_index_lists(const elsaa_params *params,
+                             const void *workspace, size_t workspace_bytes,
+                             int32_t *lists, void *stream);
 
 /*
  * Token-wise gates and query-dependent lambda, the learned inputs of the

@@ -49,15 +49,19 @@ def exact_causal(Q, K, V, scale, eps):
     return O, logd
 
 
-def sortlsh_pair(Q, K, V, hq, hk, b, scale, eps):
+def sortlsh_pair(Q, K, V, hq, hk, b, scale, eps, orders=None):
     """Algorithm sortLSH on queries Q and keys K, V of the same length m
     with codes hq, hk: stable sort of both, blocks of b consecutive sorted
     positions (the last one shorter if b does not divide m, CR3), query
     block t attends key block t. Returns (O, log d) in the original query
-    order."""
+    order. When `orders` is a list, the two sorted orders (pq, pk; sorted
+    position -> local row) are appended to it: they fix which keys each
+    query attends."""
     m = Q.shape[0]
     pq = orc.stable_argsort(hq)
     pk = orc.stable_argsort(hk)
+    if orders is not None:
+        orders.append((pq, pk))
     O = np.zeros_like(Q)
     logd = np.zeros(m)
     for t0 in range(0, m, b):
@@ -84,10 +88,14 @@ def merge_lse(O1, ld1, O2, ld2, eps):
     return O, mu + np.log(s + eps)
 
 
-def causal_sparse(Q, K, V, hq, hk, pad_code, b, N0, scale, eps):
+def causal_sparse(Q, K, V, hq, hk, pad_code, b, N0, scale, eps, trace=None,
+                  _start=0, _level=1):
     """CausalSparse(Q, K, V): the recursion of Algorithm "Causal sortLSH"
     over rows [0, n). hq, hk: sort codes of the rows; pad_code: the code of
-    a zero row (CR2). Returns (O [n, d], log d [n])."""
+    a zero row (CR2). Returns (O [n, d], log d [n]). When `trace` is a
+    list, every SortLSH call of the recursion appends (level, first row of
+    its node, sorted future-half query rows, sorted past-half key rows),
+    rows counted from the start of the sequence, level 1 = the top."""
     n, d = Q.shape
     if n <= N0:
         return exact_causal(Q, K, V, scale, eps)
@@ -100,11 +108,17 @@ def causal_sparse(Q, K, V, hq, hk, pad_code, b, N0, scale, eps):
         n += 1
     m = n // 2
     O_top, ld_top = causal_sparse(Q[:m], K[:m], V[:m], hq[:m], hk[:m],
-                                  pad_code, b, N0, scale, eps)
+                                  pad_code, b, N0, scale, eps, trace,
+                                  _start, _level + 1)
     O_diag, ld_diag = causal_sparse(Q[m:], K[m:], V[m:], hq[m:], hk[m:],
-                                    pad_code, b, N0, scale, eps)
+                                    pad_code, b, N0, scale, eps, trace,
+                                    _start + m, _level + 1)
+    orders = [] if trace is not None else None
     O_off, ld_off = sortlsh_pair(Q[m:], K[:m], V[:m], hq[m:], hk[:m], b,
-                                 scale, eps)
+                                 scale, eps, orders)
+    if trace is not None:
+        pq, pk = orders[0]
+        trace.append((_level, _start, _start + m + pq, _start + pk))
     O_bot, ld_bot = merge_lse(O_diag, ld_diag, O_off, ld_off, eps)
     O = np.vstack([O_top, O_bot])
     ld = np.concatenate([ld_top, ld_bot])
@@ -191,8 +205,10 @@ def forward_head(q32, k32, v32, w_sort, w_race, p: dict, lam=None,
     V = v32.astype(np.float64)
     O_lr, d_lr = causal_race(Q, K, V, w_race, p["beta"], p["causal_chunk"],
                              p["eps"])
+    trace = []
     O_s, log_d_s = causal_sparse(Q, K, V, hq, hk, pad_code, p["block"],
-                                 p["causal_base_len"], scale, p["eps"])
+                                 p["causal_base_len"], scale, p["eps"],
+                                 trace)
     lam_r = (np.full(N, p["lam"], np.float64) if lam is None
              else np.asarray(lam, np.float64))
     if gates is None:
@@ -206,7 +222,22 @@ def forward_head(q32, k32, v32, w_sort, w_race, p: dict, lam=None,
     O, m, m_log = orc.fuse_rows(O_s, np.exp(log_d_s), log_d_s, O_lr, d_lr,
                                 lam_r, g_s, g_lr, p["eps"], p["fusion_mode"])
     return dict(O=O, O_sparse=O_s, log_d_sparse=log_d_s, O_lr=O_lr,
-                d_lr=d_lr, m=m, m_log=m_log, keys_q=hq, keys_k=hk)
+                d_lr=d_lr, m=m, m_log=m_log, keys_q=hq, keys_k=hk,
+                index_lists=index_lists(trace))
+
+
+def index_lists(trace):
+    """The SortLSH orders of a trace of causal_sparse as per-level arrays:
+    {level: (queries, keys)}, each the concatenation over the level's nodes
+    (in row order) of the sorted row indices of the node's future-half
+    queries and past-half keys."""
+    out = {}
+    for level in sorted({t[0] for t in trace}):
+        nodes = sorted((t for t in trace if t[0] == level),
+                       key=lambda t: t[1])
+        out[level] = (np.concatenate([t[2] for t in nodes]),
+                      np.concatenate([t[3] for t in nodes]))
+    return out
 
 
 def forward(inputs: dict, p: dict, lam=None, gates=None, heads=None) -> dict:

@@ -147,6 +147,8 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
         return bad(ELSAA_ERR_INVALID_ARG, "impl must be AUTO or SIMT");
     if (p->neighbor_blocks < 0)
         return bad(ELSAA_ERR_INVALID_ARG, "neighbor_blocks must be >= 0");
+    if (p->out_fp32 != 0 && p->out_fp32 != 1)
+        return bad(ELSAA_ERR_INVALID_ARG, "out_fp32 must be 0 or 1");
     if ((long)p->B * p->H > 65535)
         return bad(ELSAA_ERR_UNSUPPORTED, "B * H must be at most 65535");
     if ((long)p->B * p->H * p->N > (1L << 31) - 1)
@@ -176,6 +178,7 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     Q.scale = p->scale > 0.f ? p->scale : 1.0f / sqrtf((float)p->d_h);
     Q.lambda = p->lambda;
     Q.fusion_mode = p->fusion_mode;
+    Q.o32 = p->dtype == ELSAA_BF16 && p->out_fp32 == 1;
     // neighbour windows wider than the sequence change nothing: clip
     Q.nb = p->neighbor_blocks < Q.N / Q.b ? p->neighbor_blocks : Q.N / Q.b;
     Q.impl = 1;
@@ -621,14 +624,6 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                    m_sparse, status, st);
                            }),
                            "block_attn_ws");
-    } else if (P.impl == 2 && P.nb == 0) {
-        ELSAA_CHECK_LAUNCH(timed("block_attn_tc", st, [&] {
-                               return launch_block_attn_tc(
-                                   P, q, k, v, w_race, pq, pk, A, Bh,
-                                   lambda_tok, gates, o, log_d_sparse, d_lr,
-                                   m_sparse, status, st);
-                           }),
-                           "block_attn_tc");
     } else {
         ELSAA_CHECK_LAUNCH(timed("block_attn_simt", st, [&] {
                                return launch_block_attn_simt(
@@ -751,6 +746,47 @@ extern "C" int elsaa_forward_race_summaries(const elsaa_params *params,
                         (size_t)P.BH * P.r * P.d * sizeof(float),
                         cudaMemcpyDeviceToDevice, st),
         "copy of B");
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_causal_levels(const elsaa_params *params,
+                                   int *levels) {
+    g_err[0] = 0;
+    if (!levels) return fail(ELSAA_ERR_INVALID_ARG, "levels is NULL");
+    if (!params || params->causal != 1)
+        return fail(ELSAA_ERR_INVALID_ARG, "params must have causal = 1");
+    CausalPlan C;
+    const char *msg = "";
+    int rc = make_causal_plan(params, &C, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    *levels = C.Lv;
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_causal_index_lists(const elsaa_params *params,
+                                        const void *workspace,
+                                        size_t workspace_bytes,
+                                        int32_t *lists, void *stream) {
+    g_err[0] = 0;
+    if (!params || params->causal != 1)
+        return fail(ELSAA_ERR_INVALID_ARG, "params must have causal = 1");
+    CausalPlan C;
+    const char *msg = "";
+    int rc = make_causal_plan(params, &C, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    if (C.Lv == 0) return ELSAA_OK;  // one segment: nothing is sorted
+    if (!lists) return fail(ELSAA_ERR_INVALID_ARG, "lists is NULL");
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if (workspace_bytes < C.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, C.total);
+    const char *ws = (const char *)workspace;
+    ELSAA_CHECK_LAUNCH(
+        cudaMemcpyAsync(lists, ws + C.off_perms,
+                        (size_t)C.Lv * C.P.BH * C.P.N * sizeof(int32_t),
+                        cudaMemcpyDeviceToDevice, (cudaStream_t)stream),
+        "copy of the index lists");
     return ELSAA_OK;
 }
 

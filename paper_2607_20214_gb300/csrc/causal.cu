@@ -748,7 +748,8 @@ __global__ void __launch_bounds__(kCaThreads, 1)
                      const float *__restrict__ lambda_tok,
                      const float *__restrict__ gates, int N, int H, float beta,
                      float eps, float lambda, int mode,
-                     uint16_t *__restrict__ ox, float *__restrict__ log_ds_out,
+                     uint16_t *__restrict__ ox, float *__restrict__ o32,
+                     float *__restrict__ log_ds_out,
                      float *__restrict__ dlr_out, float *__restrict__ m_out,
                      DeviceStatus *status) {
     constexpr int R = 16, G = 4;
@@ -1011,6 +1012,13 @@ __global__ void __launch_bounds__(kCaThreads, 1)
 #pragma unroll
                 for (int e = 0; e < 8; ++e)
                     y[e] = cs * sv[e] + cl * __uint_as_float(v[j + e]);
+                if (o32) {  // fp32 output: two 16-byte stores
+                    float4 *dst = reinterpret_cast<float4 *>(
+                        o32 + tok * D + half * DH + c + j);
+                    dst[0] = make_float4(y[0], y[1], y[2], y[3]);
+                    dst[1] = make_float4(y[4], y[5], y[6], y[7]);
+                    continue;
+                }
                 uint4 pk;
                 pk.x = pack_bf16x2(y[0], y[1]);
                 pk.y = pack_bf16x2(y[2], y[3]);
@@ -1164,8 +1172,8 @@ cudaError_t launch_causal_race(const Plan &P, const void *q, const void *k,
         kern<<<blocks, kCaThreads, smem, st>>>(
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
             w_bf16, sBh, sA, RO, RL, lambda_tok, gates, P.N, P.H, P.beta,
-            P.eps, P.lambda, P.fusion_mode, (uint16_t *)o, log_ds, dlr, m,
-            status);
+            P.eps, P.lambda, P.fusion_mode, P.o32 ? nullptr : (uint16_t *)o,
+            P.o32 ? (float *)o : nullptr, log_ds, dlr, m, status);
         return cudaGetLastError();
     };
     if (P.d == 128) {

@@ -47,6 +47,7 @@ struct Plan {
     int nb;          // neighbouring sorted key blocks on each side
     int impl;        // resolved: 1 = SIMT, 2 = tensor core
     int Lg_pad;      // L * gamma rounded up to 16 (projection MMA width)
+    int o32;         // write O as fp32 although the inputs are bf16
     size_t off_status, off_keyrank, off_hist, off_perm, off_part, off_A,
         off_B, off_Bh, off_W, total;
 };
@@ -90,12 +91,7 @@ cudaError_t launch_block_attn_simt(
 bool tc_supported(const Plan &P);
 // Chunks per head of the tensor-core RACE key kernel; writes tokens per chunk.
 int tc_race_chunks(const Plan &P, int *chunk);
-cudaError_t launch_block_attn_tc(
-    const Plan &P, const void *q, const void *k, const void *v,
-    const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
-    const float *A, const uint16_t *Bh, const float *lambda_tok,
-    const float *gates, void *o, float *log_d_sparse, float *d_lr,
-    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+
 
 // Backward pass (bwd.cu), CUDA cores.
 size_t bwd_block_smem(const Plan &P);

@@ -160,6 +160,7 @@ __global__ void __launch_bounds__(kBlkThreads)
                  const float *__restrict__ Ag, const float *__restrict__ Bg,
                  const float *__restrict__ lambda_tok,
                  const float *__restrict__ gates, T *__restrict__ ox,
+                 float *__restrict__ o32,
                  float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
                  float *__restrict__ m_out, int N, int d, int H, int b,
                  int L, int gamma, int tps, int nb, float beta, float eps,
@@ -335,7 +336,10 @@ __global__ void __launch_bounds__(kBlkThreads)
         float gl = gates ? gates[tok * 2 + 1] : 1.f;
         float olr = (num[j] * invL) / (s_den[row] + eps);
         float val = gs * s_m[row] * os[row * d + e] + gl * olr;
-        ox[tok * d + e] = from_f32<T>(val);
+        if (o32)
+            o32[tok * d + e] = val;
+        else
+            ox[tok * d + e] = from_f32<T>(val);
     }
 }
 
@@ -428,7 +432,8 @@ cudaError_t launch_block_attn_simt(
                              (int)smem);                                      \
         kern<<<grid, kBlkThreads, smem, st>>>(                                \
             (const T *)q, (const T *)k, (const T *)v, w_race, perm_q, perm_k, \
-            A, Bm, lambda_tok, gates, (T *)o, log_d_sparse, d_lr, m_sparse,   \
+            A, Bm, lambda_tok, gates, P.o32 ? nullptr : (T *)o,               \
+            P.o32 ? (float *)o : nullptr, log_d_sparse, d_lr, m_sparse,       \
             P.N, P.d, P.H, P.b, P.L, P.gamma, P.tables_per_slice, P.nb,       \
             P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, status);         \
     } while (0)

@@ -1,21 +1,30 @@
-// elsaa_forward_noalloc: the forward pass with scratch taken from a fixed
-// array in the library's device image, for callers that cannot allocate
-// device memory (see include/elsaa.h for the contract).
-#include <mutex>
-
+// elsaa_forward_noalloc and its companions: the forward pass with scratch
+// taken from a fixed array in the library's device image, for callers that
+// cannot allocate device memory (see include/elsaa.h for the contract).
 #include "internal.h"
 
 namespace {
 
 // The scratch array. In host code this name is only a host-side handle for
 // the device symbol, never a device address: its device address is looked
-// up with cudaGetSymbolAddress below, once per device.
+// up with cudaGetSymbolAddress below.
 static __device__ __align__(256) unsigned char
     g_static_workspace[ELSAA_STATIC_WORKSPACE_BYTES];
 
-constexpr int kMaxDevices = 64;
-void *g_static_ptr[kMaxDevices] = {};
-std::mutex g_static_mu;
+// Device address of the array on the current device. Looked up on every
+// call (a cheap query that allocates nothing), so a device reset or a new
+// primary context, which reloads the module at another address, never
+// leaves a stale pointer behind.
+int static_workspace(void **ptr) {
+    void *p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_static_workspace);
+    if (e != cudaSuccess || !p)
+        return elsaa::set_last_error(ELSAA_ERR_CUDA,
+                                     "cudaGetSymbolAddress: %s",
+                                     cudaGetErrorString(e));
+    *ptr = p;
+    return ELSAA_OK;
+}
 
 }  // namespace
 
@@ -37,31 +46,28 @@ extern "C" int elsaa_forward_noalloc(const elsaa_params *params,
             "problem needs %zu bytes of scratch; the static array of "
             "elsaa_forward_noalloc holds %zu",
             need, (size_t)ELSAA_STATIC_WORKSPACE_BYTES);
-    int dev = -1;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess)
-        return elsaa::set_last_error(ELSAA_ERR_CUDA, "cudaGetDevice: %s",
-                                     cudaGetErrorString(e));
-    if (dev < 0 || dev >= kMaxDevices)
-        return elsaa::set_last_error(ELSAA_ERR_UNSUPPORTED,
-                                     "device ordinal %d above %d", dev,
-                                     kMaxDevices - 1);
     void *ws = nullptr;
-    {
-        std::lock_guard<std::mutex> lk(g_static_mu);
-        if (!g_static_ptr[dev]) {
-            // set-up, once per device, with that device current
-            void *p = nullptr;
-            e = cudaGetSymbolAddress(&p, g_static_workspace);
-            if (e != cudaSuccess || !p)
-                return elsaa::set_last_error(
-                    ELSAA_ERR_CUDA, "cudaGetSymbolAddress: %s",
-                    cudaGetErrorString(e));
-            g_static_ptr[dev] = p;
-        }
-        ws = g_static_ptr[dev];
-    }
+    rc = static_workspace(&ws);
+    if (rc != ELSAA_OK) return rc;
     return elsaa_forward(params, q, k, v, w_sort, w_race, lambda_tok, gates,
                          o, log_d_sparse, d_lr, m_sparse, perm_q, perm_k, ws,
                          ELSAA_STATIC_WORKSPACE_BYTES, stream);
+}
+
+// The status word of the forward pass sits at the start of its workspace,
+// here the start of the static array.
+extern "C" int elsaa_check_status_noalloc(void *stream) {
+    void *ws = nullptr;
+    int rc = static_workspace(&ws);
+    if (rc != ELSAA_OK) return rc;
+    return elsaa_check_status(ws, stream);
+}
+
+extern "C" int elsaa_selftest_wait_timeout_noalloc(int limit_ms,
+                                                   void *stream) {
+    void *ws = nullptr;
+    int rc = static_workspace(&ws);
+    if (rc != ELSAA_OK) return rc;
+    return elsaa_selftest_wait_timeout(ws, ELSAA_STATIC_WORKSPACE_BYTES,
+                                       limit_ms, stream);
 }

@@ -348,30 +348,6 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src,
         : "memory");
 }
 
-// TMA gather of four rows (tile::gather4, 2-D map with a one-row box): the
-// box of each row index in r goes to four consecutive 128-byte lines at dst
-// (the 128-byte swizzle follows the shared-memory address).
-__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap *map,
-                                            int x, int4 r, uint64_t *bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cta.global.tile::gather4.mbarrier::"
-        "complete_tx::bytes [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(r.x), "r"(r.y),
-        "r"(r.z), "r"(r.w), "r"(smem_u32(bar))
-        : "memory");
-}
-
-// TMA scatter of four rows (tile::scatter4), the inverse of tma_gather4.
-__device__ __forceinline__ void tma_scatter4(const CUtensorMap *map, int x,
-                                             int4 r, uint32_t src) {
-    asm volatile(
-        "cp.async.bulk.tensor.2d.global.shared::cta.tile::scatter4.bulk_group"
-        " [%0, {%1, %2, %3, %4, %5}], [%6];" ::"l"(
-            reinterpret_cast<uint64_t>(map)),
-        "r"(x), "r"(r.x), "r"(r.y), "r"(r.z), "r"(r.w), "r"(src)
-        : "memory");
-}
-
 __device__ __forceinline__ void bulk_commit() {
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
 }

@@ -76,6 +76,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     const float *__restrict__ Ag,
                     const float *__restrict__ lambda_tok,
                     const float *__restrict__ gates, uint16_t *__restrict__ ox,
+                    float *__restrict__ o32,
                     float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
                     float *__restrict__ m_out, int N, int d, int H, int b,
                     int nb, int L, int Lg_pad, float beta, float eps,
@@ -709,7 +710,8 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             // O = c1 acc as bf16, this half's d / 2 columns, staged in this
             // slot's V buffer (the P V product of the tile is complete) in
             // the swizzled panel layout, then copied out by the slot's 256
-            // threads in whole rows (coalesced 16-byte stores)
+            // threads in whole rows (coalesced 16-byte stores). With an
+            // fp32 output (o32) each thread stores its half row directly.
             const uint32_t sVg = sV0 + g * tileB;
             constexpr int kMaxHalf = 64;  // d / 2 for d = 128
 #pragma unroll
@@ -718,6 +720,20 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     uint32_t v[16], ob[8];
                     tmem_ld16(so + nk + half * (d >> 1) + c, v);
                     tmem_wait_ld();
+                    if (o32) {
+                        if (qvalid) {
+                            float4 *dst = reinterpret_cast<float4 *>(
+                                o32 + tok * (size_t)d + half * (d >> 1) + c);
+#pragma unroll
+                            for (int q = 0; q < 4; ++q)
+                                dst[q] = make_float4(
+                                    c1e * __uint_as_float(v[4 * q]),
+                                    c1e * __uint_as_float(v[4 * q + 1]),
+                                    c1e * __uint_as_float(v[4 * q + 2]),
+                                    c1e * __uint_as_float(v[4 * q + 3]));
+                        }
+                        continue;
+                    }
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
                         ob[q] = pack_bf16x2(c1e * __uint_as_float(v[2 * q]),
@@ -740,7 +756,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                 }
             }
             named_sync(1 + g, 256);
-            {
+            if (!o32) {
                 const int ct = (cw & 7) * 32 + lane_id;  // 0..255
                 const int cpr = d >> 3, rpp = 256 / cpr;
                 const int crow = ct / cpr, cc = ct - crow * cpr;
@@ -816,7 +832,8 @@ cudaError_t launch_block_attn_ws(
                              (int)smem);
         kern<<<grid, kWsThreads, smem, st>>>(
             (const uint16_t *)q, (const uint16_t *)k, (const uint16_t *)v,
-            tmW, tmB, perm_q, perm_k, A, lambda_tok, gates, (uint16_t *)o,
+            tmW, tmB, perm_q, perm_k, A, lambda_tok, gates,
+            P.o32 ? nullptr : (uint16_t *)o, P.o32 ? (float *)o : nullptr,
             log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, P.nb, P.L, lg,
             P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, tiles_per_head,
             total, status);

@@ -30,7 +30,10 @@ SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_profile_stop", "elsaa_forward_noalloc",
            "elsaa_backward_workspace_size", "elsaa_backward",
            "elsaa_gates_workspace_size", "elsaa_gates",
-           "elsaa_selftest_wait_timeout", "elsaa_forward_race_summaries")
+           "elsaa_selftest_wait_timeout", "elsaa_forward_race_summaries",
+           "elsaa_check_status_noalloc",
+           "elsaa_selftest_wait_timeout_noalloc", "elsaa_causal_levels",
+           "elsaa_causal_index_lists")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -47,7 +50,7 @@ class elsaa_params(ctypes.Structure):
         ("scale", ctypes.c_float), ("lam", ctypes.c_float),
         ("fusion_mode", ctypes.c_int), ("impl", ctypes.c_int),
         ("neighbor_blocks", ctypes.c_int), ("causal_chunk", ctypes.c_int),
-        ("causal_base_len", ctypes.c_int),
+        ("causal_base_len", ctypes.c_int), ("out_fp32", ctypes.c_int),
     ]
 
 
@@ -128,6 +131,16 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
     L.elsaa_selftest_wait_timeout.argtypes = [vp, ctypes.c_size_t,
                                               ctypes.c_int, vp]
     L.elsaa_selftest_wait_timeout.restype = ctypes.c_int
+    L.elsaa_causal_levels.argtypes = [ctypes.POINTER(elsaa_params),
+                                      ctypes.POINTER(ctypes.c_int)]
+    L.elsaa_causal_levels.restype = ctypes.c_int
+    L.elsaa_causal_index_lists.argtypes = [ctypes.POINTER(elsaa_params), vp,
+                                           ctypes.c_size_t, vp, vp]
+    L.elsaa_causal_index_lists.restype = ctypes.c_int
+    L.elsaa_check_status_noalloc.argtypes = [vp]
+    L.elsaa_check_status_noalloc.restype = ctypes.c_int
+    L.elsaa_selftest_wait_timeout_noalloc.argtypes = [ctypes.c_int, vp]
+    L.elsaa_selftest_wait_timeout_noalloc.restype = ctypes.c_int
     _lib = L
     return L
 
@@ -149,13 +162,13 @@ def make_params(B, H, N, d_h, dtype="bf16", block_size=64, sort_bits=5,
                 gray_order=1, race_tables=4, race_bits=4, beta=1.0, eps=1e-6,
                 scale=0.0, lam=1.0, fusion_mode=0, causal=0,
                 impl=ELSAA_IMPL_AUTO, neighbor_blocks=0, causal_chunk=128,
-                causal_base_len=4096) -> elsaa_params:
+                causal_base_len=4096, out_fp32=0) -> elsaa_params:
     dt = {"bf16": ELSAA_BF16, "fp32": ELSAA_FP32}[dtype] if isinstance(
         dtype, str) else int(dtype)
     return elsaa_params(B, H, N, d_h, dt, causal, block_size, sort_bits,
                         gray_order, race_tables, race_bits, beta, eps, scale,
                         lam, fusion_mode, impl, neighbor_blocks, causal_chunk,
-                        causal_base_len)
+                        causal_base_len, out_fp32)
 
 
 def params_for(wl, **over) -> elsaa_params:
@@ -217,10 +230,11 @@ def elsaa_forward(params: elsaa_params, q, k, v, w_sort, w_race,
     if dev.type != "cuda":
         raise ValueError("q must be a CUDA tensor")
     tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    odt = torch.float32 if params.out_fp32 else tdt
     BHN = params.B * params.H * params.N
     nqkv = BHN * params.d_h
     if o is None:
-        o = torch.empty_like(q)
+        o = torch.empty(q.shape, dtype=odt, device=dev)
     if workspace is None:
         workspace = new_workspace(params, dev)
     if stream is None:
@@ -237,7 +251,7 @@ def elsaa_forward(params: elsaa_params, q, k, v, w_sort, w_race,
              dev),
         _ptr(lambda_tok, "lambda_tok", torch.float32, BHN, dev),
         _ptr(gates, "gates", torch.float32, 2 * BHN, dev),
-        _ptr(o, "o", tdt, nqkv, dev),
+        _ptr(o, "o", odt, nqkv, dev),
         _ptr(log_d_sparse, "log_d_sparse", torch.float32, BHN, dev),
         _ptr(d_lr, "d_lr", torch.float32, BHN, dev),
         _ptr(m_sparse, "m_sparse", torch.float32, BHN, dev),
@@ -446,8 +460,9 @@ def elsaa_forward_noalloc(params: elsaa_params, q, k, v, w_sort, w_race,
 
     Scratch comes from the library's fixed ELSAA_STATIC_WORKSPACE_BYTES
     array, shared by all calls: order overlapping calls on one stream. The
-    first call on a device looks up that array and should precede any
-    stream capture. `o` must be given (nothing is allocated here either).
+    first call on a device may load the library's module there and should
+    precede any stream capture. `o` must be given (nothing is allocated here
+    either). elsaa_check_status_noalloc reads the call's status word.
     """
     lib = load_library()
     if o is None:
@@ -455,6 +470,7 @@ def elsaa_forward_noalloc(params: elsaa_params, q, k, v, w_sort, w_race,
                          "nothing")
     dev = q.device
     tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    odt = torch.float32 if params.out_fp32 else tdt
     BHN = params.B * params.H * params.N
     nqkv = BHN * params.d_h
     if stream is None:
@@ -471,7 +487,7 @@ def elsaa_forward_noalloc(params: elsaa_params, q, k, v, w_sort, w_race,
              dev),
         _ptr(lambda_tok, "lambda_tok", torch.float32, BHN, dev),
         _ptr(gates, "gates", torch.float32, 2 * BHN, dev),
-        _ptr(o, "o", tdt, nqkv, dev),
+        _ptr(o, "o", odt, nqkv, dev),
         _ptr(log_d_sparse, "log_d_sparse", torch.float32, BHN, dev),
         _ptr(d_lr, "d_lr", torch.float32, BHN, dev),
         _ptr(m_sparse, "m_sparse", torch.float32, BHN, dev),
@@ -480,3 +496,50 @@ def elsaa_forward_noalloc(params: elsaa_params, q, k, v, w_sort, w_race,
     ]
     _check(lib.elsaa_forward_noalloc(ctypes.byref(params), *args, sp))
     return o
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return stream.cuda_stream if hasattr(stream, "cuda_stream") else stream
+
+
+def elsaa_check_status_noalloc(stream=None):
+    """elsaa_check_status for elsaa_forward_noalloc: synchronise and raise
+    ElsaaError if a kernel recorded a fault in the static array's status
+    word."""
+    _check(load_library().elsaa_check_status_noalloc(_stream_ptr(stream)))
+
+
+def elsaa_selftest_wait_timeout_noalloc(limit_ms=100, stream=None):
+    """The bounded-wait self-test on the static array's status word."""
+    _check(load_library().elsaa_selftest_wait_timeout_noalloc(
+        int(limit_ms), _stream_ptr(stream)))
+
+
+def elsaa_causal_levels(params: elsaa_params) -> int:
+    """Halving levels Lv of the causal sparse branch for params."""
+    n = ctypes.c_int(0)
+    _check(load_library().elsaa_causal_levels(ctypes.byref(params),
+                                              ctypes.byref(n)))
+    return n.value
+
+
+def elsaa_causal_index_lists(params: elsaa_params, workspace, lists=None,
+                             stream=None):
+    """Sorted orders of every SortLSH call of the last causal forward on
+    `workspace`: int32 [Lv, 2, B, H, N / 2] (allocated here when not
+    given; None when Lv = 0). See include/elsaa.h for the layout."""
+    lv = elsaa_causal_levels(params)
+    if lv == 0:
+        return None
+    dev = workspace.device
+    shape = (lv, 2, params.B, params.H, params.N // 2)
+    if lists is None:
+        lists = torch.empty(shape, dtype=torch.int32, device=dev)
+    n = lv * params.B * params.H * params.N
+    _check(load_library().elsaa_causal_index_lists(
+        ctypes.byref(params), _ptr(workspace, "workspace", None, None, dev),
+        workspace.numel() * workspace.element_size(),
+        _ptr(lists, "lists", torch.int32, n, dev), _stream_ptr(stream)))
+    return lists

@@ -80,6 +80,21 @@ def causal_flop_model(wl: Workload) -> dict:
             "bytes": 4 * N * d * wl.elt * heads}
 
 
+def backward_flop_model(wl: Workload) -> dict:
+    """Tensor FLOPs and algorithmic HBM bytes of one backward pass (dQ, dK,
+    dV in fp32), per head: sparse blocks 10 N b d_h (recomputed scores, P V
+    for O_s, and the products for dV, dP, dQ, dK), RACE 8 N r d_h (Num
+    recomputed, gB and gA sums, dL/dphi of queries and keys, dV of the
+    summaries), projections 8 N d_h L_s gamma (recomputed and
+    back-propagated for queries and keys). Bytes: Q, K, V and dO read once,
+    dQ, dK, dV written once in fp32."""
+    N, b, d, r = wl.N, keys_per_query(wl), wl.d_h, wl.r
+    per_head = (10 * N * b * d + 8 * N * r * d
+                + 8 * N * d * wl.race_tables * wl.race_bits)
+    return {"tensor_flops": per_head * wl.heads,
+            "bytes": (4 * N * d * wl.elt + 3 * N * d * 4) * wl.heads}
+
+
 def keys_per_query(wl: Workload) -> int:
     """Keys each query attends to in the sparse branch: its block and the
     neighbouring sorted blocks, (2 r + 1) b (Section 5), at most N (the

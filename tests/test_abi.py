@@ -58,7 +58,7 @@ def test_params_struct_matches_header():
 
 
 def test_abi_version(lib):
-    assert elsaa.elsaa_abi_version() == 4
+    assert elsaa.elsaa_abi_version() == 5
 
 
 @pytest.mark.parametrize("name", sorted(WORKLOADS))
@@ -95,7 +95,24 @@ BAD = [
     (dict(fusion_mode=3), elsaa.ELSAA_ERR_INVALID_ARG, "fusion_mode"),
     (dict(B=0), elsaa.ELSAA_ERR_INVALID_ARG, "positive"),
     (dict(neighbor_blocks=-1), elsaa.ELSAA_ERR_INVALID_ARG, "neighbor"),
+    (dict(out_fp32=2), elsaa.ELSAA_ERR_INVALID_ARG, "out_fp32"),
 ]
+
+
+@pytest.mark.parametrize("N,N0,levels", [(16384, 4096, 2), (1024, 256, 2),
+                                         (2048, 300, 3), (512, 4096, 0)])
+def test_causal_levels(lib, N, N0, levels):
+    p = elsaa.make_params(B=1, H=2, N=N, d_h=128, block_size=128,
+                          race_tables=16, causal=1, causal_base_len=N0)
+    assert elsaa.elsaa_causal_levels(p) == levels
+
+
+def test_causal_index_lists_rejects_non_causal(lib):
+    p = elsaa.make_params(B=1, H=2, N=256, d_h=64, block_size=64,
+                          race_tables=4)
+    rc = lib.elsaa_causal_index_lists(ctypes.byref(p), None, 0, None, None)
+    assert rc == elsaa.ELSAA_ERR_INVALID_ARG
+    assert "causal" in elsaa.elsaa_last_error()
 
 
 @pytest.mark.parametrize("over,code,word", BAD)

@@ -111,6 +111,25 @@ def _split_rule_sets(n, b, N0):
     return sets
 
 
+def _trace_sets(mod, n, hq, hk, b, N0):
+    """Each row's key set rebuilt from the SortLSH orders the recursion
+    records (its trace) alone: the row's base-segment prefix, plus at every
+    recorded call the past-half keys of the block holding the row's sorted
+    position. Needs n = n_leaf 2^k (no padding)."""
+    trace = []
+    Q = np.zeros((n, 2))
+    mod.causal_sparse(Q, Q, Q, hq, hk, 0, b, N0, 1.0, 0.0, trace)
+    leaf = n
+    while leaf > N0:
+        leaf //= 2
+    sets = [set(range(i - i % leaf, i + 1)) for i in range(n)]
+    for _, _, qrows, krows in trace:
+        for p, i in enumerate(qrows):
+            t = p // b
+            sets[int(i)] |= set(int(j) for j in krows[t * b:(t + 1) * b])
+    return sets
+
+
 def check_sparse_pins(mod):
     scale = 0.7
     # (1) n <= N0: exact causal attention
@@ -138,10 +157,40 @@ def check_sparse_pins(mod):
                            b, N0)
         for i, ks in want.items():
             assert got[i] == ks, (name, i, got[i], ks)
+        # the recorded sorted orders give the same sets
+        got = _trace_sets(mod, 8, codes.get("q", z8), codes.get("k", z8), b,
+                          N0)
+        for i, ks in want.items():
+            assert got[i] == ks, (name, "trace", i, got[i], ks)
     for n, b, N0 in [(64, 8, 8), (50, 4, 6), (41, 8, 5), (96, 16, 12)]:
         zn = np.zeros(n, np.uint16)
         assert _attend_sets(mod, n, zn, zn, 0, b, N0) == \
             _split_rule_sets(n, b, N0), (n, b, N0)
+    for n, b, N0 in [(64, 8, 8), (96, 16, 12)]:
+        zn = np.zeros(n, np.uint16)
+        assert _trace_sets(mod, n, zn, zn, b, N0) == \
+            _split_rule_sets(n, b, N0), (n, b, N0)
+    # with random codes: the trace's orders are stable argsorts of each
+    # half's codes, and rebuild the sets the one-hot run shows
+    rng = np.random.default_rng(17)
+    n, b, N0 = 64, 4, 8
+    hq = rng.integers(0, 4, n).astype(np.uint16)
+    hk = rng.integers(0, 4, n).astype(np.uint16)
+    trace = []
+    Q = np.zeros((n, 2))
+    mod.causal_sparse(Q, Q, Q, hq, hk, 0, b, N0, 1.0, 0.0, trace)
+    assert sorted((t[0], t[1]) for t in trace) == [
+        (1, 0), (2, 0), (2, 32), (3, 0), (3, 16), (3, 32), (3, 48)]
+    for level, start, qrows, krows in trace:
+        m = n >> level
+        fut = np.arange(start + m, start + 2 * m)
+        past = np.arange(start, start + m)
+        np.testing.assert_array_equal(
+            qrows, fut[np.argsort(hq[fut], kind="stable")])
+        np.testing.assert_array_equal(
+            krows, past[np.argsort(hk[past], kind="stable")])
+    assert _trace_sets(mod, n, hq, hk, b, N0) == \
+        _attend_sets(mod, n, hq, hk, 0, b, N0)
     # ... and with real scores, softmax over exactly those sets
     n, b, N0 = 50, 4, 6
     Q, K, V = _qkv(n, seed=5, temp=2.0)

@@ -51,7 +51,13 @@ def run_gpu(wl, x, gates=None, lam=None, impl=elsaa.ELSAA_IMPL_AUTO, **over):
     torch.cuda.synchronize()
     res = {k: v.cpu() for k, v in out.items()}
     res["O"] = o.float().cpu()
+    res["O_raw"] = o.cpu()
     return res
+
+
+def rel_l2(got, ref):
+    """Relative error ||got - ref|| / ||ref|| (reported beside max-abs)."""
+    return float(np.linalg.norm(got - ref) / np.linalg.norm(ref))
 
 
 def run_oracle(wl, x, gates=None, lam=None, heads=None, rows=None, **over):
@@ -71,7 +77,11 @@ def compare(wl, g, ref, rows=None, label=""):
         O = g["O"][b, h].numpy()[idx]
         err = np.abs(O - r["O"]).max()
         worst = max(worst, err)
+        rel = rel_l2(O, r["O"])
+        print("%s head (%d, %d): max |O - O_ref| = %.3e, relative (l2) "
+              "%.3e" % (label, b, h, err, rel))
         assert err <= TOL_O[wl.dtype], (label, b, h, "O", err)
+        assert rel <= TOL_O[wl.dtype], (label, b, h, "O relative", rel)
         e_logd = np.abs(g["log_d_sparse"][b, h].numpy()[idx] -
                         r["log_d_sparse"]).max()
         assert e_logd <= TOL_LOGD[wl.dtype], (label, b, h, "logd", e_logd)
@@ -114,6 +124,28 @@ def test_shapes(d_h, b, L, gamma):
                N=b * 7, H=2, B=2)
     x = make_inputs(wl)
     compare(wl, run_gpu(wl, x), run_oracle(wl, x), label="shape")
+
+
+@pytest.mark.parametrize("d_h,b,nb,impl", [
+    (128, 128, 0, elsaa.ELSAA_IMPL_AUTO),   # one key pass
+    (64, 64, 0, elsaa.ELSAA_IMPL_AUTO),
+    (128, 256, 0, elsaa.ELSAA_IMPL_AUTO),   # two key passes
+    (128, 128, 1, elsaa.ELSAA_IMPL_AUTO),   # neighbour window
+    (64, 64, 0, elsaa.ELSAA_IMPL_SIMT),     # CUDA cores
+])
+def test_fp32_output_of_bf16_inputs(d_h, b, nb, impl):
+    """out_fp32 = 1: the same arithmetic without the final rounding of O to
+    bf16. O within the bf16-input bound of the oracle, and the bf16 output
+    of the same call equals it rounded to bf16."""
+    wl = small("bf16", d_h=d_h, block=b, race_tables=8, N=b * 9, H=2, B=2,
+               neighbor_blocks=nb)
+    x = make_inputs(wl)
+    ref = run_oracle(wl, x)
+    g32 = run_gpu(wl, x, impl=impl, out_fp32=1)
+    assert g32["O_raw"].dtype == torch.float32
+    compare(wl, g32, ref, label="fp32 out")
+    g16 = run_gpu(wl, x, impl=impl)
+    assert torch.equal(g16["O_raw"], g32["O_raw"].to(torch.bfloat16))
 
 
 def test_gates_and_per_token_lambda():

@@ -2,17 +2,23 @@
 device memory (for example a plug-in whose host application owns all device
 buffers and offers no allocator, or a path that must not risk the
 device-wide synchronisation of cudaMalloc / cudaFree). Its scratch is a fixed
-array inside the library, so these checks compare it with elsaa_forward
-(caller-provided workspace) on two calls in a row, and check that a problem
-larger than the array is refused.
+array inside the library, shared by every call, so these checks compare it
+with elsaa_forward (caller-provided workspace) on calls in a row, including a
+larger problem followed by a smaller one of another shape (stale scratch from
+the first must not reach the second), read its status word through
+elsaa_check_status_noalloc, and check that a problem larger than the array is
+refused.
 
 This file is named so that pytest collects it last.
 """
 import ctypes
+import time
 
+import numpy as np
 import pytest
 import torch
 
+from oracle import oracle as orc
 from paper_2607_20214_gb300 import build, elsaa
 from paper_2607_20214_gb300.workloads import Workload, make_inputs
 
@@ -27,34 +33,79 @@ def _lib():
     elsaa.load_library()
 
 
-def _case(dtype):
-    return Workload("noalloc", B=2, H=2, N=1184, d_h=64, dtype=dtype,
-                    block=32, race_tables=4, recipe="plain", temperature=2.0,
-                    seed=21, plane_seed=1021)
+def _case(dtype, N=1184, block=32, seed=21):
+    return Workload("noalloc", B=2, H=2, N=N, d_h=64, dtype=dtype,
+                    block=block, race_tables=4, recipe="plain",
+                    temperature=2.0, seed=seed, plane_seed=1000 + seed)
 
 
-@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
-def test_noalloc_matches_workspace_entry_point_twice(dtype):
-    wl = _case(dtype)
-    dev = torch.device("cuda:0")
+def _compare(wl, dev):
+    """One elsaa_forward_noalloc call against elsaa_forward on the same
+    inputs: O within the dtype's bound, both sort orders identical."""
+    dtype = wl.dtype
     x = {k: t.to(dev) for k, t in make_inputs(wl).items()}
     p = elsaa.params_for(wl)
     assert elsaa.elsaa_workspace_size(p) <= \
         elsaa.ELSAA_STATIC_WORKSPACE_BYTES
     BHN = (wl.B, wl.H, wl.N)
-    ref_perm = torch.empty(BHN, dtype=torch.int32, device=dev)
+    ref_pq = torch.empty(BHN, dtype=torch.int32, device=dev)
+    ref_pk = torch.empty(BHN, dtype=torch.int32, device=dev)
     ref = elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
-                              x["w_race"], perm_q=ref_perm)
+                              x["w_race"], perm_q=ref_pq, perm_k=ref_pk)
     torch.cuda.synchronize()
-    for call in range(2):
-        o = torch.full_like(x["q"], float("nan"))
-        perm = torch.full(BHN, -1, dtype=torch.int32, device=dev)
-        elsaa.elsaa_forward_noalloc(p, x["q"], x["k"], x["v"], x["w_sort"],
-                                    x["w_race"], o=o, perm_q=perm)
-        torch.cuda.synchronize()
-        err = (o.float() - ref.float()).abs().max().item()
-        assert err <= TOL[dtype], (call, err)
-        assert torch.equal(perm, ref_perm), call
+    o = torch.full_like(x["q"], float("nan"))
+    pq = torch.full(BHN, -1, dtype=torch.int32, device=dev)
+    pk = torch.full(BHN, -1, dtype=torch.int32, device=dev)
+    elsaa.elsaa_forward_noalloc(p, x["q"], x["k"], x["v"], x["w_sort"],
+                                x["w_race"], o=o, perm_q=pq, perm_k=pk)
+    elsaa.elsaa_check_status_noalloc()
+    err = (o.float() - ref.float()).abs().max().item()
+    assert err <= TOL[dtype], err
+    assert torch.equal(pq, ref_pq)
+    assert torch.equal(pk, ref_pk)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_noalloc_matches_workspace_entry_point_twice(dtype):
+    dev = torch.device("cuda:0")
+    for _ in range(2):
+        _compare(_case(dtype), dev)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "fp32"])
+def test_noalloc_larger_then_smaller_problem(dtype):
+    """The shared array keeps the previous call's contents: a smaller call
+    of another N and block size after a larger one must match the
+    workspace entry point exactly in its sort orders."""
+    dev = torch.device("cuda:0")
+    _compare(_case(dtype, N=4096, block=64, seed=23), dev)
+    _compare(_case(dtype, N=1184, block=32, seed=24), dev)
+
+
+def test_noalloc_status_word_reports_timeout_then_clears():
+    """The static array's status word is readable without its address: the
+    bounded-wait self-test records a timeout there, and the next forward
+    clears it and matches the oracle."""
+    dev = torch.device("cuda:0")
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    elsaa.elsaa_selftest_wait_timeout_noalloc(limit_ms=100)
+    with pytest.raises(elsaa.ElsaaError) as e:
+        elsaa.elsaa_check_status_noalloc()
+    assert time.perf_counter() - t0 >= 0.1
+    assert e.value.code == elsaa.ELSAA_ERR_DEVICE
+    assert "status 3" in str(e.value)
+    assert "site %d" % 0x7E57 in str(e.value)
+    wl = _case("bf16", seed=25)
+    x = make_inputs(wl)
+    xd = {k: v.to(dev) for k, v in x.items()}
+    o = torch.empty_like(xd["q"])
+    elsaa.elsaa_forward_noalloc(elsaa.params_for(wl), xd["q"], xd["k"],
+                                xd["v"], xd["w_sort"], xd["w_race"], o=o)
+    elsaa.elsaa_check_status_noalloc()
+    ref = orc.forward(x, orc.params_from_workload(wl), heads=[(1, 0)])
+    err = np.abs(o[1, 0].float().cpu().numpy() - ref[(1, 0)]["O"]).max()
+    assert err <= TOL["bf16"]
 
 
 def test_noalloc_refuses_problem_larger_than_its_array():
