@@ -363,3 +363,145 @@ void elsaa_oracle_dense_rows(const double *Q, const double *K,
     }
     free(z);
 }
+
+/* ------------------------------------------------------ top-k selector */
+/*
+ * An alternative selector for the sparse branch. Section 3 ("sorted Hamming
+ * LSH") names learned top-k, sliding windows and global tokens as selectors
+ * a future version could use in place of the sorted blocks; the paper
+ * defines none of them. Reading taken here (each step also listed in the
+ * design notes):
+ *   1. after the hash and the stable sort of Algorithm sortLSH, block t of
+ *      the sorted queries (positions [t b, (t+1) b)) and block u of the
+ *      sorted keys are summarised by their sums qbar_t, kbar_u (fp32,
+ *      sequential over increasing sorted position from +0.0f);
+ *   2. block score s(t, u) = <qbar_t, kbar_u> (the canonical fp32 FMA chain
+ *      of the sort hash); query block t takes its own key block t and the
+ *      c - 1 other key blocks of largest score (equal scores: lower u);
+ *   3. query i of block t scores every key j of those c blocks with
+ *      <q_i, k_j> (the same chain, unscaled) and keeps the k of largest
+ *      score (equal scores: lower original key index j);
+ *   4. the sparse branch is the block step of Algorithm sortLSH over that
+ *      set: d_s,i = sum_j exp(z_ij), O_s,i = sum_j exp(z_ij) V_j /
+ *      (d_s,i + eps); RACE and the fusion are unchanged.
+ * With c = 1 and k = b every query keeps its whole block: the sorted-block
+ * branch. With c = N / b and k = N every query attends every key.
+ */
+
+/* The canonical fp32 chain sum_e a[e] b[e] over e = 0 .. d-1 (one rounding
+ * per fused multiply-add, from +0.0f): the precision in which both this
+ * oracle and the device take every selection decision. */
+static float select_dot(const float *a, const float *b, int d) {
+    float acc = 0.0f;
+    for (int e = 0; e < d; ++e) acc = fmaf(a[e], b[e], acc);
+    return acc;
+}
+
+/* Step 1: sums[t][e] = sum over sorted positions p = t b .. t b + b - 1 (in
+ * that order) of x[perm[p]][e], fp32, for the N / b blocks. */
+void elsaa_oracle_block_sums(const float *x, int N, int d_h,
+                             const int32_t *perm, int b, float *sums) {
+    int T = N / b;
+    for (int t = 0; t < T; ++t)
+        for (int e = 0; e < d_h; ++e) {
+            float acc = 0.0f;
+            for (int p = t * b; p < (t + 1) * b; ++p)
+                acc = acc + x[(size_t)perm[p] * d_h + e];
+            sums[(size_t)t * d_h + e] = acc;
+        }
+}
+
+/* Step 2: cand[t][0] = t; cand[t][1 .. c) = the c - 1 blocks u != t of
+ * largest s(t, u), in order of decreasing score (equal scores: lower u). */
+void elsaa_oracle_topk_candidates(const float *qsum, const float *ksum,
+                                  int T, int d_h, int c, int32_t *cand) {
+    float *s = (float *)malloc(sizeof(float) * (size_t)T);
+    char *taken = (char *)malloc((size_t)T);
+    for (int t = 0; t < T; ++t) {
+        for (int u = 0; u < T; ++u) {
+            s[u] = select_dot(qsum + (size_t)t * d_h, ksum + (size_t)u * d_h,
+                              d_h);
+            taken[u] = 0;
+        }
+        cand[(size_t)t * c] = t;
+        taken[t] = 1;
+        for (int m = 1; m < c; ++m) {
+            int best = -1;
+            for (int u = 0; u < T; ++u)  /* strict >: lower u wins ties */
+                if (!taken[u] && (best < 0 || s[u] > s[best])) best = u;
+            cand[(size_t)t * c + m] = best;
+            taken[best] = 1;
+        }
+    }
+    free(taken);
+    free(s);
+}
+
+/* Step 3 for the queries rows[0 .. n_rows) (original indices): query i at
+ * sorted position p (block t = p / b) keeps the k candidate keys of largest
+ * <q_i, k_j>, equal scores by lower j; sel[m][0 .. k) lists the keys of
+ * rows[m] by increasing j. */
+void elsaa_oracle_topk_select_rows(const float *q, const float *kx, int N,
+                                   int d_h, const int32_t *perm_q,
+                                   const int32_t *perm_k, int b,
+                                   const int32_t *cand, int c, int k,
+                                   const int32_t *rows, int n_rows,
+                                   int32_t *sel) {
+    int nc = c * b;
+    int32_t *pos = (int32_t *)malloc(sizeof(int32_t) * (size_t)N);
+    int32_t *idx = (int32_t *)malloc(sizeof(int32_t) * (size_t)nc);
+    float *sc = (float *)malloc(sizeof(float) * (size_t)nc);
+    char *keep = (char *)malloc((size_t)nc);
+    for (int p = 0; p < N; ++p) pos[perm_q[p]] = p;
+    for (int r = 0; r < n_rows; ++r) {
+        int i = rows[r], t = pos[i] / b;
+        const float *qi = q + (size_t)i * d_h;
+        for (int m = 0; m < c; ++m) {
+            int u = cand[(size_t)t * c + m];
+            for (int o = 0; o < b; ++o) {
+                int j = perm_k[u * b + o];
+                idx[m * b + o] = j;
+                sc[m * b + o] = select_dot(qi, kx + (size_t)j * d_h, d_h);
+            }
+        }
+        /* candidate a beats candidate x when its score is larger, or equal
+         * with a lower key index: keep a when fewer than k candidates beat
+         * it (the order is total: each key appears once) */
+        for (int a = 0; a < nc; ++a) {
+            int beaten = 0;
+            for (int x = 0; x < nc; ++x)
+                if (sc[x] > sc[a] || (sc[x] == sc[a] && idx[x] < idx[a]))
+                    ++beaten;
+            keep[a] = beaten < k;
+        }
+        /* the kept keys by increasing index */
+        int32_t *out = sel + (size_t)r * k;
+        int n = 0;
+        for (int a = 0; a < nc; ++a)
+            if (keep[a]) out[n++] = idx[a];
+        for (int x = 1; x < n; ++x)  /* insertion sort */
+            for (int y = x; y > 0 && out[y - 1] > out[y]; --y) {
+                int32_t tmp = out[y];
+                out[y] = out[y - 1];
+                out[y - 1] = tmp;
+            }
+    }
+    free(keep);
+    free(sc);
+    free(idx);
+    free(pos);
+}
+
+/* Step 4 for rows[0 .. n_rows): the block step of Algorithm sortLSH over
+ * each row's selected keys sel[m][0 .. k) (as step 3 lists them). */
+void elsaa_oracle_sparse_sets_rows(const double *Q, const double *K,
+                                   const double *V, int d_h,
+                                   const int32_t *sel, int k, double scale,
+                                   double eps, const int32_t *rows,
+                                   int n_rows, double *O_rows,
+                                   double *d_rows, double *logd_rows) {
+    for (int m = 0; m < n_rows; ++m)
+        block_row(Q + (size_t)rows[m] * d_h, K, V, d_h, sel + (size_t)m * k,
+                  k, scale, eps, O_rows + (size_t)m * d_h, d_rows + m,
+                  logd_rows + m);
+}

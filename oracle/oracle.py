@@ -70,6 +70,16 @@ def configure(L):
     L.elsaa_oracle_fuse_rows.argtypes = [
         ctypes.c_int, ctypes.c_int, _dp, _dp, _dp, _dp, _dp, _dp, _dp,
         _dp, ctypes.c_double, ctypes.c_int, _dp, _dp, _dp]
+    L.elsaa_oracle_block_sums.argtypes = [
+        _fp, ctypes.c_int, ctypes.c_int, _ip, ctypes.c_int, _fp]
+    L.elsaa_oracle_topk_candidates.argtypes = [
+        _fp, _fp, ctypes.c_int, ctypes.c_int, ctypes.c_int, _ip]
+    L.elsaa_oracle_topk_select_rows.argtypes = [
+        _fp, _fp, ctypes.c_int, ctypes.c_int, _ip, _ip, ctypes.c_int, _ip,
+        ctypes.c_int, ctypes.c_int, _ip, ctypes.c_int, _ip]
+    L.elsaa_oracle_sparse_sets_rows.argtypes = [
+        _dp, _dp, _dp, ctypes.c_int, _ip, ctypes.c_int, ctypes.c_double,
+        ctypes.c_double, _ip, ctypes.c_int, _dp, _dp, _dp]
     L.elsaa_oracle_dense_rows.argtypes = [
         _dp, _dp, _dp, ctypes.c_int, ctypes.c_int, ctypes.c_double, _ip,
         ctypes.c_int, _dp, _dp]
@@ -199,6 +209,64 @@ def sortlsh_rows(Q, K, V, perm_q, perm_k, b, scale, eps, rows, nb=0):
     return O, ds, lds
 
 
+def block_sums(x32, perm, b):
+    """Top-k selector step 1: fp32 sums of each sorted block, [N / b, d]."""
+    x32 = _c(x32, np.float32)
+    N, d = x32.shape
+    out = np.zeros((N // b, d), dtype=np.float32)
+    lib().elsaa_oracle_block_sums(_ptr(x32, _fp), N, d,
+                                  _ptr(_c(perm, np.int32), _ip), b,
+                                  _ptr(out, _fp))
+    return out
+
+
+def topk_candidates(qsum, ksum, c):
+    """Top-k selector step 2: candidate key blocks [T, c] of every query
+    block (its own block first)."""
+    qsum = _c(qsum, np.float32)
+    ksum = _c(ksum, np.float32)
+    T, d = qsum.shape
+    cand = np.zeros((T, c), dtype=np.int32)
+    lib().elsaa_oracle_topk_candidates(_ptr(qsum, _fp), _ptr(ksum, _fp), T,
+                                       d, c, _ptr(cand, _ip))
+    return cand
+
+
+def topk_select_rows(q32, k32, perm_q, perm_k, b, cand, k, rows):
+    """Top-k selector step 3: the k selected key indices of each of the
+    query rows, [len(rows), k], increasing."""
+    q32 = _c(q32, np.float32)
+    k32 = _c(k32, np.float32)
+    N, d = q32.shape
+    cand = _c(cand, np.int32)
+    rows = _c(rows, np.int32)
+    sel = np.zeros((rows.shape[0], k), dtype=np.int32)
+    lib().elsaa_oracle_topk_select_rows(
+        _ptr(q32, _fp), _ptr(k32, _fp), N, d, _ptr(_c(perm_q, np.int32), _ip),
+        _ptr(_c(perm_k, np.int32), _ip), b, _ptr(cand, _ip), cand.shape[1],
+        k, _ptr(rows, _ip), rows.shape[0], _ptr(sel, _ip))
+    return sel
+
+
+def sparse_sets_rows(Q, K, V, sel, scale, eps, rows):
+    """Top-k selector step 4: the sparse branch over each row's set."""
+    Q = _c(Q, np.float64)
+    K = _c(K, np.float64)
+    V = _c(V, np.float64)
+    d = Q.shape[1]
+    sel = _c(sel, np.int32)
+    rows = _c(rows, np.int32)
+    n = rows.shape[0]
+    O = np.zeros((n, d), dtype=np.float64)
+    ds = np.zeros(n, dtype=np.float64)
+    lds = np.zeros(n, dtype=np.float64)
+    lib().elsaa_oracle_sparse_sets_rows(
+        _ptr(Q, _dp), _ptr(K, _dp), _ptr(V, _dp), d, _ptr(sel, _ip),
+        sel.shape[1], scale, eps, _ptr(rows, _ip), n, _ptr(O, _dp),
+        _ptr(ds, _dp), _ptr(lds, _dp))
+    return O, ds, lds
+
+
 def fuse_rows(O_s, d_s, log_d_s, O_lr, d_lr, lam, g_s, g_lr, eps, mode):
     O_s = _c(O_s, np.float64)
     n, d = O_s.shape
@@ -262,10 +330,23 @@ def forward_head(q32, k32, v32, w_sort, w_race, p: dict, lam=None,
     if rows is None:
         rows = np.arange(N, dtype=np.int32)
     rows = _c(rows, np.int32)
-    # Algorithm sortLSH: block attention, un-permuted to the requested rows.
-    O_s, d_s, log_d_s = sortlsh_rows(Q, K, V, perm_q, perm_k, p["block"],
-                                     scale, p["eps"], rows,
-                                     nb=p.get("neighbors", 0))
+    extra = {}
+    if p.get("selector", 0) == 1:
+        # top-k selector: block sums, candidate blocks, per-query top-k,
+        # then the block step over each query's selected keys
+        b = p["block"]
+        cand = topk_candidates(block_sums(q32, perm_q, b),
+                               block_sums(k32, perm_k, b), p["topk_blocks"])
+        sel = topk_select_rows(q32, k32, perm_q, perm_k, b, cand, p["topk"],
+                               rows)
+        O_s, d_s, log_d_s = sparse_sets_rows(Q, K, V, sel, scale, p["eps"],
+                                             rows)
+        extra = dict(cand=cand, sel=sel)
+    else:
+        # Algorithm sortLSH: block attention, un-permuted to the rows.
+        O_s, d_s, log_d_s = sortlsh_rows(Q, K, V, perm_q, perm_k, p["block"],
+                                         scale, p["eps"], rows,
+                                         nb=p.get("neighbors", 0))
     # Algorithm RACE: key-side summaries over all keys, query readout.
     A, Bs = race_summaries(K, V, w_race, p["beta"])
     O_lr, d_lr = race_readout_rows(Q, w_race, p["beta"], p["eps"], A, Bs,
@@ -285,7 +366,7 @@ def forward_head(q32, k32, v32, w_sort, w_race, p: dict, lam=None,
     return dict(O=O, O_sparse=O_s, d_sparse=d_s, log_d_sparse=log_d_s,
                 O_lr=O_lr, d_lr=d_lr, m=m, m_log=m_log, perm_q=perm_q,
                 perm_k=perm_k, keys_q=keys_q, keys_k=keys_k, A=A, B=Bs,
-                hash_fp64_mismatch=mis_q + mis_k, rows=rows)
+                hash_fp64_mismatch=mis_q + mis_k, rows=rows, **extra)
 
 
 def params_from_workload(wl, **over) -> dict:
@@ -297,6 +378,9 @@ def params_from_workload(wl, **over) -> dict:
     p["neighbors"] = getattr(wl, "neighbor_blocks", 0)
     p["causal_chunk"] = getattr(wl, "causal_chunk", 128)
     p["causal_base_len"] = getattr(wl, "causal_base_len", 4096)
+    p["selector"] = getattr(wl, "selector", 0)
+    p["topk"] = getattr(wl, "topk", 0)
+    p["topk_blocks"] = getattr(wl, "topk_blocks", 1)
     p.update(over)
     return p
 

@@ -43,6 +43,9 @@ class Workload:
     causal_chunk: int = 128  # C of causal RACE
     causal_base_len: int = 4096  # N_0 of CausalSparse (Table 7, text: 4096)
     neighbor_blocks: int = 0  # r neighbouring sorted key blocks per side
+    selector: int = 0  # 0: sorted blocks; 1: per-query top-k (candidates)
+    topk: int = 0  # k keys per query with selector 1
+    topk_blocks: int = 1  # c candidate key blocks per query block
     recipe: str = "plain"  # input recipe, see make_inputs
     temperature: float = 1.0
     seed: int = 0

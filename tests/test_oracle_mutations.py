@@ -13,6 +13,7 @@ import pytest
 
 from oracle import oracle as orc
 import test_oracle_pins as pins
+import test_oracle_topk as topk_pins
 
 MUTATIONS = [
     # (name, original text, planted mistake, pin expected to fail, args)
@@ -52,6 +53,31 @@ MUTATIONS = [
     ("gate_swapped", "g_lr[k] * O_lr[(size_t)k * d_h + e]",
      "g_s[k] * O_lr[(size_t)k * d_h + e]",
      pins.test_gates_select_branches_and_ablation_sets_m_to_one, ()),
+    # top-k selector
+    ("topk_tie_break_reversed",
+     "(sc[x] == sc[a] && idx[x] < idx[a])",
+     "(sc[x] == sc[a] && idx[x] > idx[a])",
+     topk_pins.test_hand_worked_example, ()),
+    ("topk_keeps_one_too_many", "keep[a] = beaten < k;",
+     "keep[a] = beaten <= k;",
+     topk_pins.test_integer_inputs_match_brute_force,
+     (64, 4, 8, 2, 8, 2, 0)),
+    ("topk_own_block_not_forced", "taken[t] = 1;", "taken[t] = 0;",
+     topk_pins.test_integer_inputs_match_brute_force,
+     (64, 4, 8, 3, 5, 1, 1)),
+    ("topk_block_tie_higher_u",
+     "if (!taken[u] && (best < 0 || s[u] > s[best])) best = u;",
+     "if (!taken[u] && (best < 0 || s[u] >= s[best])) best = u;",
+     topk_pins.test_hand_worked_example, ()),
+    ("topk_block_sum_skips_last_row",
+     "for (int p = t * b; p < (t + 1) * b; ++p)",
+     "for (int p = t * b; p < (t + 1) * b - 1; ++p)",
+     topk_pins.test_hand_worked_example, ()),
+    ("topk_scores_keys_against_keys",
+     "sc[m * b + o] = select_dot(qi, kx + (size_t)j * d_h, d_h);",
+     "sc[m * b + o] = select_dot(kx + (size_t)i * d_h, kx + (size_t)j * d_h, d_h);",
+     topk_pins.test_integer_inputs_match_brute_force,
+     (96, 6, 16, 2, 20, 2, 2)),
 ]
 
 
