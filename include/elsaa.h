@@ -45,7 +45,7 @@
 extern "C" {
 #endif
 
-#define ELSAA_ABI_VERSION 5
+#define ELSAA_ABI_VERSION 6
 
 /* Return codes. */
 #define ELSAA_OK 0
@@ -115,6 +115,27 @@ typedef struct elsaa_params {
                            not rounded to bf16 (the same arithmetic, with
                            the final rounding of a bf16 O left out). Not
                            used by elsaa_backward or elsaa_gates          */
+    int selector;       /* keys of the sparse branch. 0: the sorted key
+                           block (Algorithm sortLSH). 1: per-query top-k, a
+                           selector Section 3 names as future work, read
+                           here as: after the hash and stable sort, block
+                           sums qbar_t, kbar_u of the sorted blocks (fp32,
+                           sequential in sorted order); block scores
+                           <qbar_t, kbar_u>; query block t takes key block
+                           t and the topk_blocks - 1 other blocks of largest
+                           score (ties: lower block); each query keeps the
+                           topk candidate keys of largest <q_i, k_j> (ties:
+                           lower key index) and runs the block step over
+                           them. Every score is the sequential fp32 FMA
+                           chain of the sort hash, so the selected sets
+                           are exact. Requires causal = 0, neighbor_blocks
+                           = 0, topk_blocks * block_size <= 512 and at most
+                           8192 blocks per head; elsaa_backward returns
+                           ELSAA_ERR_UNSUPPORTED                           */
+    int topk;           /* selector 1: keys per query, 1 <= topk <=
+                           topk_blocks * block_size                        */
+    int topk_blocks;    /* selector 1: candidate key blocks per query
+                           block, 1 <= topk_blocks <= N / block_size       */
 } elsaa_params;
 
 /*
@@ -315,6 +336,18 @@ int elsaa_causal_levels(const elsaa_params *params, int *levels);
 int elsaa_causal_index_lists(const elsaa_params *params,
                              const void *workspace, size_t workspace_bytes,
                              int32_t *lists, void *stream);
+
+/*
+ * The key sets of the last elsaa_forward with params->selector = 1 enqueued
+ * with this `params` and `workspace`: keys[b][h][i][0 .. topk) = the
+ * original indices of the keys query i attends, increasing (device, int32,
+ * written, stream-ordered after that forward on `stream`).
+ * ELSAA_ERR_INVALID_ARG unless params->selector = 1; other errors as for
+ * elsaa_forward_race_summaries.
+ */
+int elsaa_forward_selected_keys(const elsaa_params *params,
+                                const void *workspace, size_t workspace_bytes,
+                                int32_t *keys, void *stream);
 
 /*
  * Token-wise gates and query-dependent lambda, the learned inputs of the

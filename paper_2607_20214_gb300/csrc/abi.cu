@@ -149,6 +149,24 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
         return bad(ELSAA_ERR_INVALID_ARG, "neighbor_blocks must be >= 0");
     if (p->out_fp32 != 0 && p->out_fp32 != 1)
         return bad(ELSAA_ERR_INVALID_ARG, "out_fp32 must be 0 or 1");
+    if (p->selector != 0 && p->selector != 1)
+        return bad(ELSAA_ERR_INVALID_ARG, "selector must be 0 or 1");
+    if (p->selector == 1) {
+        if (p->topk_blocks < 1 || p->topk_blocks > p->N / p->block_size)
+            return bad(ELSAA_ERR_INVALID_ARG,
+                       "selector 1: topk_blocks must be in [1, N / block_size]");
+        if (p->topk < 1 || (long)p->topk > (long)p->topk_blocks * p->block_size)
+            return bad(ELSAA_ERR_INVALID_ARG,
+                       "selector 1: topk must be in [1, topk_blocks * "
+                       "block_size]");
+        if (p->neighbor_blocks != 0)
+            return bad(ELSAA_ERR_INVALID_ARG,
+                       "selector 1: neighbor_blocks must be 0 (the candidate "
+                       "blocks replace the neighbour window)");
+        if (p->causal != 0)
+            return bad(ELSAA_ERR_UNSUPPORTED,
+                       "selector 1 is not built for the causal variant");
+    }
     if ((long)p->B * p->H > 65535)
         return bad(ELSAA_ERR_UNSUPPORTED, "B * H must be at most 65535");
     if ((long)p->B * p->H * p->N > (1L << 31) - 1)
@@ -179,6 +197,9 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     Q.lambda = p->lambda;
     Q.fusion_mode = p->fusion_mode;
     Q.o32 = p->dtype == ELSAA_BF16 && p->out_fp32 == 1;
+    Q.sel = p->selector;
+    Q.tk_k = Q.sel ? p->topk : 0;
+    Q.tk_c = Q.sel ? p->topk_blocks : 0;
     // neighbour windows wider than the sequence change nothing: clip
     Q.nb = p->neighbor_blocks < Q.N / Q.b ? p->neighbor_blocks : Q.N / Q.b;
     Q.impl = 1;
@@ -219,6 +240,18 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
     off = align_up(off + (size_t)Q.BH * Q.r * Q.d * sizeof(uint16_t), 256);
     Q.off_W = off;
     off = align_up(off + (size_t)Q.H * Q.Lg_pad * Q.d * sizeof(uint16_t), 256);
+    Q.off_sums = Q.off_cand = Q.off_mask = off;
+    if (Q.sel) {
+        if (!topk_supported(Q, msg)) return ELSAA_ERR_UNSUPPORTED;
+        const size_t T = (size_t)(Q.N / Q.b);
+        Q.off_sums = off;  // [2][BH][T][d] fp32 block sums
+        off = align_up(off + 2 * Q.BH * T * Q.d * sizeof(float), 256);
+        Q.off_cand = off;  // [BH][T][c] candidate blocks
+        off = align_up(off + Q.BH * T * Q.tk_c * sizeof(int32_t), 256);
+        Q.off_mask = off;  // [BH][N][c b / 32] selected candidates
+        off = align_up(off + BHN * (Q.tk_c * Q.b / 32) * sizeof(uint32_t),
+                       256);
+    }
     Q.total = off;
     *msg = "";
     return ELSAA_OK;
@@ -559,9 +592,12 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     DeviceStatus *status = (DeviceStatus *)(ws + P.off_status);
     uint32_t *keyrank = (uint32_t *)(ws + P.off_keyrank);
     int *hist = (int *)(ws + P.off_hist);
-    int32_t *pq = perm_q ? perm_q : (int32_t *)(ws + P.off_perm);
-    int32_t *pk = perm_k ? perm_k
-                         : (int32_t *)(ws + P.off_perm) + (size_t)P.BH * P.N;
+    // the top-k selector keeps the sorted orders in the workspace (the
+    // selected-key export reads them); the caller's copies follow
+    int32_t *pq = perm_q && !P.sel ? perm_q : (int32_t *)(ws + P.off_perm);
+    int32_t *pk = perm_k && !P.sel
+                      ? perm_k
+                      : (int32_t *)(ws + P.off_perm) + (size_t)P.BH * P.N;
     float *part = (float *)(ws + P.off_part);
     float *A = (float *)(ws + P.off_A);
     float *Bm = (float *)(ws + P.off_B);
@@ -612,11 +648,32 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                                       pk, status, st);
                        }),
                        "sort_scatter");
+    int32_t *cand = nullptr;
+    uint32_t *selmask = nullptr;
+    if (P.sel) {
+        cand = (int32_t *)(ws + P.off_cand);
+        selmask = (uint32_t *)(ws + P.off_mask);
+        ELSAA_CHECK_LAUNCH(timed("topk_select", st, [&] {
+                               return launch_topk(P, q, k, pq, pk,
+                                                  (float *)(ws + P.off_sums),
+                                                  cand, selmask, status, st);
+                           }),
+                           "topk_select");
+        const size_t pb = (size_t)P.BH * P.N * sizeof(int32_t);
+        if (perm_q)
+            ELSAA_CHECK_LAUNCH(cudaMemcpyAsync(perm_q, pq, pb,
+                                               cudaMemcpyDeviceToDevice, st),
+                               "copy of perm_q");
+        if (perm_k)
+            ELSAA_CHECK_LAUNCH(cudaMemcpyAsync(perm_k, pk, pb,
+                                               cudaMemcpyDeviceToDevice, st),
+                               "copy of perm_k");
+    }
     ELSAA_CHECK_LAUNCH(cudaStreamWaitEvent(st, side->join, 0), "join wait");
     // neighbouring key blocks (nb > 0) run in the persistent kernel for
     // b of 128 or 256 and nb = 1, otherwise in the CUDA-core block kernel;
     // the RACE key side above does not depend on them
-    if (P.impl == 2 && ws_supported(P)) {
+    if (P.impl == 2 && ws_supported(P) && !P.sel) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_ws", st, [&] {
                                return launch_block_attn_ws(
                                    P, q, k, v, Wbf, pq, pk, A, Bh,
@@ -629,7 +686,7 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                return launch_block_attn_simt(
                                    P, q, k, v, w_race, pq, pk, A, Bm,
                                    lambda_tok, gates, o, log_d_sparse, d_lr,
-                                   m_sparse, status, st);
+                                   m_sparse, status, st, cand, selmask);
                            }),
                            "block_attn_simt");
     }
@@ -655,6 +712,10 @@ struct BwdPlan {
 int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     if (p && p->causal) {
         *msg = "elsaa_backward: the causal variant has no backward pass here";
+        return ELSAA_ERR_UNSUPPORTED;
+    }
+    if (p && p->selector != 0) {
+        *msg = "elsaa_backward: built for the sorted-block selector only";
         return ELSAA_ERR_UNSUPPORTED;
     }
     elsaa_params q = *p;
@@ -746,6 +807,35 @@ extern "C" int elsaa_forward_race_summaries(const elsaa_params *params,
                         (size_t)P.BH * P.r * P.d * sizeof(float),
                         cudaMemcpyDeviceToDevice, st),
         "copy of B");
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_forward_selected_keys(const elsaa_params *params,
+                                           const void *workspace,
+                                           size_t workspace_bytes,
+                                           int32_t *keys, void *stream) {
+    g_err[0] = 0;
+    if (!params || params->selector != 1)
+        return fail(ELSAA_ERR_INVALID_ARG, "params must have selector = 1");
+    Plan P;
+    const char *msg = "";
+    int rc = make_plan(params, &P, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    if (!keys) return fail(ELSAA_ERR_INVALID_ARG, "keys is NULL");
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if (workspace_bytes < P.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, P.total);
+    char *ws = (char *)workspace;
+    const int32_t *pq = (const int32_t *)(ws + P.off_perm);
+    ELSAA_CHECK_LAUNCH(
+        launch_topk_export(P, pq, pq + (size_t)P.BH * P.N,
+                           (const int32_t *)(ws + P.off_cand),
+                           (const uint32_t *)(ws + P.off_mask), keys,
+                           (DeviceStatus *)(ws + P.off_status),
+                           (cudaStream_t)stream),
+        "topk_export");
     return ELSAA_OK;
 }
 

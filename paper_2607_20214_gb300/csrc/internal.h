@@ -48,8 +48,10 @@ struct Plan {
     int impl;        // resolved: 1 = SIMT, 2 = tensor core
     int Lg_pad;      // L * gamma rounded up to 16 (projection MMA width)
     int o32;         // write O as fp32 although the inputs are bf16
+    int sel;         // 0: sorted blocks; 1: per-query top-k selector
+    int tk_k, tk_c;  // top-k: keys per query, candidate blocks per block
     size_t off_status, off_keyrank, off_hist, off_perm, off_part, off_A,
-        off_B, off_Bh, off_W, total;
+        off_B, off_Bh, off_W, off_sums, off_cand, off_mask, total;
 };
 
 // Records a one-line error for elsaa_last_error() and returns `code`.
@@ -85,7 +87,19 @@ cudaError_t launch_block_attn_simt(
     const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const float *Bm, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
-    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+    float *m_sparse, DeviceStatus *status, cudaStream_t st,
+    const int32_t *cand = nullptr, const uint32_t *selmask = nullptr);
+
+// Per-query top-k selector (topk.cu).
+bool topk_supported(const Plan &P, const char **msg);
+cudaError_t launch_topk(const Plan &P, const void *q, const void *k,
+                        const int32_t *perm_q, const int32_t *perm_k,
+                        float *sums, int32_t *cand, uint32_t *selmask,
+                        DeviceStatus *status, cudaStream_t st);
+cudaError_t launch_topk_export(const Plan &P, const int32_t *perm_q,
+                               const int32_t *perm_k, const int32_t *cand,
+                               const uint32_t *selmask, int32_t *out,
+                               DeviceStatus *status, cudaStream_t st);
 
 // Tensor-core (tcgen05) path for bf16 inputs.
 bool tc_supported(const Plan &P);

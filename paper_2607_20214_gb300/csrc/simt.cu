@@ -164,7 +164,9 @@ __global__ void __launch_bounds__(kBlkThreads)
                  float *__restrict__ log_ds_out, float *__restrict__ dlr_out,
                  float *__restrict__ m_out, int N, int d, int H, int b,
                  int L, int gamma, int tps, int nb, float beta, float eps,
-                 float scale, float lambda, int mode, DeviceStatus *status) {
+                 float scale, float lambda, int mode, DeviceStatus *status,
+                 const int32_t *__restrict__ cand,
+                 const uint32_t *__restrict__ selmask, int tk_c) {
     extern __shared__ float smem[];
     const int bh = blockIdx.y, h = bh % H;
     const int pos0 = blockIdx.x * kSimtQT;
@@ -209,16 +211,33 @@ __global__ void __launch_bounds__(kBlkThreads)
         for (int c = 0; c < 4; ++c) o_acc[qq][c] = 0.f;
     }
     // key block blk and its nb neighbouring sorted blocks on each side,
-    // clipped to the N / b blocks: sorted positions [lo b, (hi + 1) b)
+    // clipped to the N / b blocks: sorted positions [lo b, (hi + 1) b).
+    // With the top-k selector: the tk_c candidate blocks of the query
+    // block, each key masked unless the query selected it.
     const int nblk = N / b;
     const int lo = blk - nb > 0 ? blk - nb : 0;
     const int hi = blk + nb < nblk - 1 ? blk + nb : nblk - 1;
-    const int kbase = lo * b, nkeys = (hi - lo + 1) * b;
+    const int kbase = lo * b;
+    const int nkeys = cand ? tk_c * b : (hi - lo + 1) * b;
+    const int32_t *cb = cand ? cand + ((size_t)bh * nblk + blk) * tk_c
+                             : nullptr;
+    const int W = tk_c * b / 32;  // mask words per query (selector 1)
     for (int c0 = 0; c0 < nkeys; c0 += kKC) {
         __syncthreads();
+        // sorted key position of chunk c0 (chunks never straddle a block:
+        // b is a multiple of kKC)
+        int kp0 = kbase + c0;
+        if (cb) {
+            int u = cb[c0 / b];
+            if (u < 0 || u >= nblk) {
+                report(status, kDevPermRange, 3, bh, u);
+                u = blk;
+            }
+            kp0 = u * b + c0 % b;
+        }
         for (int i = tid; i < kKC * d; i += kBlkThreads) {
             int row = i / d, col = i - row * d;
-            int j = pk[kbase + c0 + row];
+            int j = pk[kp0 + row];
             if (j < 0 || j >= N) {
                 if (col == 0) report(status, kDevPermRange, 2, bh, j);
                 j = 0;
@@ -234,9 +253,15 @@ __global__ void __launch_bounds__(kBlkThreads)
             float z = 0.f;
             for (int e = 0; e < d; ++e) z = fmaf(qr[e], kr[e], z);
             z *= scale;
+            bool keep = true;
+            if (selmask)
+                keep = (selmask[((size_t)bh * N + pos0 + wid * kQPerWarp +
+                                 qq) * W + c0 / 32] >> lane) & 1u;
+            if (!keep) z = -INFINITY;
             float mnew = fmaxf(m_run[qq], warp_max(z));
-            float alpha = expf(m_run[qq] - mnew);
-            float p = expf(z - mnew);
+            // nothing kept yet (mnew = -inf): no change
+            float alpha = mnew == -INFINITY ? 1.0f : expf(m_run[qq] - mnew);
+            float p = keep ? expf(z - mnew) : 0.0f;
             l_run[qq] = l_run[qq] * alpha + warp_sum(p);
 #pragma unroll
             for (int c = 0; c < 4; ++c) o_acc[qq][c] *= alpha;
@@ -414,7 +439,8 @@ cudaError_t launch_block_attn_simt(
     const float *w_race, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const float *Bm, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
-    float *m_sparse, DeviceStatus *status, cudaStream_t st) {
+    float *m_sparse, DeviceStatus *status, cudaStream_t st,
+    const int32_t *cand, const uint32_t *selmask) {
     dim3 grid(P.N / kSimtQT, P.BH);
     // phase 1: qs + ks(padded) + vs; phase 2 reuses ks, vs for outputs,
     // features and planes.
@@ -435,7 +461,8 @@ cudaError_t launch_block_attn_simt(
             A, Bm, lambda_tok, gates, P.o32 ? nullptr : (T *)o,               \
             P.o32 ? (float *)o : nullptr, log_d_sparse, d_lr, m_sparse,       \
             P.N, P.d, P.H, P.b, P.L, P.gamma, P.tables_per_slice, P.nb,       \
-            P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, status);         \
+            P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, status, cand,    \
+            selmask, P.tk_c);                                                 \
     } while (0)
     if (P.dtype == ELSAA_FP32)
         ELSAA_LAUNCH_BLK(float);

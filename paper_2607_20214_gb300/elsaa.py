@@ -33,7 +33,7 @@ SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_selftest_wait_timeout", "elsaa_forward_race_summaries",
            "elsaa_check_status_noalloc",
            "elsaa_selftest_wait_timeout_noalloc", "elsaa_causal_levels",
-           "elsaa_causal_index_lists")
+           "elsaa_causal_index_lists", "elsaa_forward_selected_keys")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -51,6 +51,8 @@ class elsaa_params(ctypes.Structure):
         ("fusion_mode", ctypes.c_int), ("impl", ctypes.c_int),
         ("neighbor_blocks", ctypes.c_int), ("causal_chunk", ctypes.c_int),
         ("causal_base_len", ctypes.c_int), ("out_fp32", ctypes.c_int),
+        ("selector", ctypes.c_int), ("topk", ctypes.c_int),
+        ("topk_blocks", ctypes.c_int),
     ]
 
 
@@ -137,6 +139,9 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
     L.elsaa_causal_index_lists.argtypes = [ctypes.POINTER(elsaa_params), vp,
                                            ctypes.c_size_t, vp, vp]
     L.elsaa_causal_index_lists.restype = ctypes.c_int
+    L.elsaa_forward_selected_keys.argtypes = [
+        ctypes.POINTER(elsaa_params), vp, ctypes.c_size_t, vp, vp]
+    L.elsaa_forward_selected_keys.restype = ctypes.c_int
     L.elsaa_check_status_noalloc.argtypes = [vp]
     L.elsaa_check_status_noalloc.restype = ctypes.c_int
     L.elsaa_selftest_wait_timeout_noalloc.argtypes = [ctypes.c_int, vp]
@@ -162,13 +167,15 @@ def make_params(B, H, N, d_h, dtype="bf16", block_size=64, sort_bits=5,
                 gray_order=1, race_tables=4, race_bits=4, beta=1.0, eps=1e-6,
                 scale=0.0, lam=1.0, fusion_mode=0, causal=0,
                 impl=ELSAA_IMPL_AUTO, neighbor_blocks=0, causal_chunk=128,
-                causal_base_len=4096, out_fp32=0) -> elsaa_params:
+                causal_base_len=4096, out_fp32=0, selector=0, topk=0,
+                topk_blocks=1) -> elsaa_params:
     dt = {"bf16": ELSAA_BF16, "fp32": ELSAA_FP32}[dtype] if isinstance(
         dtype, str) else int(dtype)
     return elsaa_params(B, H, N, d_h, dt, causal, block_size, sort_bits,
                         gray_order, race_tables, race_bits, beta, eps, scale,
                         lam, fusion_mode, impl, neighbor_blocks, causal_chunk,
-                        causal_base_len, out_fp32)
+                        causal_base_len, out_fp32, selector, topk,
+                        topk_blocks)
 
 
 def params_for(wl, **over) -> elsaa_params:
@@ -180,7 +187,9 @@ def params_for(wl, **over) -> elsaa_params:
               lam=wl.lam, fusion_mode=wl.fusion_mode, causal=wl.causal,
               neighbor_blocks=wl.neighbor_blocks,
               causal_chunk=wl.causal_chunk,
-              causal_base_len=wl.causal_base_len)
+              causal_base_len=wl.causal_base_len,
+              selector=wl.selector, topk=wl.topk,
+              topk_blocks=wl.topk_blocks)
     kw.update(over)
     return make_params(**kw)
 
@@ -543,3 +552,20 @@ def elsaa_causal_index_lists(params: elsaa_params, workspace, lists=None,
         workspace.numel() * workspace.element_size(),
         _ptr(lists, "lists", torch.int32, n, dev), _stream_ptr(stream)))
     return lists
+
+
+def elsaa_forward_selected_keys(params: elsaa_params, workspace, keys=None,
+                                stream=None):
+    """The key sets of the last top-k forward (selector = 1) on `workspace`:
+    int32 [B, H, N, topk], each row's original key indices increasing
+    (allocated here when not given)."""
+    dev = workspace.device
+    shape = (params.B, params.H, params.N, params.topk)
+    if keys is None:
+        keys = torch.empty(shape, dtype=torch.int32, device=dev)
+    n = params.B * params.H * params.N * params.topk
+    _check(load_library().elsaa_forward_selected_keys(
+        ctypes.byref(params), _ptr(workspace, "workspace", None, None, dev),
+        workspace.numel() * workspace.element_size(),
+        _ptr(keys, "keys", torch.int32, n, dev), _stream_ptr(stream)))
+    return keys

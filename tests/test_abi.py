@@ -58,7 +58,7 @@ def test_params_struct_matches_header():
 
 
 def test_abi_version(lib):
-    assert elsaa.elsaa_abi_version() == 5
+    assert elsaa.elsaa_abi_version() == 6
 
 
 @pytest.mark.parametrize("name", sorted(WORKLOADS))
@@ -96,7 +96,33 @@ BAD = [
     (dict(B=0), elsaa.ELSAA_ERR_INVALID_ARG, "positive"),
     (dict(neighbor_blocks=-1), elsaa.ELSAA_ERR_INVALID_ARG, "neighbor"),
     (dict(out_fp32=2), elsaa.ELSAA_ERR_INVALID_ARG, "out_fp32"),
+    (dict(selector=2), elsaa.ELSAA_ERR_INVALID_ARG, "selector"),
+    (dict(selector=1, topk=8, topk_blocks=0), elsaa.ELSAA_ERR_INVALID_ARG,
+     "topk_blocks"),
+    (dict(selector=1, topk=8, topk_blocks=5), elsaa.ELSAA_ERR_INVALID_ARG,
+     "topk_blocks"),
+    (dict(selector=1, topk=129, topk_blocks=2), elsaa.ELSAA_ERR_INVALID_ARG,
+     "topk"),
+    (dict(selector=1, topk=0, topk_blocks=2), elsaa.ELSAA_ERR_INVALID_ARG,
+     "topk"),
+    (dict(selector=1, topk=8, topk_blocks=2, neighbor_blocks=1),
+     elsaa.ELSAA_ERR_INVALID_ARG, "neighbor_blocks"),
+    (dict(selector=1, topk=8, topk_blocks=2, causal=1),
+     elsaa.ELSAA_ERR_UNSUPPORTED, "causal"),
+    (dict(selector=1, topk=8, topk_blocks=9, N=1024),
+     elsaa.ELSAA_ERR_UNSUPPORTED, "512"),
 ]
+
+
+def test_selector_workspace_grows_and_backward_refuses(lib):
+    base = dict(B=1, H=2, N=1024, d_h=64, block_size=64, race_tables=4)
+    a = elsaa.elsaa_workspace_size(elsaa.make_params(**base))
+    p = elsaa.make_params(selector=1, topk=64, topk_blocks=2, **base)
+    assert elsaa.elsaa_workspace_size(p) > a
+    n = ctypes.c_size_t(0)
+    rc = lib.elsaa_backward_workspace_size(ctypes.byref(p), ctypes.byref(n))
+    assert rc == elsaa.ELSAA_ERR_UNSUPPORTED
+    assert "selector" in elsaa.elsaa_last_error()
 
 
 @pytest.mark.parametrize("N,N0,levels", [(16384, 4096, 2), (1024, 256, 2),
