@@ -228,9 +228,12 @@ def workload_config(wl):
                             ("causal (C=%d, N_0=%d)" % (
                                 wl.causal_chunk, wl.causal_base_len))
                             if wl.causal else "non-causal",
-                            (", %d neighbour blocks per side" %
-                             wl.neighbor_blocks) if wl.neighbor_blocks
-                            else ""),
+                            ((", %d neighbour blocks per side" %
+                              wl.neighbor_blocks) if wl.neighbor_blocks
+                             else "") +
+                            ((", top-k selector: k=%d over %d candidate "
+                              "blocks" % (wl.topk, wl.topk_blocks))
+                             if wl.selector else "")),
             "B": wl.B, "H": wl.H, "N": wl.N, "d_h": wl.d_h,
             "block": wl.block, "r": wl.r, "global_batch": wl.B,
             "seq_len": wl.N,
@@ -342,6 +345,37 @@ def extra_workloads(args, dev, stream, peaks):
         "err_vs_oracle": dict(forward_errors(wl, x, o, [(0, 0), (0, 31)],
                                              rows=rows),
                               sample="512 rows of heads (0, 0), (0, 31)"),
+    }
+    del x, o, ws
+    # -- c3 with the per-query top-k selector (k = 128 over two candidate
+    # blocks per query block)
+    wl = WORKLOADS["c3"].with_(selector=1, topk=128, topk_blocks=2)
+    x = make_inputs(wl, device=dev)
+    p = elsaa.params_for(wl)
+    ws = elsaa.new_workspace(p, dev)
+    o = torch.empty_like(x["q"])
+
+    def step():
+        elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
+                            x["w_race"], o=o, workspace=ws, stream=stream)
+
+    ms, prof = measure(step, args.steps, args.warmup, dev, stream)
+    elsaa.elsaa_check_status(ws)
+    fm = perfmodel.flop_model(wl)
+    rows = np.random.default_rng(6).choice(wl.N, 256, replace=False)
+    rows.sort()
+    out["c3_topk"] = {
+        "config": workload_config(wl), "ms_per_step": ms,
+        "value": wl.tokens / (ms / 1e3), "unit": "tokens/s",
+        "step_roofline_frac": max(
+            fm["tensor_flops"] / (peaks["bf16_tflops"] * 1e12),
+            fm["bytes"] / (peaks["hbm_gbs"] * 1e9)) / (ms / 1e3),
+        "roofline": dominant_roofline(wl, prof, peaks, ms, args.steps),
+        "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n}
+                    for k, (n, t) in sorted(prof.items())},
+        "gpu_launches": sum(n for n, _ in prof.values()),
+        "err_vs_oracle": dict(forward_errors(wl, x, o, [(1, 7)], rows=rows),
+                              sample="256 rows of head (1, 7)"),
     }
     del x, o, ws
     # -- c5: training step, forward + backward
@@ -711,7 +745,7 @@ def run_ours(args, wl):
     if rank == 0 and world == 1 and not args.no_extra and \
             args.workload == "c3" and not (args.backward or args.gate_mlp or
                                            args.batch or args.heads or
-                                           args.neighbors):
+                                           args.neighbors or args.topk):
         extra = extra_workloads(args, dev, stream, peaks)
 
     if rank != 0:
@@ -763,6 +797,11 @@ def main():
     ap.add_argument("--neighbors", type=int, default=0, metavar="R",
                     help="R neighbouring sorted key blocks per side "
                          "(sparse branch on CUDA cores when R > 0)")
+    ap.add_argument("--topk", type=int, default=0, metavar="K",
+                    help="per-query top-k selector with K keys per query "
+                         "(default: the sorted-block selector)")
+    ap.add_argument("--topk-blocks", type=int, default=2, metavar="C",
+                    help="candidate key blocks per query block for --topk")
     ap.add_argument("--heads", type=int, default=0,
                     help="override H (smaller cases for profiler captures)")
     ap.add_argument("--no-preroll", action="store_true",
@@ -784,6 +823,9 @@ def main():
         wl = wl.with_(H=args.heads)
     if args.neighbors:
         wl = wl.with_(neighbor_blocks=args.neighbors)
+    if args.topk:
+        wl = wl.with_(selector=1, topk=args.topk,
+                      topk_blocks=args.topk_blocks)
     if args.impl == "reference":
         return run_reference(args, wl)
     return run_ours(args, wl)

@@ -653,12 +653,16 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     if (P.sel) {
         cand = (int32_t *)(ws + P.off_cand);
         selmask = (uint32_t *)(ws + P.off_mask);
-        ELSAA_CHECK_LAUNCH(timed("topk_select", st, [&] {
-                               return launch_topk(P, q, k, pq, pk,
-                                                  (float *)(ws + P.off_sums),
-                                                  cand, selmask, status, st);
-                           }),
-                           "topk_select");
+        static const char *const kStage[3] = {"topk_sums", "topk_cand",
+                                              "topk_select"};
+        for (int sg = 0; sg < 3; ++sg)
+            ELSAA_CHECK_LAUNCH(timed(kStage[sg], st, [&] {
+                                   return launch_topk(
+                                       sg, P, q, k, pq, pk,
+                                       (float *)(ws + P.off_sums), cand,
+                                       selmask, status, st);
+                               }),
+                               kStage[sg]);
         const size_t pb = (size_t)P.BH * P.N * sizeof(int32_t);
         if (perm_q)
             ELSAA_CHECK_LAUNCH(cudaMemcpyAsync(perm_q, pq, pb,
@@ -673,12 +677,12 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
     // neighbouring key blocks (nb > 0) run in the persistent kernel for
     // b of 128 or 256 and nb = 1, otherwise in the CUDA-core block kernel;
     // the RACE key side above does not depend on them
-    if (P.impl == 2 && ws_supported(P) && !P.sel) {
+    if (P.impl == 2 && ws_supported(P)) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_ws", st, [&] {
                                return launch_block_attn_ws(
                                    P, q, k, v, Wbf, pq, pk, A, Bh,
                                    lambda_tok, gates, o, log_d_sparse, d_lr,
-                                   m_sparse, status, st);
+                                   m_sparse, status, st, cand, selmask);
                            }),
                            "block_attn_ws");
     } else {

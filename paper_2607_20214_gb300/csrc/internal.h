@@ -92,10 +92,12 @@ cudaError_t launch_block_attn_simt(
 
 // Per-query top-k selector (topk.cu).
 bool topk_supported(const Plan &P, const char **msg);
-cudaError_t launch_topk(const Plan &P, const void *q, const void *k,
-                        const int32_t *perm_q, const int32_t *perm_k,
-                        float *sums, int32_t *cand, uint32_t *selmask,
-                        DeviceStatus *status, cudaStream_t st);
+// stage 0: block sums; 1: candidate blocks; 2: per-query selection
+cudaError_t launch_topk(int stage, const Plan &P, const void *q,
+                        const void *k, const int32_t *perm_q,
+                        const int32_t *perm_k, float *sums, int32_t *cand,
+                        uint32_t *selmask, DeviceStatus *status,
+                        cudaStream_t st);
 cudaError_t launch_topk_export(const Plan &P, const int32_t *perm_q,
                                const int32_t *perm_k, const int32_t *cand,
                                const uint32_t *selmask, int32_t *out,
@@ -220,6 +222,7 @@ cudaError_t launch_block_attn_ws(
     const uint16_t *w_bf16, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const uint16_t *Bh, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
-    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+    float *m_sparse, DeviceStatus *status, cudaStream_t st,
+    const int32_t *cand = nullptr, const uint32_t *selmask = nullptr);
 
 }  // namespace elsaa

@@ -62,9 +62,12 @@ struct WsBars {
 // NPASS 128-key passes per query tile, online softmax across them: 1 for
 // b <= 128; b / 128 for larger blocks; with nb neighbouring sorted key
 // blocks per side (b >= 128), (2 nb + 1) b / 128 passes over the window.
-// WIN: the passes walk a neighbour window (nb > 0), whose passes past
-// either end of the sequence are masked; false compiles those checks out.
-template <int G, int NPASS, bool WIN>
+// KM: which keys the passes walk. 0: the query block's own key block.
+// 1 (WIN): a neighbour window (nb > 0), whose passes past either end of
+// the sequence are masked. 2 (SEL): the top-k selector's candidate blocks
+// (cand, tk_c per query block), each key masked unless the row's bit in
+// selmask is set. The checks of the other modes are compiled out.
+template <int G, int NPASS, int KM>
 __global__ void __launch_bounds__(kWsThreads, 1)
     k_block_attn_ws(const uint16_t *__restrict__ qx,
                     const uint16_t *__restrict__ kx,
@@ -82,7 +85,10 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     int nb, int L, int Lg_pad, float beta, float eps,
                     float scale,
                     float lambda, int mode, int tiles_per_head,
-                    long total_tiles, DeviceStatus *status) {
+                    long total_tiles, DeviceStatus *status,
+                    const int32_t *__restrict__ cand,
+                    const uint32_t *__restrict__ selmask, int tk_c) {
+    constexpr bool WIN = KM == 1, SEL = KM == 2;
     constexpr int R = 1 << G;
     constexpr int nk = kWsNK;
     extern __shared__ unsigned char smem_raw[];
@@ -153,16 +159,24 @@ __global__ void __launch_bounds__(kWsThreads, 1)
     // query block (the block and nb neighbouring blocks per side) in
     // 128-key steps. A pass past either end of the sequence holds no keys:
     // its rows are read from a valid position and its scores are masked.
-    auto key_pos_raw = [=](int p0, int p) {
+    // SEL: pass p holds candidate keys [128 p, 128 p + 128) of the query
+    // block, i.e. keys of candidate block 128 p / b (b >= 128)
+    auto key_pos_raw = [=](int bh, int p0, int p) {
+        if (SEL) {
+            const int T = N / b, t = p0 / b;
+            int u = cand[((size_t)bh * T + t) * tk_c + (128 * p) / b];
+            u = (u < 0 || u >= T) ? t : u;
+            return u * b + (128 * p) % b;
+        }
         return NPASS == 1 ? p0 : (p0 / b - (WIN ? nb : 0)) * b + 128 * p;
     };
     auto pass_valid = [=](int p0, int p) {
         if (!WIN) return true;
-        const int k0 = key_pos_raw(p0, p);
+        const int k0 = key_pos_raw(0, p0, p);
         return k0 >= 0 && k0 < N;
     };
-    auto key_pos = [=](int p0, int p) {
-        const int k0 = key_pos_raw(p0, p);
+    auto key_pos = [=](int bh, int p0, int p) {
+        const int k0 = key_pos_raw(bh, p0, p);
         if (NPASS == 1) return k0;  // the tile's own keys (ragged end kept)
         return k0 < 0 ? 0 : (k0 > N - 128 ? N - 128 : k0);
     };
@@ -213,7 +227,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                 for (int ps = 0; ps < NPASS; ++ps)
                     *reinterpret_cast<int4 *>(&qkrow[t][1 + ps][4 * lt]) =
                         rows4(perm_k + (size_t)bh * N,
-                              key_pos(p0, ps) + 4 * lt, bh * N);
+                              key_pos(bh, p0, ps) + 4 * lt, bh * N);
                 __syncwarp();
                 mbar_arrive(&bars.idx_full[t]);
             }
@@ -249,7 +263,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     __syncwarp();  // the previous rows are all read
                     *reinterpret_cast<int4 *>(&vrow[4 * lt]) =
                         rows4(perm_k + (size_t)bh * N,
-                              key_pos(p0, ps) + 4 * lt, bh * N);
+                              key_pos(bh, p0, ps) + 4 * lt, bh * N);
                     __syncwarp();
                     // buffer i & 1 serves the passes of tiles i, i + 2, ...
                     // in turn; a pass's V goes in once the previous user is
@@ -519,6 +533,17 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             const bool masked = b < 128;
             // pass 0 of a tile whose window starts before the sequence
             const bool valid0 = !WIN || pass_valid(p0, 0);
+            // SEL: this row's selected candidates among this half's 64 keys
+            // of pass ps (bit k of the 64-bit word: key kbeg + k)
+            const size_t selrow = (size_t)bh * N + (size_t)min(qpos, N - 1);
+            const int selw = tk_c * b / 32;
+            auto selbits = [&](int ps) -> unsigned long long {
+                if (!SEL) return ~0ull;
+                const uint32_t *w = selmask + selrow * selw + 4 * ps + 2 * half;
+                return (unsigned long long)w[0] |
+                       ((unsigned long long)w[1] << 32);
+            };
+            const unsigned long long sb0 = selbits(0);
 #pragma unroll
             for (int c = 0; c < nk / 2; c += 16) {
                 uint32_t v[16];
@@ -528,7 +553,8 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                 for (int jj = 0; jj < 16; ++jj) {
                     const int key = kbeg + c + jj;
                     if ((!WIN || valid0) &&
-                        (!masked || (key >= klo && key < khi)))
+                        (!masked || (key >= klo && key < khi)) &&
+                        (!SEL || ((sb0 >> (c + jj)) & 1ull)))
                         mxa[jj & 3] = fmaxf(mxa[jj & 3], __uint_as_float(v[jj]));
                 }
             }
@@ -561,6 +587,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                             a1 = (key + 1 >= klo && key + 1 < khi) ? a1 : 0.0f;
                         }
                         if (WIN && !valid0) a0 = a1 = 0.0f;
+                        if (SEL) {
+                            const int kl = c + 16 * hh + jj;  // in the half
+                            a0 = ((sb0 >> kl) & 1ull) ? a0 : 0.0f;
+                            a1 = ((sb0 >> (kl + 1)) & 1ull) ? a1 : 0.0f;
+                        }
                         ls[(jj >> 1) & 3] += a0 + a1;
                         pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
                     }
@@ -599,6 +630,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     break;
                 }
                 const bool pvalid = !WIN || pass_valid(p0, ps);
+                const unsigned long long sbp = selbits(ps);
                 float mxb[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
                 if (!WIN || pvalid) {
 #pragma unroll
@@ -608,8 +640,9 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                         tmem_wait_ld();
 #pragma unroll
                         for (int jj = 0; jj < 16; ++jj)
-                            mxb[jj & 3] =
-                                fmaxf(mxb[jj & 3], __uint_as_float(v[jj]));
+                            if (!SEL || ((sbp >> (c + jj)) & 1ull))
+                                mxb[jj & 3] = fmaxf(mxb[jj & 3],
+                                                    __uint_as_float(v[jj]));
                     }
                 }
                 xmax[g][half][row] =
@@ -658,6 +691,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                             float a1 = ex2_approx(
                                 fmaf(__uint_as_float(v[jj + 1]), sl2e, -M2));
                             if (WIN && !pvalid) a0 = a1 = 0.0f;
+                            if (SEL) {
+                                const int kl = c + 16 * hh + jj;
+                                a0 = ((sbp >> kl) & 1ull) ? a0 : 0.0f;
+                                a1 = ((sbp >> (kl + 1)) & 1ull) ? a1 : 0.0f;
+                            }
                             lb[(jj >> 1) & 3] += a0 + a1;
                             pk16[8 * hh + (jj >> 1)] = pack_bf16x2(a0, a1);
                         }
@@ -787,6 +825,11 @@ __global__ void __launch_bounds__(kWsThreads, 1)
 // 128 or 256, gamma = 4): the (2 nb + 1) b / 128 passes of the window, 3 or
 // 6 for nb = 1.
 static int ws_passes(const Plan &P) {
+    if (P.sel) {  // the candidate blocks, 128 keys per pass (b >= 128)
+        if (P.gamma != 4 || (P.b != 128 && P.b != 256)) return 0;
+        const int n = P.tk_c * P.b / 128;
+        return n <= 4 ? n : 0;
+    }
     if (P.nb == 0) return P.b <= 128 ? 1 : (P.b == 256 ? 2 : 0);
     if (P.nb != 1 || P.gamma != 4 || (P.b != 128 && P.b != 256)) return 0;
     return 3 * (P.b / 128);
@@ -806,7 +849,8 @@ cudaError_t launch_block_attn_ws(
     const uint16_t *w_bf16, const int32_t *perm_q, const int32_t *perm_k,
     const float *A, const uint16_t *Bh, const float *lambda_tok,
     const float *gates, void *o, float *log_d_sparse, float *d_lr,
-    float *m_sparse, DeviceStatus *status, cudaStream_t st) {
+    float *m_sparse, DeviceStatus *status, cudaStream_t st,
+    const int32_t *cand, const uint32_t *selmask) {
     const int lg_pad = (P.L * P.gamma + 15) / 16 * 16;
     const size_t tileB = (size_t)kWsNK * P.d * 2;
     const size_t smem = 1024 + 4 * tileB + ((size_t)lg_pad * P.d * 2 + 1023) /
@@ -836,19 +880,28 @@ cudaError_t launch_block_attn_ws(
             P.o32 ? nullptr : (uint16_t *)o, P.o32 ? (float *)o : nullptr,
             log_d_sparse, d_lr, m_sparse, P.N, P.d, P.H, P.b, P.nb, P.L, lg,
             P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, tiles_per_head,
-            total, status);
+            total, status, cand, selmask, P.tk_c);
         return cudaGetLastError();
     };
     const int passes = ws_passes(P);
-    if (passes == 3) return launch(k_block_attn_ws<4, 3, true>);
-    if (passes == 6) return launch(k_block_attn_ws<4, 6, true>);
+    if (P.sel) {
+        switch (passes) {
+            case 1: return launch(k_block_attn_ws<4, 1, 2>);
+            case 2: return launch(k_block_attn_ws<4, 2, 2>);
+            case 3: return launch(k_block_attn_ws<4, 3, 2>);
+            case 4: return launch(k_block_attn_ws<4, 4, 2>);
+            default: return cudaErrorInvalidValue;
+        }
+    }
+    if (passes == 3) return launch(k_block_attn_ws<4, 3, 1>);
+    if (passes == 6) return launch(k_block_attn_ws<4, 6, 1>);
     switch (P.gamma) {
-        case 1: return P.b > 128 ? launch(k_block_attn_ws<1, 2, false>) : launch(k_block_attn_ws<1, 1, false>);
-        case 2: return P.b > 128 ? launch(k_block_attn_ws<2, 2, false>) : launch(k_block_attn_ws<2, 1, false>);
-        case 3: return P.b > 128 ? launch(k_block_attn_ws<3, 2, false>) : launch(k_block_attn_ws<3, 1, false>);
-        case 4: return P.b > 128 ? launch(k_block_attn_ws<4, 2, false>) : launch(k_block_attn_ws<4, 1, false>);
-        case 5: return P.b > 128 ? launch(k_block_attn_ws<5, 2, false>) : launch(k_block_attn_ws<5, 1, false>);
-        case 6: return P.b > 128 ? launch(k_block_attn_ws<6, 2, false>) : launch(k_block_attn_ws<6, 1, false>);
+        case 1: return P.b > 128 ? launch(k_block_attn_ws<1, 2, 0>) : launch(k_block_attn_ws<1, 1, 0>);
+        case 2: return P.b > 128 ? launch(k_block_attn_ws<2, 2, 0>) : launch(k_block_attn_ws<2, 1, 0>);
+        case 3: return P.b > 128 ? launch(k_block_attn_ws<3, 2, 0>) : launch(k_block_attn_ws<3, 1, 0>);
+        case 4: return P.b > 128 ? launch(k_block_attn_ws<4, 2, 0>) : launch(k_block_attn_ws<4, 1, 0>);
+        case 5: return P.b > 128 ? launch(k_block_attn_ws<5, 2, 0>) : launch(k_block_attn_ws<5, 1, 0>);
+        case 6: return P.b > 128 ? launch(k_block_attn_ws<6, 2, 0>) : launch(k_block_attn_ws<6, 1, 0>);
         default: return cudaErrorInvalidValue;
     }
 }

@@ -27,7 +27,6 @@ namespace {
 
 constexpr int kSelThreads = 256;
 constexpr int kSelWarps = kSelThreads / 32;
-constexpr int kSelPad = 4;  // fp32 row padding of the staged keys
 
 // Order-preserving map of fp32 scores to uint32 (larger score, larger key).
 // -0.0 is taken as +0.0, as the float comparison of the oracle does.
@@ -49,14 +48,23 @@ __global__ void k_topk_sums(const X *__restrict__ qx, const X *__restrict__ kx,
     const int T = gridDim.x, BH = gridDim.y, e = threadIdx.x;
     const X *x = (w ? kx : qx) + (size_t)bh * N * d;
     const int32_t *pm = (w ? perm_k : perm_q) + (size_t)bh * N;
+    // rows 16 at a time: the loads are issued together, the additions stay
+    // in sorted order
+    constexpr int kU = 16;
     float acc = 0.0f;
-    for (int p = t * b; p < (t + 1) * b; ++p) {
-        int i = pm[p];
-        if (i < 0 || i >= N) {
-            if (e == 0) report(status, kDevPermRange, 20, bh, i);
-            i = 0;
+    for (int p0 = t * b; p0 < (t + 1) * b; p0 += kU) {
+        float v[kU];
+#pragma unroll
+        for (int u = 0; u < kU; ++u) {
+            int i = pm[p0 + u];
+            if (i < 0 || i >= N) {
+                if (e == 0) report(status, kDevPermRange, 20, bh, i);
+                i = 0;
+            }
+            v[u] = to_f32<X>(x[(size_t)i * d + e]);
         }
-        acc = __fadd_rn(acc, to_f32<X>(x[(size_t)i * d + e]));
+#pragma unroll
+        for (int u = 0; u < kU; ++u) acc = __fadd_rn(acc, v[u]);
     }
     sums[(((size_t)w * BH + bh) * T + t) * d + e] = acc;
 }
@@ -81,9 +89,21 @@ __global__ void __launch_bounds__(kSelThreads)
     for (int e = tid; e < d; e += kSelThreads) qs[e] = qsum[e];
     __syncthreads();
     for (int u = tid; u < T; u += kSelThreads) {
-        const float *kr = ksum + (size_t)u * d;
+        const float4 *kr = reinterpret_cast<const float4 *>(ksum +
+                                                             (size_t)u * d);
         float acc = 0.0f;
-        for (int e = 0; e < d; ++e) acc = fmaf(qs[e], kr[e], acc);
+        for (int e = 0; e < d; e += 16) {
+            float4 kv[4];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) kv[x] = kr[e / 4 + x];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+                acc = fmaf(qs[e + 4 * x], kv[x].x, acc);
+                acc = fmaf(qs[e + 4 * x + 1], kv[x].y, acc);
+                acc = fmaf(qs[e + 4 * x + 2], kv[x].z, acc);
+                acc = fmaf(qs[e + 4 * x + 3], kv[x].w, acc);
+            }
+        }
         sc[u] = acc;
         taken[u] = u == t;
     }
@@ -129,9 +149,85 @@ __global__ void __launch_bounds__(kSelThreads)
     }
 }
 
+// Candidate-key staging element: bf16 inputs stay bf16 in shared memory
+// (widened exactly when read), fp32 inputs stay fp32.
+template <typename X>
+struct SelStage;
+template <>
+struct SelStage<float> {
+    using T = float;
+    static constexpr int kPer16 = 4;  // values per 16-byte load
+    __device__ static void widen(const uint4 &u, float *f) {
+        f[0] = __uint_as_float(u.x);
+        f[1] = __uint_as_float(u.y);
+        f[2] = __uint_as_float(u.z);
+        f[3] = __uint_as_float(u.w);
+    }
+};
+template <>
+struct SelStage<__nv_bfloat16> {
+    using T = __nv_bfloat16;
+    static constexpr int kPer16 = 8;
+    __device__ static void widen(const uint4 &u, float *f) {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            f[2 * i] = __uint_as_float(w[i] << 16);
+            f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+        }
+    }
+};
+
+// Rows of staged candidate keys: d + 16 bytes of padding keep 16-byte
+// alignment and spread a quarter-warp's 16-byte loads over all banks.
+template <typename X>
+__host__ __device__ constexpr int sel_row_bytes(int d) {
+    return d * (int)sizeof(X) + 16;
+}
+
+constexpr int kSelQB = 4;  // queries per warp sharing each key load
+
+// 16-byte global -> shared copy that does not block the thread
+// (cp.async.cg), and the wait for all of this thread's copies.
+__device__ __forceinline__ void sel_cp16(void *dst, const void *src) {
+    const uint32_t d =
+        static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d),
+                 "l"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void sel_cp_wait() {
+    asm volatile("cp.async.wait_all;" ::: "memory");
+}
+
+// Two fp32 lanes per instruction (fma.rn.f32x2): lane by lane d = a b + c,
+// one rounding each, so each lane is an ordinary fmaf.
+__device__ __forceinline__ unsigned long long sel_fma2(unsigned long long a,
+                                                       unsigned long long b,
+                                                       unsigned long long c) {
+    unsigned long long r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+__device__ __forceinline__ unsigned long long sel_pack(float lo, float hi) {
+    unsigned long long r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+    return r;
+}
+__device__ __forceinline__ float sel_lo(unsigned long long v) {
+    return __uint_as_float((uint32_t)v);
+}
+__device__ __forceinline__ float sel_hi(unsigned long long v) {
+    return __uint_as_float((uint32_t)(v >> 32));
+}
+
 // Grid (T, BH), kSelThreads threads, M = c b / 32 candidate words (<= 16).
-// Dynamic shared memory: the candidate keys as fp32 rows of d + kSelPad,
-// their original indices, one query row per warp.
+// Dynamic shared memory: the candidate keys and the block's b queries (both
+// in the input type, rows padded), the candidates' original indices. All
+// rows are copied at once (indices first, then every 16-byte piece with
+// cp.async). Each warp scores kSelQB queries at a time: every staged key
+// value feeds two packed chains (queries 0|1 and 2|3), then the four radix
+// selects run interleaved.
 template <typename X, int M>
 __global__ void __launch_bounds__(kSelThreads)
     k_topk_select(const X *__restrict__ qx, const X *__restrict__ kx,
@@ -140,111 +236,194 @@ __global__ void __launch_bounds__(kSelThreads)
                   const int32_t *__restrict__ cand, int N, int d, int b,
                   int c, int k, uint32_t *__restrict__ selmask,
                   DeviceStatus *status) {
-    extern __shared__ __align__(16) float ssm[];
+    using S = SelStage<X>;
+    extern __shared__ __align__(16) unsigned char sel_smem[];
     const int t = blockIdx.x, bh = blockIdx.y, T = gridDim.x;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int nc = 32 * M, ds = d + kSelPad;
-    float *kc = ssm;                                    // [nc][ds]
-    int *cidx = reinterpret_cast<int *>(kc + (size_t)nc * ds);  // [nc]
-    float *qrow = reinterpret_cast<float *>(cidx + nc) + warp * d;  // [d]
+    const int nc = 32 * M, rb = sel_row_bytes<X>(d);
+    unsigned char *kc = sel_smem;                                 // [nc][rb]
+    unsigned char *qs = kc + (size_t)nc * rb;                     // [b][rb]
+    int *cidx = reinterpret_cast<int *>(qs + (size_t)b * rb);     // [nc]
+    int *qidx = cidx + nc;                                        // [b]
     const X *qh = qx + (size_t)bh * N * d;
     const X *kh = kx + (size_t)bh * N * d;
     const int32_t *pq = perm_q + (size_t)bh * N;
     const int32_t *pk = perm_k + (size_t)bh * N;
     const int32_t *cb = cand + ((size_t)bh * T + t) * c;
-    // stage the c b candidate keys (candidate r = key r % b of block r / b)
-    for (int r = warp; r < nc; r += kSelWarps) {
+    // the c b candidate keys (candidate r = key r % b of block r / b) and
+    // the block's queries: original indices first, then the rows
+    for (int r = tid; r < nc; r += kSelThreads) {
         int u = cb[r / b];
         if (u < 0 || u >= T) u = t;
         int j = pk[u * b + r % b];
         if (j < 0 || j >= N) {
-            if (lane == 0) report(status, kDevPermRange, 21, bh, j);
+            report(status, kDevPermRange, 21, bh, j);
             j = 0;
         }
-        if (lane == 0) cidx[r] = j;
-        for (int e = lane; e < d; e += 32)
-            kc[(size_t)r * ds + e] = to_f32<X>(kh[(size_t)j * d + e]);
+        cidx[r] = j;
     }
-    __syncthreads();
-    const int W = M;  // mask words per query
-    for (int qq = warp; qq < b; qq += kSelWarps) {
-        const int p = t * b + qq;
-        int i = pq[p];
+    for (int r = tid; r < b; r += kSelThreads) {
+        int i = pq[t * b + r];
         if (i < 0 || i >= N) {
-            if (lane == 0) report(status, kDevPermRange, 22, bh, i);
+            report(status, kDevPermRange, 22, bh, i);
             i = 0;
         }
-        __syncwarp();
-        for (int e = lane; e < d; e += 32)
-            qrow[e] = to_f32<X>(qh[(size_t)i * d + e]);
-        __syncwarp();
-        // canonical chains: candidate lane + 32 m, e = 0 .. d - 1 in order
-        float acc[M];
+        qidx[r] = i;
+    }
+    __syncthreads();
+    const int cpr = d * (int)sizeof(X) / 16;  // 16-byte chunks per row
+    for (int x = tid; x < nc * cpr; x += kSelThreads) {
+        const int r = x / cpr, ch = x - r * cpr;
+        sel_cp16(kc + (size_t)r * rb + 16 * ch,
+                 reinterpret_cast<const unsigned char *>(
+                     kh + (size_t)cidx[r] * d) + 16 * ch);
+    }
+    for (int x = tid; x < b * cpr; x += kSelThreads) {
+        const int r = x / cpr, ch = x - r * cpr;
+        sel_cp16(qs + (size_t)r * rb + 16 * ch,
+                 reinterpret_cast<const unsigned char *>(
+                     qh + (size_t)qidx[r] * d) + 16 * ch);
+    }
+    sel_cp_wait();
+    __syncthreads();
+    int cj[M];  // original index of each of this lane's candidates
 #pragma unroll
-        for (int m = 0; m < M; ++m) acc[m] = 0.0f;
-        for (int e = 0; e < d; e += 4) {
-            const float4 qv = *reinterpret_cast<const float4 *>(qrow + e);
+    for (int m = 0; m < M; ++m) cj[m] = cidx[lane + 32 * m];
+    const int W = M;  // mask words per query
+    for (int q0 = warp * kSelQB; q0 < b; q0 += kSelWarps * kSelQB) {
+        const int nq = min(kSelQB, b - q0);
+        // query rows of this group (rows past the block repeat row q0)
+        const unsigned char *qr[kSelQB];
+#pragma unroll
+        for (int qq = 0; qq < kSelQB; ++qq)
+            qr[qq] = qs + (size_t)(q0 + (qq < nq ? qq : 0)) * rb;
+        // canonical chains: query qq, candidate lane + 32 m, e = 0 .. d - 1
+        // in order (each lane of a packed fma rounds once, from +0.0f)
+        unsigned long long acc01[M], acc23[M];
+#pragma unroll
+        for (int m = 0; m < M; ++m) acc01[m] = acc23[m] = 0ull;
+        for (int e0 = 0; e0 < d; e0 += S::kPer16) {
+            unsigned long long q01[S::kPer16], q23[S::kPer16];
+            {
+                float qv[kSelQB][S::kPer16];
+#pragma unroll
+                for (int qq = 0; qq < kSelQB; ++qq)
+                    S::widen(*reinterpret_cast<const uint4 *>(
+                                 qr[qq] + e0 * (int)sizeof(X)),
+                             qv[qq]);
+#pragma unroll
+                for (int x = 0; x < S::kPer16; ++x) {
+                    q01[x] = sel_pack(qv[0][x], qv[1][x]);
+                    q23[x] = sel_pack(qv[2][x], qv[3][x]);
+                }
+            }
 #pragma unroll
             for (int m = 0; m < M; ++m) {
-                const float4 kv = *reinterpret_cast<const float4 *>(
-                    kc + (size_t)(lane + 32 * m) * ds + e);
-                acc[m] = fmaf(qv.x, kv.x, acc[m]);
-                acc[m] = fmaf(qv.y, kv.y, acc[m]);
-                acc[m] = fmaf(qv.z, kv.z, acc[m]);
-                acc[m] = fmaf(qv.w, kv.w, acc[m]);
-            }
-        }
-        uint32_t key[M];
+                const uint4 u = *reinterpret_cast<const uint4 *>(
+                    kc + (size_t)(lane + 32 * m) * rb +
+                    e0 * (int)sizeof(X));
+                float kv[S::kPer16];
+                S::widen(u, kv);
 #pragma unroll
-        for (int m = 0; m < M; ++m) key[m] = ordered_key(acc[m]);
-        // the k-th largest key: MSB-first radix select
-        uint32_t pre = 0, msk = 0;
-        int above = 0;
-        for (int bit = 31; bit >= 0; --bit) {
-            const uint32_t bm = 1u << bit, want = pre | bm, mk = msk | bm;
-            int cnt = 0;
-#pragma unroll
-            for (int m = 0; m < M; ++m) cnt += (key[m] & mk) == want;
-            cnt = __reduce_add_sync(0xffffffffu, cnt);
-            if (above + cnt >= k)
-                pre = want;
-            else
-                above += cnt;
-            msk = mk;
-        }
-        // keys equal to the threshold: the need lowest original indices
-        const int need = k - above;
-        int ties = 0;
-#pragma unroll
-        for (int m = 0; m < M; ++m) ties += key[m] == pre;
-        ties = __reduce_add_sync(0xffffffffu, ties);
-        int jmax = 0x7fffffff;
-        if (ties > need) {
-            uint32_t jp = 0, jm = 0;
-            int below = 0;
-            for (int bit = 30; bit >= 0; --bit) {
-                const uint32_t bm = 1u << bit, mk = jm | bm;
-                int cnt = 0;  // ties whose index has this bit clear
-#pragma unroll
-                for (int m = 0; m < M; ++m)
-                    cnt += key[m] == pre &&
-                           ((uint32_t)cidx[lane + 32 * m] & mk) == jp;
-                cnt = __reduce_add_sync(0xffffffffu, cnt);
-                if (below + cnt < need) {
-                    below += cnt;
-                    jp |= bm;
+                for (int x = 0; x < S::kPer16; ++x) {
+                    const unsigned long long kk = sel_pack(kv[x], kv[x]);
+                    acc01[m] = sel_fma2(q01[x], kk, acc01[m]);
+                    acc23[m] = sel_fma2(q23[x], kk, acc23[m]);
                 }
-                jm = mk;
             }
-            jmax = (int)jp;
         }
-        uint32_t *out = selmask + ((size_t)bh * N + p) * W;
+        uint32_t key[kSelQB][M];
 #pragma unroll
         for (int m = 0; m < M; ++m) {
-            const bool s = key[m] > pre ||
-                           (key[m] == pre && cidx[lane + 32 * m] <= jmax);
-            const uint32_t word = __ballot_sync(0xffffffffu, s);
-            if (lane == m) out[m] = word;
+            key[0][m] = ordered_key(sel_lo(acc01[m]));
+            key[1][m] = ordered_key(sel_hi(acc01[m]));
+            key[2][m] = ordered_key(sel_lo(acc23[m]));
+            key[3][m] = ordered_key(sel_hi(acc23[m]));
+        }
+        // the k-th largest key of each query: the largest value T with at
+        // least k keys >= T, built MSB first (a bit stays set when enough
+        // keys reach it); the four searches run together, two counts packed
+        // per warp reduction
+        uint32_t pre[kSelQB] = {0u, 0u, 0u, 0u};
+        for (int bit = 31; bit >= 0; --bit) {
+            const uint32_t bm = 1u << bit;
+            int cnt[kSelQB];
+#pragma unroll
+            for (int qq = 0; qq < kSelQB; ++qq) {
+                const uint32_t want = pre[qq] | bm;
+                int n = 0;
+#pragma unroll
+                for (int m = 0; m < M; ++m) n += key[qq][m] >= want;
+                cnt[qq] = n;
+            }
+            const int c01 = __reduce_add_sync(0xffffffffu,
+                                              cnt[0] | (cnt[1] << 16));
+            const int c23 = __reduce_add_sync(0xffffffffu,
+                                              cnt[2] | (cnt[3] << 16));
+            cnt[0] = c01 & 0xffff;
+            cnt[1] = c01 >> 16;
+            cnt[2] = c23 & 0xffff;
+            cnt[3] = c23 >> 16;
+#pragma unroll
+            for (int qq = 0; qq < kSelQB; ++qq)
+                if (cnt[qq] >= k) pre[qq] |= bm;
+        }
+        // keys strictly above each threshold
+        int above[kSelQB];
+        {
+            int cnt[kSelQB];
+#pragma unroll
+            for (int qq = 0; qq < kSelQB; ++qq) {
+                int n = 0;
+#pragma unroll
+                for (int m = 0; m < M; ++m) n += key[qq][m] > pre[qq];
+                cnt[qq] = n;
+            }
+            const int c01 = __reduce_add_sync(0xffffffffu,
+                                              cnt[0] | (cnt[1] << 16));
+            const int c23 = __reduce_add_sync(0xffffffffu,
+                                              cnt[2] | (cnt[3] << 16));
+            above[0] = c01 & 0xffff;
+            above[1] = c01 >> 16;
+            above[2] = c23 & 0xffff;
+            above[3] = c23 >> 16;
+        }
+        for (int qq = 0; qq < nq; ++qq) {
+            const int p = t * b + q0 + qq;
+            // keys equal to the threshold: the need lowest original indices
+            const int need = k - above[qq];
+            int ties = 0;
+#pragma unroll
+            for (int m = 0; m < M; ++m) ties += key[qq][m] == pre[qq];
+            ties = __reduce_add_sync(0xffffffffu, ties);
+            int jmax = 0x7fffffff;
+            if (ties > need) {
+                uint32_t jp = 0, jm = 0;
+                int below = 0;
+                for (int bit = 30; bit >= 0; --bit) {
+                    const uint32_t bm = 1u << bit, mk = jm | bm;
+                    int cnt = 0;  // ties whose index has this bit clear
+#pragma unroll
+                    for (int m = 0; m < M; ++m)
+                        cnt += key[qq][m] == pre[qq] &&
+                               ((uint32_t)cj[m] & mk) == jp;
+                    cnt = __reduce_add_sync(0xffffffffu, cnt);
+                    if (below + cnt < need) {
+                        below += cnt;
+                        jp |= bm;
+                    }
+                    jm = mk;
+                }
+                jmax = (int)jp;
+            }
+            uint32_t *out = selmask + ((size_t)bh * N + p) * W;
+#pragma unroll
+            for (int m = 0; m < M; ++m) {
+                const bool sl = key[qq][m] > pre[qq] ||
+                                (key[qq][m] == pre[qq] && cj[m] <= jmax);
+                const uint32_t word = __ballot_sync(0xffffffffu, sl);
+                if (lane == m) out[m] = word;
+            }
         }
     }
 }
@@ -297,8 +476,9 @@ __global__ void __launch_bounds__(kSelThreads)
 
 size_t select_smem(const Plan &P) {
     const int nc = P.tk_c * P.b;
-    return (size_t)nc * (P.d + kSelPad) * 4 + (size_t)nc * 4 +
-           (size_t)kSelWarps * P.d * 4;
+    const int rb = P.dtype == ELSAA_FP32 ? sel_row_bytes<float>(P.d)
+                                         : sel_row_bytes<__nv_bfloat16>(P.d);
+    return (size_t)(nc + P.b) * rb + (size_t)(nc + P.b) * 4;
 }
 
 }  // namespace
@@ -315,17 +495,20 @@ bool topk_supported(const Plan &P, const char **msg) {
     }
     if (select_smem(P) > 200 * 1024) {
         *msg = "selector 1: the candidate keys of a block (topk_blocks * "
-               "block_size rows of d_h fp32) exceed 200 KiB of shared memory";
+               "block_size rows of d_h values) exceed 200 KiB of shared "
+               "memory";
         return false;
     }
     return true;
 }
 
-cudaError_t launch_topk(const Plan &P, const void *q, const void *k,
-                        const int32_t *perm_q, const int32_t *perm_k,
-                        float *sums, int32_t *cand, uint32_t *selmask,
-                        DeviceStatus *status, cudaStream_t st) {
+cudaError_t launch_topk(int stage, const Plan &P, const void *q,
+                        const void *k, const int32_t *perm_q,
+                        const int32_t *perm_k, float *sums, int32_t *cand,
+                        uint32_t *selmask, DeviceStatus *status,
+                        cudaStream_t st) {
     const int T = P.N / P.b;
+    if (stage == 0) {
     dim3 gs(T, P.BH, 2);
     if (P.dtype == ELSAA_FP32)
         k_topk_sums<float><<<gs, P.d, 0, st>>>(
@@ -335,17 +518,18 @@ cudaError_t launch_topk(const Plan &P, const void *q, const void *k,
         k_topk_sums<__nv_bfloat16><<<gs, P.d, 0, st>>>(
             (const __nv_bfloat16 *)q, (const __nv_bfloat16 *)k, perm_q,
             perm_k, P.N, P.d, P.b, sums, status);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    const size_t csm = (size_t)P.d * 4 + (size_t)T * 8;
-    if (csm > 48 * 1024)
-        cudaFuncSetAttribute(k_topk_cand,
-                             cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)csm);
-    k_topk_cand<<<dim3(T, P.BH), kSelThreads, csm, st>>>(sums, P.d, P.tk_c,
-                                                         cand);
-    e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
+        return cudaGetLastError();
+    }
+    if (stage == 1) {
+        const size_t csm = (size_t)P.d * 4 + (size_t)T * 8;
+        if (csm > 48 * 1024)
+            cudaFuncSetAttribute(k_topk_cand,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)csm);
+        k_topk_cand<<<dim3(T, P.BH), kSelThreads, csm, st>>>(sums, P.d,
+                                                             P.tk_c, cand);
+        return cudaGetLastError();
+    }
     const size_t smem = select_smem(P);
     auto run = [&](auto kern, auto *qp, auto *kp) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,

@@ -98,7 +98,11 @@ def backward_flop_model(wl: Workload) -> dict:
 def keys_per_query(wl: Workload) -> int:
     """Keys each query attends to in the sparse branch: its block and the
     neighbouring sorted blocks, (2 r + 1) b (Section 5), at most N (the
-    clipped windows at the two ends are counted as full)."""
+    clipped windows at the two ends are counted as full). With the top-k
+    selector the tensor cores score all c b candidate keys of a query
+    block (the unselected ones are masked)."""
+    if getattr(wl, "selector", 0) == 1:
+        return min(wl.N, wl.topk_blocks * wl.block)
     return min(wl.N, (2 * getattr(wl, "neighbor_blocks", 0) + 1) * wl.block)
 
 
@@ -182,6 +186,16 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
     elif kernel.startswith("race_reduce"):
         by = H * r * (d + 1) * 4  # the summaries A and B, written once
         fl = 0
+        simt = True
+    elif kernel.startswith("topk_select"):
+        # block sums (Q and K read through the sort orders), block scores,
+        # and per query the canonical fp32 chains over the c b candidate
+        # keys (each query block stages its candidates once): reads Q once
+        # and the candidate keys c times, writes the bitmask
+        c = getattr(wl, "topk_blocks", 1)
+        by = H * (2 * N * d * e + N * d * e + c * N * d * e + N * c * wl.block
+                  // 8)
+        fl = H * (2 * N * c * wl.block * d + 2 * (N // wl.block) ** 2 * d)
         simt = True
     elif kernel.startswith("sort_hash"):
         by = H * 2 * N * d * e

@@ -99,12 +99,28 @@ def oracle(wl, x, heads=None, rows=None, **kw):
     ("bf16", 64, 64, 2, 64), ("bf16", 128, 128, 2, 128),
     ("bf16", 128, 32, 4, 50), ("fp32", 128, 128, 2, 200),
     ("bf16", 64, 256, 2, 300), ("bf16", 64, 64, 1, 10),
+    ("bf16", 128, 128, 1, 64), ("bf16", 64, 128, 3, 200),
+    ("bf16", 128, 256, 1, 100), ("bf16", 64, 128, 4, 128),
 ])
 def test_topk_matches_oracle(dtype, d_h, b, c, k):
     wl = small(dtype, d_h=d_h, block=b, topk_blocks=c, topk=k,
                N=max(1024, 4 * b))
     x = make_inputs(wl)
     compare(wl, run_gpu(wl, x), oracle(wl, x), label=(dtype, d_h, b, c, k))
+
+
+def test_tensor_core_path_runs_for_bf16_blocks_of_128():
+    """bf16 with blocks of 128 or 256 and gamma = 4: the persistent
+    tensor-core block kernel walks the candidate blocks (no CUDA-core
+    fallback)."""
+    wl = small("bf16", d_h=128, block=128, topk_blocks=2, topk=100)
+    x = make_inputs(wl)
+    elsaa.elsaa_profile_start()
+    g = run_gpu(wl, x)
+    prof = elsaa.elsaa_profile_stop()
+    assert "block_attn_ws" in prof and "block_attn_simt" not in prof, prof
+    assert "topk_select" in prof
+    compare(wl, g, oracle(wl, x), label="tc path")
 
 
 def test_topk_ties_on_integer_inputs():
