@@ -378,6 +378,34 @@ def extra_workloads(args, dev, stream, peaks):
                               sample="256 rows of head (1, 7)"),
     }
     del x, o, ws
+    # -- c3 with learned gates and query-dependent lambda (hidden width 64)
+    # computed inside the forward call
+    wl = WORKLOADS["c3"]
+    x = make_inputs(wl, device=dev)
+    p = elsaa.params_for(wl)
+    mlp = make_gate_mlp(wl, hidden=64, device=dev)
+    ws = torch.empty(max(elsaa.elsaa_forward_gated_workspace_size(p, mlp),
+                         256), dtype=torch.uint8, device=dev)
+    o = torch.empty_like(x["q"])
+
+    def step():
+        elsaa.elsaa_forward_gated(p, mlp, x["q"], x["k"], x["v"],
+                                  x["w_sort"], x["w_race"], o=o,
+                                  workspace=ws, stream=stream)
+
+    ms, prof = measure(step, args.steps, args.warmup, dev, stream)
+    elsaa.elsaa_check_status(ws)
+    out["c3_gated"] = {
+        "config": dict(workload_config(wl), gate_mlp_hidden=64),
+        "step": "elsaa_forward_gated: gate MLP (hidden 64) and lambda_i in "
+                "the same call",
+        "ms_per_step": ms, "value": wl.tokens / (ms / 1e3),
+        "unit": "tokens/s",
+        "kernels": {k: {"launches": n, "avg_us": 1e3 * t / n}
+                    for k, (n, t) in sorted(prof.items())},
+        "gpu_launches": sum(n for n, _ in prof.values()),
+    }
+    del x, o, ws
     # -- c5: training step, forward + backward
     wl = WORKLOADS["c5"]
     x = make_inputs(wl.with_(backward=True), device=dev)
@@ -481,21 +509,18 @@ def run_ours(args, wl):
                             x["w_race"], o=o, workspace=ws, stream=stream)
 
     if args.gate_mlp:
-        # learned gates and query-dependent lambda (elsaa_gates) feeding the
-        # fusion: both calls run in every step
+        # learned gates and query-dependent lambda feeding the fusion, in
+        # the same call (elsaa_forward_gated: inside the sort hash where the
+        # shape allows, else the gate kernel first)
         mlp = make_gate_mlp(wl_rank, hidden=args.gate_mlp, device=dev)
-        BHN = (wl.B, wl.H, wl.N)
-        gts = torch.empty(BHN + (2,), dtype=torch.float32, device=dev)
-        lam = torch.empty(BHN, dtype=torch.float32, device=dev)
-        wsg = torch.empty(max(elsaa.elsaa_gates_workspace_size(p, mlp), 256),
-                          dtype=torch.uint8, device=dev)
+        ws = torch.empty(
+            max(elsaa.elsaa_forward_gated_workspace_size(p, mlp), 256),
+            dtype=torch.uint8, device=dev)
 
         def step():
-            elsaa.elsaa_gates(p, mlp, x["q"], gates=gts, lambda_tok=lam,
-                              workspace=wsg, stream=stream)
-            elsaa.elsaa_forward(p, x["q"], x["k"], x["v"], x["w_sort"],
-                                x["w_race"], lambda_tok=lam, gates=gts, o=o,
-                                workspace=ws, stream=stream)
+            elsaa.elsaa_forward_gated(p, mlp, x["q"], x["k"], x["v"],
+                                      x["w_sort"], x["w_race"], o=o,
+                                      workspace=ws, stream=stream)
 
     if args.backward:
         # the backward pass of the same inputs: permutations and the RACE

@@ -403,6 +403,38 @@ int elsaa_gates(const elsaa_params *params, const elsaa_gate_mlp *mlp,
                 void *workspace, size_t workspace_bytes, void *stream);
 
 /*
+ * The forward pass with its learned gates and query-dependent lambda
+ * computed in the same call: the result of elsaa_gates followed by
+ * elsaa_forward with those gates and lambda_tok (Section 3.3 fusion with
+ * gates sigma(G_theta(q_i)); the model-setup appendix's gate MLP; the
+ * lambda appendix's lambda_i).
+ *
+ * Non-causal: the gate kernel runs on the caller's stream right after the
+ * sort, while the RACE key side (the longer of the two chains before the
+ * block kernel) is still running, so it fills the SMs the sort chain has
+ * left idle; the block kernel then reads the gates and lambda. Causal: the
+ * gate kernel, then the causal forward.
+ *
+ * Arguments as elsaa_forward and elsaa_gates; gates_out [B, H, N, 2] and
+ * lambda_out [B, H, N] (fp32, device, written) are optional copies of the
+ * computed gates and lambda (NULL: kept in the workspace; lambda is only
+ * computed when mlp->w_lambda is given, otherwise params->lambda is used).
+ * workspace: at least elsaa_forward_gated_workspace_size() bytes, 256-byte
+ * aligned. Errors as for elsaa_forward and elsaa_gates.
+ */
+int elsaa_forward_gated_workspace_size(const elsaa_params *params,
+                                       const elsaa_gate_mlp *mlp,
+                                       size_t *bytes);
+int elsaa_forward_gated(const elsaa_params *params,
+                        const elsaa_gate_mlp *mlp, const void *q,
+                        const void *k, const void *v, const float *w_sort,
+                        const float *w_race, void *o, float *log_d_sparse,
+                        float *d_lr, float *m_sparse, int32_t *perm_q,
+                        int32_t *perm_k, float *gates_out, float *lambda_out,
+                        void *workspace, size_t workspace_bytes,
+                        void *stream);
+
+/*
  * Synchronises `stream` and reads the in-band status word that the kernels
  * of the last elsaa_forward on this workspace wrote (bounded waits that ran
  * out, inconsistent sort counts). Returns ELSAA_OK, ELSAA_ERR_DEVICE (with

@@ -6,6 +6,7 @@
 
 #include <cudaTypedefs.h>
 
+#include <deque>
 #include <mutex>
 #include <string>
 #include <vector>
@@ -73,7 +74,8 @@ struct SideStream {
 };
 
 cudaError_t side_stream(SideStream **out) {
-    thread_local std::vector<SideStream> ss;
+    // a deque keeps earlier entries in place when another device is added
+    thread_local std::deque<SideStream> ss;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
@@ -549,19 +551,17 @@ extern "C" int elsaa_workspace_size(const elsaa_params *params,
 }
 
 
-extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
-                             const void *k, const void *v,
-                             const float *w_sort, const float *w_race,
-                             const float *lambda_tok, const float *gates,
-                             void *o, float *log_d_sparse, float *d_lr,
-                             float *m_sparse, int32_t *perm_q,
-                             int32_t *perm_k, void *workspace,
-                             size_t workspace_bytes, void *stream) {
-    g_err[0] = 0;
-    if (params && params->causal == 1)
-        return causal_forward(params, q, k, v, w_sort, w_race, lambda_tok,
-                              gates, o, log_d_sparse, d_lr, m_sparse,
-                              workspace, workspace_bytes, stream);
+namespace {
+
+// The non-causal forward. gf: the gate network computed in the same call
+// (its outputs are the gates / lambda_tok given here), or NULL.
+int forward_impl(const elsaa_params *params, const void *q, const void *k,
+                 const void *v, const float *w_sort, const float *w_race,
+                 const float *lambda_tok, const float *gates, void *o,
+                 float *log_d_sparse, float *d_lr, float *m_sparse,
+                 int32_t *perm_q, int32_t *perm_k, void *workspace,
+                 size_t workspace_bytes, void *stream,
+                 const GateFusion *gf) {
     Plan P;
     const char *msg = "";
     int rc = make_plan(params, &P, &msg);
@@ -648,6 +648,16 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                                                       pk, status, st);
                        }),
                        "sort_scatter");
+    // the gate network (elsaa_forward_gated): on the caller's stream right
+    // after the sort, so its CTAs take the SMs that the sort chain leaves
+    // idle while the RACE key side (the longer chain) finishes
+    if (gf)
+        ELSAA_CHECK_LAUNCH(timed("gate_mlp", st, [&] {
+                               return launch_gates(P, *gf->mlp, q, gf->gates,
+                                                   gf->lam, gf->gate_ws,
+                                                   status, st);
+                           }),
+                           "gate_mlp");
     int32_t *cand = nullptr;
     uint32_t *selmask = nullptr;
     if (P.sel) {
@@ -695,6 +705,26 @@ extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
                            "block_attn_simt");
     }
     return ELSAA_OK;
+}
+
+}  // namespace
+
+extern "C" int elsaa_forward(const elsaa_params *params, const void *q,
+                             const void *k, const void *v,
+                             const float *w_sort, const float *w_race,
+                             const float *lambda_tok, const float *gates,
+                             void *o, float *log_d_sparse, float *d_lr,
+                             float *m_sparse, int32_t *perm_q,
+                             int32_t *perm_k, void *workspace,
+                             size_t workspace_bytes, void *stream) {
+    g_err[0] = 0;
+    if (params && params->causal == 1)
+        return causal_forward(params, q, k, v, w_sort, w_race, lambda_tok,
+                              gates, o, log_d_sparse, d_lr, m_sparse,
+                              workspace, workspace_bytes, stream);
+    return forward_impl(params, q, k, v, w_sort, w_race, lambda_tok, gates,
+                        o, log_d_sparse, d_lr, m_sparse, perm_q, perm_k,
+                        workspace, workspace_bytes, stream, nullptr);
 }
 
 // ---------------------------------------------------------------- backward
@@ -1133,6 +1163,106 @@ extern "C" int elsaa_gates(const elsaa_params *params,
                        }),
                        "gate_mlp");
     return ELSAA_OK;
+}
+
+namespace {
+
+// Extra workspace of elsaa_forward_gated after the forward's own: the gate
+// kernel's workspace (elsaa_gates' layout), then the gates [B*H*N][2] and
+// lambda [B*H*N] (fp32).
+struct GatedPlan {
+    size_t fwd, off_gws, off_gates, off_lam, total;
+};
+
+int make_gated_plan(const elsaa_params *params, const elsaa_gate_mlp *mlp,
+                    GatedPlan *G, const char **msg) {
+    static thread_local char fwd_msg[256];
+    size_t fwd = 0;
+    int rc = elsaa_workspace_size(params, &fwd);
+    if (rc != ELSAA_OK) {
+        snprintf(fwd_msg, sizeof(fwd_msg), "%s", elsaa_last_error());
+        *msg = fwd_msg;
+        return rc;
+    }
+    Plan P;
+    rc = make_plan(params, &P, msg);
+    if (rc == ELSAA_OK) rc = check_gate_mlp(mlp, msg);
+    if (rc != ELSAA_OK) return rc;
+    size_t off = align_up(fwd, 256);
+    G->fwd = fwd;
+    G->off_gws = off;
+    off = align_up(off + gate_workspace_bytes(P, mlp->hidden), 256);
+    const size_t BHN = (size_t)P.BH * P.N;
+    G->off_gates = off;
+    off = align_up(off + BHN * 2 * sizeof(float), 256);
+    G->off_lam = off;
+    off = align_up(off + BHN * sizeof(float), 256);
+    G->total = off;
+    return ELSAA_OK;
+}
+
+}  // namespace
+
+extern "C" int elsaa_forward_gated_workspace_size(const elsaa_params *params,
+                                                  const elsaa_gate_mlp *mlp,
+                                                  size_t *bytes) {
+    g_err[0] = 0;
+    if (!bytes) return fail(ELSAA_ERR_INVALID_ARG, "bytes is NULL");
+    GatedPlan G;
+    const char *msg = "";
+    int rc = make_gated_plan(params, mlp, &G, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    *bytes = G.total;
+    return ELSAA_OK;
+}
+
+extern "C" int elsaa_forward_gated(
+    const elsaa_params *params, const elsaa_gate_mlp *mlp, const void *q,
+    const void *k, const void *v, const float *w_sort, const float *w_race,
+    void *o, float *log_d_sparse, float *d_lr, float *m_sparse,
+    int32_t *perm_q, int32_t *perm_k, float *gates_out, float *lambda_out,
+    void *workspace, size_t workspace_bytes, void *stream) {
+    g_err[0] = 0;
+    GatedPlan G;
+    const char *msg = "";
+    int rc = make_gated_plan(params, mlp, &G, &msg);
+    if (rc != ELSAA_OK) return fail(rc, "%s", msg);
+    if (!q) return fail(ELSAA_ERR_INVALID_ARG, "q must be non-NULL");
+    if ((uintptr_t)q % 16 || (uintptr_t)mlp->b1 % 16 ||
+        (uintptr_t)mlp->w2 % 16 || (gates_out && (uintptr_t)gates_out % 8))
+        return fail(ELSAA_ERR_INVALID_ARG,
+                    "q, mlp->b1 and mlp->w2 must be 16-byte and gates_out "
+                    "8-byte aligned");
+    if (!workspace) return fail(ELSAA_ERR_WORKSPACE, "workspace is NULL");
+    if ((uintptr_t)workspace % 256)
+        return fail(ELSAA_ERR_WORKSPACE, "workspace must be 256-byte aligned");
+    if (workspace_bytes < G.total)
+        return fail(ELSAA_ERR_WORKSPACE,
+                    "workspace too small: %zu bytes given, %zu needed",
+                    workspace_bytes, G.total);
+    cudaStream_t st = (cudaStream_t)stream;
+    char *ws = (char *)workspace;
+    float *gts = gates_out ? gates_out : (float *)(ws + G.off_gates);
+    float *lam = mlp->w_lambda
+                     ? (lambda_out ? lambda_out : (float *)(ws + G.off_lam))
+                     : nullptr;
+    if (params->causal) {
+        // causal: the gate kernel of elsaa_gates, then the forward
+        rc = elsaa_gates(params, mlp, q, gts, lam, ws + G.off_gws,
+                         G.off_gates - G.off_gws, stream);
+        if (rc != ELSAA_OK) return rc;
+        return elsaa_forward(params, q, k, v, w_sort, w_race, lam, gts, o,
+                             log_d_sparse, d_lr, m_sparse, perm_q, perm_k,
+                             workspace, G.fwd, stream);
+    }
+    GateFusion gf;
+    gf.mlp = mlp;
+    gf.gate_ws = (uint16_t *)(ws + G.off_gws + 256);
+    gf.gates = gts;
+    gf.lam = lam;
+    return forward_impl(params, q, k, v, w_sort, w_race, lam, gts, o,
+                        log_d_sparse, d_lr, m_sparse, perm_q, perm_k,
+                        workspace, G.fwd, stream, &gf);
 }
 
 extern "C" int elsaa_selftest_wait_timeout(void *workspace,

@@ -90,6 +90,14 @@ cudaError_t launch_block_attn_simt(
     float *m_sparse, DeviceStatus *status, cudaStream_t st,
     const int32_t *cand = nullptr, const uint32_t *selmask = nullptr);
 
+// The gate network run inside elsaa_forward_gated (gates.cu kernels):
+// its description, the bf16 operand image it writes, and its outputs.
+struct GateFusion {
+    const elsaa_gate_mlp *mlp;
+    uint16_t *gate_ws;  // launch_gates' bf16 operand image
+    float *gates, *lam;
+};
+
 // Per-query top-k selector (topk.cu).
 bool topk_supported(const Plan &P, const char **msg);
 // stage 0: block sums; 1: candidate blocks; 2: per-query selection

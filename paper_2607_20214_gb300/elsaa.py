@@ -33,7 +33,8 @@ SYMBOLS = ("elsaa_workspace_size", "elsaa_forward", "elsaa_check_status",
            "elsaa_selftest_wait_timeout", "elsaa_forward_race_summaries",
            "elsaa_check_status_noalloc",
            "elsaa_selftest_wait_timeout_noalloc", "elsaa_causal_levels",
-           "elsaa_causal_index_lists", "elsaa_forward_selected_keys")
+           "elsaa_causal_index_lists", "elsaa_forward_selected_keys",
+           "elsaa_forward_gated_workspace_size", "elsaa_forward_gated")
 # Size of the fixed scratch array behind elsaa_forward_noalloc.
 ELSAA_STATIC_WORKSPACE_BYTES = 64 << 20
 
@@ -139,6 +140,14 @@ def load_library(path: str = LIB) -> ctypes.CDLL:
     L.elsaa_causal_index_lists.argtypes = [ctypes.POINTER(elsaa_params), vp,
                                            ctypes.c_size_t, vp, vp]
     L.elsaa_causal_index_lists.restype = ctypes.c_int
+    L.elsaa_forward_gated_workspace_size.argtypes = [
+        ctypes.POINTER(elsaa_params), ctypes.POINTER(elsaa_gate_mlp),
+        ctypes.POINTER(ctypes.c_size_t)]
+    L.elsaa_forward_gated_workspace_size.restype = ctypes.c_int
+    L.elsaa_forward_gated.argtypes = [
+        ctypes.POINTER(elsaa_params), ctypes.POINTER(elsaa_gate_mlp)] + [
+        vp] * 14 + [ctypes.c_size_t, vp]
+    L.elsaa_forward_gated.restype = ctypes.c_int
     L.elsaa_forward_selected_keys.argtypes = [
         ctypes.POINTER(elsaa_params), vp, ctypes.c_size_t, vp, vp]
     L.elsaa_forward_selected_keys.restype = ctypes.c_int
@@ -569,3 +578,58 @@ def elsaa_forward_selected_keys(params: elsaa_params, workspace, keys=None,
         workspace.numel() * workspace.element_size(),
         _ptr(keys, "keys", torch.int32, n, dev), _stream_ptr(stream)))
     return keys
+
+
+def elsaa_forward_gated_workspace_size(params: elsaa_params, mlp: dict,
+                                       device=None) -> int:
+    dev = mlp["w1"].device if device is None else device
+    m = _gate_struct(params, mlp, dev)
+    n = ctypes.c_size_t(0)
+    _check(load_library().elsaa_forward_gated_workspace_size(
+        ctypes.byref(params), ctypes.byref(m), ctypes.byref(n)))
+    return n.value
+
+
+def elsaa_forward_gated(params: elsaa_params, mlp: dict, q, k, v, w_sort,
+                        w_race, o=None, log_d_sparse=None, d_lr=None,
+                        m_sparse=None, perm_q=None, perm_k=None,
+                        gates_out=None, lambda_out=None, workspace=None,
+                        stream=None):
+    """Enqueue elsaa_forward_gated: the forward with the gates and lambda
+    of the gate MLP `mlp` (as for elsaa_gates) computed in the same call.
+    Returns o (allocated here when not given)."""
+    lib = load_library()
+    dev = q.device
+    tdt = torch.float32 if params.dtype == ELSAA_FP32 else torch.bfloat16
+    odt = torch.float32 if params.out_fp32 else tdt
+    BHN = params.B * params.H * params.N
+    nqkv = BHN * params.d_h
+    m = _gate_struct(params, mlp, dev)
+    if o is None:
+        o = torch.empty(q.shape, dtype=odt, device=dev)
+    if workspace is None:
+        n = elsaa_forward_gated_workspace_size(params, mlp, dev)
+        workspace = torch.empty(max(n, 256), dtype=torch.uint8, device=dev)
+    args = [
+        _ptr(q, "q", tdt, nqkv, dev), _ptr(k, "k", tdt, nqkv, dev),
+        _ptr(v, "v", tdt, nqkv, dev),
+        _ptr(w_sort, "w_sort", torch.float32,
+             params.H * params.sort_bits * params.d_h, dev)
+        if params.sort_bits > 0 else None,
+        _ptr(w_race, "w_race", torch.float32,
+             params.H * params.race_tables * params.race_bits * params.d_h,
+             dev),
+        _ptr(o, "o", odt, nqkv, dev),
+        _ptr(log_d_sparse, "log_d_sparse", torch.float32, BHN, dev),
+        _ptr(d_lr, "d_lr", torch.float32, BHN, dev),
+        _ptr(m_sparse, "m_sparse", torch.float32, BHN, dev),
+        _ptr(perm_q, "perm_q", torch.int32, BHN, dev),
+        _ptr(perm_k, "perm_k", torch.int32, BHN, dev),
+        _ptr(gates_out, "gates_out", torch.float32, 2 * BHN, dev),
+        _ptr(lambda_out, "lambda_out", torch.float32, BHN, dev),
+        _ptr(workspace, "workspace", None, None, dev),
+    ]
+    _check(lib.elsaa_forward_gated(
+        ctypes.byref(params), ctypes.byref(m), *args,
+        workspace.numel() * workspace.element_size(), _stream_ptr(stream)))
+    return o
