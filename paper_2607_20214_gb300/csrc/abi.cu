@@ -1037,7 +1037,8 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                                return launch_bwd_block(
                                    P, q, k, v, d_o, w_race, A, Bm, perm_q,
                                    perm_k, lambda_tok, gates, dq, dk, dv,
-                                   d_gates, d_lambda, gnum, gden, st);
+                                   d_gates, d_lambda, gnum, gden, status,
+                                   st);
                            }),
                            "bwd_block");
     }

@@ -132,7 +132,8 @@ __global__ void __launch_bounds__(kBwdThreads)
                 float lambda, int mode, float *__restrict__ dq,
                 float *__restrict__ dk, float *__restrict__ dv,
                 float *__restrict__ d_gates, float *__restrict__ d_lambda,
-                float *__restrict__ gnum, float *__restrict__ gden) {
+                float *__restrict__ gnum, float *__restrict__ gden,
+                DeviceStatus *status) {
     extern __shared__ float sm[];
     __shared__ int qi[kBwdMaxB], ki[kBwdMaxB];
     const int t = blockIdx.x, bh = blockIdx.y, h = bh % H, tid = threadIdx.x;
@@ -154,8 +155,19 @@ __global__ void __launch_bounds__(kBwdThreads)
 
     const size_t base = (size_t)bh * N;
     for (int i = tid; i < b; i += kBwdThreads) {
-        qi[i] = perm_q[base + (size_t)t * b + i];
-        ki[i] = perm_k[base + (size_t)t * b + i];
+        // entries outside [0, N) are recorded and read as row 0
+        int a = perm_q[base + (size_t)t * b + i];
+        int c = perm_k[base + (size_t)t * b + i];
+        if (a < 0 || a >= N) {
+            report(status, kDevPermRange, 12, bh, a);
+            a = 0;
+        }
+        if (c < 0 || c >= N) {
+            report(status, kDevPermRange, 13, bh, c);
+            c = 0;
+        }
+        qi[i] = a;
+        ki[i] = c;
     }
     __syncthreads();
     for (int x = tid; x < b * d; x += kBwdThreads) {
@@ -366,7 +378,8 @@ cudaError_t launch_bwd_block(const Plan &P, const void *q, const void *k,
                              const int32_t *perm_k, const float *lambda_tok,
                              const float *gates, float *dq, float *dk,
                              float *dv, float *d_gates, float *d_lambda,
-                             float *gnum, float *gden, cudaStream_t st) {
+                             float *gnum, float *gden, DeviceStatus *status,
+                             cudaStream_t st) {
     dim3 grid(P.N / P.b, P.BH);
     const size_t smem = bwd_block_smem(P);
 #define ELSAA_LAUNCH_BWD(T)                                                    \
@@ -379,7 +392,7 @@ cudaError_t launch_bwd_block(const Plan &P, const void *q, const void *k,
             (const T *)q, (const T *)k, (const T *)v, (const T *)d_o, w_race,  \
             A, Bm, perm_q, perm_k, lambda_tok, gates, P.N, P.d, P.H, P.b, P.L, \
             P.gamma, P.beta, P.eps, P.scale, P.lambda, P.fusion_mode, dq, dk,  \
-            dv, d_gates, d_lambda, gnum, gden);                                \
+            dv, d_gates, d_lambda, gnum, gden, status);                        \
     } while (0)
     if (P.dtype == ELSAA_FP32)
         ELSAA_LAUNCH_BWD(float);

@@ -179,8 +179,15 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             const size_t hb = (size_t)bh * N;
             const int p0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
             int qi = perm_q[hb + p0 + tid], ki = perm_k[hb + p0 + tid];
-            qi = (qi < 0 || qi >= N) ? 0 : qi;
-            ki = (ki < 0 || ki >= N) ? 0 : ki;
+            // entries outside [0, N) are recorded and read as row 0
+            if (qi < 0 || qi >= N) {
+                report(status, kDevPermRange, 10, bh, qi);
+                qi = 0;
+            }
+            if (ki < 0 || ki >= N) {
+                report(status, kDevPermRange, 11, bh, ki);
+                ki = 0;
+            }
             qrow2[tt & 1][tid] = (int)(hb + qi);
             krow2[tt & 1][tid] = (int)(hb + ki);
         }

@@ -246,8 +246,12 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         // from the level's index list into krow_s[kt & 1] (then a barrier)
         auto stage_rows = [&](int kt) {
             if (MODE == 1 && tid < 128) {
-                const int t = kl[kt * 128 + tid];
-                krow_s[kt & 1][tid] = (t < 0 || t >= N) ? 0 : t;
+                int t = kl[kt * 128 + tid];
+                if (t < 0 || t >= N) {  // recorded, read as row 0
+                    report(status, kDevPermRange, 14, bh, t);
+                    t = 0;
+                }
+                krow_s[kt & 1][tid] = t;
             }
         };
         auto load_tile = [&](uint32_t dst, const uint16_t *src, int kt) {
@@ -270,7 +274,10 @@ __global__ void __launch_bounds__(kCaThreads, 2)
                 t = seg0 + qt * 128 + tid;
             } else {
                 t = ql[qt * 128 + tid];
-                t = (t < 0 || t >= N) ? 0 : t;
+                if (t < 0 || t >= N) {  // recorded, read as row 0
+                    report(status, kDevPermRange, 15, bh, t);
+                    t = 0;
+                }
             }
             qrow_s[tid] = t;
         }

@@ -128,7 +128,8 @@ cudaError_t launch_bwd_block(const Plan &P, const void *q, const void *k,
                              const int32_t *perm_k, const float *lambda_tok,
                              const float *gates, float *dq, float *dk,
                              float *dv, float *d_gates, float *d_lambda,
-                             float *gnum, float *gden, cudaStream_t st);
+                             float *gnum, float *gden, DeviceStatus *status,
+                             cudaStream_t st);
 cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
                             const float *w_race, const float *gA,
                             const float *gB, float *dk, float *dv,

@@ -192,8 +192,13 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             r.z = pm[min(pos + 2, N - 1)];
             r.w = pm[min(pos + 3, N - 1)];
         }
+        // an entry outside [0, N) is recorded and read as row 0
         auto fix = [=](int v) {
-            return rowbase + ((v < 0 || v >= N) ? 0 : v);
+            if (v < 0 || v >= N) {
+                report(status, kDevPermRange, 4, rowbase / N, v);
+                v = 0;
+            }
+            return rowbase + v;
         };
         return make_int4(fix(r.x), fix(r.y), fix(r.z), fix(r.w));
     };
