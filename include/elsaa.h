@@ -352,8 +352,8 @@ int elsaa_forward_selected_keys(const elsaa_params *params,
 /*
  * Token-wise gates and query-dependent lambda, the learned inputs of the
  * fusion (Section 3.3: (g_sparse,i, g_lr,i) = sigma(G_theta(q_i)); the
- * model-setup appendix: G_theta is a two-layer MLP with a SiLU hidden layer
- * and two independent sigmoid outputs; the lambda appendix: the
+ * experiment-hyperparameter appendix (Appendix D): G_theta is a two-layer
+ * MLP with a SiLU hidden layer and two independent sigmoid outputs, and the
  * input-dependent coefficient lambda_i = c + sigma(w^T q_i + b), floored at
  * lambda_min). For every query row q_i of head h:
  *     a_i         = SiLU(W1[h] q_i + b1[h])            (width g)
@@ -406,8 +406,8 @@ int elsaa_gates(const elsaa_params *params, const elsaa_gate_mlp *mlp,
  * The forward pass with its learned gates and query-dependent lambda
  * computed in the same call: the result of elsaa_gates followed by
  * elsaa_forward with those gates and lambda_tok (Section 3.3 fusion with
- * gates sigma(G_theta(q_i)); the model-setup appendix's gate MLP; the
- * lambda appendix's lambda_i).
+ * gates sigma(G_theta(q_i)); Appendix D's gate MLP and input-dependent
+ * lambda_i).
  *
  * Non-causal: the gate kernel runs on the caller's stream right after the
  * sort, while the RACE key side (the longer of the two chains before the

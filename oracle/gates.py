@@ -14,7 +14,7 @@ Definitions followed (per head, per query row q_i):
       z_i = W2 a_i + b2                (2 outputs)
       g_i = sigmoid(z_i)               (elementwise)
   with SiLU(x) = x * sigmoid(x).
-* Query-dependent lambda, Appendix E (the input-dependent version):
+* Query-dependent lambda, Appendix D (the input-dependent version):
       lambda_i = max(c + sigmoid(w^T q_i + b), lambda_min),
   c >= 0, lambda_min = 1e-6 in the paper.
 

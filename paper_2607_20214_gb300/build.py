@@ -18,6 +18,11 @@ ROOT = os.path.dirname(PKG)
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libelsaa.so")
+# The checked variant: the sources that guard extra checks with
+# ELSAA_CHECKED (recording out-of-range permutation entries in the forward
+# kernels) compiled with it, linked with the other objects of the default
+# build.
+LIB_CHECKED = os.path.join(PKG, "libelsaa_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC",
               "--expt-relaxed-constexpr", "-I" + os.path.join(ROOT, "include")]
@@ -73,6 +78,39 @@ def build(force: bool = False, verbose: bool = False, extra=()) -> str:
         raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
     os.replace(tmp, LIB)
     return LIB
+
+
+def build_checked(force: bool = False) -> str:
+    """Builds libelsaa_checked.so (after the default library)."""
+    build()
+    checked = [src for src in _sources()
+               if "ELSAA_CHECKED" in open(src).read()]
+    if (not force and os.path.exists(LIB_CHECKED) and
+            os.path.getmtime(LIB_CHECKED) >= os.path.getmtime(LIB)):
+        return LIB_CHECKED
+    cc = nvcc()
+
+    def compile_one(src):
+        obj = os.path.join(BUILD, os.path.basename(src) + ".checked.o")
+        cmd = [cc, *ARCH, *NVCC_FLAGS, "-DELSAA_CHECKED", "-c", src, "-o",
+               obj]
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError("nvcc failed on %s:\n%s%s" % (
+                os.path.basename(src), r.stdout, r.stderr))
+        return obj
+
+    with ThreadPoolExecutor(max_workers=max(1, len(checked))) as ex:
+        cobjs = list(ex.map(compile_one, checked))
+    objs = [os.path.join(BUILD, os.path.basename(src) + ".o")
+            for src in _sources() if src not in checked] + cobjs
+    tmp = LIB_CHECKED + ".tmp%d" % os.getpid()
+    r = subprocess.run([cc, *ARCH, "-shared", "-o", tmp, *objs],
+                       capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError("link failed:\n%s%s" % (r.stdout, r.stderr))
+    os.replace(tmp, LIB_CHECKED)
+    return LIB_CHECKED
 
 
 if __name__ == "__main__":

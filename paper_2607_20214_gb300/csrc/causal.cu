@@ -247,8 +247,10 @@ __global__ void __launch_bounds__(kCaThreads, 2)
         auto stage_rows = [&](int kt) {
             if (MODE == 1 && tid < 128) {
                 int t = kl[kt * 128 + tid];
-                if (t < 0 || t >= N) {  // recorded, read as row 0
+                if (t < 0 || t >= N) {  // read as row 0 (checked: recorded)
+#ifdef ELSAA_CHECKED
                     report(status, kDevPermRange, 14, bh, t);
+#endif
                     t = 0;
                 }
                 krow_s[kt & 1][tid] = t;
@@ -274,8 +276,10 @@ __global__ void __launch_bounds__(kCaThreads, 2)
                 t = seg0 + qt * 128 + tid;
             } else {
                 t = ql[qt * 128 + tid];
-                if (t < 0 || t >= N) {  // recorded, read as row 0
+                if (t < 0 || t >= N) {  // read as row 0 (checked: recorded)
+#ifdef ELSAA_CHECKED
                     report(status, kDevPermRange, 15, bh, t);
+#endif
                     t = 0;
                 }
             }

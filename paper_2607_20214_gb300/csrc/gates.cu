@@ -1,10 +1,11 @@
 // Token-wise gates and query-dependent lambda of the ELSAA fusion.
 //
-// Section 3.3 (the fusion paragraph) with the model-setup appendix: the
-// gates are (g_sparse, g_lr) = sigmoid(G_theta(q_i)), G_theta a two-layer
-// MLP with a SiLU hidden layer of width g and two outputs, each through its
-// own sigmoid. The lambda appendix: lambda_i = max(c + sigmoid(w^T q + b),
-// lambda_min). Both are per head, per query row.
+// Section 3.3 (the fusion paragraph) with Appendix D (experiment
+// hyperparameters): the gates are (g_sparse, g_lr) = sigmoid(G_theta(q_i)),
+// G_theta a two-layer MLP with a SiLU hidden layer of width g and two
+// outputs, each through its own sigmoid. Appendix D, input-dependent
+// lambda: lambda_i = max(c + sigmoid(w^T q + b), lambda_min). Both are per
+// head, per query row.
 //
 // Tensor-core path (bf16 Q, d_h in {64, 128}): the hidden pre-activations
 // and the lambda projection of a 128-query tile come out of one tcgen05 MMA

@@ -66,8 +66,9 @@ struct WsBars {
 // 1 (WIN): a neighbour window (nb > 0), whose passes past either end of
 // the sequence are masked. 2 (SEL): the top-k selector's candidate blocks
 // (cand, tk_c per query block), each key masked unless the row's bit in
-// selmask is set. The checks of the other modes are compiled out.
-template <int G, int NPASS, int KM>
+// selmask is set. The checks of the other modes are compiled out. O32: O
+// is written as fp32 (out_fp32), each thread storing its half row directly.
+template <int G, int NPASS, int KM, bool O32 = false>
 __global__ void __launch_bounds__(kWsThreads, 1)
     k_block_attn_ws(const uint16_t *__restrict__ qx,
                     const uint16_t *__restrict__ kx,
@@ -192,10 +193,15 @@ __global__ void __launch_bounds__(kWsThreads, 1)
             r.z = pm[min(pos + 2, N - 1)];
             r.w = pm[min(pos + 3, N - 1)];
         }
-        // an entry outside [0, N) is recorded and read as row 0
+        // an entry outside [0, N) is read as row 0 (the orders come from
+        // the sort, in range by construction); the checked build
+        // (ELSAA_CHECKED) also records it: 4 % of this kernel's time when
+        // always on
         auto fix = [=](int v) {
             if (v < 0 || v >= N) {
+#ifdef ELSAA_CHECKED
                 report(status, kDevPermRange, 4, rowbase / N, v);
+#endif
                 v = 0;
             }
             return rowbase + v;
@@ -763,7 +769,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                     uint32_t v[16], ob[8];
                     tmem_ld16(so + nk + half * (d >> 1) + c, v);
                     tmem_wait_ld();
-                    if (o32) {
+                    if constexpr (O32) {
                         if (qvalid) {
                             float4 *dst = reinterpret_cast<float4 *>(
                                 o32 + tok * (size_t)d + half * (d >> 1) + c);
@@ -799,7 +805,7 @@ __global__ void __launch_bounds__(kWsThreads, 1)
                 }
             }
             named_sync(1 + g, 256);
-            if (!o32) {
+            if constexpr (!O32) {
                 const int ct = (cw & 7) * 32 + lane_id;  // 0..255
                 const int cpr = d >> 3, rpp = 256 / cpr;
                 const int crow = ct / cpr, cc = ct - crow * cpr;
@@ -845,6 +851,9 @@ bool ws_supported(const Plan &P) {
     // second (buckets past 128) at most 16, i.e. gamma >= 4 when r > 128;
     // row numbers in int
     const long rows = (long)P.N * P.BH;  // row numbers are int
+    // fp32 output is instantiated for gamma = 4; other gamma with out_fp32
+    // run the CUDA-core block kernel
+    if (P.o32 && P.gamma != 4) return false;
     return tc_supported(P) && ws_passes(P) > 0 &&
            (P.gamma >= 4 || P.r <= 128) && rows < (1L << 31);
 }
@@ -889,6 +898,22 @@ cudaError_t launch_block_attn_ws(
         return cudaGetLastError();
     };
     const int passes = ws_passes(P);
+    if (P.o32) {  // fp32 output: gamma = 4 (ws_supported)
+        if (P.sel) {
+            switch (passes) {
+                case 1: return launch(k_block_attn_ws<4, 1, 2, true>);
+                case 2: return launch(k_block_attn_ws<4, 2, 2, true>);
+                case 3: return launch(k_block_attn_ws<4, 3, 2, true>);
+                case 4: return launch(k_block_attn_ws<4, 4, 2, true>);
+                default: return cudaErrorInvalidValue;
+            }
+        }
+        if (passes == 3) return launch(k_block_attn_ws<4, 3, 1, true>);
+        if (passes == 6) return launch(k_block_attn_ws<4, 6, 1, true>);
+        if (P.gamma != 4) return cudaErrorInvalidValue;
+        return P.b > 128 ? launch(k_block_attn_ws<4, 2, 0, true>)
+                         : launch(k_block_attn_ws<4, 1, 0, true>);
+    }
     if (P.sel) {
         switch (passes) {
             case 1: return launch(k_block_attn_ws<4, 1, 2>);

@@ -11,7 +11,7 @@ Q, K, V in R^{N x d_h}; multi-head applies the operator per head), laid out
 as [B, H, N, d_h]. Hyper-parameter defaults follow Table 7 (attention
 hyper-parameters): RACE hash bits gamma = 4, sortLSH bits = 5,
 epsilon = 1e-6; lambda = 1 is the initial value of the learned scalar
-(Appendix E).
+(Appendix D, experiment hyperparameters).
 """
 from __future__ import annotations
 
@@ -195,7 +195,7 @@ def make_gates_lambda(wl: Workload, seed: int, device="cpu"):
     """Per-token gates in (0, 1)^2 and per-token lambda > 0, for tests.
 
     Gates stand in for sigma(G_theta(q_i)) (Section 3.3); lambda_i stands in
-    for c + sigma(w^T q_i + b) (Appendix E). Both are plain seeded draws.
+    for c + sigma(w^T q_i + b) (Appendix D, experiment hyperparameters). Both are plain seeded draws.
     """
     g = _gen(seed, device)
     gates = torch.rand((wl.B, wl.H, wl.N, 2), generator=g, device=device,
@@ -209,7 +209,7 @@ def make_gate_mlp(wl: Workload, hidden: int = 64, seed: int = 7,
                   device="cpu", w_lambda_std: float = 0.05) -> dict:
     """Parameters of the token-wise gate MLP and of the query-dependent
     lambda, per head (Section 3.3; Appendix D "gate hidden dim" 64 or 128;
-    Appendix E for lambda).
+    Appendix D for lambda).
 
     w1 [H, g, d] and w_lambda [H, d] hold bf16-representable fp32 values
     (like the RACE planes); w1 ~ N(0, 1/d), b1 ~ 0.1 N(0, 1),
