@@ -424,9 +424,52 @@ cudaError_t launch_race_partial_weighted(const Plan &P, const void *x,
     return cudaGetLastError();
 }
 
+// k_race_reduce four values per thread (per and r d multiples of 4): the
+// same sums in the same chunk order, 16-byte loads and stores.
+__global__ void k_race_reduce4(const float *__restrict__ part, int S, int r,
+                               int d, float *__restrict__ A,
+                               float *__restrict__ Bm,
+                               uint16_t *__restrict__ Bh) {
+    const int bh = blockIdx.y;
+    const size_t per = (size_t)r * d + r, rd = (size_t)r * d;
+    for (size_t i = 4 * ((size_t)blockIdx.x * blockDim.x + threadIdx.x);
+         i < per; i += 4 * (size_t)gridDim.x * blockDim.x) {
+        const float *p = part + (size_t)bh * S * per + i;
+        float4 s = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int c = 0; c < S; ++c) {
+            const float4 x =
+                *reinterpret_cast<const float4 *>(p + (size_t)c * per);
+            s.x += x.x;
+            s.y += x.y;
+            s.z += x.z;
+            s.w += x.w;
+        }
+        if (i < rd) {
+            *reinterpret_cast<float4 *>(Bm + (size_t)bh * rd + i) = s;
+            if (Bh) {
+                const __nv_bfloat162 lo = __floats2bfloat162_rn(s.x, s.y);
+                const __nv_bfloat162 hi = __floats2bfloat162_rn(s.z, s.w);
+                uint2 w;
+                w.x = *reinterpret_cast<const uint32_t *>(&lo);
+                w.y = *reinterpret_cast<const uint32_t *>(&hi);
+                *reinterpret_cast<uint2 *>(Bh + (size_t)bh * rd + i) = w;
+            }
+        } else {
+            *reinterpret_cast<float4 *>(A + (size_t)bh * r + (i - rd)) = s;
+        }
+    }
+}
+
 cudaError_t launch_race_reduce(const Plan &P, const float *part, float *A,
                                float *Bm, uint16_t *Bh, cudaStream_t st) {
     size_t per = (size_t)P.r * P.d + P.r;
+    if (per % 4 == 0 && ((size_t)P.r * P.d) % 4 == 0 && P.r % 4 == 0) {
+        int gx = (int)((per / 4 + 255) / 256);
+        if (gx > 1024) gx = 1024;
+        k_race_reduce4<<<dim3(gx, P.BH), 256, 0, st>>>(part, P.S, P.r, P.d,
+                                                        A, Bm, Bh);
+        return cudaGetLastError();
+    }
     int gx = (int)((per + 255) / 256);
     if (gx > 1024) gx = 1024;
     dim3 grid(gx, P.BH);
