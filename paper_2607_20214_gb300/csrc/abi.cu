@@ -687,7 +687,16 @@ int forward_impl(const elsaa_params *params, const void *q, const void *k,
     // neighbouring key blocks (nb > 0) run in the persistent kernel for
     // b of 128 or 256 and nb = 1, otherwise in the CUDA-core block kernel;
     // the RACE key side above does not depend on them
-    if (P.impl == 2 && ws_supported(P)) {
+    if (P.impl == 2 && pair_supported(P)) {
+        // key blocks of 256: the two query tiles of a block on a CTA pair
+        ELSAA_CHECK_LAUNCH(timed("block_attn_pair", st, [&] {
+                               return launch_block_attn_pair(
+                                   P, q, k, v, Wbf, pq, pk, A, Bh,
+                                   lambda_tok, gates, o, log_d_sparse, d_lr,
+                                   m_sparse, status, st);
+                           }),
+                           "block_attn_pair");
+    } else if (P.impl == 2 && ws_supported(P)) {
         ELSAA_CHECK_LAUNCH(timed("block_attn_ws", st, [&] {
                                return launch_block_attn_ws(
                                    P, q, k, v, Wbf, pq, pk, A, Bh,

@@ -234,4 +234,15 @@ cudaError_t launch_block_attn_ws(
     float *m_sparse, DeviceStatus *status, cudaStream_t st,
     const int32_t *cand = nullptr, const uint32_t *selmask = nullptr);
 
+// Block attention for key blocks of 256 on CTA pairs (cta_group::2 MMAs):
+// bf16, d_h = 128, gamma = 4, no neighbours or selector, N a multiple of 256.
+bool pair_supported(const Plan &P);
+size_t pair_smem(const Plan &P);
+cudaError_t launch_block_attn_pair(
+    const Plan &P, const void *q, const void *k, const void *v,
+    const uint16_t *w_bf16, const int32_t *perm_q, const int32_t *perm_k,
+    const float *A, const uint16_t *Bh, const float *lambda_tok,
+    const float *gates, void *o, float *log_d_sparse, float *d_lr,
+    float *m_sparse, DeviceStatus *status, cudaStream_t st);
+
 }  // namespace elsaa

@@ -485,5 +485,90 @@ __device__ __forceinline__ float tanh_approx(float x) {
     return y;
 }
 
+// ------------------------------------------------- CTA pairs (clusters of 2)
+//
+// A cta_group::2 MMA is issued by one thread of the even CTA of the pair and
+// reads both CTAs' shared memory (and tensor memory) at the same addresses:
+// A rows [0, M/2) from the even CTA, [M/2, M) from the odd one; B columns
+// [0, N/2) from the even CTA, [N/2, N) from the odd one. With M = 256 each
+// CTA's tensor memory receives its 128 rows (lane = row) and all N columns.
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Every thread of both CTAs; orders shared-memory writes and barrier
+// initialisation before the peer's accesses.
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile(
+        "barrier.cluster.arrive.release.aligned;\n"
+        "barrier.cluster.wait.acquire.aligned;" ::
+            : "memory");
+}
+
+// One warp of each CTA of the pair, collectively: the same columns in both.
+__device__ __forceinline__ void tmem_alloc_pair(uint32_t *dst,
+                                                uint32_t ncols) {
+    asm volatile(
+        "tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::
+            "r"(smem_u32(dst)),
+        "r"(ncols)
+        : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;");
+}
+
+__device__ __forceinline__ void tmem_dealloc_pair(uint32_t taddr,
+                                                  uint32_t ncols) {
+    asm volatile(
+        "tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(taddr),
+        "r"(ncols)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_pair_ss(uint32_t d_tmem, uint64_t a_desc,
+                                            uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(
+            d_tmem),
+        "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_pair_ts(uint32_t d_tmem, uint32_t a_tmem,
+                                            uint64_t b_desc, uint32_t idesc,
+                                            uint32_t accumulate) {
+    asm volatile(
+        "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+        " tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(
+            d_tmem),
+        "r"(a_tmem), "l"(b_desc), "r"(idesc), "r"(accumulate));
+}
+
+// Arrives once on `bar` in both CTAs of the pair when every MMA issued so
+// far by this thread is complete.
+__device__ __forceinline__ void mma_commit_pair(uint64_t *bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster."
+        "multicast::cluster.b64 [%0], %1;" ::"r"(smem_u32(bar)),
+        "h"((uint16_t)3)
+        : "memory");
+}
+
+// Arrival on the barrier at the same shared-memory offset in CTA `rank`.
+__device__ __forceinline__ void mbar_arrive_remote(uint64_t *bar,
+                                                   uint32_t rank) {
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;"
+                 : "=r"(remote)
+                 : "r"(smem_u32(bar)), "r"(rank));
+    asm volatile(
+        "mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(
+            remote)
+        : "memory");
+}
+
 }  // namespace tc
 }  // namespace elsaa

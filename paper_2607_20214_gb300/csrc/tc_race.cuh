@@ -68,13 +68,10 @@ __device__ __forceinline__ void race_bits32(uint32_t taddr, int ncols,
     }
 }
 
-// race_bits32 over 16 projection columns: sp[j] for j < 16, entries past
-// `ncols` set to 1/2. The TMEM load is waited for inside.
-__device__ __forceinline__ void race_bits16(uint32_t taddr, int ncols,
-                                           float beta, float *sp) {
-    uint32_t pr[16];
-    tmem_ld16(taddr, pr);
-    tmem_wait_ld();
+// The per-bit factors of 16 projections already loaded from TMEM (fp32
+// bits in pr): sp[j] for j < 16, entries past `ncols` set to 1/2.
+__device__ __forceinline__ void race_factors16(const uint32_t *pr, int ncols,
+                                               float beta, float *sp) {
 #pragma unroll
     for (int j = 0; j < 16; ++j) {
         if (j < ncols) {
@@ -84,6 +81,16 @@ __device__ __forceinline__ void race_bits16(uint32_t taddr, int ncols,
             sp[j] = 0.5f;
         }
     }
+}
+
+// race_bits32 over 16 projection columns: sp[j] for j < 16, entries past
+// `ncols` set to 1/2. The TMEM load is waited for inside.
+__device__ __forceinline__ void race_bits16(uint32_t taddr, int ncols,
+                                           float beta, float *sp) {
+    uint32_t pr[16];
+    tmem_ld16(taddr, pr);
+    tmem_wait_ld();
+    race_factors16(pr, ncols, beta, sp);
 }
 
 // Features of table l from its G per-bit factors: phi[r] = prod_b (bit b of
@@ -301,6 +308,14 @@ __device__ __forceinline__ void write_phi_chunk(const float *sp, int nt,
                 tmem_st16(taddr + (uint32_t)(k - 15), buf);
         }
     }
+}
+
+// TMEM column of K-step k (16 keys or buckets = 8 packed bf16 columns) of
+// the quarter pair starting at col0: quarters (col0, col0 + 64) of 32
+// columns each, the A operand of the P V and Phi'B products in the block
+// kernels' slots.
+__device__ __forceinline__ uint32_t quarter_col(int k, int col0) {
+    return (uint32_t)(col0 + (k < 4 ? 8 * k : 64 + 8 * (k - 4)));
 }
 
 }  // namespace tc

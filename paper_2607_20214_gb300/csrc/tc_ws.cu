@@ -46,10 +46,6 @@ constexpr int kWsNK = 128;        // keys per query tile
 // the scores already read; the pre-scaled RACE features of buckets
 // [0, 128) go to quarters 1 and 3, buckets [128, 256) to quarters 0 and 2
 // once the P V product is done.
-__device__ __forceinline__ uint32_t quarter_col(int k, int col0) {
-    // K-step k (16 keys or buckets = 8 columns) of a quarter pair
-    return (uint32_t)(col0 + (k < 4 ? 8 * k : 64 + 8 * (k - 4)));
-}
 
 struct WsBars {
     uint64_t qk_full, wb_full, head_done;
