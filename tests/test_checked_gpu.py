@@ -40,11 +40,12 @@ def _forward(lib_swap, wl, x, **over):
     return o.cpu()
 
 
-@pytest.mark.parametrize("causal", [0, 1])
-def test_checked_build_computes_the_same(checked, causal):
+@pytest.mark.parametrize("causal,block", [(0, 128), (1, 128), (0, 256)])
+def test_checked_build_computes_the_same(checked, causal, block):
+    """block 256: the CTA-pair kernel."""
     wl = Workload(name="chk", B=1, H=2, N=1024, d_h=128, dtype="bf16",
-                  block=128, race_tables=16, recipe="plain", temperature=2.0,
-                  seed=51, plane_seed=1051, causal=causal,
+                  block=block, race_tables=16, recipe="plain",
+                  temperature=2.0, seed=51, plane_seed=1051, causal=causal,
                   causal_base_len=256)
     x = make_inputs(wl)
     got = _forward(checked, wl, x)
