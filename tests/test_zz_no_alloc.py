@@ -33,9 +33,9 @@ def _lib():
     elsaa.load_library()
 
 
-def _case(dtype, N=1184, block=32, seed=21):
-    return Workload("noalloc", B=2, H=2, N=N, d_h=64, dtype=dtype,
-                    block=block, race_tables=4, recipe="plain",
+def _case(dtype, N=1184, block=32, seed=21, d_h=64, race_tables=4):
+    return Workload("noalloc", B=2, H=2, N=N, d_h=d_h, dtype=dtype,
+                    block=block, race_tables=race_tables, recipe="plain",
                     temperature=2.0, seed=seed, plane_seed=1000 + seed)
 
 
@@ -80,6 +80,16 @@ def test_noalloc_larger_then_smaller_problem(dtype):
     dev = torch.device("cuda:0")
     _compare(_case(dtype, N=4096, block=64, seed=23), dev)
     _compare(_case(dtype, N=1184, block=32, seed=24), dev)
+
+
+def test_noalloc_tensor_core_kernels():
+    """bf16 shapes that take the one-CTA tensor-core block kernel (b = 128)
+    and the CTA-pair kernel (b = 256, d_h = 128) through the static array."""
+    dev = torch.device("cuda:0")
+    _compare(_case("bf16", N=2048, block=128, seed=25, d_h=128,
+                   race_tables=16), dev)
+    _compare(_case("bf16", N=2048, block=256, seed=26, d_h=128,
+                   race_tables=16), dev)
 
 
 def test_noalloc_status_word_reports_timeout_then_clears():
