@@ -418,6 +418,16 @@ __device__ __forceinline__ void load_rows(uint32_t dst, const uint16_t *src,
     }
 }
 
+// One 32-byte global store (a whole sector) of 8 words; `p` 32-byte
+// aligned.
+__device__ __forceinline__ void st_global_v8(void *p, const uint32_t (&w)[8]) {
+    asm volatile(
+        "st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p),
+        "r"(w[0]), "r"(w[1]), "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]),
+        "r"(w[6]), "r"(w[7])
+        : "memory");
+}
+
 // Stores 8 fp32 values as 8 bf16 (one 16-byte chunk) at a shared address.
 __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
     uint4 v;

@@ -63,7 +63,7 @@ struct PrBars {
     uint64_t s_full[2], pv0_done[2], pv_done[2], o_full[2], v_empty[kPrNP];
     uint64_t head_done;
     // local
-    uint64_t idx_full[2], idx_empty[2], o_free;
+    uint64_t idx_full[2], idx_empty[2];
 };
 constexpr int kPrRelayed = 2 + kPrNP + kPrNP + 1;  // copy barriers
 
@@ -96,7 +96,6 @@ __global__ void __launch_bounds__(kPrThreads, 1)
     __shared__ __align__(16) int qrow[2][128];
     __shared__ __align__(16) int krow[2][NP][64];
     __shared__ __align__(16) int vrow[128];  // value loader: the pass's keys
-    __shared__ int orow[128];                // epilogue: output row or -1
     volatile int *abort = &abort_flag;
     const int tid = threadIdx.x, warp = tid >> 5, lane_id = tid & 31;
     const uint32_t crank = cluster_rank();  // 0: issues the MMAs
@@ -122,7 +121,7 @@ __global__ void __launch_bounds__(kPrThreads, 1)
     // shared memory: two query tiles, the pass-0 key buffer (64 keys and
     // this CTA's 32 plane rows), the pass-1 key buffer, one value buffer per
     // pass (128 keys x this CTA's 64 columns), this CTA's 64 columns of the
-    // B summary, the A summary, the output staging tile
+    // B summary, the A summary
     const uint32_t tileQ = (uint32_t)nk * d * 2u;
     const uint32_t base = align1k(smem_u32(smem_raw));
     const uint32_t sQ = base;
@@ -131,7 +130,6 @@ __global__ void __launch_bounds__(kPrThreads, 1)
     const uint32_t sV = sK1 + kPrKRows1 * d * 2;
     const uint32_t sB = sV + NP * 16384u;
     const uint32_t sA = sB + align1k((uint32_t)r * 128u);
-    const uint32_t sO = sA + align1k((uint32_t)r * 4u);
     const float *Asm = reinterpret_cast<const float *>(
         smem_raw + (sA - smem_u32(smem_raw)));
     auto kbuf = [=](int p) { return p == 0 ? sK0 : sK1; };
@@ -159,7 +157,6 @@ __global__ void __launch_bounds__(kPrThreads, 1)
         }
         mbar_init(&bars.wb_full, 1 + x);
         mbar_init(&bars.head_done, 1);
-        mbar_init(&bars.o_free, 256);
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -753,12 +750,10 @@ __global__ void __launch_bounds__(kPrThreads, 1)
             }
             if (!wwait(&bars.o_full[g], k & 1, 81)) break;
             tc_fence_after();
-            // O = c1 acc, this half's 64 columns: fp32 straight from the
-            // registers, bf16 staged in sO (shared by the slots, taken in
-            // block order) and copied out in whole rows
-            if constexpr (!O32) {
-                if (j >= 1 && !wwait(&bars.o_free, (j - 1) & 1, 82)) break;
-            }
+            // O = c1 acc, this half's 64 columns, straight from the
+            // registers: fp32, or bf16 in 32-byte stores (a whole sector
+            // each) when O is 32-byte aligned
+            const bool o_a32 = ((uintptr_t)ox & 31u) == 0;
 #pragma unroll
             for (int c = 0; c < 64; c += 16) {
                 uint32_t v[16];
@@ -779,29 +774,22 @@ __global__ void __launch_bounds__(kPrThreads, 1)
                     for (int q = 0; q < 8; ++q)
                         ob[q] = pack_bf16x2(c1e * __uint_as_float(v[2 * q]),
                                             c1e * __uint_as_float(v[2 * q + 1]));
-                    const int cidx = (half * 64 + c) >> 3;  // 16-byte chunk
-                    st_shared_v4(sO + panel_offset(row, cidx, nk), ob[0],
-                                 ob[1], ob[2], ob[3]);
-                    st_shared_v4(sO + panel_offset(row, cidx + 1, nk), ob[4],
-                                 ob[5], ob[6], ob[7]);
+                    uint16_t *dst = ox + tok * (size_t)d + half * 64 + c;
+                    if (o_a32) {
+                        st_global_v8(dst, ob);
+                    } else {
+                        uint4 *d4 = reinterpret_cast<uint4 *>(dst);
+                        d4[0] = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+                        d4[1] = make_uint4(ob[4], ob[5], ob[6], ob[7]);
+                    }
                 }
             }
             tc_fence_before();
             signal(&bars.tmem_empty[g]);
             if (half == 0) {
-                if constexpr (!O32) orow[row] = (int)tok;
                 if (log_ds_out) log_ds_out[tok] = log_ds;
                 if (dlr_out) dlr_out[tok] = denf;
                 if (m_out) m_out[tok] = msp;
-            }
-            if constexpr (!O32) {
-                named_sync(1 + g, 256);
-                for (int rr = crow; rr < nk; rr += 16) {
-                    const uint4 val = ld_shared_v4(sO + panel_offset(rr, cc, nk));
-                    *reinterpret_cast<uint4 *>(ox + (size_t)orow[rr] * d +
-                                               cc * 8) = val;
-                }
-                mbar_arrive(&bars.o_free);  // this thread's reads are done
             }
         }
         cp_async_wait<0>();
@@ -825,8 +813,7 @@ size_t pair_smem(const Plan &P) {
     const size_t r = (size_t)P.r;
     return 1024 + 2 * (size_t)kPrNK * kPrD * 2 +
            (size_t)(kPrKRows0 + kPrKRows1) * kPrD * 2 + kPrNP * 16384 +
-           (r * 128 + 1023) / 1024 * 1024 + (r * 4 + 1023) / 1024 * 1024 +
-           (size_t)kPrNK * kPrD * 2;
+           (r * 128 + 1023) / 1024 * 1024 + (r * 4 + 1023) / 1024 * 1024;
 }
 
 cudaError_t launch_block_attn_pair(
