@@ -86,3 +86,15 @@ def test_pair_rows_of_a_large_head():
     g = run_gpu(wl, x)
     compare(wl, g, run_oracle(wl, x, heads=[(0, 1), (0, 3)], rows=rows),
             label="pair N=16384")
+
+
+@pytest.mark.parametrize("over", [dict(fusion_mode=1), dict(beta=4.0),
+                                  dict(lam=0.25), dict(eps=1e-2),
+                                  dict(sort_bits=0)])
+def test_pair_parameter_variants(over):
+    """Fusion mode, RACE temperature, lambda, epsilon and the identity
+    order (no sort bits: every block is a run of consecutive tokens)."""
+    wl = pair_wl(H=4, N=2048, seed=74).with_(**over)
+    x = make_inputs(wl)
+    compare(wl, run_gpu(wl, x), run_oracle(wl, x, heads=[(0, 0), (0, 3)]),
+            label=str(over))
