@@ -168,6 +168,30 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         unpack_bf16x8(ld_shared_v4(region + panel_offset(rr, chunk, rows)),
                       v);
     };
+    // fp32 gradient rows leave through shared memory: each thread stages
+    // its 32 TMEM columns into its row (256 bytes, the 16-byte chunks
+    // XOR-permuted by row & 7 so that eight consecutive rows hit eight
+    // bank groups), then every warp writes whole rows, two per
+    // instruction, to their original positions.
+    static_assert(kBtD == 64, "staged rows are 256 bytes");
+    auto stage_f32 = [&](uint32_t region, const uint32_t *v) {
+        const uint32_t rb = region + (uint32_t)row * 256;
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            st_shared_v4(rb + ((uint32_t)((8 * half + q) ^ (row & 7)) << 4),
+                         v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+    };
+    auto flush_f32 = [&](uint32_t region, float *dst, const int *rows) {
+        const int c = lane_id & 15;
+#pragma unroll
+        for (int it = 0; it < kBtT / (2 * kBtThreads / 32); ++it) {
+            const int i = (2 * kBtThreads / 32) * it + 2 * warp + (lane_id >> 4);
+            const uint4 w =
+                ld_shared_v4(region + (uint32_t)i * 256 +
+                             ((uint32_t)(c ^ (i & 7)) << 4));
+            *reinterpret_cast<uint4 *>(dst + (size_t)rows[i] * d + 4 * c) = w;
+        }
+    };
 
     // Rows of tile tt (sorted positions -> original rows) into the index
     // arrays of parity tt & 1. The next tile's copies start as soon as
@@ -551,18 +575,11 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             for (int q = 0; q < TL * G / 8; ++q)
                 st8(sDU, row, (half * TL * G) / 8 + q, kBtT, du + 8 * q);
         }
-        {
+        {  // dV staged in sX, sGN (their last readers, phase 5, are done)
             uint32_t v[32];
             tmem_ld32(tm + lane + kCdV + 32 * half, v);
             tmem_wait_ld();
-            float4 *o4 =
-                reinterpret_cast<float4 *>(dv + (size_t)krow_s[row] * d + 32 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                o4[q] = make_float4(__uint_as_float(v[4 * q]),
-                                    __uint_as_float(v[4 * q + 1]),
-                                    __uint_as_float(v[4 * q + 2]),
-                                    __uint_as_float(v[4 * q + 3]));
+            stage_f32(sX, v);
         }
         fence_proxy_async_smem();
         tc_fence_before();
@@ -591,33 +608,25 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 mma_ss(tm + kCN, smem_desc(sE + k * 2048, 16384, 1024),
                        smem_desc(sQ + k * 2048, 16384, 1024), id_k, k > 0);
         }
+        flush_f32(sX, dv, krow_s);  // beside the MMAs, which do not read sX
         if (!(ok = mma_done(83))) break;
         if (more) load_qk(tt + 1);  // Q and K's last readers are done
         cp_async_commit();
 
         // ------------------------------------------- phase 8: dQ, dK stores
-        {
+        {  // dQ staged in sE, dK in sX, sGN (phase 7's MMAs are done)
             uint32_t v[32];
             tmem_ld32(tm + lane + kCO + 32 * half, v);
             tmem_wait_ld();
-            float4 *q4 = reinterpret_cast<float4 *>(dq + (size_t)qrow * d + 32 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                q4[q] = make_float4(__uint_as_float(v[4 * q]),
-                                    __uint_as_float(v[4 * q + 1]),
-                                    __uint_as_float(v[4 * q + 2]),
-                                    __uint_as_float(v[4 * q + 3]));
+            stage_f32(sE, v);
             tmem_ld32(tm + lane + kCN + 32 * half, v);
             tmem_wait_ld();
-            float4 *k4 = reinterpret_cast<float4 *>(dk + (size_t)krow_s[row] * d + 32 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                k4[q] = make_float4(__uint_as_float(v[4 * q]),
-                                    __uint_as_float(v[4 * q + 1]),
-                                    __uint_as_float(v[4 * q + 2]),
-                                    __uint_as_float(v[4 * q + 3]));
+            stage_f32(sX, v);
         }
         tc_fence_before();
+        __syncthreads();
+        flush_f32(sE, dq, qrow_s);
+        flush_f32(sX, dk, krow_s);
         __syncthreads();  // TMEM and shared memory are reused by the next tile
     }
     cp_async_wait<0>();
