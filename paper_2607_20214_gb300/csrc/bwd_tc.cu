@@ -110,7 +110,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     constexpr int TL = L / 2;          // tables per row half
     constexpr int d = kBtD;
     extern __shared__ unsigned char smem_raw[];
-    __shared__ uint64_t mma_bar;
+    __shared__ uint64_t mma_bar, sums_bar;
     __shared__ uint32_t tbase;
     __shared__ int abort_flag;
     __shared__ float xa[2][kBtT], xb[2][kBtT], xc[2][kBtT];
@@ -122,17 +122,19 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     const uint32_t lane = (uint32_t)((warp & 3) * 32) << 16;
 
     const uint32_t base = align1k(smem_u32(smem_raw));
-    const uint32_t sQ = base;                       // [128 x 64]
-    const uint32_t sG = sQ + 16384;                 // dO rows
-    const uint32_t sKW = sG + 16384;                // [NR x 64]: K, then W
-    const uint32_t sV = sKW + align1k(NR * 128);    // [128 x 64]
+    // Q [128 x 64] and [K ; W] [NR x 64] of two tiles, by tile parity: the
+    // next tile's rows land while this one computes
+    const uint32_t kQKW = 16384 + align1k(NR * 128);
+    // [128 x r]; the bucket-sum MMA reads 128 bucket columns, so with
+    // r = 64 its unused upper half reads the 16 KB after sPhi (sG)
+    const uint32_t sPhi = base + 2 * kQKW;
+    const uint32_t sG = sPhi + align1k(kBtT * r * 2);  // dO, then X = c_x dO
+    const uint32_t sGN = sG + 16384;                // [128 x 64]
+    const uint32_t sDU = sGN + 16384;  // dL/dDen (columns 0-15), dL/du (32-63)
+    const uint32_t sV = sDU + 16384;                // [128 x 64]
     const uint32_t sE = sV + 16384;                 // [128 x 128]: E, dZ
-    const uint32_t sPhi = sE + 32768;               // [128 x r]
-    const uint32_t sB = sPhi + align1k(kBtT * r * 2);  // [r x 64]
-    const uint32_t sX = sB + align1k(r * 128);      // [128 x 64]
-    const uint32_t sGN = sX + 16384;                // [128 x 64]
-    const uint32_t sDU = sGN + 16384;               // [128 x 64] (Lg_pad used)
-    const uint32_t sAo = sDU + 16384;               // fp32 [r]
+    const uint32_t sB = sE + 32768;                 // [r x 64]
+    const uint32_t sAo = sB + align1k(r * 128);     // fp32 [r]
     const float *Asm =
         reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
 
@@ -142,6 +144,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     if (warp == 0) tmem_alloc(&tbase, 512);
     if (tid == 0) {
         mbar_init(&mma_bar, 1);
+        mbar_init(&sums_bar, 1);
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -149,15 +152,18 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tm = tbase;
-    uint32_t mph = 0;  // MMA barrier phases completed
+    uint32_t mph = 0, sph = 0;  // barrier phases completed
+    // everyone waits for a commit of thread 0
+    auto mma_wait = [&](uint64_t *bar, uint32_t &ph, int site) -> bool {
+        const bool ok = mbar_wait_or_abort(bar, ph & 1, abort, status, site);
+        ++ph;
+        tc_fence_after();
+        return __syncthreads_and(ok);
+    };
     // thread 0 issues, everyone waits for the commit
     auto mma_done = [&](int site) -> bool {
         if (tid == 0) mma_commit(&mma_bar);
-        const bool ok = mbar_wait_or_abort(&mma_bar, mph & 1, abort, status,
-                                           site);
-        ++mph;
-        tc_fence_after();
-        return __syncthreads_and(ok);
+        return mma_wait(&mma_bar, mph, site);
     };
     // 16-byte chunk (8 bf16) at (row, chunk) of a panel region of `rows`
     auto st8 = [&](uint32_t region, int rr, int chunk, int rows,
@@ -194,15 +200,27 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     };
 
     // Rows of tile tt (sorted positions -> original rows) into the index
-    // arrays of parity tt & 1. The next tile's copies start as soon as
-    // their buffers are free: dO after phase 4, V after phase 5, Q and K
-    // after phase 7; the top of each tile waits for every copy.
+    // arrays of parity tt & 1, from permutation entries fetched into
+    // registers a tile earlier. The next tile's copies start as soon as
+    // their buffers are free: Q and K (other parity) in phase 1, V after
+    // phase 5, the head's B and A and then dO in phase 7. The top of a tile
+    // waits for all but the newest copy group (dO), phase 4 for dO.
+    int qi_next = 0, ki_next = 0;
+    auto fetch_rows = [&](long tt) {
+        if (tid < kBtT) {
+            const int bh = (int)(tt / tiles_per_head);
+            const size_t p = (size_t)bh * N +
+                             (size_t)(tt - (long)bh * tiles_per_head) * kBtT +
+                             tid;
+            qi_next = perm_q[p];
+            ki_next = perm_k[p];
+        }
+    };
     auto stage_rows = [&](long tt) {
         if (tid < kBtT) {
             const int bh = (int)(tt / tiles_per_head);
             const size_t hb = (size_t)bh * N;
-            const int p0 = (int)(tt - (long)bh * tiles_per_head) * kBtT;
-            int qi = perm_q[hb + p0 + tid], ki = perm_k[hb + p0 + tid];
+            int qi = qi_next, ki = ki_next;
             // entries outside [0, N) are recorded and read as row 0
             if (qi < 0 || qi >= N) {
                 report(status, kDevPermRange, 10, bh, qi);
@@ -216,15 +234,39 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             krow2[tt & 1][tid] = (int)(hb + ki);
         }
     };
+    // Q, K of tile tt into the buffers of parity tt & 1, and the head's
+    // planes below K when that buffer holds another head's
+    int planes_h0 = -1, planes_h1 = -1;  // head of each buffer's planes
     auto load_qk = [&](long tt) {
         const int *qr = qrow2[tt & 1], *kr = krow2[tt & 1];
+        const uint32_t q_s = base + (uint32_t)(tt & 1) * kQKW;
+        const uint32_t k_s = q_s + 16384;
         for (int i = tid; i < kBtT * 8; i += kBtThreads) {
             const int rr = i >> 3, c = i & 7;
-            cp_async16(sQ + panel_offset(rr, c, kBtT),
+            cp_async16(q_s + panel_offset(rr, c, kBtT),
                        qx + (size_t)qr[rr] * d + c * 8);
-            cp_async16(sKW + panel_offset(rr, c, NR),
+            cp_async16(k_s + panel_offset(rr, c, NR),
                        kx + (size_t)kr[rr] * d + c * 8);
         }
+        const int hh = (int)(tt / tiles_per_head) % H;
+        int &ph = (tt & 1) ? planes_h1 : planes_h0;
+        if (ph != hh) {
+            for (int i = tid; i < Lg_pad * 8; i += kBtThreads) {
+                const int rr = i >> 3, c = i & 7;
+                cp_async16(k_s + panel_offset(kBtT + rr, c, NR),
+                           w_bf16 + ((size_t)hh * Lg_pad + rr) * d + c * 8);
+            }
+            ph = hh;
+        }
+    };
+    auto load_sums = [&](int bh) {  // the head's B summary (bf16) and A
+        for (int i = tid; i < r * 8; i += kBtThreads) {
+            const int rr = i >> 3, c = i & 7;
+            cp_async16(sB + panel_offset(rr, c, r),
+                       Bh + ((size_t)bh * r + rr) * d + c * 8);
+        }
+        for (int i = tid; i < r / 4; i += kBtThreads)
+            cp_async16(sAo + 16 * i, Ag + (size_t)bh * r + 4 * i);
     };
     auto load_g = [&](long tt) {
         const int *qr = qrow2[tt & 1];
@@ -243,40 +285,29 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         }
     };
     if (t_begin < t_end) {
+        fetch_rows(t_begin);
         stage_rows(t_begin);
+        if (t_begin + 1 < t_end) fetch_rows(t_begin + 1);
         __syncthreads();
         load_qk(t_begin);
-        load_g(t_begin);
         load_v(t_begin);
+        load_sums((int)(t_begin / tiles_per_head));
         cp_async_commit();
+        load_g(t_begin);
     }
+    cp_async_commit();
 
-    int cur_bh = -1;
     bool ok = true;
     for (long tt = t_begin; tt < t_end && ok; ++tt) {
         const int bh = (int)(tt / tiles_per_head);
-        const int h = bh % H;
+        const uint32_t sQ = base + (uint32_t)(tt & 1) * kQKW;
+        const uint32_t sKW = sQ + 16384;  // [NR x 64]: K, then W
         const int *qrow_s = qrow2[tt & 1], *krow_s = krow2[tt & 1];
         const bool more = tt + 1 < t_end;
         // ---------------------------------------------------- phase 0: load
-        if (bh != cur_bh) {  // the head's planes, B summary (bf16) and A
-            for (int i = tid; i < Lg_pad * 8; i += kBtThreads) {
-                const int rr = i >> 3, c = i & 7;
-                cp_async16(sKW + panel_offset(kBtT + rr, c, NR),
-                           w_bf16 + ((size_t)h * Lg_pad + rr) * d + c * 8);
-            }
-            for (int i = tid; i < r * 8; i += kBtThreads) {
-                const int rr = i >> 3, c = i & 7;
-                cp_async16(sB + panel_offset(rr, c, r),
-                           Bh + ((size_t)bh * r + rr) * d + c * 8);
-            }
-            for (int i = tid; i < r / 4; i += kBtThreads)
-                cp_async16(sAo + 16 * i, Ag + (size_t)bh * r + 4 * i);
-            cur_bh = bh;
-        }
-        cp_async_commit();
-        cp_async_wait<0>();
+        cp_async_wait<1>();  // all but this tile's dO
         if (more) stage_rows(tt + 1);  // the next tile's rows, parity flips
+        if (tt + 2 < t_end) fetch_rows(tt + 2);
         fence_proxy_async_smem();
         __syncthreads();
 
@@ -288,8 +319,11 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             for (int k = 0; k < d / 16; ++k)
                 mma_ss(tm + kCS, smem_desc(sQ + k * 32, 16, 1024),
                        smem_desc(sKW + k * 32, 16, 1024), id, k > 0);
+            mma_commit(&mma_bar);
         }
-        if (!(ok = mma_done(80))) break;
+        if (more) load_qk(tt + 1);  // the other parity's readers are done
+        cp_async_commit();
+        if (!(ok = mma_wait(&mma_bar, mph, 80))) break;
 
         // ---------------------- phase 2: E on the query's own block, phi, Den
         const int blk = row >> 6;
@@ -383,6 +417,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        smem_desc(sB + k * 2048, (uint32_t)r * 128, 1024), id,
                        k > 0);
         }
+        cp_async_wait<1>();  // this tile's dO (the barrier below shares it)
         if (!(ok = mma_done(81))) break;
 
         // ------------------------------------- phase 4: per-query scalars
@@ -452,16 +487,14 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 nv[j] = cn * gv[j];
             }
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                st8(sX, row, 4 * half + q, kBtT, xv + 8 * q);
+            for (int q = 0; q < 4; ++q) {  // X over the dO this thread read
+                st8(sG, row, 4 * half + q, kBtT, xv + 8 * q);
                 st8(sGN, row, 4 * half + q, kBtT, nv + 8 * q);
             }
         }
         fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
-        if (more) load_g(tt + 1);  // dO of this tile was read in phase 4
-        cp_async_commit();
 
         // ------------- phase 5: E^T X, X V^T, gNum B^T, phi^T [gNum | gDen]
         const bool seg_first = tt == t_begin || (tt % tiles_per_head) == 0;
@@ -469,21 +502,24 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             tt + 1 == t_end || ((tt + 1) % tiles_per_head) == 0;
         if (tid == 0) {
             tc_fence_after();
-            const uint32_t id_v = idesc_bf16(128, d, true, true);
-#pragma unroll
-            for (int k = 0; k < kBtT / 16; ++k)  // dV = E^T X (K = queries)
-                mma_ss(tm + kCdV, smem_desc(sE + k * 2048, 16384, 1024),
-                       smem_desc(sX + k * 2048, 16384, 1024), id_v, k > 0);
             const uint32_t id_p = idesc_bf16(128, kBtT, false, false);
 #pragma unroll
             for (int k = 0; k < d / 16; ++k)  // P = X V^T (K = d)
-                mma_ss(tm + kCS, smem_desc(sX + k * 32, 16, 1024),
+                mma_ss(tm + kCS, smem_desc(sG + k * 32, 16, 1024),
                        smem_desc(sV + k * 32, 16, 1024), id_p, k > 0);
             const uint32_t id_g = idesc_bf16(128, r, false, false);
 #pragma unroll
             for (int k = 0; k < d / 16; ++k)  // Gphi = gNum B^T (K = d)
                 mma_ss(tm + kCG, smem_desc(sGN + k * 32, 16, 1024),
                        smem_desc(sB + k * 32, 16, 1024), id_g, k > 0);
+            mma_commit(&mma_bar);
+            // dV and the bucket sums run beside phase 6, which writes
+            // none of their operands before it waits for them
+            const uint32_t id_v = idesc_bf16(128, d, true, true);
+#pragma unroll
+            for (int k = 0; k < kBtT / 16; ++k)  // dV = E^T X (K = queries)
+                mma_ss(tm + kCdV, smem_desc(sE + k * 2048, 16384, 1024),
+                       smem_desc(sG + k * 2048, 16384, 1024), id_v, k > 0);
             // bucket sums (K = queries; M = 128 buckets, rows past r unused;
             // the B operand is gNum followed by the dL/dDen panel)
             const uint32_t id_s = idesc_bf16(128, d + 16, true, true);
@@ -492,47 +528,21 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 mma_ss(tm + kCAcc, smem_desc(sPhi + k * 2048, 16384, 1024),
                        smem_desc(sGN + k * 2048, 16384, 1024), id_s,
                        (k > 0 || !seg_first) ? 1u : 0u);
+            mma_commit(&sums_bar);
         }
-        if (!(ok = mma_done(82))) break;
+        if (!(ok = mma_wait(&mma_bar, mph, 82))) break;
         if (more) load_v(tt + 1);  // V's last reader (P = X V^T) is done
         cp_async_commit();
-        if (seg_last && row < r) {  // this CTA's share of the head's sums
-            const long j = (long)blockIdx.x -
-                           tile_owner((long)bh * tiles_per_head, total_tiles,
-                                      gridDim.x);
-            float *out =
-                part + ((size_t)bh * S_seg + j) * ((size_t)r * d + r);
-            uint32_t v[32];
-            tmem_ld32(tm + lane + kCAcc + 32 * half, v);
-            tmem_wait_ld();
-            float4 *o4 =
-                reinterpret_cast<float4 *>(out + (size_t)row * d + 32 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                o4[q] = make_float4(__uint_as_float(v[4 * q]),
-                                    __uint_as_float(v[4 * q + 1]),
-                                    __uint_as_float(v[4 * q + 2]),
-                                    __uint_as_float(v[4 * q + 3]));
-            if (half == 0) {
-                uint32_t a16[16];
-                tmem_ld16(tm + lane + kCAcc + d, a16);
-                tmem_wait_ld();
-                out[(size_t)r * d + row] = __uint_as_float(a16[0]);
-            }
-        }
 
         // ------------- phase 6: dZ, back through the features, dV stores
+        float dz[32];  // into sE once dV = E^T X is done
         {
             uint32_t v[32];
             tmem_ld32(tm + lane + kCS + c0, v);
             tmem_wait_ld();
-            float dz[32];
 #pragma unroll
             for (int j = 0; j < 32; ++j)
                 dz[j] = scale * e[j] * (__uint_as_float(v[j]) + gdsE);
-#pragma unroll
-            for (int q = 0; q < 4; ++q)
-                st8(sE, row, (c0 >> 3) + q, kBtT, dz + 8 * q);
         }
         {
             float du[2 * L > 16 ? 16 : 2 * L];
@@ -573,13 +583,43 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             }
 #pragma unroll
             for (int q = 0; q < TL * G / 8; ++q)
-                st8(sDU, row, (half * TL * G) / 8 + q, kBtT, du + 8 * q);
+                st8(sDU, row, 4 + (half * TL * G) / 8 + q, kBtT, du + 8 * q);
         }
-        {  // dV staged in sX, sGN (their last readers, phase 5, are done)
+        // dV and the bucket sums read sE, sG, sPhi, sGN and the dL/dDen
+        // columns of sDU
+        if (!(ok = mma_wait(&sums_bar, sph, 86))) break;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) st8(sE, row, (c0 >> 3) + q, kBtT, dz + 8 * q);
+        if (seg_last && row < r) {  // this CTA's share of the head's sums
+            const long j = (long)blockIdx.x -
+                           tile_owner((long)bh * tiles_per_head, total_tiles,
+                                      gridDim.x);
+            float *out =
+                part + ((size_t)bh * S_seg + j) * ((size_t)r * d + r);
+            uint32_t v[32];
+            tmem_ld32(tm + lane + kCAcc + 32 * half, v);
+            tmem_wait_ld();
+            float4 *o4 =
+                reinterpret_cast<float4 *>(out + (size_t)row * d + 32 * half);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                o4[q] = make_float4(__uint_as_float(v[4 * q]),
+                                    __uint_as_float(v[4 * q + 1]),
+                                    __uint_as_float(v[4 * q + 2]),
+                                    __uint_as_float(v[4 * q + 3]));
+            if (half == 0) {
+                uint32_t a16[16];
+                tmem_ld16(tm + lane + kCAcc + d, a16);
+                tmem_wait_ld();
+                out[(size_t)r * d + row] = __uint_as_float(a16[0]);
+            }
+        }
+
+        {  // dV staged in sG, sGN (their last readers are done)
             uint32_t v[32];
             tmem_ld32(tm + lane + kCdV + 32 * half, v);
             tmem_wait_ld();
-            stage_f32(sX, v);
+            stage_f32(sG, v);
         }
         fence_proxy_async_smem();
         tc_fence_before();
@@ -598,7 +638,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        id_q, k > 0);
 #pragma unroll
             for (int k = 0; k < Lg_pad / 16; ++k)  // K = projections
-                mma_ss(tm + kCO, smem_desc(sDU + k * 32, 16, 1024),
+                mma_ss(tm + kCO, smem_desc(sDU + 64 + k * 32, 16, 1024),
                        smem_desc(sKW + kBtT * 128 + k * 2048,
                                  (uint32_t)NR * 128, 1024),
                        id_q, 1);
@@ -607,26 +647,32 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             for (int k = 0; k < kBtT / 16; ++k)  // K = queries
                 mma_ss(tm + kCN, smem_desc(sE + k * 2048, 16384, 1024),
                        smem_desc(sQ + k * 2048, 16384, 1024), id_k, k > 0);
+            mma_commit(&mma_bar);
         }
-        flush_f32(sX, dv, krow_s);  // beside the MMAs, which do not read sX
-        if (!(ok = mma_done(83))) break;
-        if (more) load_qk(tt + 1);  // Q and K's last readers are done
+        flush_f32(sG, dv, krow_s);  // beside the MMAs, which do not read sG
+        // a new head's B and A: their last readers (Gphi, phase 6) are done
+        if (more && (tt + 1) / tiles_per_head != bh)
+            load_sums((int)((tt + 1) / tiles_per_head));
+        cp_async_commit();
+        if (!(ok = mma_wait(&mma_bar, mph, 83))) break;
+        if (more) load_g(tt + 1);  // dV's rows have left sG
         cp_async_commit();
 
         // ------------------------------------------- phase 8: dQ, dK stores
-        {  // dQ staged in sE, dK in sX, sGN (phase 7's MMAs are done)
+        {  // dQ staged in sE, dK over this tile's Q and K rows (phase 7's
+           // MMAs are done; the planes after K stay)
             uint32_t v[32];
             tmem_ld32(tm + lane + kCO + 32 * half, v);
             tmem_wait_ld();
             stage_f32(sE, v);
             tmem_ld32(tm + lane + kCN + 32 * half, v);
             tmem_wait_ld();
-            stage_f32(sX, v);
+            stage_f32(sQ, v);
         }
         tc_fence_before();
         __syncthreads();
         flush_f32(sE, dq, qrow_s);
-        flush_f32(sX, dk, krow_s);
+        flush_f32(sQ, dk, krow_s);
         __syncthreads();  // TMEM and shared memory are reused by the next tile
     }
     cp_async_wait<0>();
@@ -747,6 +793,34 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     auto st8 = [&](uint32_t region, int rr, int chunk, int rows,
                    const float *v) {
         st_shared_bf16x8(region + panel_offset(rr, chunk, rows), v);
+    };
+    // this thread's 32 TMEM columns added into its padded old row
+    auto add_old = [&](uint32_t region, const uint32_t *v) {
+        const uint32_t rb = region + (uint32_t)row * kOldRow + 128 * half;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+            const uint4 a = ld_shared_v4(rb + 16 * q);
+            st_shared_v4(rb + 16 * q,
+                         __float_as_uint(__uint_as_float(a.x) +
+                                         __uint_as_float(v[4 * q])),
+                         __float_as_uint(__uint_as_float(a.y) +
+                                         __uint_as_float(v[4 * q + 1])),
+                         __float_as_uint(__uint_as_float(a.z) +
+                                         __uint_as_float(v[4 * q + 2])),
+                         __float_as_uint(__uint_as_float(a.w) +
+                                         __uint_as_float(v[4 * q + 3])));
+        }
+    };
+    // the tile's 128 rows (contiguous in global memory) written out by
+    // whole rows, two per warp instruction
+    auto flush_rows = [&](uint32_t region, float *dst) {
+        const int c = lane_id & 15;
+#pragma unroll
+        for (int it = 0; it < kBtT / (2 * kBtThreads / 32); ++it) {
+            const int i = (2 * kBtThreads / 32) * it + 2 * warp + (lane_id >> 4);
+            *reinterpret_cast<uint4 *>(dst + (size_t)i * d + 4 * c) =
+                ld_shared_v4(region + (uint32_t)i * kOldRow + 16 * c);
+        }
     };
 
     // cp.async groups, in commit order: K and V of the first tile; then per
@@ -889,24 +963,11 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         if (tt + 1 < t_end) load_v(tt + 1);  // this tile's V is consumed
         cp_async_commit();
 
-        const size_t key = row0 + row;
         {
             uint32_t v[32];
             tmem_ld32(tm + lane + kKdV + 32 * half, v);
             tmem_wait_ld();
-            float4 *o4 = reinterpret_cast<float4 *>(dv + key * d + 32 * half);
-            const float4 *p4 = reinterpret_cast<const float4 *>(
-                smem_raw + (sDVo - smem_u32(smem_raw)) + row * kOldRow +
-                128 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                float4 a = p4[q];
-                a.x += __uint_as_float(v[4 * q]);
-                a.y += __uint_as_float(v[4 * q + 1]);
-                a.z += __uint_as_float(v[4 * q + 2]);
-                a.w += __uint_as_float(v[4 * q + 3]);
-                o4[q] = a;
-            }
+            add_old(sDVo, v);
         }
         {
             float du[2 * L > 16 ? 16 : 2 * L];
@@ -963,27 +1024,18 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                                  (uint32_t)NR * 128, 1024),
                        id_q, k > 0);
         }
+        flush_rows(sDVo, dv + row0 * d);  // dV's sums, beside the MMAs
         if (!(ok = mma_done(92))) break;
         {
             uint32_t v[32];
             tmem_ld32(tm + lane + kKdK + 32 * half, v);
             tmem_wait_ld();
-            float4 *o4 = reinterpret_cast<float4 *>(dk + key * d + 32 * half);
-            const float4 *p4 = reinterpret_cast<const float4 *>(
-                smem_raw + (sDKo - smem_u32(smem_raw)) + row * kOldRow +
-                128 * half);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-                float4 a = p4[q];
-                a.x += __uint_as_float(v[4 * q]);
-                a.y += __uint_as_float(v[4 * q + 1]);
-                a.z += __uint_as_float(v[4 * q + 2]);
-                a.w += __uint_as_float(v[4 * q + 3]);
-                o4[q] = a;
-            }
+            add_old(sDKo, v);
         }
         tc_fence_before();
         __syncthreads();
+        flush_rows(sDKo, dk + row0 * d);
+        __syncthreads();  // the next tile's old rows land in sDVo, sDKo
     }
     cp_async_wait<0>();
     tc_fence_before();
@@ -1003,8 +1055,8 @@ size_t bwd_tc_smem(const Plan &P) {
     const size_t r = (size_t)P.L * 16;
     const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
     auto a1k = [](size_t x) { return (x + 1023) / 1024 * 1024; };
-    return 1024 + 16384 * 2 + a1k((kBtT + lg_pad) * 128) + 16384 + 32768 +
-           a1k(kBtT * r * 2) + a1k(r * 128) + 16384 * 3 + r * 4;
+    return 1024 + 2 * (16384 + a1k((kBtT + lg_pad) * 128)) + 16384 * 4 +
+           32768 + a1k(kBtT * r * 2) + a1k(r * 128) + r * 4;
 }
 
 int bwd_tc_grid(const Plan &P) {
