@@ -261,9 +261,10 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
 
 namespace {
 
-cudaError_t encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t rows,
-                           uint64_t cols, uint32_t box_cols,
-                           uint32_t box_rows, CUtensorMapSwizzle swizzle) {
+cudaError_t encode_2d(CUtensorMap *map, CUtensorMapDataType type,
+                      uint32_t esize, const void *base, uint64_t rows,
+                      uint64_t cols, uint32_t box_cols, uint32_t box_rows,
+                      CUtensorMapSwizzle swizzle) {
     static PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     static std::once_flag once;
     std::call_once(once, [] {
@@ -276,10 +277,10 @@ cudaError_t encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t rows,
     });
     if (!encode) return cudaErrorNotSupported;
     cuuint64_t dims[2] = {cols, rows};
-    cuuint64_t strides[1] = {cols * 2};
+    cuuint64_t strides[1] = {cols * esize};
     cuuint32_t box[2] = {box_cols, box_rows};
     cuuint32_t estr[2] = {1, 1};
-    CUresult r = encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2,
+    CUresult r = encode(map, type, 2,
                         const_cast<void *>(base), dims, strides, box, estr,
                         CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -292,8 +293,16 @@ cudaError_t encode_bf16_2d(CUtensorMap *map, const void *base, uint64_t rows,
 cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
                               uint64_t rows, uint64_t cols,
                               uint32_t box_rows) {
-    return encode_bf16_2d(map, base, rows, cols, 64, box_rows,
-                          CU_TENSOR_MAP_SWIZZLE_128B);
+    return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, rows,
+                     cols, 64, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+cudaError_t make_tma_map_f32(CUtensorMap *map, const void *base,
+                             uint64_t rows, uint64_t cols, uint32_t box_cols,
+                             uint32_t box_rows) {
+    if (box_cols != 32) return cudaErrorInvalidValue;
+    return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, base, rows,
+                     cols, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 cudaError_t make_tma_map_bf16_narrow(CUtensorMap *map, const void *base,
@@ -306,7 +315,8 @@ cudaError_t make_tma_map_bf16_narrow(CUtensorMap *map, const void *base,
         case 64: sw = CU_TENSOR_MAP_SWIZZLE_128B; break;
         default: return cudaErrorInvalidValue;
     }
-    return encode_bf16_2d(map, base, rows, cols, box_cols, box_rows, sw);
+    return encode_2d(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, rows,
+                     cols, box_cols, box_rows, sw);
 }
 
 int set_last_error(int code, const char *fmt, ...) {

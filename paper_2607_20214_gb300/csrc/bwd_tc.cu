@@ -721,22 +721,25 @@ __global__ void k_bwd_sums_reduce(const float *__restrict__ part, int S_seg,
 //   MMA  dK_k = dL/d(W k) W
 //   CUDA dK += dK_k
 // Each key belongs to one tile: plain read-modify-write of dV and dK (the
-// sparse parts were stored by the block kernel before).
+// sparse parts were stored by the block kernel before). A tile's 128 keys
+// are consecutive rows, so K, V and the old dV, dK rows arrive by TMA (the
+// fp32 rows as two boxes of 32 columns in the 128-byte swizzle) and the
+// updated dV, dK rows leave by TMA stores from the same boxes.
 constexpr uint32_t kKU = 0;     // projections [0, 32)
 constexpr uint32_t kKdV = 32;   // phi gB
 constexpr uint32_t kKG = 96;    // V gB^T (r <= 128)
 constexpr uint32_t kKdK = 224;  // dL/du W
-constexpr uint32_t kOldRow = 272; // bytes per staged fp32 dV / dK row
 
 template <int L>
 __global__ void __launch_bounds__(kBtThreads, 1)
-    k_bwd_keys_tc(const uint16_t *__restrict__ kx,
-                  const uint16_t *__restrict__ vx,
+    k_bwd_keys_tc(const __grid_constant__ CUtensorMap tmK,
+                  const __grid_constant__ CUtensorMap tmV,
+                  const __grid_constant__ CUtensorMap tmDK,
+                  const __grid_constant__ CUtensorMap tmDV,
                   const uint16_t *__restrict__ w_bf16,
                   const uint16_t *__restrict__ gBh,
                   const float *__restrict__ gAg, int N, int H, float beta,
                   int tiles_per_head, long total_tiles,
-                  float *__restrict__ dk, float *__restrict__ dv,
                   DeviceStatus *status) {
     constexpr int R = 16, G = 4;
     constexpr int r = L * R, Lg = L * G;
@@ -745,7 +748,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     constexpr int TL = L / 2;
     constexpr int d = kBtD;
     extern __shared__ unsigned char smem_raw[];
-    __shared__ uint64_t mma_bar;
+    __shared__ uint64_t mma_bar, k_bar, v_bar, old_bar;
     __shared__ uint32_t tbase;
     __shared__ int abort_flag;
     volatile int *abort = &abort_flag;
@@ -760,12 +763,12 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     const uint32_t sPhi = sV + 16384;                 // [128 x r]
     const uint32_t sgB = sPhi + align1k(kBtT * r * 2);  // [r x 64]
     const uint32_t sDU = sgB + align1k(r * 128);      // [128 x 64]
-    const uint32_t sAo = sDU + 16384;                 // fp32 gA [r]
-    // fp32 dV, dK rows of the tile as the block kernel left them, rows of
-    // 272 bytes (16-byte pad: a warp's 16-byte reads of 8 rows hit distinct
-    // bank groups)
-    const uint32_t sDVo = sAo + (uint32_t)r * 4;
-    const uint32_t sDKo = sDVo + kBtT * kOldRow;
+    // fp32 dV, dK rows of the tile as the block kernel left them: per
+    // matrix two boxes [128 x 32] of 128-byte rows, the 16-byte chunk c of
+    // row j at chunk c ^ (j & 7)
+    const uint32_t sDVo = sDU + 16384;
+    const uint32_t sDKo = sDVo + 32768;
+    const uint32_t sAo = sDKo + 32768;                 // fp32 gA [r]
     const float *gAs =
         reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
 
@@ -774,6 +777,9 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     if (warp == 0) tmem_alloc(&tbase, 512);
     if (tid == 0) {
         mbar_init(&mma_bar, 1);
+        mbar_init(&k_bar, 1);
+        mbar_init(&v_bar, 1);
+        mbar_init(&old_bar, 1);
         abort_flag = 0;
         fence_mbar_init();
     }
@@ -782,6 +788,12 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     tc_fence_after();
     const uint32_t tm = tbase;
     uint32_t mph = 0;
+    // every thread waits for a copy barrier; all leave if any wait ran out
+    auto copy_wait = [&](uint64_t *bar, long tt, int site) -> bool {
+        const bool ok = mbar_wait_or_abort(bar, (uint32_t)(tt - t_begin) & 1,
+                                           abort, status, site);
+        return __syncthreads_and(ok);
+    };
     auto mma_done = [&](int site) -> bool {
         if (tid == 0) mma_commit(&mma_bar);
         const bool ok = mbar_wait_or_abort(&mma_bar, mph & 1, abort, status,
@@ -794,13 +806,14 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                    const float *v) {
         st_shared_bf16x8(region + panel_offset(rr, chunk, rows), v);
     };
-    // this thread's 32 TMEM columns added into its padded old row
+    // this thread's 32 TMEM columns (box `half`) added into its old row
     auto add_old = [&](uint32_t region, const uint32_t *v) {
-        const uint32_t rb = region + (uint32_t)row * kOldRow + 128 * half;
+        const uint32_t rb = region + 16384u * half + (uint32_t)row * 128;
 #pragma unroll
         for (int q = 0; q < 8; ++q) {
-            const uint4 a = ld_shared_v4(rb + 16 * q);
-            st_shared_v4(rb + 16 * q,
+            const uint32_t a16 = rb + ((uint32_t)(q ^ (row & 7)) << 4);
+            const uint4 a = ld_shared_v4(a16);
+            st_shared_v4(a16,
                          __float_as_uint(__uint_as_float(a.x) +
                                          __uint_as_float(v[4 * q])),
                          __float_as_uint(__uint_as_float(a.y) +
@@ -811,48 +824,28 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                                          __uint_as_float(v[4 * q + 3])));
         }
     };
-    // the tile's 128 rows (contiguous in global memory) written out by
-    // whole rows, two per warp instruction
-    auto flush_rows = [&](uint32_t region, float *dst) {
-        const int c = lane_id & 15;
-#pragma unroll
-        for (int it = 0; it < kBtT / (2 * kBtThreads / 32); ++it) {
-            const int i = (2 * kBtThreads / 32) * it + 2 * warp + (lane_id >> 4);
-            *reinterpret_cast<uint4 *>(dst + (size_t)i * d + 4 * c) =
-                ld_shared_v4(region + (uint32_t)i * kOldRow + 16 * c);
-        }
-    };
-
-    // cp.async groups, in commit order: K and V of the first tile; then per
-    // tile t: [planes, gB, gA on a head change,] old dV, dK of t; K of
-    // t + 1; V of t + 1 (empty past the last tile). "All but the newest
-    // group" is then always the operand about to be used.
     auto tile_row0 = [&](long tt) {
         const int bh = (int)(tt / tiles_per_head);
         return (size_t)bh * N +
                (size_t)(tt - (long)bh * tiles_per_head) * kBtT;
     };
+    // thread 0 issues every TMA copy; the last tile a copy was issued for,
+    // per barrier, lets an aborted CTA drain its copies before it exits
+    long k_last = -1, v_last = -1, old_last = -1;
     auto load_k = [&](long tt) {
-        const size_t r0 = tile_row0(tt);
-        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
-            const int rr = i >> 3, c = i & 7;
-            cp_async16(sKW + panel_offset(rr, c, NR),
-                       kx + (r0 + rr) * d + c * 8);
-        }
+        mbar_expect_tx(&k_bar, 16384);
+        tma_load_2d(sKW, &tmK, 0, (int)tile_row0(tt), &k_bar);
+        k_last = tt;
     };
     auto load_v = [&](long tt) {
-        const size_t r0 = tile_row0(tt);
-        for (int i = tid; i < kBtT * 8; i += kBtThreads) {
-            const int rr = i >> 3, c = i & 7;
-            cp_async16(sV + panel_offset(rr, c, kBtT),
-                       vx + (r0 + rr) * d + c * 8);
-        }
+        mbar_expect_tx(&v_bar, 16384);
+        tma_load_2d(sV, &tmV, 0, (int)tile_row0(tt), &v_bar);
+        v_last = tt;
     };
-    if (t_begin < t_end) {
+    if (tid == 0 && t_begin < t_end) {
         load_k(t_begin);
         load_v(t_begin);
     }
-    cp_async_commit();
 
     int cur_bh = -1;
     bool ok = true;
@@ -877,21 +870,19 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             cp_async_commit();
             cur_bh = bh;
         }
-        // old dV, dK rows of this tile (read back in the epilogues)
-        for (int i = tid; i < kBtT * 16; i += kBtThreads) {
-            const int rr = i >> 4, c = i & 15;
-            cp_async16(sDVo + rr * kOldRow + c * 16,
-                       dv + (row0 + rr) * d + c * 4);
-            cp_async16(sDKo + rr * kOldRow + c * 16,
-                       dk + (row0 + rr) * d + c * 4);
+        if (tid == 0) {  // old dV, dK rows of this tile (read back later)
+            bulk_wait_read();  // the last tile's stores have read the boxes
+            mbar_expect_tx(&old_bar, 65536);
+            const int y = (int)row0;
+            tma_load_2d(sDVo, &tmDV, 0, y, &old_bar);
+            tma_load_2d(sDVo + 16384, &tmDV, 32, y, &old_bar);
+            tma_load_2d(sDKo, &tmDK, 0, y, &old_bar);
+            tma_load_2d(sDKo + 16384, &tmDK, 32, y, &old_bar);
+            old_last = tt;
         }
-        cp_async_commit();
-        if (new_head)
-            cp_async_wait<0>();
-        else
-            cp_async_wait<1>();  // K and V of this tile
+        cp_async_wait<0>();  // planes, gB, gA on a head change
         fence_proxy_async_smem();
-        __syncthreads();
+        if (!(ok = copy_wait(&k_bar, tt, 93))) break;  // K of this tile
 
         // projections U = K W^T
         if (tid == 0) {
@@ -904,8 +895,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        k > 0);
         }
         if (!(ok = mma_done(90))) break;
-        if (tt + 1 < t_end) load_k(tt + 1);  // this tile's K is consumed
-        cp_async_commit();
+        if (tid == 0 && tt + 1 < t_end) load_k(tt + 1);  // K is consumed
 
         // features of this half's tables
         float u[2 * L > 16 ? 16 : 2 * L];
@@ -938,7 +928,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         }
         fence_proxy_async_smem();
         tc_fence_before();
-        __syncthreads();
+        if (!(ok = copy_wait(&v_bar, tt, 94))) break;  // V of this tile
 
         // dV_k = phi gB, Gphi = V gB^T
         if (tid == 0) {
@@ -958,10 +948,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                        smem_desc(sgB + k * 32, 16, 1024), id_g, k > 0);
         }
         if (!(ok = mma_done(91))) break;
-        cp_async_wait<1>();  // old dV, dK rows of this tile
-        __syncthreads();
-        if (tt + 1 < t_end) load_v(tt + 1);  // this tile's V is consumed
-        cp_async_commit();
+        if (tid == 0 && tt + 1 < t_end) load_v(tt + 1);  // V is consumed
+        if (!(ok = copy_wait(&old_bar, tt, 95))) break;
 
         {
             uint32_t v[32];
@@ -1009,12 +997,15 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             for (int q = 0; q < TL * G / 8; ++q)
                 st8(sDU, row, (half * TL * G) / 8 + q, kBtT, du + 8 * q);
         }
-        fence_proxy_async_smem();
+        fence_proxy_async_smem();  // the dV sums, for the TMA store
         tc_fence_before();
         __syncthreads();
 
         // dK_k = dL/du W
         if (tid == 0) {
+            tma_store_2d(&tmDV, 0, (int)row0, sDVo);
+            tma_store_2d(&tmDV, 32, (int)row0, sDVo + 16384);
+            bulk_commit();
             tc_fence_after();
             const uint32_t id_q = idesc_bf16(128, d, false, true);
 #pragma unroll
@@ -1024,7 +1015,6 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                                  (uint32_t)NR * 128, 1024),
                        id_q, k > 0);
         }
-        flush_rows(sDVo, dv + row0 * d);  // dV's sums, beside the MMAs
         if (!(ok = mma_done(92))) break;
         {
             uint32_t v[32];
@@ -1032,12 +1022,27 @@ __global__ void __launch_bounds__(kBtThreads, 1)
             tmem_wait_ld();
             add_old(sDKo, v);
         }
+        fence_proxy_async_smem();
         tc_fence_before();
         __syncthreads();
-        flush_rows(sDKo, dk + row0 * d);
-        __syncthreads();  // the next tile's old rows land in sDVo, sDKo
+        if (tid == 0) {
+            tma_store_2d(&tmDK, 0, (int)row0, sDKo);
+            tma_store_2d(&tmDK, 32, (int)row0, sDKo + 16384);
+            bulk_commit();
+        }
     }
     cp_async_wait<0>();
+    if (tid == 0) {
+        if (!ok) {  // an abort: the copies issued last may still be landing
+            uint64_t *bars[3] = {&k_bar, &v_bar, &old_bar};
+            const long last[3] = {k_last, v_last, old_last};
+            for (int i = 0; i < 3; ++i)
+                if (last[i] >= 0)
+                    mbar_wait(bars[i], (uint32_t)(last[i] - t_begin) & 1,
+                              status, 96);
+        }
+        bulk_wait_all();  // the last stores are complete
+    }
     tc_fence_before();
     __syncthreads();
     if (warp == 0) tmem_dealloc(tm, 512);
@@ -1126,7 +1131,7 @@ size_t bwd_keys_tc_smem(const Plan &P) {
     const size_t lg_pad = ((size_t)P.L * 4 + 15) / 16 * 16;
     auto a1k = [](size_t x) { return (x + 1023) / 1024 * 1024; };
     return 1024 + a1k((kBtT + lg_pad) * 128) + 16384 + a1k(kBtT * r * 2) +
-           a1k(r * 128) + 16384 + r * 4 + 2 * kBtT * kOldRow;
+           a1k(r * 128) + 16384 + 2 * 32768 + r * 4;
 }
 
 cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
@@ -1140,12 +1145,21 @@ cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = (int)(total < sms ? total : sms);
     const size_t smem = bwd_keys_tc_smem(P);
+    const uint64_t rows = (uint64_t)P.BH * P.N;
+    CUtensorMap tmK, tmV, tmDK, tmDV;
+    cudaError_t e = make_tma_map_bf16(&tmK, k, rows, kBtD, kBtT);
+    if (e == cudaSuccess) e = make_tma_map_bf16(&tmV, v, rows, kBtD, kBtT);
+    if (e == cudaSuccess)
+        e = make_tma_map_f32(&tmDK, dk, rows, kBtD, 32, kBtT);
+    if (e == cudaSuccess)
+        e = make_tma_map_f32(&tmDV, dv, rows, kBtD, 32, kBtT);
+    if (e != cudaSuccess) return e;
     auto launch = [&](auto kern) {
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
-        kern<<<grid, kBtThreads, smem, st>>>(
-            (const uint16_t *)k, (const uint16_t *)v, w_bf16, gBh, gA, P.N,
-            P.H, P.beta, tiles_per_head, total, dk, dv, status);
+        kern<<<grid, kBtThreads, smem, st>>>(tmK, tmV, tmDK, tmDV, w_bf16,
+                                             gBh, gA, P.N, P.H, P.beta,
+                                             tiles_per_head, total, status);
         return cudaGetLastError();
     };
     return P.L == 8 ? launch(k_bwd_keys_tc<8>) : launch(k_bwd_keys_tc<4>);

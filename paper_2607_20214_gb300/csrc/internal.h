@@ -204,7 +204,13 @@ cudaError_t launch_gates(const Plan &P, const elsaa_gate_mlp &m,
 // the encoding is rejected.
 cudaError_t make_tma_map_bf16(CUtensorMap *map, const void *base,
                               uint64_t rows, uint64_t cols, uint32_t box_rows);
-// The same with boxes of box_cols = 16, 32 or 64 columns (32, 64 or 128
+// Row-major fp32 matrix [rows x cols] with boxes of box_cols = 32 columns
+// (128 bytes) x box_rows rows and 128-byte swizzle: the 16-byte chunk c of
+// box row j lands at chunk c ^ (j mod 8).
+cudaError_t make_tma_map_f32(CUtensorMap *map, const void *base,
+                             uint64_t rows, uint64_t cols, uint32_t box_cols,
+                             uint32_t box_rows);
+// The same (bf16) with boxes of box_cols = 16, 32 or 64 columns (32, 64 or 128
 // bytes per row) and the swizzle of that width (32, 64 or 128 bytes): the
 // 16-byte chunk c of box row r lands at chunk c ^ ((r / (8 / (box_cols / 8)))
 // mod (box_cols / 8)).

@@ -337,6 +337,20 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// 2-D tiled TMA store of the box at (x = column, y = row) from shared
+// memory, in this thread's bulk async-group (bulk_commit, then
+// bulk_wait_read before the box is overwritten). x * element size must be
+// a multiple of 16 bytes and neither coordinate negative; the writes of
+// other threads to the box need fence_proxy_async_smem and a barrier first.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, int x,
+                                             int y, uint32_t src) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.global.shared::cta.bulk_group"
+        " [%0, {%1, %2}], [%3];" ::"l"(reinterpret_cast<uint64_t>(map)),
+        "r"(x), "r"(y), "r"(src)
+        : "memory");
+}
+
 // Bulk copy of `bytes` contiguous bytes (16-byte aligned, a multiple of 16)
 // from global to shared memory, completing on an mbarrier.
 __device__ __forceinline__ void bulk_load(uint32_t dst, const void *src,

@@ -170,6 +170,22 @@ def test_tensor_core_backward_shapes():
         compare(wl, g, x, [(0, 0), (0, wl.H - 1)])
 
 
+@pytest.mark.parametrize("L", [4, 8])
+def test_tensor_core_backward_several_tiles_per_cta(L):
+    """260 tiles (26 per head) over the 152 persistent CTAs: 108 CTAs take
+    two tiles, four of them across a head change (tiles 25-26, 51-52,
+    155-156, 181-182), so the second Q/K buffer, the planes kept per
+    buffer, the per-head sums reloaded mid-CTA and the bucket-sum partials
+    of a head split over several CTAs are all exercised; every head is
+    compared."""
+    wl = small("bf16", H=10, N=3328, race_tables=L, seed=31 + L)
+    x = make_inputs(wl)
+    gates, lam = make_gates_lambda(wl, seed=5) if L == 8 else (None, None)
+    g = run_gpu(wl, x, gates, lam)
+    assert g["tc"]
+    compare(wl, g, x, [(0, h) for h in range(wl.H)], gates, lam)
+
+
 @pytest.mark.parametrize("over", [dict(fusion_mode=1), dict(block=32),
                                   dict(d_h=32, race_bits=3, race_tables=6),
                                   dict(block=128, d_h=32, race_tables=2)])
