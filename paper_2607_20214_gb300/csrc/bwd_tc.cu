@@ -57,6 +57,20 @@ __host__ __device__ __forceinline__ long tile_owner(long t, long total,
     return ((t + 1) * grid + total - 1) / total - 1;
 }
 
+// The 16 entries of one table's summary (a 64-byte aligned run in shared
+// memory) in four 16-byte loads.
+__device__ __forceinline__ void load_table16(const float *a, float (&x)[16]) {
+    const float4 *p = reinterpret_cast<const float4 *>(a);
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const float4 w = p[q];
+        x[4 * q] = w.x;
+        x[4 * q + 1] = w.y;
+        x[4 * q + 2] = w.z;
+        x[4 * q + 3] = w.w;
+    }
+}
+
 __device__ __forceinline__ void unpack_bf16x8(const uint4 &u, float *x) {
     const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
@@ -386,9 +400,10 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 phi[rr] = p;
             }
             const int tg = half * TL + t;
+            float at[R];
+            load_table16(Asm + tg * R, at);
 #pragma unroll
-            for (int rr = 0; rr < R; ++rr)
-                denp = fmaf(phi[rr], Asm[tg * R + rr], denp);
+            for (int rr = 0; rr < R; ++rr) denp = fmaf(phi[rr], at[rr], denp);
             st8(sPhi, row, tg * 2, kBtT, phi);
             st8(sPhi, row, tg * 2 + 1, kBtT, phi + 8);
         }
@@ -558,7 +573,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                     bit_factors_fast(u[t * G + b], beta, sp[b], sn[b],
                                      uu[b]);
                 }
-                float s = 0.0f;
+                float s = 0.0f, at[R];
+                load_table16(Asm + tg * R, at);
 #pragma unroll
                 for (int rr = 0; rr < R; ++rr) {
                     float p = 1.0f;
@@ -566,7 +582,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                     for (int b = 0; b < G; ++b)
                         p *= ((rr >> b) & 1) ? sp[b] : sn[b];
                     phi[rr] = p;
-                    gp[rr] = (__uint_as_float(v[rr]) + Asm[tg * R + rr] * gDen) *
+                    gp[rr] = (__uint_as_float(v[rr]) + at[rr] * gDen) *
                              (1.0f / (float)L);
                     s = fmaf(p, gp[rr], s);
                 }
@@ -971,7 +987,8 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                     bit_factors_fast(u[t * G + b], beta, sp[b], sn[b],
                                      uu[b]);
                 }
-                float s = 0.0f;
+                float s = 0.0f, at[R];
+                load_table16(gAs + tg * R, at);
 #pragma unroll
                 for (int rr = 0; rr < R; ++rr) {
                     float p = 1.0f;
@@ -979,7 +996,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                     for (int b = 0; b < G; ++b)
                         p *= ((rr >> b) & 1) ? sp[b] : sn[b];
                     phi[rr] = p;
-                    gp[rr] = __uint_as_float(v[rr]) + gAs[tg * R + rr];
+                    gp[rr] = __uint_as_float(v[rr]) + at[rr];
                     s = fmaf(p, gp[rr], s);
                 }
 #pragma unroll
