@@ -389,47 +389,12 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() {
     asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
-// Bulk prefetch of [src, src + bytes) into L2 (16-byte aligned, bytes a
-// multiple of 16); no completion to wait for.
-__device__ __forceinline__ void prefetch_l2(const void *src, uint32_t bytes) {
-    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(src),
-                 "r"(bytes)
-                 : "memory");
-}
-
 // The mbarrier receives one arrival (not counted in advance) once every
 // cp.async this thread issued so far has completed; the thread goes on.
 __device__ __forceinline__ void cp_async_mbar_arrive(uint64_t *bar) {
     asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(
                      smem_u32(bar))
                  : "memory");
-}
-
-// Gathers `nrows` rows of `cols` bf16 elements (cols % 64 == 0) into the
-// panel layout at `dst` (1024-byte aligned). Row i is read from
-// src + idx[i] * ld (elements). All `nthreads` threads of the group take part.
-__device__ __forceinline__ void gather_rows(uint32_t dst, const uint16_t *src,
-                                            const int32_t *idx, int nrows,
-                                            int cols, size_t ld, int tid,
-                                            int nthreads) {
-    const int chunks = cols >> 3;  // 16-byte chunks per row
-    for (int i = tid; i < nrows * chunks; i += nthreads) {
-        int row = i / chunks, c = i - row * chunks;
-        const uint16_t *g = src + (size_t)idx[row] * ld + c * 8;
-        cp_async16(dst + panel_offset(row, c, nrows), g);
-    }
-}
-
-// Same for contiguous rows [0, nrows) of a row-major matrix.
-__device__ __forceinline__ void load_rows(uint32_t dst, const uint16_t *src,
-                                          int nrows, int cols, size_t ld,
-                                          int tid, int nthreads) {
-    const int chunks = cols >> 3;
-    for (int i = tid; i < nrows * chunks; i += nthreads) {
-        int row = i / chunks, c = i - row * chunks;
-        cp_async16(dst + panel_offset(row, c, nrows), src + (size_t)row * ld +
-                                                          c * 8);
-    }
 }
 
 // One 32-byte global store (a whole sector) of 8 words; `p` 32-byte
@@ -442,7 +407,6 @@ __device__ __forceinline__ void st_global_v8(void *p, const uint32_t (&w)[8]) {
         : "memory");
 }
 
-// Stores 8 fp32 values as 8 bf16 (one 16-byte chunk) at a shared address.
 __device__ __forceinline__ uint4 ld_shared_v4(uint32_t addr) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
@@ -460,6 +424,7 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a,
                  : "memory");
 }
 
+// Stores 8 fp32 values as 8 bf16 (one 16-byte chunk) at a shared address.
 __device__ __forceinline__ void st_shared_bf16x8(uint32_t addr,
                                                  const float *v) {
     uint32_t a, b, c, d;

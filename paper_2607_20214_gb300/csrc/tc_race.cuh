@@ -195,56 +195,6 @@ __device__ __forceinline__ void write_phi_tmem(const float (&sp)[32], int l0,
     }
 }
 
-// Same as write_phi_tmem, but the 32-bucket groups of [lo, hi) go to the
-// column groups col0 + 64 * (gi / 2) + 16 * (gi % 2) of a 128-column TMEM
-// region (gi = group index from lo), i.e. quarters col0 and col0 + 64.
-template <int G>
-__device__ __forceinline__ void write_phi_tmem_q(const float (&sp)[32], int l0,
-                                                 int l1, int r, float scale,
-                                                 int lo, int hi,
-                                                 uint32_t taddr_col0) {
-    constexpr int R = 1 << G;
-    uint32_t buf[16];
-#pragma unroll
-    for (int lt = 0; lt < 32 / G; ++lt) {
-        if (l0 + lt < l1) {
-            uint32_t pk[R / 2];
-            if constexpr (G == 4) {
-                float u[4], w[4];
-                table_uw4(&sp[lt * G], scale, u, w);
-                table_pack4(u, w, pk);
-            } else {
-                float phi[R];
-                table_phi<G>(&sp[lt * G], phi, scale);
-#pragma unroll
-                for (int q = 0; q < R; q += 2)
-                    pk[q >> 1] = pack_bf16x2(phi[q], phi[q + 1]);
-            }
-#pragma unroll
-            for (int q = 0; q < R; q += 2) {
-                const int prel = lt * R + q;
-                const int slot = (prel >> 1) & 15;
-                buf[slot] = pk[q >> 1];
-                const int p = l0 * R + prel;
-                const bool last = p + 2 == r;
-                if (slot == 15 || last) {
-                    if (last) {
-#pragma unroll
-                        for (int z = 0; z < 16; ++z)
-                            if (z > slot) buf[z] = 0u;
-                    }
-                    const int g = p - 2 * slot;
-                    if (g >= lo && g < hi) {
-                        const int gi = (g - lo) >> 5;
-                        tmem_st16(taddr_col0 + 64 * (gi >> 1) + 16 * (gi & 1),
-                                  buf);
-                    }
-                }
-            }
-        }
-    }
-}
-
 // sum over tables t < nt of phi_t . A_t for the tables of one 64-bucket
 // chunk (at most TT of them; per-bit factors sp[t * G ..], A of the chunk's
 // first table at A). Four independent partial sums in acc.
