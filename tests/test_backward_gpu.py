@@ -3,7 +3,11 @@ analytic fp64 gradient on the same seeded inputs.
 
 The permutations come from the GPU forward and must equal the oracle's
 (integer work, bit-exact). Gradients are compared relative to the largest
-reference magnitude of each tensor. The CUDA-core path keeps every operand
+reference magnitude of each tensor, by their relative l2 error, and row by
+row: the relative l2 error of each row on its own scale, 99 % of rows
+within five times the bound (the others are rows whose terms cancel
+under the softmax gradient: such a row is far smaller than its terms, and
+so than their rounding errors). The CUDA-core path keeps every operand
 in fp32 and accumulates over at most b + r terms per element (b <= 128,
 r <= 256): its error stays near 1e-6 of that magnitude; its bound is 1e-3.
 The tensor-core path (bf16 inputs, b = 64, d_h = 64) rounds its MMA
@@ -123,9 +127,21 @@ def compare(wl, g, x, heads, gates=None, lam=None):
         assert np.array_equal(g["perm_k"][b, h].numpy(), r["perm_k"])
         for name in ("dQ", "dK", "dV"):
             ref = r[name]
-            err = np.abs(g[name][b, h].numpy() - ref).max() / np.abs(ref).max()
+            got = g[name][b, h].numpy().astype(np.float64)
+            err = np.abs(got - ref).max() / np.abs(ref).max()
             worst[name] = max(worst.get(name, 0.0), err)
             assert err <= tol, (name, b, h, err)
+            # spread-out errors: relative l2 over the tensor, and per row
+            # (a row on its own scale, so small-magnitude rows are checked
+            # too) for all but the 1 % of rows where the softmax gradient's
+            # cancellation leaves the row much smaller than its terms
+            l2 = np.linalg.norm(got - ref) / np.linalg.norm(ref)
+            assert l2 <= tol, (name, b, h, "rel l2", l2)
+            rn = np.linalg.norm(ref, axis=1)
+            live = rn > 0
+            rows = np.linalg.norm(got - ref, axis=1)[live] / rn[live]
+            q99 = np.quantile(rows, 0.99)
+            assert q99 <= 5 * tol, (name, b, h, "row rel l2 p99", q99)
         ref = r["dgates"]
         err = np.abs(g["dgates"][b, h].numpy() - ref).max() / np.abs(ref).max()
         assert err <= tol, ("dgates", b, h, err)
