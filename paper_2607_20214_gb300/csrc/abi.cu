@@ -175,6 +175,7 @@ int make_plan(const elsaa_params *p, Plan *P, const char **msg) {
         return bad(ELSAA_ERR_UNSUPPORTED, "B * H * N must fit in int32");
 
     Plan &Q = *P;
+    Q = Plan{};
     Q.B = p->B;
     Q.H = p->H;
     Q.N = p->N;
