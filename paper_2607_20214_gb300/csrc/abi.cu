@@ -759,7 +759,7 @@ struct BwdPlan {
     Plan P;    // forward geometry with CUDA-core RACE chunking
     Plan Pf;   // the forward's own plan (tensor-core key summaries if bf16)
     size_t off_status, off_part, off_A, off_B, off_gA, off_gB, off_gnum,
-        off_gden, off_W, off_Bh, off_gBh, total;
+        off_gden, off_W, off_Bh, total;
     bool tc;   // tensor-core block kernel (bf16 operands)
 };
 
@@ -804,10 +804,12 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     off = align_up(off + (size_t)P.BH * P.r * sizeof(float), 256);
     Bp->off_B = off;
     off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(float), 256);
-    Bp->off_gA = off;
-    off = align_up(off + (size_t)P.BH * P.r * sizeof(float), 256);
+    Bp->off_gA = off;  // gA, gB: CUDA-core path (the tensor-core key
+                       // kernel sums the partials itself)
+    if (!Bp->tc) off = align_up(off + (size_t)P.BH * P.r * sizeof(float), 256);
     Bp->off_gB = off;
-    off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(float), 256);
+    if (!Bp->tc)
+        off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(float), 256);
     Bp->off_gnum = off;
     if (!Bp->tc) off = align_up(off + BHN * P.d * sizeof(float), 256);
     Bp->off_gden = off;
@@ -815,10 +817,6 @@ int make_bwd_plan(const elsaa_params *p, BwdPlan *Bp, const char **msg) {
     Bp->off_W = off;
     off = align_up(off + (size_t)P.H * P.Lg_pad * P.d * sizeof(uint16_t), 256);
     Bp->off_Bh = off;
-    if (Bp->tc)
-        off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(uint16_t),
-                       256);
-    Bp->off_gBh = off;
     if (Bp->tc)
         off = align_up(off + (size_t)P.BH * P.r * P.d * sizeof(uint16_t),
                        256);
@@ -1062,14 +1060,7 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
                            }),
                            "bwd_block");
     }
-    uint16_t *gBhw = Bp.tc ? (uint16_t *)(ws + Bp.off_gBh) : nullptr;
-    if (Bp.tc) {
-        ELSAA_CHECK_LAUNCH(timed("bwd_sums_reduce", st, [&] {
-                               return launch_bwd_sums_reduce(Pf, part, gBhw,
-                                                             gA, st);
-                           }),
-                           "bwd_sums_reduce");
-    } else {
+    if (!Bp.tc) {
         ELSAA_CHECK_LAUNCH(timed("bwd_race_sums", st, [&] {
                                return launch_race_partial_weighted(
                                    P, q, gnum, gden, w_race, part, st);
@@ -1085,8 +1076,8 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
         ELSAA_CHECK_LAUNCH(timed("bwd_keys_tc", st, [&] {
                                return launch_bwd_keys_tc(
                                    Pf, k, v,
-                                   (const uint16_t *)(ws + Bp.off_W), gBhw, gA,
-                                   dk, dv, status, st);
+                                   (const uint16_t *)(ws + Bp.off_W), part, dk,
+                                   dv, status, st);
                            }),
                            "bwd_keys_tc");
     } else {

@@ -23,8 +23,8 @@
 // Every key belongs to exactly one block, so dV, dK (sparse part) are
 // plain stores; the RACE key side adds to them afterwards. The per-head
 // sums gB, gA that the key side needs leave the kernel as one partial per
-// (head, CTA that worked on the head), summed in a fixed order by
-// k_bwd_sums_reduce.
+// (head, CTA that worked on the head); the key-side kernel sums them in a
+// fixed order when it starts on the head.
 // Operands in bf16 (relative rounding 2^-9), accumulation in fp32.
 #include "device_common.cuh"
 #include "tc_common.cuh"
@@ -49,13 +49,6 @@ constexpr uint32_t kCN = 224;    // phi B, then dK
 constexpr uint32_t kCG = 160;    // gNum B^T (r <= 128 columns) between them
 constexpr uint32_t kCdV = 288;   // E^T X
 constexpr uint32_t kCAcc = 352;  // [gB | gA] of the current head, d + 16
-
-// The CTA (of `grid` over `total` tiles, CTA c taking tiles
-// [total c / grid, total (c + 1) / grid)) that works on tile t.
-__host__ __device__ __forceinline__ long tile_owner(long t, long total,
-                                                    long grid) {
-    return ((t + 1) * grid + total - 1) / total - 1;
-}
 
 // The 16 entries of one table's summary (a 64-byte aligned run in shared
 // memory) in four 16-byte loads.
@@ -608,7 +601,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
         for (int q = 0; q < 4; ++q) st8(sE, row, (c0 >> 3) + q, kBtT, dz + 8 * q);
         if (seg_last && row < r) {  // this CTA's share of the head's sums
             const long j = (long)blockIdx.x -
-                           tile_owner((long)bh * tiles_per_head, total_tiles,
+                           range_owner((long)bh * tiles_per_head, total_tiles,
                                       gridDim.x);
             float *out =
                 part + ((size_t)bh * S_seg + j) * ((size_t)r * d + r);
@@ -697,38 +690,10 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     if (warp == 0) tmem_dealloc(tm, 512);
 }
 
-// gB, gA of each head: the partials of the CTAs that worked on the head,
-// summed in CTA order, times 1 / L; gB leaves as bf16 (the key side's MMA
-// operand), gA as fp32. Grid (ceil((r d + r) / 256), B*H).
-__global__ void k_bwd_sums_reduce(const float *__restrict__ part, int S_seg,
-                                  int r, int d, int L, int tiles_per_head,
-                                  long total, int grid,
-                                  uint16_t *__restrict__ gBh,
-                                  float *__restrict__ gA) {
-    const int bh = blockIdx.y;
-    const size_t per = (size_t)r * d + r;
-    const long c0 = tile_owner((long)bh * tiles_per_head, total, grid);
-    const long c1 =
-        tile_owner((long)(bh + 1) * tiles_per_head - 1, total, grid);
-    const float inv = 1.0f / (float)L;
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < per;
-         i += (size_t)gridDim.x * blockDim.x) {
-        const float *p = part + (size_t)bh * S_seg * per + i;
-        float s = 0.f;
-        for (long c = 0; c <= c1 - c0; ++c) s += p[(size_t)c * per];
-        s *= inv;
-        if (i < (size_t)r * d) {
-            const __nv_bfloat16 hb = __float2bfloat16_rn(s);
-            gBh[(size_t)bh * r * d + i] = *reinterpret_cast<const uint16_t *>(&hb);
-        } else {
-            gA[(size_t)bh * r + (i - (size_t)r * d)] = s;
-        }
-    }
-}
-
 // RACE key side of the backward on tensor cores, per 128-key tile (keys in
 // their original order): with gB = sum_i phi(Q_i) gNum_i^T / L and
-// gA = sum_i phi(Q_i) dL/dDen_i / L (bf16 / fp32, per head),
+// gA = sum_i phi(Q_i) dL/dDen_i / L (bf16 / fp32, per head; summed from the
+// block kernel's partials, in CTA order, whenever a CTA starts on a head),
 //   MMA  U = K W^T                         projections
 //   CUDA phi(K)
 //   MMA  dV_k = phi gB,  Gphi = V gB^T
@@ -753,10 +718,9 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                   const __grid_constant__ CUtensorMap tmDK,
                   const __grid_constant__ CUtensorMap tmDV,
                   const uint16_t *__restrict__ w_bf16,
-                  const uint16_t *__restrict__ gBh,
-                  const float *__restrict__ gAg, int N, int H, float beta,
-                  int tiles_per_head, long total_tiles,
-                  DeviceStatus *status) {
+                  const float *__restrict__ part, int S_seg, int blk_grid,
+                  int N, int H, float beta, int tiles_per_head,
+                  long total_tiles, DeviceStatus *status) {
     constexpr int R = 16, G = 4;
     constexpr int r = L * R, Lg = L * G;
     constexpr int Lg_pad = (Lg + 15) / 16 * 16;
@@ -785,8 +749,7 @@ __global__ void __launch_bounds__(kBtThreads, 1)
     const uint32_t sDVo = sDU + 16384;
     const uint32_t sDKo = sDVo + 32768;
     const uint32_t sAo = sDKo + 32768;                 // fp32 gA [r]
-    const float *gAs =
-        reinterpret_cast<const float *>(smem_raw + (sAo - smem_u32(smem_raw)));
+    float *gAs = reinterpret_cast<float *>(smem_raw + (sAo - smem_u32(smem_raw)));
 
     const long t_begin = total_tiles * blockIdx.x / gridDim.x;
     const long t_end = total_tiles * (blockIdx.x + 1) / gridDim.x;
@@ -876,13 +839,58 @@ __global__ void __launch_bounds__(kBtThreads, 1)
                 cp_async16(sKW + panel_offset(kBtT + rr, c, NR),
                            w_bf16 + ((size_t)h * Lg_pad + rr) * d + c * 8);
             }
-            for (int i = tid; i < r * 8; i += kBtThreads) {
-                const int rr = i >> 3, c = i & 7;
-                cp_async16(sgB + panel_offset(rr, c, r),
-                           gBh + ((size_t)bh * r + rr) * d + c * 8);
+            // gB (bf16 panel) and gA: the block kernel's partials of the
+            // CTAs that worked on the head, summed in CTA order, times 1 / L
+            const size_t per = (size_t)r * d + r;
+            const float *p0 = part + (size_t)bh * S_seg * per;
+            const int nparts =
+                (int)(range_owner((long)(bh + 1) * tiles_per_head - 1,
+                                  total_tiles, blk_grid) -
+                      range_owner((long)bh * tiles_per_head, total_tiles,
+                                  blk_grid) +
+                      1);
+            // each thread: NC 16-byte chunks of gB (8 values each) and at
+            // most one entry of gA, all of one partial's loads in flight at
+            // once, partials in CTA order
+            constexpr int NC = r * 8 / kBtThreads;
+            static_assert(NC * kBtThreads == r * 8 && r <= kBtThreads,
+                          "gB chunks and gA entries spread evenly");
+            const float inv = 1.0f / (float)L;
+            float sum[NC][8] = {};
+            float sa = 0.f;
+            for (int j = 0; j < nparts; ++j) {
+                const float *pj = p0 + (size_t)j * per;
+                float4 a[NC], b2[NC];
+#pragma unroll
+                for (int q = 0; q < NC; ++q) {
+                    const int i = tid + q * kBtThreads;
+                    const float4 *src = reinterpret_cast<const float4 *>(
+                        pj + (size_t)(i >> 3) * d + (i & 7) * 8);
+                    a[q] = src[0];
+                    b2[q] = src[1];
+                }
+                const float av = tid < r ? pj[(size_t)r * d + tid] : 0.f;
+#pragma unroll
+                for (int q = 0; q < NC; ++q) {
+                    sum[q][0] += a[q].x;
+                    sum[q][1] += a[q].y;
+                    sum[q][2] += a[q].z;
+                    sum[q][3] += a[q].w;
+                    sum[q][4] += b2[q].x;
+                    sum[q][5] += b2[q].y;
+                    sum[q][6] += b2[q].z;
+                    sum[q][7] += b2[q].w;
+                }
+                sa += av;
             }
-            for (int i = tid; i < r / 4; i += kBtThreads)
-                cp_async16(sAo + 16 * i, gAg + (size_t)bh * r + 4 * i);
+#pragma unroll
+            for (int q = 0; q < NC; ++q) {
+                const int i = tid + q * kBtThreads;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) sum[q][e] *= inv;
+                st8(sgB, i >> 3, i & 7, r, sum[q]);
+            }
+            if (tid < r) gAs[tid] = sa * inv;
             cp_async_commit();
             cur_bh = bh;
         }
@@ -1092,8 +1100,8 @@ int bwd_tc_segments(const Plan &P) {
     const long grid = bwd_tc_grid(P);
     long most = 1;
     for (long bh = 0; bh < P.BH; ++bh) {
-        const long n = tile_owner((bh + 1) * T - 1, total, grid) -
-                       tile_owner(bh * T, total, grid) + 1;
+        const long n = range_owner((bh + 1) * T - 1, total, grid) -
+                       range_owner(bh * T, total, grid) + 1;
         if (n > most) most = n;
     }
     return (int)most;
@@ -1127,18 +1135,6 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
     return P.L == 8 ? launch(k_bwd_block_tc<8>) : launch(k_bwd_block_tc<4>);
 }
 
-cudaError_t launch_bwd_sums_reduce(const Plan &P, const float *part,
-                                   uint16_t *gBh, float *gA, cudaStream_t st) {
-    const int tiles_per_head = P.N / kBtT;
-    const long total = (long)tiles_per_head * P.BH;
-    const int per = P.r * P.d + P.r;
-    dim3 grid((per + 255) / 256, P.BH);
-    k_bwd_sums_reduce<<<grid, 256, 0, st>>>(part, bwd_tc_segments(P), P.r,
-                                            P.d, P.L, tiles_per_head, total,
-                                            bwd_tc_grid(P), gBh, gA);
-    return cudaGetLastError();
-}
-
 }  // namespace elsaa
 
 namespace elsaa {
@@ -1152,9 +1148,9 @@ size_t bwd_keys_tc_smem(const Plan &P) {
 }
 
 cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
-                               const uint16_t *w_bf16, const uint16_t *gBh,
-                               const float *gA, float *dk, float *dv,
-                               DeviceStatus *status, cudaStream_t st) {
+                               const uint16_t *w_bf16, const float *part,
+                               float *dk, float *dv, DeviceStatus *status,
+                               cudaStream_t st) {
     const int tiles_per_head = P.N / kBtT;
     const long total = (long)tiles_per_head * P.BH;
     int dev = 0, sms = 148;
@@ -1162,6 +1158,7 @@ cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const int grid = (int)(total < sms ? total : sms);
     const size_t smem = bwd_keys_tc_smem(P);
+    const int S_seg = bwd_tc_segments(P), blk_grid = bwd_tc_grid(P);
     const uint64_t rows = (uint64_t)P.BH * P.N;
     CUtensorMap tmK, tmV, tmDK, tmDV;
     cudaError_t e = make_tma_map_bf16(&tmK, k, rows, kBtD, kBtT);
@@ -1175,8 +1172,9 @@ cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
         cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
         kern<<<grid, kBtThreads, smem, st>>>(tmK, tmV, tmDK, tmDV, w_bf16,
-                                             gBh, gA, P.N, P.H, P.beta,
-                                             tiles_per_head, total, status);
+                                             part, S_seg, blk_grid, P.N, P.H,
+                                             P.beta, tiles_per_head, total,
+                                             status);
         return cudaGetLastError();
     };
     return P.L == 8 ? launch(k_bwd_keys_tc<8>) : launch(k_bwd_keys_tc<4>);

@@ -31,6 +31,12 @@ constexpr int kDevPermRange = 2;     // a permutation entry fell outside [0, N)
 constexpr int kDevWaitTimeout = 3;   // a bounded mbarrier wait ran out
 constexpr int kDevTmem = 4;          // tensor-memory allocation failed
 
+// The CTA (of `grid` over `total` work items, CTA c taking items
+// [total c / grid, total (c + 1) / grid)) that works on item t.
+__host__ __device__ inline long range_owner(long t, long total, long grid) {
+    return ((t + 1) * grid + total - 1) / total - 1;
+}
+
 // Resolved problem geometry and workspace layout (all offsets in bytes).
 struct Plan {
     int B, H, N, d, BH;
@@ -137,7 +143,7 @@ cudaError_t launch_bwd_keys(const Plan &P, const void *k, const void *v,
 
 // Tensor-core backward (bwd_tc.cu): the block kernel also sums gB, gA per
 // head into bwd_tc_segments(P) partials per head (layout of the RACE chunk
-// partials), which launch_bwd_sums_reduce folds into bf16 gB and fp32 gA.
+// partials), which the key-side kernel adds up when it starts on a head.
 bool bwd_tc_supported(const Plan &P);
 size_t bwd_tc_smem(const Plan &P);
 int bwd_tc_grid(const Plan &P);
@@ -145,8 +151,6 @@ int bwd_tc_grid(const Plan &P);
 cudaError_t launch_bf16_image(const float *x, uint16_t *y, size_t n,
                               cudaStream_t st);
 int bwd_tc_segments(const Plan &P);
-cudaError_t launch_bwd_sums_reduce(const Plan &P, const float *part,
-                                   uint16_t *gBh, float *gA, cudaStream_t st);
 cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 const void *v, const void *d_o,
                                 const uint16_t *w_bf16, const uint16_t *Bh,
@@ -159,9 +163,9 @@ cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
 
 size_t bwd_keys_tc_smem(const Plan &P);
 cudaError_t launch_bwd_keys_tc(const Plan &P, const void *k, const void *v,
-                               const uint16_t *w_bf16, const uint16_t *gBh,
-                               const float *gA, float *dk, float *dv,
-                               DeviceStatus *status, cudaStream_t st);
+                               const uint16_t *w_bf16, const float *part,
+                               float *dk, float *dv, DeviceStatus *status,
+                               cudaStream_t st);
 
 // Causal variant (causal.cu).
 bool causal_tc_supported(const Plan &P, int n_leaf);

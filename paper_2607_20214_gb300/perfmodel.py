@@ -136,7 +136,8 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
                   (2 * N * r * (d + 1) if tc else 0))
         simt = not tc
     elif kernel.startswith("bwd_keys"):
-        # reads K, V, adds into dK, dV (fp32 read + write)
+        # reads K, V, adds into dK, dV (fp32 read + write); the tensor-core
+        # kernel also reads the block kernel's gB, gA partials (about 1 %)
         by = H * (2 * N * d * e + 4 * N * d * 4)
         fl = H * (4 * N * r * d + 4 * N * d * Lg)
         simt = not kernel.endswith("_tc")
@@ -170,10 +171,6 @@ def kernel_work(wl: Workload, kernel: str) -> dict:
         by = H * (2 * N * d * e + nc * r * (d * 2 + 4))
         fl = H * (2 * N * r * (d + 16) + 2 * N * d * Lg)
         simt = False
-    elif kernel.startswith("bwd_sums_reduce"):
-        by = H * r * (d + 1) * 4
-        fl = 0
-        simt = True
     elif kernel.startswith("bwd_race_sums"):
         by = H * (N * d * e + N * d * 4)
         fl = H * (2 * N * r * d + 2 * N * r + 2 * N * d * Lg)
