@@ -1006,7 +1006,17 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
     const Plan &Pf = Bp.Pf;
     uint16_t *Wbf = (uint16_t *)(ws + Bp.off_W);
     uint16_t *Bhw = Bp.tc ? (uint16_t *)(ws + Bp.off_Bh) : nullptr;
-    if (Pf.impl == 2)
+    const size_t nB = (size_t)P.BH * P.r * P.d;
+    // the bf16 planes and, with saved summaries, the bf16 image of B: one
+    // launch where both are needed
+    const bool images = Pf.impl == 2 && race_A && Bhw && nB % 4 == 0;
+    if (images)
+        ELSAA_CHECK_LAUNCH(timed("planes_and_image", st, [&] {
+                               return launch_planes_and_image(
+                                   Pf, w_race, Wbf, race_B, Bhw, nB, st);
+                           }),
+                           "planes_and_image");
+    else if (Pf.impl == 2)
         ELSAA_CHECK_LAUNCH(timed("prep_planes", st, [&] {
                                return launch_prep_planes(Pf, w_race, Wbf, st);
                            }),
@@ -1014,11 +1024,10 @@ extern "C" int elsaa_backward(const elsaa_params *params, const void *q,
     if (race_A) {
         A = const_cast<float *>(race_A);
         Bm = const_cast<float *>(race_B);
-        if (Bhw)
+        if (Bhw && !images)
             ELSAA_CHECK_LAUNCH(timed("bf16_image", st, [&] {
-                                   return launch_bf16_image(
-                                       race_B, Bhw,
-                                       (size_t)P.BH * P.r * P.d, st);
+                                   return launch_bf16_image(race_B, Bhw, nB,
+                                                            st);
                                }),
                                "bf16_image");
     } else {

@@ -150,6 +150,11 @@ int bwd_tc_grid(const Plan &P);
 // bf16 copy (round to nearest even) of n fp32 values.
 cudaError_t launch_bf16_image(const float *x, uint16_t *y, size_t n,
                               cudaStream_t st);
+// launch_prep_planes and launch_bf16_image in one launch (n a multiple of
+// 4, x 16-byte and y 8-byte aligned; cudaErrorInvalidValue otherwise).
+cudaError_t launch_planes_and_image(const Plan &P, const float *w_race,
+                                    uint16_t *w_bf16, const float *x,
+                                    uint16_t *y, size_t n, cudaStream_t st);
 int bwd_tc_segments(const Plan &P);
 cudaError_t launch_bwd_block_tc(const Plan &P, const void *q, const void *k,
                                 const void *v, const void *d_o,
